@@ -1,0 +1,28 @@
+import os
+import sys
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+
+def pytest_configure(config):
+    config.addinivalue_line("markers", "gpu: needs a GB300 and the built CUDA library")
+
+
+def micro_config(**overrides):
+    """A very small model for fast CPU tests of the oracle's logic."""
+    from paper_2609_34608_gb300.inputs import METHOD_DEFAULTS
+    cfg = dict(METHOD_DEFAULTS)
+    cfg.update(n_layers=3, d_model=16, n_heads=2, mlp_ratio=4, n_obs=4, n_video=6,
+               video_dim=4, n_action=5, action_dim=3, n_steps=4, precision="fp32", batch=1,
+               tr_entry_stage=2, tr_retain_stage=-1, rr_policy=0, rr_q=0, rr_s=0, rr_e=0)
+    cfg.update(overrides)
+    return cfg
+
+
+@pytest.fixture
+def micro():
+    return micro_config

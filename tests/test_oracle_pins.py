@@ -1,0 +1,458 @@
+"""Pins of the CPU oracle against what the paper and the mathematics fix.
+
+Each test ties one oracle function to something other than itself: a value printed in the
+paper (tests/golden/), a closed form, an invariant, a library routine computing the same
+textbook operation, or brute force on tiny inputs.
+"""
+import math
+import os
+
+import numpy as np
+import pytest
+import torch
+import torch.nn.functional as TF
+
+from oracle import wam_oracle as O
+from paper_2609_34608_gb300 import inputs as I
+from tests.conftest import micro_config
+
+GOLDEN = os.path.join(os.path.dirname(__file__), "golden")
+
+
+def _golden(name):
+    rows = []
+    with open(os.path.join(GOLDEN, name)) as f:
+        for line in f:
+            line = line.strip()
+            if line and not line.startswith("#"):
+                rows.append(line.split())
+    return rows
+
+
+def _setup(cfg_dict, seed=0, std=0.02):
+    W = I.make_weights(cfg_dict, seed=seed, std=std)
+    return W, O.OracleConfig.from_dict(cfg_dict)
+
+
+# ----------------------------------------------------------------------------- schedule
+def test_schedule_matches_fastwam_values_printed_in_paper():
+    for n_steps, shift, stage, sigma in _golden("fastwam_schedule.txt"):
+        sig = O.schedule(int(n_steps), float(shift))
+        assert round(float(sig[int(stage)]), 5) == pytest.approx(float(sigma), abs=0.5e-5)
+
+
+def test_linear_schedule_endpoints():
+    sig = O.schedule(8, 1.0)
+    assert sig[0] == 1.0 and sig[-1] == 0.0
+    assert np.allclose(np.diff(sig), -1.0 / 8)
+
+
+# ----------------------------------------------------------------------------- Euler
+@pytest.mark.parametrize("shift", [1.0, 5.0])
+def test_euler_constant_field_closed_form(shift):
+    rng = np.random.default_rng(3)
+    x0, v = rng.standard_normal(11), rng.standard_normal(11)
+    xs = O.euler_integrate(x0, O.schedule(10, shift), lambda x, s: v)
+    # sum of (sigma_{k+1} - sigma_k) telescopes to sigma_K - sigma_0 = -1
+    assert np.allclose(xs[-1], x0 - v, atol=1e-14)
+
+
+def test_euler_linear_field_product_form():
+    sig = O.schedule(6, 1.0)
+    a = 0.7
+    xs = O.euler_integrate(np.array([2.0]), sig, lambda x, s: a * x)
+    expect = 2.0 * np.prod([1.0 + a * (sig[k + 1] - sig[k]) for k in range(6)])
+    assert xs[-1][0] == pytest.approx(expect, rel=1e-14)
+
+
+# ----------------------------------------------------------------------------- attention
+def _attention_bruteforce(q, k, v, n_heads):
+    n, d = len(q), len(q[0])
+    dh = d // n_heads
+    out = [[0.0] * d for _ in range(n)]
+    for h in range(n_heads):
+        c0 = h * dh
+        for i in range(n):
+            logits = []
+            for j in range(n):
+                s = 0.0
+                for c in range(dh):
+                    s += q[i][c0 + c] * k[j][c0 + c]
+                logits.append(s / math.sqrt(dh))
+            mx = max(logits)
+            w = [math.exp(x - mx) for x in logits]
+            z = sum(w)
+            for c in range(dh):
+                out[i][c0 + c] = sum(w[j] * v[j][c0 + c] for j in range(n)) / z
+    return np.array(out)
+
+
+def test_attention_vs_bruteforce_loops():
+    rng = np.random.default_rng(0)
+    q, k, v = (rng.standard_normal((7, 8)) for _ in range(3))
+    ref = _attention_bruteforce(q.tolist(), k.tolist(), v.tolist(), 2)
+    assert np.allclose(O.attention(q, k, v, 2), ref, atol=1e-13)
+
+
+def test_attention_vs_torch_sdpa():
+    rng = np.random.default_rng(1)
+    n, d, H = 13, 24, 3
+    q, k, v = (rng.standard_normal((n, d)) for _ in range(3))
+    t = lambda a: torch.from_numpy(a).reshape(n, H, d // H).permute(1, 0, 2)
+    ref = TF.scaled_dot_product_attention(t(q), t(k), t(v)).permute(1, 0, 2).reshape(n, d)
+    assert np.allclose(O.attention(q, k, v, H), ref.numpy(), atol=1e-12)
+
+
+def test_attention_zero_queries_average_values():
+    rng = np.random.default_rng(2)
+    k, v = rng.standard_normal((5, 6)), rng.standard_normal((5, 6))
+    out = O.attention(np.zeros((5, 6)), k, v, 3)
+    assert np.allclose(out, np.broadcast_to(v.mean(axis=0), (5, 6)), atol=1e-14)
+
+
+# ----------------------------------------------------------------------------- elementwise
+def test_layer_norm_vs_torch():
+    x = np.random.default_rng(4).standard_normal((5, 33)) * 3 + 1
+    ref = TF.layer_norm(torch.from_numpy(x), (33,), eps=1e-6).numpy()
+    assert np.allclose(O.layer_norm(x), ref, atol=1e-12)
+
+
+def test_gelu_tanh_vs_torch_and_known_value():
+    x = np.linspace(-6, 6, 101)
+    ref = TF.gelu(torch.from_numpy(x), approximate="tanh").numpy()
+    assert np.allclose(O.gelu_tanh(x), ref, atol=1e-14)
+    assert O.gelu_tanh(np.array(1.0)) == pytest.approx(0.8411919906082768, abs=1e-15)
+
+
+def test_silu_vs_torch():
+    x = np.linspace(-8, 8, 77)
+    assert np.allclose(O.silu(x), TF.silu(torch.from_numpy(x)).numpy(), atol=1e-15)
+
+
+def test_timestep_features_at_zero_and_one_frequency():
+    e0 = O.timestep_features(0.0)
+    assert e0.shape == (256,) and np.all(e0[:128] == 1.0) and np.all(e0[128:] == 0.0)
+    e = O.timestep_features(0.37)
+    assert e[0] == pytest.approx(math.cos(370.0)) and e[128] == pytest.approx(math.sin(370.0))
+    assert e[64] == pytest.approx(math.cos(370.0 * 10000 ** (-0.5)))
+
+
+# ----------------------------------------------------------------------------- DiT layer
+def _torch_block(W, cfg, h, l, mod):
+    """The same adaLN-DiT block from torch library modules (float64)."""
+    d = cfg.d_model
+    p = f"layers.{l}."
+    g = lambda n: torch.from_numpy(np.asarray(W[p + n], dtype=np.float64))
+    mha = torch.nn.MultiheadAttention(d, cfg.n_heads, batch_first=True, dtype=torch.float64)
+    with torch.no_grad():
+        mha.in_proj_weight.copy_(g("qkv_w").T)
+        mha.in_proj_bias.copy_(g("qkv_b"))
+        mha.out_proj.weight.copy_(g("out_w").T)
+        mha.out_proj.bias.copy_(g("out_b"))
+        m = torch.from_numpy(mod)
+        ht = torch.from_numpy(h)[None]
+        x = TF.layer_norm(ht, (d,), eps=1e-6) * (1 + m[1]) + m[0]
+        a, _ = mha(x, x, x, need_weights=False)
+        ht = ht + m[2] * a
+        x = TF.layer_norm(ht, (d,), eps=1e-6) * (1 + m[4]) + m[3]
+        u = TF.gelu(TF.linear(x, g("up_w").T, g("up_b")), approximate="tanh")
+        ht = ht + m[5] * TF.linear(u, g("down_w").T, g("down_b"))
+    return ht[0].numpy()
+
+
+def test_dit_layer_vs_torch_modules():
+    cfgd = micro_config(d_model=24, n_heads=3)
+    W, cfg = _setup(cfgd, std=0.2)
+    rng = np.random.default_rng(5)
+    h = rng.standard_normal((cfg.n_tokens, cfg.d_model))
+    mod = rng.standard_normal((6, cfg.d_model)) * 0.5
+    out = O.dit_layer(W, cfg, h, 1, mod)
+    assert np.allclose(out, _torch_block(W, cfg, h, 1, mod), atol=1e-11)
+
+
+def test_dit_layer_zero_gates_is_identity():
+    W, cfg = _setup(micro_config(), std=0.3)
+    rng = np.random.default_rng(6)
+    h = rng.standard_normal((cfg.n_tokens, cfg.d_model))
+    mod = rng.standard_normal((6, cfg.d_model))
+    mod[2] = 0.0
+    mod[5] = 0.0
+    assert np.array_equal(O.dit_layer(W, cfg, h, 0, mod), h)
+
+
+def test_conditioning_vs_torch_linear_chain():
+    W, cfg = _setup(micro_config(), std=0.3)
+    mods, fin = O.conditioning(W, cfg, 0.6)
+    g = lambda n: torch.from_numpy(np.asarray(W[n], dtype=np.float64))
+    e = torch.from_numpy(O.timestep_features(0.6))
+    c = TF.linear(TF.silu(TF.linear(e, g("t_w1").T, g("t_b1"))), g("t_w2").T, g("t_b2"))
+    m2 = TF.linear(TF.silu(c), g("layers.2.ada_w").T, g("layers.2.ada_b")).reshape(6, -1)
+    assert np.allclose(mods[2], m2.numpy(), atol=1e-13)
+    f = TF.linear(TF.silu(c), g("final_ada_w").T, g("final_ada_b")).reshape(2, -1)
+    assert np.allclose(fin, f.numpy(), atol=1e-13)
+
+
+def test_velocity_is_token_permutation_equivariant_without_positions():
+    cfgd = micro_config()
+    W, cfg = _setup(cfgd, std=0.3)
+    W["pos"][:] = 0.0
+    rng = np.random.default_rng(7)
+    x = rng.standard_normal(cfg.traj_len)
+    obs = rng.standard_normal((cfg.n_obs, cfg.d_model))
+    v = O.velocity(W, cfg, x, obs, 0.4)
+    pv = rng.permutation(cfg.n_video)
+    pa = rng.permutation(cfg.n_action)
+    xv = x[:cfg.video_len].reshape(cfg.n_video, -1)[pv].reshape(-1)
+    xa = x[cfg.video_len:].reshape(cfg.n_action, -1)[pa].reshape(-1)
+    po = rng.permutation(cfg.n_obs)
+    v2 = O.velocity(W, cfg, np.concatenate([xv, xa]), obs[po], 0.4)
+    vv = v[:cfg.video_len].reshape(cfg.n_video, -1)[pv].reshape(-1)
+    va = v[cfg.video_len:].reshape(cfg.n_action, -1)[pa].reshape(-1)
+    assert np.allclose(v2, np.concatenate([vv, va]), atol=1e-12)
+
+
+def test_velocity_output_rows_match_token_rows():
+    """Changing only the last action token's input changes its own output most directly:
+    with zero attention weights on the output path the map is strictly per token."""
+    cfgd = micro_config()
+    W, cfg = _setup(cfgd, std=0.3)
+    for l in range(cfg.n_layers):  # switch off both residual branches: tokens stay independent
+        W[f"layers.{l}.ada_w"][:] = 0.0
+        W[f"layers.{l}.ada_b"][:] = 0.0
+    rng = np.random.default_rng(8)
+    x = rng.standard_normal(cfg.traj_len)
+    obs = rng.standard_normal((cfg.n_obs, cfg.d_model))
+    v = O.velocity(W, cfg, x, obs, 0.3)
+    x2 = x.copy()
+    x2[-1] += 1.0
+    v2 = O.velocity(W, cfg, x2, obs, 0.3)
+    changed = np.nonzero(np.abs(v2 - v) > 1e-14)[0]
+    ad = cfg.action_dim
+    assert set(changed.tolist()) <= set(range(cfg.traj_len - ad, cfg.traj_len))
+    assert len(changed) > 0
+
+
+# ----------------------------------------------------------------------------- TR
+def test_rms_normaliser_has_unit_mean_square():
+    v = np.random.default_rng(9).standard_normal(1000) * 7.3
+    assert np.mean(O.normalize_rms(v) ** 2) == pytest.approx(1.0, abs=1e-14)
+    assert np.all(O.normalize_rms(np.zeros(5)) == 0.0)
+
+
+def test_tr_remap_slot_indices_bruteforce():
+    cfgd = micro_config(tr_normalize=1)
+    cfg = O.OracleConfig.from_dict(cfgd)
+    T, V, ad = cfg.traj_len, cfg.video_len, cfg.action_dim
+    x_bar = np.arange(T, dtype=np.float64)
+    eps = -1.0 - np.arange(T, dtype=np.float64)
+    for shift in range(0, cfg.n_action + 2):
+        out = O.tr_remap(cfg, x_bar, x_bar, 0.5, 0.25, shift, eps)  # x^r == x_bar -> d = 0
+        assert np.array_equal(out[:V], x_bar[:V])
+        for j in range(cfg.n_action):
+            for c in range(ad):
+                src = j + shift
+                want = x_bar[V + src * ad + c] if src < cfg.n_action else 0.25 * eps[V + j * ad + c]
+                assert out[V + j * ad + c] == want
+
+
+def test_tr_remap_closed_form_and_fresh_video_mode():
+    cfgd = micro_config(tr_video_mode=1)
+    cfg = O.OracleConfig.from_dict(cfgd)
+    rng = np.random.default_rng(10)
+    x_bar, x_r, eps = (rng.standard_normal(cfg.traj_len) for _ in range(3))
+    out = O.tr_remap(cfg, x_bar, x_r, 0.6, 0.7, 0, eps)
+    V = cfg.video_len
+    assert np.array_equal(out[:V], 0.7 * eps[:V])
+    u = (x_r[V:] - x_bar[V:]) / 0.6
+    assert np.allclose(out[V:], x_bar[V:] + 0.7 * u / np.sqrt(np.mean(u * u)), atol=1e-14)
+
+
+def test_tr_identity_normaliser_recovers_retained_latent():
+    cfg = O.OracleConfig.from_dict(micro_config(tr_normalize=0))
+    rng = np.random.default_rng(11)
+    x_bar, x_r, eps = (rng.standard_normal(cfg.traj_len) for _ in range(3))
+    out = O.tr_remap(cfg, x_bar, x_r, 0.4, 0.4, 0, eps)
+    assert np.allclose(out, x_r, atol=1e-14)
+
+
+def _episode(cfgd, std=0.3, seed=0):
+    W, cfg = _setup(cfgd, std=std, seed=seed)
+    return W, cfg, O.OracleEpisode(W, cfg)
+
+
+def test_invariant_zero_shift_identity_rescale_equals_plain_continuation():
+    cfgd = micro_config(tr_normalize=0, tr_entry_stage=2, tr_retain_stage=-1)
+    W, cfg, ep = _episode(cfgd)
+    rng = np.random.default_rng(12)
+    obs = rng.standard_normal((cfg.n_obs, cfg.d_model))
+    noise = rng.standard_normal(cfg.traj_len)
+    ep.sample_cold(obs, noise, cfg.n_steps)
+    x2 = ep.hist[2].copy()
+    final = ep.hist[cfg.n_steps].copy()
+    assert ep.adapt(obs, 0, rng.standard_normal(cfg.traj_len)) == O.ADAPT_TR_INIT
+    assert np.allclose(ep.x, x2, atol=1e-13)
+    ep.advance(cfg.n_steps - 2)
+    assert np.allclose(ep.hist[cfg.n_steps], final, atol=1e-12)
+
+
+def test_invariant_empty_target_set_entry_zero_equals_cold():
+    cfgd = micro_config(tr_video_mode=1, tr_entry_stage=0)
+    W, cfg, ep = _episode(cfgd)
+    rng = np.random.default_rng(13)
+    obs = rng.standard_normal((cfg.n_obs, cfg.d_model))
+    ep.sample_cold(obs, rng.standard_normal(cfg.traj_len), cfg.n_steps)
+    eps = rng.standard_normal(cfg.traj_len)
+    obs2 = rng.standard_normal((cfg.n_obs, cfg.d_model))
+    ep.adapt(obs2, cfg.n_action, eps)        # shift covers the whole action horizon
+    assert np.array_equal(ep.x, eps)         # sigma_0 = 1: pure fresh noise
+    warm = ep.advance(cfg.n_steps)
+    cold = O.OracleEpisode(W, cfg).sample_cold(obs2, eps, cfg.n_steps)
+    assert np.array_equal(warm, cold)
+
+
+# ----------------------------------------------------------------------------- OR
+def test_or_score_closed_forms():
+    cfg = O.OracleConfig.from_dict(micro_config(n_obs=4, or_n_components=2,
+                                                or_deltas=(2.0, 0.5, 1, 1),
+                                                or_weights=(3.0, 1.0, 1, 1)))
+    P = np.zeros((4, 16))
+    R = np.zeros((4, 16))
+    R[:2] = 1.0      # component 0: diff -1, / delta 2 -> e0 = 0.5
+    R[2] = -0.25     # component 1: diffs 0.25 and 0.75, / delta 0.5 -> 0.5 and 1.5
+    R[3] = -0.75     #   e1 = sqrt((0.25 + 2.25) / 2)
+    e0, e1 = 0.5, math.sqrt(1.25)
+    assert O.or_score(cfg, P, R) == pytest.approx(math.sqrt((3 * e0 ** 2 + e1 ** 2) / 4))
+    assert O.or_score(cfg, R, R) == 0.0
+
+
+def _kappa_run(cfgd, n_replans, real_offsets):
+    W, cfg, ep = _episode(cfgd)
+    rng = np.random.default_rng(14)
+    obs = rng.standard_normal((cfg.n_obs, cfg.d_model))
+    ep.sample_cold(obs, rng.standard_normal(cfg.traj_len), cfg.n_steps)
+    seq = []
+    for t in range(n_replans):
+        eps = rng.standard_normal(cfg.traj_len)
+        st = ep.adapt(obs, 1, eps)
+        seq.append(st)
+        x_b0 = ep.x.copy()
+        if st == O.ADAPT_TR_INIT:
+            ep.advance(1)
+        st2 = ep.adapt(obs + real_offsets[t], 0, None)
+        seq.append(st2)
+        if st2 == O.ADAPT_REBIND_RESTART:
+            assert np.array_equal(ep.x, x_b0) and ep.stage == cfg.tr_entry_stage
+        ep.advance(cfg.n_steps - ep.stage)
+    return seq, ep
+
+
+def test_kappa_cap_forces_refresh_and_skips_prefix():
+    A, R, T, N, F = (O.ADAPT_REBIND_ACCEPT, O.ADAPT_REBIND_RESTART, O.ADAPT_TR_INIT,
+                     O.ADAPT_TR_INIT_NO_PREFIX, O.ADAPT_REFRESH)
+    seq, ep = _kappa_run(micro_config(or_tau=0.5, or_kappa_max=3), 6, [0.1] * 6)
+    assert seq == [T, A, T, A, T, A, N, F, T, A, T, A]
+    st = ep.stats.rates()
+    assert ep.stats.n_start == 5 and ep.stats.n_bind == 5 and ep.stats.n_noninitial == 6
+    assert st["r_or"] == 1.0 and st["coverage"] == pytest.approx(5 / 6)
+    seq, _ = _kappa_run(micro_config(or_tau=0.5, or_kappa_max=3), 3, [0.1, 0.7, 0.1])
+    assert seq == [T, A, T, R, T, A]
+
+
+# ----------------------------------------------------------------------------- RR
+@pytest.mark.parametrize("c", [0.5, 1.0, 1.1, 1.25, 2.0, -1.0])
+def test_rr_scaled_probe_closed_form(c):
+    cfg = O.OracleConfig.from_dict(micro_config())
+    p_a = np.random.default_rng(15).standard_normal(200)
+    chk = O.rr_check(c * p_a, p_a, cfg)
+    alpha = min(max(c, 1.0), 1.25)
+    assert chk.alpha == pytest.approx(alpha, abs=1e-14)
+    assert chk.cos == pytest.approx(math.copysign(1.0, c), abs=1e-14)
+    assert chk.fit == pytest.approx(abs(c - alpha) / abs(c), abs=1e-13)
+    assert chk.passed == (chk.fit <= 0.40 and chk.cos >= 0.95)
+
+
+def test_rr_gate_vs_bruteforce_loops():
+    cfg = O.OracleConfig.from_dict(micro_config(rr_gamma_cos=0.5, rr_gamma_fit=0.9))
+    rng = np.random.default_rng(16)
+    for trial in range(20):
+        p_a = rng.standard_normal(30).tolist()
+        p_i = [a * 1.1 + 0.4 * rng.standard_normal() for a in p_a]
+        n = len(p_a)
+        num = sum(x * y for x, y in zip(p_i, p_a)) / n
+        den = max(sum(y * y for y in p_a) / n, 1e-8)
+        alpha = min(max(num / den, 1.0), 1.25)
+        ni = math.sqrt(sum(x * x for x in p_i))
+        na = math.sqrt(sum(y * y for y in p_a))
+        cos = sum(x * y for x, y in zip(p_i, p_a)) / (ni * na)
+        fit = math.sqrt(sum((x - alpha * y) ** 2 for x, y in zip(p_i, p_a))) / ni
+        chk = O.rr_check(np.array(p_i), np.array(p_a), cfg)
+        assert (chk.alpha, chk.cos, chk.fit) == pytest.approx((alpha, cos, fit), abs=1e-12)
+        assert chk.passed == (cos >= 0.5 and fit <= 0.9)
+
+
+def test_rr_zero_probe_fails_gate():
+    cfg = O.OracleConfig.from_dict(micro_config())
+    assert not O.rr_check(np.zeros(10), np.ones(10), cfg).passed
+    assert not O.rr_check(np.ones(10), np.zeros(10), cfg).passed
+
+
+def test_rr_reuse_on_identical_input_reproduces_full_forward():
+    cfgd = micro_config(n_layers=6, rr_policy=1, rr_q=1, rr_s=2, rr_e=5)
+    W, cfg = _setup(cfgd, std=0.3)
+    rng = np.random.default_rng(17)
+    x = rng.standard_normal(cfg.traj_len)
+    obs = rng.standard_normal((cfg.n_obs, cfg.d_model))
+    full = O.velocity(W, cfg, x, obs, 0.5)
+    v1, st, rec1 = O.velocity_rr(W, cfg, x, obs, 0.5, None, True)
+    assert not rec1.rr_attempt and np.allclose(v1, full, atol=1e-13)
+    v2, st2, rec2 = O.velocity_rr(W, cfg, x, obs, 0.5, st, True)
+    assert rec2.rr_attempt and rec2.rr_accept and st2 is st
+    for c in rec2.checks:
+        assert c.alpha == 1.0 and c.cos == pytest.approx(1.0) and c.fit == pytest.approx(0.0, abs=1e-7)
+    assert np.allclose(v2, full, atol=1e-12)
+
+
+def test_rr_disabled_equals_full_forward():
+    cfgd = micro_config(n_layers=6, rr_policy=0, rr_q=1, rr_s=2, rr_e=5)
+    W, cfg, ep = _episode(cfgd)
+    rng = np.random.default_rng(18)
+    obs = rng.standard_normal((cfg.n_obs, cfg.d_model))
+    noise = rng.standard_normal(cfg.traj_len)
+    out = ep.sample_cold(obs, noise, cfg.n_steps)
+    sig = O.schedule(cfg.n_steps)
+    xs = O.euler_integrate(noise, sig, lambda x, s: O.velocity(W, cfg, x, obs, s))
+    assert np.array_equal(out, xs[-1])
+    assert ep.stats.n_attempt == 0 and ep.stats.b_dense == 0
+
+
+def test_rr_rejected_step_refreshes_state_and_counts():
+    cfgd = micro_config(n_layers=6, rr_policy=1, rr_q=1, rr_s=2, rr_e=5,
+                        rr_gamma_cos=1.1)       # unreachable: every check fails
+    W, cfg, ep = _episode(cfgd)
+    rng = np.random.default_rng(19)
+    obs = rng.standard_normal((cfg.n_obs, cfg.d_model))
+    ep.sample_cold(obs, rng.standard_normal(cfg.traj_len), cfg.n_steps)
+    assert ep.stats.n_attempt == cfg.n_steps - 1 and ep.stats.n_reuse == 0
+    assert ep.stats.b_dense == cfg.n_steps * cfg.n_layers and ep.stats.b_skip == 0
+
+
+def test_rr_layer_evaluation_counts_match_table6():
+    for _, name, L, q, s, e, evaluated in (r for r in _golden("profiles.txt") if r[0] == "rr"):
+        L, q, s, e = int(L), int(q), int(s), int(e)
+        assert 0 < q < s < e < L
+        assert L - (e - s) == int(evaluated)
+
+
+def test_method_defaults_match_paper_tables():
+    rows = _golden("profiles.txt")
+    alpha = [r for r in rows if r[0] == "alpha"][0]
+    d = I.METHOD_DEFAULTS
+    assert (d["rr_alpha_min"], d["rr_alpha_max"], d["rr_eps"]) == tuple(float(a) for a in alpha[1:])
+    motus = [r for r in rows if r[0] == "gate" and r[1] == "motus"][0]
+    assert (d["rr_gamma_cos"], d["rr_gamma_fit"]) == (float(motus[2]), float(motus[3]))
+
+
+def test_reuse_rates_definitions():
+    s = O.Stats(n_attempt=8, n_reuse=6, b_skip=24, b_dense=96, n_start=5, n_bind=4, n_noninitial=9)
+    r = s.rates()
+    assert r == dict(r_rr=0.75, f_skip=0.25, r_or=0.8, coverage=4 / 9)
