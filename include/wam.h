@@ -1,0 +1,258 @@
+/*
+ * wam.h — C ABI of the GB300-native WAMachine hot path.
+ *
+ * The library runs the iterative flow denoising loop of a World Action Model: a DiT-style
+ * transformer over the joint [observation ; future-video-latent ; action] token sequence,
+ * integrated with explicit Euler steps, and the three state-adaptation mechanisms of
+ * "Efficient World Action Model Inference with Adaptive Intermediate States"
+ * (arXiv 2609.34608):
+ *   - Trajectory Remapping (TR), §3.1, Eqs. 1-2 and App. B.1 Eq. 12,
+ *   - Observation Rebinding (OR), §3.2, Eq. 4 and the kappa rule,
+ *   - Residual Rescaling (RR), §3.3, Eqs. 5-9,
+ * coordinated as described in §3.4.  The paper does not define the denoiser (it cites DiT);
+ * the network implemented here is fixed by the weight layout documented below.
+ *
+ * Conventions for every call
+ *   - Return value: WAM_OK or one WAM_ERR_* code.  No call aborts or throws across the ABI;
+ *     wam_last_error() returns a message for the last failure on a context.
+ *   - Buffers are owned by the caller.  Each buffer argument may be a host pointer or a device
+ *     pointer of the current device; the library detects which (CUDA pointer attributes).
+ *     Host buffers are copied in / out inside the call; a call with a host output returns
+ *     only after the output has been written.  With device buffers only, a call returns
+ *     once its work is enqueued on the context's stream.
+ *   - Contexts and states own their device memory.  A context is used from one host thread
+ *     at a time; it is not thread-safe.
+ *   - All float buffers are IEEE float32, row-major, contiguous.
+ *
+ * Layouts (B = episodes in a state, No/Nv/Na = observation/video/action tokens,
+ *          d = model width, T = Nv*video_dim + Na*action_dim)
+ *   obs        [B, No, d]   already-encoded observation tokens (the condition c of §3.2)
+ *   trajectory [B, T]       video values (token-major, video_dim each) then action values
+ *   actions    [B, Na, action_dim]
+ *   video      [B, Nv, video_dim]
+ */
+#ifndef WAM_H_
+#define WAM_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* ---- status codes ------------------------------------------------------------------- */
+#define WAM_OK 0
+#define WAM_ERR_INVALID_ARG 1  /* null / mis-sized / out-of-range argument */
+#define WAM_ERR_BAD_STATE 2    /* call not valid for the state's current phase */
+#define WAM_ERR_OOM 3          /* device allocation failed */
+#define WAM_ERR_CUDA 4         /* a CUDA runtime call or kernel launch failed */
+#define WAM_ERR_TIMEOUT 5      /* a bounded device-side wait gave up (kernel returned early) */
+#define WAM_ERR_UNSUPPORTED 6  /* configuration outside what the kernels implement */
+
+/* ---- precision ---------------------------------------------------------------------- */
+#define WAM_PREC_FP32 0  /* SIMT float32 everywhere */
+#define WAM_PREC_BF16 1  /* bf16 tensor-core GEMMs / attention, float32 residual stream */
+
+/* ---- RR policies (App. B.1, paragraph after Table 5) -------------------------------- */
+#define WAM_RR_OFF 0         /* every step runs all layers */
+#define WAM_RR_ALL_PATHS 1   /* reuse allowed on every step once a layer state exists */
+#define WAM_RR_PREFIX_PATH 2 /* reuse only on the anticipatory path after its first full step */
+
+/* ---- adapt statuses (per episode, written by wam_adapt_state) ------------------------ */
+#define WAM_ADAPT_TR_INIT 1           /* remapped init at b0; an anticipatory prefix may run */
+#define WAM_ADAPT_TR_INIT_NO_PREFIX 2 /* remapped init; kappa reached kappa_max: skip the prefix */
+#define WAM_ADAPT_COLD_INIT 3         /* fresh episode: noise at stage 0 */
+#define WAM_ADAPT_REBIND_ACCEPT 4     /* consistency passed: real condition bound, state kept */
+#define WAM_ADAPT_REBIND_RESTART 5    /* consistency failed: restart from the remapped init */
+#define WAM_ADAPT_REFRESH 6           /* no prefix ran: real condition bound at b0, kappa = 0 */
+
+/* entry_stage value that starts an episode afresh from noise (the first replan, §3.1) */
+#define WAM_ENTRY_COLD (-1)
+
+/*
+ * Model + method profile.  Plain values, copied by wam_create.
+ *
+ * Schedule: sigma_k = s t_k / (1 + (s-1) t_k), t_k = 1 - k/K, k = 0..K (s = sched_shift;
+ * s = 1 is linear flow time).  Step k integrates x_{k+1} = x_k + (sigma_{k+1}-sigma_k) v_k.
+ *
+ * TR (§3.1): the retained stage r (tr_retain_stage, -1 = same as the entry stage) and entry
+ * stage b0 (tr_entry_stage, per-episode override in wam_adapt_state) with r >= b0 of the
+ * replan that produced the state and r < K.  tr_normalize = 1 uses the unit-RMS normaliser of
+ * Eq. 12, 0 the identity.  tr_video_mode = 0 remaps video without a temporal shift, 1 fills
+ * video with fresh noise (the Motus profile of App. B.1).  Action slots shift by the executed
+ * count; uncovered tail slots get fresh noise sigma_b0 * eps.
+ *
+ * RR (§3.3): boundaries 0 < rr_q < rr_s < rr_e < n_layers; factor clamp [alpha_min, alpha_max]
+ * and epsilon of Eq. 7; gate thresholds of Eq. 8.  Branches (joint execution): observation and
+ * video rows form one branch, action rows the other; each gets its own alpha and the middle
+ * layers are skipped only if both pass.
+ *
+ * OR (§3.2): Eq. 4 over or_n_components (1..4) equal contiguous blocks of observation tokens
+ * with per-component scale or_deltas[m] and weight or_weights[m]; accept iff S < or_tau and
+ * kappa < or_kappa_max.
+ */
+typedef struct wam_config {
+  int32_t n_layers, d_model, n_heads, mlp_ratio;
+  int32_t n_obs, n_video, video_dim, n_action, action_dim;
+  int32_t n_steps;   /* K native solver steps */
+  int32_t precision; /* WAM_PREC_* */
+  int32_t batch_max; /* largest state batch this context will run */
+  float sched_shift;
+  int32_t tr_entry_stage, tr_retain_stage, tr_normalize, tr_video_mode;
+  int32_t rr_policy, rr_q, rr_s, rr_e;
+  float rr_alpha_min, rr_alpha_max, rr_eps, rr_gamma_cos, rr_gamma_fit;
+  float or_tau;
+  int32_t or_kappa_max, or_n_components;
+  float or_deltas[4];
+  float or_weights[4];
+} wam_config;
+
+/* Reuse statistics, App. D.2 Eqs. 14-15 (counts; rates are ratios of these). */
+typedef struct wam_stats {
+  int64_t n_attempt;     /* RR checks evaluated against a retained layer state */
+  int64_t n_reuse;       /* accepted checks that skipped the middle layers */
+  int64_t b_skip;        /* skipped layer evaluations */
+  int64_t b_dense;       /* full-depth layer count of RR-enabled steps */
+  int64_t n_start;       /* anticipatory prefixes started (rebinding attempts) */
+  int64_t n_bind;        /* prefixes accepted and used */
+  int64_t n_noninitial;  /* replans after the first (TR inits) */
+  int64_t n_episode_steps;  /* denoising steps executed, summed over episodes */
+  int64_t n_layer_evals;    /* transformer layer evaluations, summed over episodes */
+  int64_t n_kernel_launches;/* kernels launched by this context */
+} wam_stats;
+
+/* One record per (episode, denoising step) of the latest wam_sample_cold / wam_continue. */
+typedef struct wam_step_record {
+  int32_t episode, stage;
+  int32_t rr_active;  /* step ran on an RR-enabled path */
+  int32_t rr_attempt; /* gate evaluated */
+  int32_t rr_accept;  /* middle layers skipped */
+  int32_t pad_;
+  float alpha[2], cos[2], fit[2]; /* per branch: 0 = obs+video rows, 1 = action rows */
+} wam_step_record;
+
+typedef struct wam_ctx wam_ctx;
+typedef struct wam_state wam_state;
+
+/*
+ * Number of floats in the flat weight buffer for cfg, or 0 if cfg is invalid.
+ * Weight order (matrices [in, out], y = x W + b):
+ *   obs_w[d,d] obs_b[d] vid_w[video_dim,d] vid_b[d] act_w[action_dim,d] act_b[d] pos[N,d]
+ *   t_w1[256,d] t_b1[d] t_w2[d,d] t_b2[d]
+ *   per layer: ada_w[d,6d] ada_b[6d] qkv_w[d,3d] qkv_b[3d] out_w[d,d] out_b[d]
+ *              up_w[d,r d] up_b[r d] down_w[r d,d] down_b[d]          (r = mlp_ratio)
+ *   final_ada_w[d,2d] final_ada_b[2d] vout_w[d,video_dim] vout_b[video_dim]
+ *   aout_w[d,action_dim] aout_b[action_dim]
+ * Network: tokens [obs W_o + b_o ; x_video W_v + b_v ; x_action W_a + b_a] + pos.
+ * Conditioning c = SiLU(e W_t1 + b_t1) W_t2 + b_t2 with e = [cos(1000 sigma f), sin(1000 sigma f)],
+ * f_j = 10000^(-j/128).  Layer modulations (shift1, scale1, gate1, shift2, scale2, gate2)
+ * = SiLU(c) ada_w + ada_b; h += gate1 * Attn(LN(h)(1+scale1)+shift1) W_out;
+ * h += gate2 * GELU_tanh(LN(h)(1+scale2)+shift2 W_up) W_down (biases included, LN eps 1e-6,
+ * no affine; attention full, unmasked, scale 1/sqrt(d/heads)).  Output: LN(h)(1+scale)+shift
+ * then vout on video rows, aout on action rows.
+ */
+size_t wam_weight_count(const wam_config* cfg);
+
+/*
+ * Create a context: validates cfg, uploads and converts the weights (host or device pointer,
+ * n_weights == wam_weight_count(cfg)), allocates activation buffers for batch_max episodes.
+ * stream: a cudaStream_t (NULL = legacy default stream).
+ * Errors: INVALID_ARG (cfg or weights), UNSUPPORTED (shape the kernels cannot run), OOM, CUDA.
+ */
+int wam_create(const wam_config* cfg, const float* weights, size_t n_weights, void* stream,
+               wam_ctx** out);
+void wam_destroy(wam_ctx* ctx);
+const char* wam_last_error(const wam_ctx* ctx);
+int wam_set_stream(wam_ctx* ctx, void* stream);
+
+/* Per-episode replan / denoising / layer state for `batch` episodes (1..batch_max). */
+int wam_state_create(wam_ctx* ctx, int32_t batch, wam_state** out);
+void wam_state_destroy(wam_state* st);
+
+/*
+ * First replan of every episode (§3.1: it starts from fresh noise): x_0 = noise [B,T] at stage 0
+ * under obs [B,No,d], then n_steps (1..K) Euler steps.  Resets kappa and the RR layer state.
+ * actions_out [B,Na,action_dim] (nullable) receives the latent's action part after the
+ * last step (the denoised actions when n_steps == K).
+ */
+int wam_sample_cold(wam_ctx* ctx, wam_state* st, const float* obs, const float* noise,
+                    int32_t n_steps, float* actions_out);
+
+/*
+ * Adapt the retained state to a new planning context, per episode:
+ *   finished replan (stage K): Trajectory Remapping, Eqs. 1-2 — direction from x^r and x_bar,
+ *       remapped init at b0 = entry_stage[b] (NULL: cfg.tr_entry_stage) with the action
+ *       horizon shifted by executed_shift[b] (>= 0), fresh slots sigma_b0 * fresh_noise;
+ *       new_obs becomes the bound condition (a prediction, for an anticipatory prefix, or the
+ *       real observation).  Status TR_INIT, or TR_INIT_NO_PREFIX when kappa == kappa_max.
+ *   replan in flight: Observation Rebinding, §3.2 — executed_shift[b] must be 0; if a prefix
+ *       ran since the last binding, S (Eq. 4) compares the bound condition with new_obs;
+ *       S < tau and kappa < kappa_max binds new_obs and keeps the denoising state
+ *       (REBIND_ACCEPT, kappa+1), otherwise the episode restarts from its remapped init
+ *       under new_obs (REBIND_RESTART, kappa = 0).  With no prefix steps: REFRESH.
+ *   entry_stage[b] == WAM_ENTRY_COLD: fresh episode, x_0 = fresh_noise[b] at stage 0 (COLD_INIT).
+ * new_obs [B,No,d]; executed_shift [B] (NULL = all 0); fresh_noise [B,T] standard normal
+ * (required when any episode remaps or starts cold); status_out [B] (nullable).
+ * Errors: INVALID_ARG, BAD_STATE (retained stage unavailable, shift on a rebind).
+ */
+int wam_adapt_state(wam_ctx* ctx, wam_state* st, const float* new_obs,
+                    const int32_t* executed_shift, const int32_t* entry_stage,
+                    const float* fresh_noise, int32_t* status_out);
+
+/*
+ * Advance each episode n_steps[b] (>= 0, stage + n <= K) Euler steps under its bound
+ * condition, with Residual Rescaling per cfg.rr_policy.  Episodes that reach stage K become
+ * finished replans (x_bar = x_K).  actions_out [B,Na,action_dim], video_out [B,Nv,video_dim]
+ * (both nullable) receive every episode's current latent after the call.
+ */
+int wam_continue(wam_ctx* ctx, wam_state* st, const int32_t* n_steps, float* actions_out,
+                 float* video_out);
+
+/* Reuse statistics accumulated on the context since creation / the last reset. */
+int wam_get_stats(wam_ctx* ctx, wam_stats* out);
+int wam_reset_stats(wam_ctx* ctx);
+
+/* Per-step records of the latest sampling call: copies min(capacity, available) records. */
+int wam_state_log(const wam_state* st, wam_step_record* out, int32_t capacity, int32_t* n_out);
+
+/* ---- state export / import (checkpoint + parity inspection) ------------------------- */
+#define WAM_FIELD_X 0        /* current latent            [B,T]     */
+#define WAM_FIELD_X_STAGE 1  /* latent at stage `index`   [B,T]     (index 0..K) */
+#define WAM_FIELD_V_STEP 2   /* velocity of the step from stage `index` [B,T] (index 0..K-1) */
+#define WAM_FIELD_X_INIT 3   /* remapped init x^{b0}      [B,T]     */
+#define WAM_FIELD_OBS 4      /* bound condition           [B,No,d]  */
+#define WAM_FIELD_RR_P 5     /* retained probe residual p_a  [B,N,d] */
+#define WAM_FIELD_RR_R 6     /* retained middle residual R_a [B,N,d] */
+/* Host-side per-episode scalars: 8 int32 per episode:
+ * stage, hist_from, b0, kappa, finished, since_bind, path (0 cold 1 prefix 2 refresh), rr_valid */
+#define WAM_FIELD_META 7
+int wam_state_read(wam_ctx* ctx, const wam_state* st, int32_t field, int32_t index, void* out,
+                   size_t n_bytes);
+int wam_state_write(wam_ctx* ctx, wam_state* st, int32_t field, int32_t index, const void* in,
+                    size_t n_bytes);
+
+/* Wait for the context's stream; returns a pending device-side error (e.g. TIMEOUT). */
+int wam_sync(wam_ctx* ctx);
+
+/* Kernel-class timing spans recorded with CUDA events on the context's stream. */
+#define WAM_KCLASS_GEMM 0
+#define WAM_KCLASS_ATTN 1
+#define WAM_KCLASS_NORM 2      /* LN-modulate, embed, final+Euler */
+#define WAM_KCLASS_COND 3      /* conditioning GEMVs */
+#define WAM_KCLASS_ADAPT 4     /* TR / OR / RR kernels */
+#define WAM_KCLASS_COUNT 5
+typedef struct wam_kclass_timing {
+  int64_t launches;
+  double ms;          /* summed event-measured duration */
+  double flops;       /* algorithmic flops of those launches */
+  double bytes;       /* algorithmic bytes of those launches */
+} wam_kclass_timing;
+/* enable != 0 starts recording (clears previous spans); reading synchronizes the stream. */
+int wam_profile_enable(wam_ctx* ctx, int32_t enable);
+int wam_profile_read(wam_ctx* ctx, wam_kclass_timing* out /* [WAM_KCLASS_COUNT] */);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* WAM_H_ */

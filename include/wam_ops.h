@@ -1,0 +1,66 @@
+/*
+ * wam_ops.h — kernel-level entry points of the WAMachine library.
+ *
+ * These expose single hot-path kernels for parity tests and kernel benchmarks.  Every pointer
+ * is a device pointer of the current device; nothing is allocated except where noted, and
+ * every call is asynchronous on `stream` (a cudaStream_t, NULL = legacy default stream).
+ * Return value: 0 on success or a WAM_ERR_* code from wam.h; wam_op_last_error() returns the
+ * message of the calling thread's last failure.
+ */
+#ifndef WAM_OPS_H_
+#define WAM_OPS_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* GEMM epilogues (C = A W^T + bias, fused into the accumulator read-back) */
+#define WAM_EPI_BF16 0       /* C_bf16[m,n] = acc + bias[n] */
+#define WAM_EPI_GELU_BF16 1  /* C_bf16[m,n] = GELU_tanh(acc + bias[n]) (DiT MLP up-projection) */
+#define WAM_EPI_RESID_F32 2  /* C_f32[m,n] += gate[item(m), n] * (acc + bias[n]) (adaLN gated
+                                residual, item(m) = m / rows_per_item) */
+#define WAM_EPI_F32 3        /* C_f32[m,n] = acc + bias[n] */
+
+/*
+ * Dense projection of the DiT block (QKV, attention output, MLP up / down):
+ *   A  [M, K] bf16 row-major (activations), Wt [N, K] bf16 row-major (weight, K-major),
+ *   bias [N] float32 (nullable), gate rows of `gate_stride` floats (RESID only).
+ * Runs on the fifth-generation tensor cores (tcgen05.mma, TMEM accumulators, TMA loads).
+ * Requires K % 64 == 0, N % 128 == 0, 16-byte aligned pointers.  M >= 1 is arbitrary.
+ */
+int wam_op_gemm_bf16(const void* A, const void* Wt, const float* bias, void* C, int32_t M,
+                     int32_t N, int32_t K, int32_t epilogue, const float* gate,
+                     int64_t gate_stride, int32_t rows_per_item, void* stream);
+
+/* Same contraction in float32 SIMT (the library's fp32 precision mode). */
+int wam_op_gemm_f32(const float* A, const float* Wt, const float* bias, float* C, int32_t M,
+                    int32_t N, int32_t K, int32_t epilogue, const float* gate,
+                    int64_t gate_stride, int32_t rows_per_item, void* stream);
+
+/*
+ * Full bidirectional multi-head attention over the joint token sequence of each item:
+ *   qkv [B*N, 3d] (q | k | v column blocks, head h owns columns h*dh .. h*dh+dh-1 of each),
+ *   out [B*N, d].  softmax(q k^T / sqrt(dh)) v, no mask.
+ * precision WAM_PREC_BF16: bf16 in / out, fp32 accumulation, head dim 64 or 72.
+ * precision WAM_PREC_FP32: float32 in / out, head dim <= 128 and a multiple of 32... any dh <= 128.
+ */
+int wam_op_attention(const void* qkv, void* out, int32_t B, int32_t N, int32_t d,
+                     int32_t n_heads, int32_t precision, void* stream);
+
+/*
+ * adaLN modulate: out[m,:] = LN(h[m,:]) * (1 + scale[item(m),:]) + shift[item(m),:]
+ * h [M, d] float32; shift/scale rows of `mod_stride` floats; out bf16 (precision BF16) or f32.
+ */
+int wam_op_ln_modulate(const float* h, const float* shift, const float* scale,
+                       int64_t mod_stride, void* out, int32_t M, int32_t d,
+                       int32_t rows_per_item, int32_t precision, void* stream);
+
+const char* wam_op_last_error(void);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* WAM_OPS_H_ */

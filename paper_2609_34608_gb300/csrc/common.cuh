@@ -1,0 +1,96 @@
+// Shared helpers of the WAMachine CUDA library (device utilities, launch bookkeeping and the
+// internal interfaces between translation units).  Nothing here is part of the public ABI.
+#pragma once
+
+#include <cuda.h>
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#define WAM_DEV __device__ __forceinline__
+
+namespace wam {
+
+using bf16 = __nv_bfloat16;
+
+// Bits of the device error word a context hands to kernels with bounded waits.
+constexpr int kDevErrTimeout = 1;
+// A bounded wait gives up after this long (ns of %globaltimer).
+constexpr uint64_t kWaitLimitNs = 2000000000ull;
+
+WAM_DEV uint64_t globaltimer_ns() {
+  uint64_t t;
+  asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+  return t;
+}
+
+WAM_DEV float warp_sum(float v) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+  return v;
+}
+
+WAM_DEV double warp_sum_d(double v) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+  return v;
+}
+
+WAM_DEV float silu_f(float x) { return x / (1.0f + expf(-x)); }
+
+WAM_DEV float gelu_tanh_f(float x) {
+  // 0.5 x (1 + tanh(sqrt(2/pi) (x + 0.044715 x^3)))
+  const float k0 = 0.7978845608028654f;
+  return 0.5f * x * (1.0f + tanhf(k0 * (x + 0.044715f * x * x * x)));
+}
+
+// ---- activation storage type helpers ---------------------------------------------------
+template <typename T> struct Act;
+template <> struct Act<float> {
+  static WAM_DEV void store4(float* p, float a, float b, float c, float d) {
+    *reinterpret_cast<float4*>(p) = make_float4(a, b, c, d);
+  }
+  static WAM_DEV float load(const float* p) { return *p; }
+};
+template <> struct Act<bf16> {
+  static WAM_DEV void store4(bf16* p, float a, float b, float c, float d) {
+    __nv_bfloat162 lo = __floats2bfloat162_rn(a, b);
+    __nv_bfloat162 hi = __floats2bfloat162_rn(c, d);
+    uint2 u;
+    u.x = *reinterpret_cast<uint32_t*>(&lo);
+    u.y = *reinterpret_cast<uint32_t*>(&hi);
+    *reinterpret_cast<uint2*>(p) = u;
+  }
+  static WAM_DEV float load(const bf16* p) { return __bfloat162float(*p); }
+};
+
+// ---- GEMM epilogue description (shared by the tensor-core and SIMT GEMMs) ---------------
+enum EpiMode { kEpiBf16 = 0, kEpiGeluBf16 = 1, kEpiResidF32 = 2, kEpiF32 = 3 };
+
+struct EpiArgs {
+  const float* bias;     // [N] or null
+  void* C;               // output (bf16 or f32, row-major, leading dim N)
+  const float* gate;     // RESID: gate rows
+  int64_t gate_stride;   // floats between gate rows of consecutive items
+  int rows_per_item;     // rows of one item (tokens of one episode)
+  const int* item_map;   // nullable: gate row of local item i = item_map[i]
+};
+
+// ---- internal interfaces -----------------------------------------------------------------
+// tcgen05 GEMM (gemm_tc.cu).  CUtensorMap is the driver's 128-byte opaque descriptor.
+int tc_encode_kmajor_bf16(CUtensorMap* map, const void* base, uint64_t rows, uint64_t K);
+cudaError_t tc_gemm(const CUtensorMap& ta, const CUtensorMap& tb, int M, int N, int K, int epi,
+                    const EpiArgs& e, int num_sms, int* dev_err, cudaStream_t s);
+
+// float32 SIMT GEMM (gemm_simt.cu): C = A[M,K] Wt[N,K]^T
+cudaError_t simt_gemm(const float* A, const float* Wt, int M, int N, int K, int epi,
+                      const EpiArgs& e, cudaStream_t s);
+
+// attention (attention.cu)
+cudaError_t attention_bf16(const bf16* qkv, bf16* out, int B, int N, int d, int H,
+                           cudaStream_t s);
+cudaError_t attention_f32(const float* qkv, float* out, int B, int N, int d, int H,
+                          cudaStream_t s);
+bool attention_bf16_supported(int head_dim);
+
+}  // namespace wam

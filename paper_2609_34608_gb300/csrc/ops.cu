@@ -1,0 +1,118 @@
+// Kernel-level entry points (wam_ops.h): single hot-path kernels on caller-owned device
+// buffers, for parity tests and kernel benchmarks.  They allocate nothing.
+#include <string>
+
+#include "kernels.cuh"
+#include "wam.h"
+#include "wam_ops.h"
+
+using namespace wam;
+
+namespace {
+
+thread_local std::string g_op_err;
+
+int op_fail(int code, const std::string& msg) {
+  g_op_err = msg;
+  return code;
+}
+
+int op_cuda(const char* what, cudaError_t e) {
+  return op_fail(WAM_ERR_CUDA, std::string(what) + ": " + cudaGetErrorString(e));
+}
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+EpiArgs make_epi(const float* bias, void* C, const float* gate, int64_t gstride, int rpi) {
+  EpiArgs e;
+  e.bias = bias;
+  e.C = C;
+  e.gate = gate;
+  e.gate_stride = gstride;
+  e.rows_per_item = rpi > 0 ? rpi : 1;
+  e.item_map = nullptr;
+  return e;
+}
+
+int check_gemm_args(const void* A, const void* Wt, void* C, int M, int N, int K, int epi,
+                    const float* gate, int rpi) {
+  if (A == nullptr || Wt == nullptr || C == nullptr) return op_fail(WAM_ERR_INVALID_ARG, "null operand");
+  if (M < 0 || N <= 0 || K <= 0) return op_fail(WAM_ERR_INVALID_ARG, "bad GEMM shape");
+  if (epi < WAM_EPI_BF16 || epi > WAM_EPI_F32) return op_fail(WAM_ERR_INVALID_ARG, "unknown epilogue");
+  if (epi == WAM_EPI_RESID_F32 && (gate == nullptr || rpi <= 0)) return op_fail(WAM_ERR_INVALID_ARG, "RESID needs gate and rows_per_item");
+  return WAM_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+const char* wam_op_last_error(void) { return g_op_err.c_str(); }
+
+int wam_op_gemm_bf16(const void* A, const void* Wt, const float* bias, void* C, int32_t M, int32_t N,
+                     int32_t K, int32_t epilogue, const float* gate, int64_t gate_stride,
+                     int32_t rows_per_item, void* stream) {
+  int r = check_gemm_args(A, Wt, C, M, N, K, epilogue, gate, rows_per_item);
+  if (r != WAM_OK) return r;
+  if (K % 64 != 0 || N % 128 != 0) return op_fail(WAM_ERR_UNSUPPORTED, "needs K % 64 == 0 and N % 128 == 0");
+  if (!aligned16(A) || !aligned16(Wt) || !aligned16(C) || (bias && !aligned16(bias)) || (gate && !aligned16(gate)) ||
+      (gate && gate_stride % 4 != 0))
+    return op_fail(WAM_ERR_INVALID_ARG, "operands must be 16-byte aligned");
+  int dev = 0, sms = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e == cudaSuccess) e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  if (e != cudaSuccess) return op_cuda("device query", e);
+  CUtensorMap ta, tb;
+  if (tc_encode_kmajor_bf16(&ta, A, static_cast<uint64_t>(M > 0 ? M : 1), K) != 0 ||
+      tc_encode_kmajor_bf16(&tb, Wt, N, K) != 0)
+    return op_fail(WAM_ERR_CUDA, "cuTensorMapEncodeTiled failed");
+  e = tc_gemm(ta, tb, M, N, K, epilogue, make_epi(bias, C, gate, gate_stride, rows_per_item), sms, nullptr,
+              static_cast<cudaStream_t>(stream));
+  return e == cudaSuccess ? WAM_OK : op_cuda("tcgen05 GEMM launch", e);
+}
+
+int wam_op_gemm_f32(const float* A, const float* Wt, const float* bias, float* C, int32_t M, int32_t N,
+                    int32_t K, int32_t epilogue, const float* gate, int64_t gate_stride,
+                    int32_t rows_per_item, void* stream) {
+  int r = check_gemm_args(A, Wt, C, M, N, K, epilogue, gate, rows_per_item);
+  if (r != WAM_OK) return r;
+  cudaError_t e = simt_gemm(A, Wt, M, N, K, epilogue, make_epi(bias, C, gate, gate_stride, rows_per_item),
+                            static_cast<cudaStream_t>(stream));
+  return e == cudaSuccess ? WAM_OK : op_cuda("SIMT GEMM launch", e);
+}
+
+int wam_op_attention(const void* qkv, void* out, int32_t B, int32_t N, int32_t d, int32_t n_heads,
+                     int32_t precision, void* stream) {
+  if (qkv == nullptr || out == nullptr || B < 0 || N < 0 || d <= 0 || n_heads <= 0 || d % n_heads != 0)
+    return op_fail(WAM_ERR_INVALID_ARG, "bad attention arguments");
+  cudaError_t e;
+  if (precision == WAM_PREC_BF16) {
+    if (!attention_bf16_supported(d / n_heads)) return op_fail(WAM_ERR_UNSUPPORTED, "head dim must be 64 or 72");
+    if (!aligned16(qkv) || !aligned16(out)) return op_fail(WAM_ERR_INVALID_ARG, "16-byte alignment required");
+    e = attention_bf16(static_cast<const bf16*>(qkv), static_cast<bf16*>(out), B, N, d, n_heads,
+                       static_cast<cudaStream_t>(stream));
+  } else if (precision == WAM_PREC_FP32) {
+    if (d / n_heads > 128) return op_fail(WAM_ERR_UNSUPPORTED, "head dim must be <= 128");
+    e = attention_f32(static_cast<const float*>(qkv), static_cast<float*>(out), B, N, d, n_heads,
+                      static_cast<cudaStream_t>(stream));
+  } else {
+    return op_fail(WAM_ERR_INVALID_ARG, "unknown precision");
+  }
+  return e == cudaSuccess ? WAM_OK : op_cuda("attention launch", e);
+}
+
+int wam_op_ln_modulate(const float* h, const float* shift, const float* scale, int64_t mod_stride, void* out,
+                       int32_t M, int32_t d, int32_t rows_per_item, int32_t precision, void* stream) {
+  if (h == nullptr || shift == nullptr || scale == nullptr || out == nullptr || M < 0 || rows_per_item <= 0)
+    return op_fail(WAM_ERR_INVALID_ARG, "bad LN arguments");
+  if (d % 128 != 0 || d > 1536) return op_fail(WAM_ERR_UNSUPPORTED, "d must be a multiple of 128, at most 1536");
+  // shift and scale are addressed as offsets from a common base (the modulation row)
+  const int64_t so = static_cast<int64_t>(shift - scale);
+  const float* base = so >= 0 ? scale : shift;
+  const int shift_off = static_cast<int>(shift - base), scale_off = static_cast<int>(scale - base);
+  cudaError_t e = ln_modulate(h, nullptr, base, mod_stride, shift_off, scale_off, nullptr, out,
+                              precision == WAM_PREC_BF16, M, d, rows_per_item, static_cast<cudaStream_t>(stream));
+  return e == cudaSuccess ? WAM_OK : op_cuda("LN-modulate launch", e);
+}
+
+}  // extern "C"

@@ -1,0 +1,1114 @@
+// C ABI of the WAMachine hot path: context / state management and the host-side orchestration
+// of one denoising step (conditioning, embedding, DiT layers with the Residual Rescaling
+// branch, final layer + Euler), of Trajectory Remapping and of Observation Rebinding.
+// Every step of the path runs in this library's kernels; the host only sequences launches,
+// keeps the per-episode bookkeeping of §3.4 and takes the two data-dependent decisions
+// (RR gate, OR acceptance) after reading their device-computed statistics.
+#include <algorithm>
+#include <cmath>
+#include <cstdio>
+#include <cstring>
+#include <new>
+#include <string>
+#include <vector>
+
+#include "kernels.cuh"
+#include "wam.h"
+#include "wam_ops.h"
+
+using namespace wam;
+
+namespace {
+
+constexpr int kRingSlots = 64;
+constexpr size_t kSlotBytes = 16384;
+constexpr int kMaxBatch = 256;
+
+struct LayerW {
+  void* qkv_wt = nullptr;
+  void* out_wt = nullptr;
+  void* up_wt = nullptr;
+  void* down_wt = nullptr;
+  float* qkv_b = nullptr;
+  float* out_b = nullptr;
+  float* up_b = nullptr;
+  float* down_b = nullptr;
+  CUtensorMap tm_qkv, tm_out, tm_up, tm_down;
+};
+
+struct ProfSpan {
+  int kclass;
+  cudaEvent_t a, b;
+  double flops, bytes;
+};
+
+enum Path : int32_t { kPathCold = 0, kPathPrefix = 1, kPathRefresh = 2 };
+
+struct EpisodeMeta {
+  int32_t stage = -1;
+  int32_t hist_from = 0;
+  int32_t b0 = 0;
+  int32_t kappa = 0;
+  int32_t finished = 0;
+  int32_t since_bind = 0;
+  int32_t path = kPathCold;
+  int32_t rr_valid = 0;
+  int32_t path_steps = 0;
+};
+
+}  // namespace
+
+struct wam_ctx {
+  wam_config cfg;
+  int L, d, H, R, No, Nv, vd, Na, ad, N, T, V, K, dff, Bmax;
+  int64_t mod_n;
+  bool bf16;
+  cudaStream_t stream = nullptr;
+  int device = 0, num_sms = 0;
+  std::string err;
+  std::vector<double> sigma;
+  std::vector<void*> allocs;
+  // weights
+  void* obs_wt = nullptr;
+  float* obs_b = nullptr;
+  float *vid_w, *vid_b, *act_w, *act_b, *pos;
+  float *t_w1, *t_b1, *t_w2, *t_b2;
+  void* mod_w = nullptr;
+  float* mod_b = nullptr;
+  std::vector<LayerW> layers;
+  float *vout_w, *vout_b, *aout_w, *aout_b;
+  CUtensorMap tm_obs_w;
+  // activations (batch_max episodes)
+  float *h = nullptr, *hq = nullptr, *hm = nullptr;
+  void *xln = nullptr, *qkv = nullptr, *att = nullptr, *u = nullptr, *obs_lp = nullptr;
+  CUtensorMap tm_xln, tm_att, tm_u, tm_obs_lp;
+  float *t1 = nullptr, *cvec = nullptr, *mods = nullptr;
+  StepItem* d_items = nullptr;
+  int* d_map = nullptr;
+  RRApply* d_rrapply = nullptr;
+  RRGate* d_gate = nullptr;
+  AdaptItem* d_adapt = nullptr;
+  double* d_part = nullptr;
+  size_t part_doubles = 0;
+  float* d_eps = nullptr;
+  float* d_obs_new = nullptr;
+  int* d_err = nullptr;
+  // pinned host staging
+  uint8_t* ring = nullptr;
+  cudaEvent_t ring_ev[kRingSlots];
+  bool ring_used[kRingSlots];
+  int ring_next = 0;
+  uint8_t* readback = nullptr;
+  size_t readback_bytes = 0;
+  wam_stats stats;
+  bool prof_on = false;
+  std::vector<ProfSpan> spans;
+  std::vector<cudaEvent_t> evpool;
+  size_t evnext = 0;
+};
+
+struct wam_state {
+  wam_ctx* ctx = nullptr;
+  int B = 0;
+  float* x = nullptr;      // [B,T]
+  float* xhist = nullptr;  // [K+1,B,T]
+  float* vhist = nullptr;  // [K,B,T]
+  float* xb0 = nullptr;    // [B,T]
+  float* obs = nullptr;    // [B,No,d]
+  float* obs_emb = nullptr;
+  float* pa = nullptr;     // [B,N,d]
+  float* ra = nullptr;
+  std::vector<void*> allocs;
+  std::vector<EpisodeMeta> meta;
+  std::vector<wam_step_record> log;
+};
+
+namespace {
+
+int fail(wam_ctx* c, int code, const std::string& msg) {
+  if (c) c->err = msg;
+  return code;
+}
+
+int fail_cuda(wam_ctx* c, const char* what, cudaError_t e) {
+  return fail(c, e == cudaErrorMemoryAllocation ? WAM_ERR_OOM : WAM_ERR_CUDA,
+              std::string(what) + ": " + cudaGetErrorString(e));
+}
+
+#define CK(x)                                           \
+  do {                                                  \
+    cudaError_t e_ = (x);                               \
+    if (e_ != cudaSuccess) return fail_cuda(c, #x, e_); \
+  } while (0)
+
+#define TRY(x)              \
+  do {                      \
+    int r_ = (x);           \
+    if (r_ != WAM_OK) return r_; \
+  } while (0)
+
+template <typename T>
+int dalloc(wam_ctx* c, std::vector<void*>& reg, T** p, size_t count) {
+  void* q = nullptr;
+  cudaError_t e = cudaMalloc(&q, count * sizeof(T) > 0 ? count * sizeof(T) : 16);
+  if (e != cudaSuccess) {
+    cudaGetLastError();
+    return fail(c, WAM_ERR_OOM, "device allocation of " + std::to_string(count * sizeof(T)) + " bytes failed");
+  }
+  reg.push_back(q);
+  *p = static_cast<T*>(q);
+  return WAM_OK;
+}
+
+bool is_device_ptr(const void* p) {
+  cudaPointerAttributes a;
+  if (cudaPointerGetAttributes(&a, p) != cudaSuccess) {
+    cudaGetLastError();
+    return false;
+  }
+  return a.type == cudaMemoryTypeDevice || a.type == cudaMemoryTypeManaged;
+}
+
+cudaEvent_t next_event(wam_ctx* c) {
+  if (c->evnext == c->evpool.size()) {
+    cudaEvent_t e;
+    cudaEventCreate(&e);
+    c->evpool.push_back(e);
+  }
+  return c->evpool[c->evnext++];
+}
+
+// Launch bookkeeping: counts every kernel and, while profiling, brackets it with events.
+struct Span {
+  wam_ctx* c;
+  int kc;
+  double fl, by;
+  cudaEvent_t a = nullptr;
+  Span(wam_ctx* c_, int kc_, double fl_ = 0.0, double by_ = 0.0) : c(c_), kc(kc_), fl(fl_), by(by_) {
+    c->stats.n_kernel_launches++;
+    if (c->prof_on) {
+      a = next_event(c);
+      cudaEventRecord(a, c->stream);
+    }
+  }
+  ~Span() {
+    if (a != nullptr) {
+      cudaEvent_t b = next_event(c);
+      cudaEventRecord(b, c->stream);
+      c->spans.push_back({kc, a, b, fl, by});
+    }
+  }
+};
+
+// Host -> device upload of a small control array through a pinned ring slot.
+int upload(wam_ctx* c, void* dst, const void* src, size_t n) {
+  if (n == 0) return WAM_OK;
+  if (n > kSlotBytes) return fail(c, WAM_ERR_INVALID_ARG, "control upload too large");
+  const int s = c->ring_next;
+  c->ring_next = (c->ring_next + 1) % kRingSlots;
+  if (c->ring_used[s]) CK(cudaEventSynchronize(c->ring_ev[s]));
+  std::memcpy(c->ring + s * kSlotBytes, src, n);
+  CK(cudaMemcpyAsync(dst, c->ring + s * kSlotBytes, n, cudaMemcpyHostToDevice, c->stream));
+  CK(cudaEventRecord(c->ring_ev[s], c->stream));
+  c->ring_used[s] = true;
+  return WAM_OK;
+}
+
+// Device -> host read of small statistics, followed by a stream synchronisation and a check of
+// the device error word.
+int readback(wam_ctx* c, void* dst, const void* src, size_t n) {
+  if (n + sizeof(int) > c->readback_bytes) return fail(c, WAM_ERR_INVALID_ARG, "readback too large");
+  CK(cudaMemcpyAsync(c->readback, src, n, cudaMemcpyDeviceToHost, c->stream));
+  CK(cudaMemcpyAsync(c->readback + n, c->d_err, sizeof(int), cudaMemcpyDeviceToHost, c->stream));
+  CK(cudaStreamSynchronize(c->stream));
+  int derr = 0;
+  std::memcpy(&derr, c->readback + n, sizeof(int));
+  if (derr != 0) {
+    cudaMemsetAsync(c->d_err, 0, sizeof(int), c->stream);
+    return fail(c, WAM_ERR_TIMEOUT, "a bounded device-side wait gave up");
+  }
+  std::memcpy(dst, c->readback, n);
+  return WAM_OK;
+}
+
+int sync_check(wam_ctx* c) {
+  int dummy = 0;
+  return readback(c, &dummy, c->d_err, sizeof(int));
+}
+
+// ---------------------------------------------------------------------------------- GEMM
+int gemm(wam_ctx* c, const CUtensorMap* ta, const void* A, const CUtensorMap* tb, const void* Wt,
+         int M, int N, int K, int epi, const EpiArgs& e) {
+  const double out_b = (epi == kEpiResidF32) ? 8.0 : (epi == kEpiF32 ? 4.0 : (c->bf16 ? 2.0 : 4.0));
+  const double in_b = c->bf16 ? 2.0 : 4.0;
+  Span sp(c, WAM_KCLASS_GEMM, 2.0 * M * N * K, in_b * (double(M) * K + double(N) * K) + out_b * double(M) * N);
+  if (c->bf16) {
+    CK(tc_gemm(*ta, *tb, M, N, K, epi, e, c->num_sms, c->d_err, c->stream));
+  } else {
+    CK(simt_gemm(static_cast<const float*>(A), static_cast<const float*>(Wt), M, N, K, epi, e, c->stream));
+  }
+  return WAM_OK;
+}
+
+EpiArgs epi_args(const float* bias, void* C, const float* gate, int64_t gstride, int rpi, const int* map) {
+  EpiArgs e;
+  e.bias = bias;
+  e.C = C;
+  e.gate = gate;
+  e.gate_stride = gstride;
+  e.rows_per_item = rpi;
+  e.item_map = map;
+  return e;
+}
+
+int ln_mod(wam_ctx* c, const float* hb, float* hcopy, int shift_off, int scale_off, const int* map, int M) {
+  const double by = double(M) * c->d * (4.0 + (c->bf16 ? 2.0 : 4.0) + (hcopy ? 4.0 : 0.0));
+  Span sp(c, WAM_KCLASS_NORM, 0.0, by);
+  CK(ln_modulate(hb, hcopy, c->mods, c->mod_n, shift_off, scale_off, map, c->xln, c->bf16, M, c->d, c->N, c->stream));
+  return WAM_OK;
+}
+
+// One adaLN DiT block on `Bw` items stored contiguously in hb.
+int run_layer(wam_ctx* c, int l, float* hb, int Bw, const int* map, float* hcopy) {
+  const int M = Bw * c->N, d = c->d;
+  const int base = l * 6 * d;
+  LayerW& w = c->layers[l];
+  TRY(ln_mod(c, hb, hcopy, base, base + d, map, M));
+  TRY(gemm(c, &c->tm_xln, c->xln, &w.tm_qkv, w.qkv_wt, M, 3 * d, d, kEpiBf16,
+           epi_args(w.qkv_b, c->qkv, nullptr, 0, c->N, nullptr)));
+  {
+    const double el = c->bf16 ? 2.0 : 4.0;
+    Span sp(c, WAM_KCLASS_ATTN, 4.0 * Bw * double(c->N) * c->N * d, el * 4.0 * M * d);
+    if (c->bf16)
+      CK(attention_bf16(static_cast<const bf16*>(c->qkv), static_cast<bf16*>(c->att), Bw, c->N, d, c->H, c->stream));
+    else
+      CK(attention_f32(static_cast<const float*>(c->qkv), static_cast<float*>(c->att), Bw, c->N, d, c->H, c->stream));
+  }
+  TRY(gemm(c, &c->tm_att, c->att, &w.tm_out, w.out_wt, M, d, d, kEpiResidF32,
+           epi_args(w.out_b, hb, c->mods + base + 2 * d, c->mod_n, c->N, map)));
+  TRY(ln_mod(c, hb, nullptr, base + 3 * d, base + 4 * d, map, M));
+  TRY(gemm(c, &c->tm_xln, c->xln, &w.tm_up, w.up_wt, M, c->dff, d, kEpiGeluBf16,
+           epi_args(w.up_b, c->u, nullptr, 0, c->N, nullptr)));
+  TRY(gemm(c, &c->tm_u, c->u, &w.tm_down, w.down_wt, M, d, c->dff, kEpiResidF32,
+           epi_args(w.down_b, hb, c->mods + base + 5 * d, c->mod_n, c->N, map)));
+  return WAM_OK;
+}
+
+int obs_embed(wam_ctx* c, wam_state* st) {
+  const int M = st->B * c->No;
+  if (c->bf16) {
+    {
+      Span sp(c, WAM_KCLASS_NORM, 0.0, 6.0 * M * c->d);
+      CK(cast_f32_bf16(st->obs, static_cast<bf16*>(c->obs_lp), int64_t(M) * c->d, c->stream));
+    }
+    TRY(gemm(c, &c->tm_obs_lp, c->obs_lp, &c->tm_obs_w, c->obs_wt, M, c->d, c->d, kEpiF32,
+             epi_args(c->obs_b, st->obs_emb, nullptr, 0, c->No, nullptr)));
+  } else {
+    TRY(gemm(c, nullptr, st->obs, nullptr, c->obs_wt, M, c->d, c->d, kEpiF32,
+             epi_args(c->obs_b, st->obs_emb, nullptr, 0, c->No, nullptr)));
+  }
+  return WAM_OK;
+}
+
+bool rr_enabled(const wam_ctx* c) {
+  const wam_config& g = c->cfg;
+  return g.rr_policy != WAM_RR_OFF && 0 < g.rr_q && g.rr_q < g.rr_s && g.rr_s < g.rr_e && g.rr_e < g.n_layers;
+}
+
+// Run every episode `n[b]` steps from its current stage (§3.2 native solver, §3.3 RR).
+int run_steps(wam_ctx* c, wam_state* st, const std::vector<int>& n) {
+  const int B = st->B;
+  const int d = c->d, N = c->N, L = c->L;
+  const int64_t stage_stride = int64_t(B) * c->T;
+  const bool rr_on = rr_enabled(c);
+  const int q = c->cfg.rr_q, s = c->cfg.rr_s, e = c->cfg.rr_e;
+  const int split_row = c->No + c->Nv;
+  TRY(obs_embed(c, st));
+  int max_n = 0;
+  for (int b = 0; b < B; ++b) max_n = std::max(max_n, n[b]);
+  st->log.clear();
+  std::vector<StepItem> items;
+  std::vector<int> rr_path, gate_ok;
+  std::vector<RRGate> gates(2 * B);
+  std::vector<RRApply> ap(B);
+  std::vector<int> midmap;
+  for (int i = 0; i < max_n; ++i) {
+    items.clear();
+    for (int b = 0; b < B; ++b) {
+      if (n[b] <= i) continue;
+      const int k = st->meta[b].stage;
+      StepItem it;
+      it.ep = b;
+      it.stage = k;
+      it.sigma = c->sigma[k];
+      it.dsigma = c->sigma[k + 1] - c->sigma[k];
+      items.push_back(it);
+    }
+    const int Bw = static_cast<int>(items.size());
+    TRY(upload(c, c->d_items, items.data(), sizeof(StepItem) * Bw));
+    // conditioning: features -> SiLU(W1) -> W2 -> SiLU -> every layer's modulation
+    {
+      Span sp(c, WAM_KCLASS_COND, 2.0 * Bw * 256 * d, 4.0 * 256 * d);
+      CK(cond_gemv(nullptr, c->d_items, c->t_w1, false, c->t_b1, c->t1, Bw, 256, d, kPreFeatures, 1, c->stream));
+    }
+    {
+      Span sp(c, WAM_KCLASS_COND, 2.0 * Bw * d * d, 4.0 * d * d);
+      CK(cond_gemv(c->t1, c->d_items, c->t_w2, false, c->t_b2, c->cvec, Bw, d, d, kPreNone, 0, c->stream));
+    }
+    {
+      Span sp(c, WAM_KCLASS_COND, 2.0 * Bw * d * c->mod_n, (c->bf16 ? 2.0 : 4.0) * d * c->mod_n);
+      CK(cond_gemv(c->cvec, c->d_items, c->mod_w, c->bf16, c->mod_b, c->mods, Bw, d, static_cast<int>(c->mod_n), kPreSilu, 0, c->stream));
+    }
+    {
+      Span sp(c, WAM_KCLASS_NORM, 0.0, 4.0 * Bw * double(N) * d * 2.0);
+      CK(embed_tokens(c->h, st->xhist, stage_stride, c->d_items, st->x, c->T, st->obs_emb, c->vid_w, c->vid_b,
+                      c->act_w, c->act_b, c->pos, Bw, c->No, c->Nv, c->vd, c->Na, c->ad, d, c->stream));
+    }
+    // RR eligibility per item (App. B.1 policies)
+    rr_path.assign(Bw, 0);
+    gate_ok.assign(Bw, 0);
+    bool any_rr = false, any_gate = false;
+    for (int w = 0; w < Bw; ++w) {
+      const EpisodeMeta& m = st->meta[items[w].ep];
+      if (!rr_on) continue;
+      const bool path_ok = c->cfg.rr_policy == WAM_RR_ALL_PATHS ||
+                           (c->cfg.rr_policy == WAM_RR_PREFIX_PATH && m.path == kPathPrefix);
+      if (!path_ok) continue;
+      rr_path[w] = 1;
+      any_rr = true;
+      const bool allowed = c->cfg.rr_policy == WAM_RR_ALL_PATHS || m.path_steps >= 1;
+      if (allowed && m.rr_valid) {
+        gate_ok[w] = 1;
+        any_gate = true;
+      }
+    }
+    std::vector<int> accepted(Bw, 0);
+    if (!any_rr) {
+      for (int l = 0; l < L; ++l) TRY(run_layer(c, l, c->h, Bw, nullptr, nullptr));
+    } else {
+      for (int l = 0; l < s; ++l) TRY(run_layer(c, l, c->h, Bw, nullptr, l == q ? c->hq : nullptr));
+      if (any_gate) {
+        const int nch = rr_num_chunks(int64_t(std::max(split_row, N - split_row)) * d);
+        {
+          Span sp(c, WAM_KCLASS_ADAPT, 0.0, 12.0 * Bw * double(N) * d);
+          CK(rr_probe_partial(c->h, c->hq, st->pa, c->d_items, Bw, N, d, split_row, nch, c->d_part, c->stream));
+        }
+        {
+          Span sp(c, WAM_KCLASS_ADAPT);
+          CK(rr_gate(c->d_part, Bw, nch, int64_t(split_row) * d, int64_t(N - split_row) * d, c->cfg.rr_alpha_min,
+                     c->cfg.rr_alpha_max, c->cfg.rr_eps, c->cfg.rr_gamma_cos, c->cfg.rr_gamma_fit, c->d_gate, c->stream));
+        }
+        TRY(readback(c, gates.data(), c->d_gate, sizeof(RRGate) * 2 * Bw));
+        for (int w = 0; w < Bw; ++w)
+          if (gate_ok[w] && gates[2 * w].pass && gates[2 * w + 1].pass) accepted[w] = 1;
+      }
+      midmap.clear();
+      for (int w = 0; w < Bw; ++w) {
+        ap[w].cidx = 0;
+        ap[w].alpha0 = ap[w].alpha1 = 0.0f;
+        if (accepted[w]) {
+          ap[w].mode = kRRInject;
+          ap[w].alpha0 = static_cast<float>(gates[2 * w].alpha);
+          ap[w].alpha1 = static_cast<float>(gates[2 * w + 1].alpha);
+        } else {
+          ap[w].mode = rr_path[w] ? kRRRefresh : kRRCopyBack;
+          ap[w].cidx = static_cast<int>(midmap.size());
+          midmap.push_back(w);
+        }
+      }
+      const int nmid = static_cast<int>(midmap.size());
+      if (nmid > 0) {
+        for (int j = 0; j < nmid; ++j)
+          CK(cudaMemcpyAsync(c->hm + int64_t(j) * N * d, c->h + int64_t(midmap[j]) * N * d,
+                             sizeof(float) * N * d, cudaMemcpyDeviceToDevice, c->stream));
+        TRY(upload(c, c->d_map, midmap.data(), sizeof(int) * nmid));
+        for (int l = s; l < e; ++l) TRY(run_layer(c, l, c->hm, nmid, c->d_map, nullptr));
+      }
+      TRY(upload(c, c->d_rrapply, ap.data(), sizeof(RRApply) * Bw));
+      {
+        Span sp(c, WAM_KCLASS_ADAPT, 0.0, 16.0 * Bw * double(N) * d);
+        CK(rr_apply(c->h, c->hm, c->hq, st->pa, st->ra, c->d_items, c->d_rrapply, Bw, N, d, split_row, c->stream));
+      }
+      for (int l = e; l < L; ++l) TRY(run_layer(c, l, c->h, Bw, nullptr, nullptr));
+    }
+    {
+      Span sp(c, WAM_KCLASS_NORM, 2.0 * Bw * double(c->Nv * c->vd + c->Na * c->ad) * d,
+              4.0 * Bw * double(c->Nv + c->Na) * d + 16.0 * Bw * c->T);
+      CK(final_euler(c->h, c->d_items, c->mods, c->mod_n, 6 * L * d, c->vout_w, c->vout_b, c->aout_w, c->aout_b,
+                     st->x, st->xhist, st->vhist, stage_stride, c->T, Bw, c->No, c->Nv, c->vd, c->Na, c->ad, d,
+                     c->stream));
+    }
+    // bookkeeping (§3.4) and reuse statistics (App. D.2)
+    for (int w = 0; w < Bw; ++w) {
+      EpisodeMeta& m = st->meta[items[w].ep];
+      wam_step_record rec;
+      std::memset(&rec, 0, sizeof(rec));
+      rec.episode = items[w].ep;
+      rec.stage = m.stage;
+      rec.rr_active = rr_path[w];
+      rec.rr_attempt = gate_ok[w];
+      rec.rr_accept = accepted[w];
+      if (gate_ok[w]) {
+        for (int br = 0; br < 2; ++br) {
+          rec.alpha[br] = static_cast<float>(gates[2 * w + br].alpha);
+          rec.cos[br] = static_cast<float>(gates[2 * w + br].cos);
+          rec.fit[br] = static_cast<float>(gates[2 * w + br].fit);
+        }
+      }
+      st->log.push_back(rec);
+      c->stats.n_episode_steps++;
+      c->stats.n_layer_evals += accepted[w] ? (L - (e - s)) : L;
+      if (rr_path[w]) {
+        c->stats.b_dense += L;
+        m.rr_valid = 1;
+      }
+      if (gate_ok[w]) c->stats.n_attempt++;
+      if (accepted[w]) {
+        c->stats.n_reuse++;
+        c->stats.b_skip += e - s;
+      }
+      m.stage++;
+      m.since_bind++;
+      m.path_steps++;
+      if (m.stage == c->K) m.finished = 1;
+    }
+  }
+  return WAM_OK;
+}
+
+int copy_out(wam_ctx* c, wam_state* st, float* actions_out, float* video_out, bool& host_out) {
+  if (actions_out != nullptr) {
+    const size_t w = sizeof(float) * c->Na * c->ad;
+    CK(cudaMemcpy2DAsync(actions_out, w, st->x + c->V, sizeof(float) * c->T, w, st->B, cudaMemcpyDefault, c->stream));
+    host_out = host_out || !is_device_ptr(actions_out);
+  }
+  if (video_out != nullptr) {
+    const size_t w = sizeof(float) * c->V;
+    CK(cudaMemcpy2DAsync(video_out, w, st->x, sizeof(float) * c->T, w, st->B, cudaMemcpyDefault, c->stream));
+    host_out = host_out || !is_device_ptr(video_out);
+  }
+  return WAM_OK;
+}
+
+int validate_cfg(const wam_config* g, std::string& why) {
+  if (g == nullptr) return why = "null config", WAM_ERR_INVALID_ARG;
+  if (g->n_layers < 1 || g->d_model < 1 || g->n_heads < 1 || g->mlp_ratio < 1 || g->n_obs < 1 ||
+      g->n_video < 1 || g->video_dim < 1 || g->n_action < 1 || g->action_dim < 1 || g->n_steps < 1 ||
+      g->batch_max < 1)
+    return why = "every size must be >= 1", WAM_ERR_INVALID_ARG;
+  if (g->d_model % g->n_heads != 0) return why = "d_model must be a multiple of n_heads", WAM_ERR_INVALID_ARG;
+  if (g->precision != WAM_PREC_FP32 && g->precision != WAM_PREC_BF16) return why = "unknown precision", WAM_ERR_INVALID_ARG;
+  if (g->batch_max > kMaxBatch) return why = "batch_max above 256", WAM_ERR_UNSUPPORTED;
+  if (g->d_model % 128 != 0 || g->d_model > 1536) return why = "d_model must be a multiple of 128, at most 1536", WAM_ERR_UNSUPPORTED;
+  if (g->video_dim > 16 || g->action_dim > 16) return why = "video_dim and action_dim must be <= 16", WAM_ERR_UNSUPPORTED;
+  const int dh = g->d_model / g->n_heads;
+  if (g->precision == WAM_PREC_BF16 && !attention_bf16_supported(dh)) return why = "bf16 attention supports head dim 64 or 72", WAM_ERR_UNSUPPORTED;
+  if (g->precision == WAM_PREC_FP32 && dh > 128) return why = "fp32 attention supports head dim <= 128", WAM_ERR_UNSUPPORTED;
+  if (!(g->sched_shift > 0.0f)) return why = "sched_shift must be > 0", WAM_ERR_INVALID_ARG;
+  if (g->tr_entry_stage < 0 || g->tr_entry_stage >= g->n_steps) return why = "tr_entry_stage outside [0, K)", WAM_ERR_INVALID_ARG;
+  if (g->tr_retain_stage >= g->n_steps || g->tr_retain_stage < -1) return why = "tr_retain_stage outside [-1, K)", WAM_ERR_INVALID_ARG;
+  if (g->rr_policy < 0 || g->rr_policy > 2) return why = "unknown rr_policy", WAM_ERR_INVALID_ARG;
+  if (g->rr_policy != WAM_RR_OFF &&
+      !(0 < g->rr_q && g->rr_q < g->rr_s && g->rr_s < g->rr_e && g->rr_e < g->n_layers))
+    return why = "RR needs 0 < q < s < e < n_layers", WAM_ERR_INVALID_ARG;
+  if (g->or_n_components < 1 || g->or_n_components > 4 || g->n_obs % g->or_n_components != 0)
+    return why = "or_n_components must be 1..4 and divide n_obs", WAM_ERR_INVALID_ARG;
+  for (int m = 0; m < g->or_n_components; ++m)
+    if (!(g->or_deltas[m] > 0.0f) || !(g->or_weights[m] >= 0.0f)) return why = "OR deltas must be > 0, weights >= 0", WAM_ERR_INVALID_ARG;
+  if (g->or_kappa_max < 0) return why = "or_kappa_max must be >= 0", WAM_ERR_INVALID_ARG;
+  const int64_t mod_n = int64_t(6 * g->n_layers + 2) * g->d_model;
+  if (mod_n % 2 != 0) return why = "modulation width must be even", WAM_ERR_UNSUPPORTED;
+  return WAM_OK;
+}
+
+size_t weight_count(const wam_config* g) {
+  const size_t d = g->d_model, L = g->n_layers, R = g->mlp_ratio, N = size_t(g->n_obs) + g->n_video + g->n_action;
+  const size_t vd = g->video_dim, ad = g->action_dim;
+  size_t n = d * d + d + vd * d + d + ad * d + d + N * d + 256 * d + d + d * d + d;
+  n += L * (d * 6 * d + 6 * d + d * 3 * d + 3 * d + d * d + d + d * R * d + R * d + R * d * d + d);
+  n += d * 2 * d + 2 * d + d * vd + vd + d * ad + ad;
+  return n;
+}
+
+int build_weights(wam_ctx* c, const float* src) {
+  const int d = c->d, L = c->L, dff = c->dff;
+  const bool b16 = c->bf16;
+  const size_t wel = b16 ? 2 : 4;
+  size_t off = 0;
+  auto take = [&](size_t n) {
+    const float* p = src + off;
+    off += n;
+    return p;
+  };
+  auto dmat = [&](void** out, size_t n) -> int {
+    void* p = nullptr;
+    if (cudaMalloc(&p, n * wel) != cudaSuccess) {
+      cudaGetLastError();
+      return fail(c, WAM_ERR_OOM, "weight allocation failed");
+    }
+    c->allocs.push_back(p);
+    *out = p;
+    return WAM_OK;
+  };
+  auto dvec = [&](float** out, const float* from, size_t n) -> int {
+    TRY(dalloc(c, c->allocs, out, n));
+    CK(cudaMemcpyAsync(*out, from, n * sizeof(float), cudaMemcpyDeviceToDevice, c->stream));
+    return WAM_OK;
+  };
+  auto tmat = [&](void** out, const float* from, int K, int Nn) -> int {  // [K,N] -> [N,K]
+    TRY(dmat(out, size_t(K) * Nn));
+    CK(transpose_cast(from, *out, b16, K, Nn, c->stream));
+    return WAM_OK;
+  };
+  TRY(tmat(&c->obs_wt, take(size_t(d) * d), d, d));
+  TRY(dvec(&c->obs_b, take(d), d));
+  TRY(dvec(&c->vid_w, take(size_t(c->vd) * d), size_t(c->vd) * d));
+  TRY(dvec(&c->vid_b, take(d), d));
+  TRY(dvec(&c->act_w, take(size_t(c->ad) * d), size_t(c->ad) * d));
+  TRY(dvec(&c->act_b, take(d), d));
+  TRY(dvec(&c->pos, take(size_t(c->N) * d), size_t(c->N) * d));
+  TRY(dvec(&c->t_w1, take(size_t(256) * d), size_t(256) * d));
+  TRY(dvec(&c->t_b1, take(d), d));
+  TRY(dvec(&c->t_w2, take(size_t(d) * d), size_t(d) * d));
+  TRY(dvec(&c->t_b2, take(d), d));
+  TRY(dmat(&c->mod_w, size_t(d) * c->mod_n));
+  TRY(dalloc(c, c->allocs, &c->mod_b, c->mod_n));
+  c->layers.resize(L);
+  for (int l = 0; l < L; ++l) {
+    LayerW& w = c->layers[l];
+    const float* ada_w = take(size_t(d) * 6 * d);
+    CK(copy_cast_2d(ada_w, 6 * d, static_cast<uint8_t*>(c->mod_w) + size_t(l) * 6 * d * wel, b16, c->mod_n, d, 6 * d, c->stream));
+    CK(cudaMemcpyAsync(c->mod_b + size_t(l) * 6 * d, take(6 * d), sizeof(float) * 6 * d, cudaMemcpyDeviceToDevice, c->stream));
+    TRY(tmat(&w.qkv_wt, take(size_t(d) * 3 * d), d, 3 * d));
+    TRY(dvec(&w.qkv_b, take(3 * d), 3 * d));
+    TRY(tmat(&w.out_wt, take(size_t(d) * d), d, d));
+    TRY(dvec(&w.out_b, take(d), d));
+    TRY(tmat(&w.up_wt, take(size_t(d) * dff), d, dff));
+    TRY(dvec(&w.up_b, take(dff), dff));
+    TRY(tmat(&w.down_wt, take(size_t(dff) * d), dff, d));
+    TRY(dvec(&w.down_b, take(d), d));
+  }
+  CK(copy_cast_2d(take(size_t(d) * 2 * d), 2 * d, static_cast<uint8_t*>(c->mod_w) + size_t(L) * 6 * d * wel, b16, c->mod_n, d, 2 * d, c->stream));
+  CK(cudaMemcpyAsync(c->mod_b + size_t(L) * 6 * d, take(2 * d), sizeof(float) * 2 * d, cudaMemcpyDeviceToDevice, c->stream));
+  TRY(dvec(&c->vout_w, take(size_t(d) * c->vd), size_t(d) * c->vd));
+  TRY(dvec(&c->vout_b, take(c->vd), c->vd));
+  TRY(dvec(&c->aout_w, take(size_t(d) * c->ad), size_t(d) * c->ad));
+  TRY(dvec(&c->aout_b, take(c->ad), c->ad));
+  if (off != weight_count(&c->cfg)) return fail(c, WAM_ERR_INVALID_ARG, "internal weight layout mismatch");
+  return WAM_OK;
+}
+
+int encode(wam_ctx* c, CUtensorMap* m, const void* base, uint64_t rows, uint64_t K) {
+  const int r = tc_encode_kmajor_bf16(m, base, rows, K);
+  if (r != 0) return fail(c, WAM_ERR_CUDA, "cuTensorMapEncodeTiled failed (" + std::to_string(r) + ")");
+  return WAM_OK;
+}
+
+int create_impl(wam_ctx* c, const wam_config* cfg, const float* weights, size_t n_weights, void* stream) {
+  std::string why;
+  const int v = validate_cfg(cfg, why);
+  if (v != WAM_OK) return fail(c, v, why);
+  if (weights == nullptr || n_weights != weight_count(cfg)) return fail(c, WAM_ERR_INVALID_ARG, "weights null or n_weights != wam_weight_count(cfg)");
+  c->cfg = *cfg;
+  c->L = cfg->n_layers;
+  c->d = cfg->d_model;
+  c->H = cfg->n_heads;
+  c->R = cfg->mlp_ratio;
+  c->No = cfg->n_obs;
+  c->Nv = cfg->n_video;
+  c->vd = cfg->video_dim;
+  c->Na = cfg->n_action;
+  c->ad = cfg->action_dim;
+  c->N = c->No + c->Nv + c->Na;
+  c->V = c->Nv * c->vd;
+  c->T = c->V + c->Na * c->ad;
+  c->K = cfg->n_steps;
+  c->dff = c->R * c->d;
+  c->Bmax = cfg->batch_max;
+  c->mod_n = int64_t(6 * c->L + 2) * c->d;
+  c->bf16 = cfg->precision == WAM_PREC_BF16;
+  c->stream = static_cast<cudaStream_t>(stream);
+  std::memset(&c->stats, 0, sizeof(c->stats));
+  for (int k = 0; k <= c->K; ++k) {
+    const double t = 1.0 - double(k) / c->K;
+    const double sft = cfg->sched_shift;
+    c->sigma.push_back(sft * t / (1.0 + (sft - 1.0) * t));
+  }
+  CK(cudaGetDevice(&c->device));
+  CK(cudaDeviceGetAttribute(&c->num_sms, cudaDevAttrMultiProcessorCount, c->device));
+  if (c->bf16) {
+    int major = 0, minor = 0;
+    CK(cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, c->device));
+    CK(cudaDeviceGetAttribute(&minor, cudaDevAttrComputeCapabilityMinor, c->device));
+    if (major != 10) return fail(c, WAM_ERR_UNSUPPORTED, "bf16 tensor-core kernels need a Blackwell (sm_10x) device");
+  }
+  if (c->bf16 && (c->dff % 128 != 0 || (3 * c->d) % 128 != 0))
+    return fail(c, WAM_ERR_UNSUPPORTED, "GEMM widths must be multiples of 128");
+  // weights: bring the flat buffer to the device once, then convert
+  const float* wdev = weights;
+  float* tmp = nullptr;
+  if (!is_device_ptr(weights)) {
+    if (cudaMalloc(&tmp, n_weights * sizeof(float)) != cudaSuccess) {
+      cudaGetLastError();
+      return fail(c, WAM_ERR_OOM, "weight staging allocation failed");
+    }
+    cudaError_t e = cudaMemcpyAsync(tmp, weights, n_weights * sizeof(float), cudaMemcpyHostToDevice, c->stream);
+    if (e != cudaSuccess) {
+      cudaFree(tmp);
+      return fail_cuda(c, "weight upload", e);
+    }
+    wdev = tmp;
+  }
+  const int rw = build_weights(c, wdev);
+  cudaError_t se = cudaStreamSynchronize(c->stream);
+  if (tmp) cudaFree(tmp);
+  if (rw != WAM_OK) return rw;
+  if (se != cudaSuccess) return fail_cuda(c, "weight conversion", se);
+  // activations
+  const size_t rows = size_t(c->Bmax) * c->N;
+  const size_t el = c->bf16 ? 2 : 4;
+  uint8_t *xln, *qkv, *att, *u, *olp;
+  TRY(dalloc(c, c->allocs, &c->h, rows * c->d));
+  TRY(dalloc(c, c->allocs, &c->hq, rows * c->d));
+  TRY(dalloc(c, c->allocs, &c->hm, rows * c->d));
+  TRY(dalloc(c, c->allocs, &xln, rows * c->d * el));
+  TRY(dalloc(c, c->allocs, &qkv, rows * 3 * c->d * el));
+  TRY(dalloc(c, c->allocs, &att, rows * c->d * el));
+  TRY(dalloc(c, c->allocs, &u, rows * c->dff * el));
+  TRY(dalloc(c, c->allocs, &olp, size_t(c->Bmax) * c->No * c->d * el));
+  c->xln = xln;
+  c->qkv = qkv;
+  c->att = att;
+  c->u = u;
+  c->obs_lp = olp;
+  TRY(dalloc(c, c->allocs, &c->t1, size_t(c->Bmax) * c->d));
+  TRY(dalloc(c, c->allocs, &c->cvec, size_t(c->Bmax) * c->d));
+  TRY(dalloc(c, c->allocs, &c->mods, size_t(c->Bmax) * c->mod_n));
+  TRY(dalloc(c, c->allocs, &c->d_items, c->Bmax));
+  TRY(dalloc(c, c->allocs, &c->d_map, c->Bmax));
+  TRY(dalloc(c, c->allocs, &c->d_rrapply, c->Bmax));
+  TRY(dalloc(c, c->allocs, &c->d_gate, 2 * c->Bmax));
+  TRY(dalloc(c, c->allocs, &c->d_adapt, c->Bmax));
+  TRY(dalloc(c, c->allocs, &c->d_eps, size_t(c->Bmax) * c->T));
+  TRY(dalloc(c, c->allocs, &c->d_obs_new, size_t(c->Bmax) * c->No * c->d));
+  TRY(dalloc(c, c->allocs, &c->d_err, 1));
+  CK(cudaMemset(c->d_err, 0, sizeof(int)));
+  // scratch for the float64 partial sums of TR / OR / RR reductions
+  const int split = c->No + c->Nv;
+  const size_t p_tr = size_t(c->Bmax) * 2 * tr_num_chunks(c->T, c->V);
+  const size_t p_or = size_t(c->Bmax) * cfg->or_n_components * or_num_chunks(int64_t(c->No / cfg->or_n_components) * c->d);
+  const size_t p_rr = size_t(c->Bmax) * 2 * 3 * rr_num_chunks(int64_t(std::max(split, c->N - split)) * c->d);
+  c->part_doubles = std::max(p_tr, std::max(p_or, p_rr));
+  TRY(dalloc(c, c->allocs, &c->d_part, c->part_doubles));
+  if (c->bf16) {
+    TRY(encode(c, &c->tm_xln, c->xln, rows, c->d));
+    TRY(encode(c, &c->tm_att, c->att, rows, c->d));
+    TRY(encode(c, &c->tm_u, c->u, rows, c->dff));
+    TRY(encode(c, &c->tm_obs_lp, c->obs_lp, size_t(c->Bmax) * c->No, c->d));
+    TRY(encode(c, &c->tm_obs_w, c->obs_wt, c->d, c->d));
+    for (LayerW& w : c->layers) {
+      TRY(encode(c, &w.tm_qkv, w.qkv_wt, 3 * c->d, c->d));
+      TRY(encode(c, &w.tm_out, w.out_wt, c->d, c->d));
+      TRY(encode(c, &w.tm_up, w.up_wt, c->dff, c->d));
+      TRY(encode(c, &w.tm_down, w.down_wt, c->d, c->dff));
+    }
+  }
+  CK(cudaHostAlloc(reinterpret_cast<void**>(&c->ring), kRingSlots * kSlotBytes, cudaHostAllocDefault));
+  for (int i = 0; i < kRingSlots; ++i) {
+    CK(cudaEventCreateWithFlags(&c->ring_ev[i], cudaEventDisableTiming));
+    c->ring_used[i] = false;
+  }
+  c->readback_bytes = std::max<size_t>(c->part_doubles * sizeof(double), sizeof(RRGate) * 2 * c->Bmax) + 64;
+  CK(cudaHostAlloc(reinterpret_cast<void**>(&c->readback), c->readback_bytes, cudaHostAllocDefault));
+  return WAM_OK;
+}
+
+void destroy_impl(wam_ctx* c) {
+  if (!c->allocs.empty()) cudaStreamSynchronize(c->stream);
+  for (void* p : c->allocs) cudaFree(p);
+  c->allocs.clear();
+  if (c->ring) {
+    cudaFreeHost(c->ring);
+    for (int i = 0; i < kRingSlots; ++i)
+      if (c->ring_ev[i]) cudaEventDestroy(c->ring_ev[i]);
+  }
+  if (c->readback) cudaFreeHost(c->readback);
+  for (cudaEvent_t e : c->evpool) cudaEventDestroy(e);
+}
+
+int field_ptr(wam_ctx* c, const wam_state* st, int field, int index, void** p, size_t* bytes) {
+  const size_t BT = size_t(st->B) * c->T;
+  switch (field) {
+    case WAM_FIELD_X: *p = st->x; *bytes = BT * 4; return WAM_OK;
+    case WAM_FIELD_X_STAGE:
+      if (index < 0 || index > c->K) return fail(c, WAM_ERR_INVALID_ARG, "stage index out of range");
+      *p = st->xhist + size_t(index) * BT; *bytes = BT * 4; return WAM_OK;
+    case WAM_FIELD_V_STEP:
+      if (index < 0 || index >= c->K) return fail(c, WAM_ERR_INVALID_ARG, "step index out of range");
+      *p = st->vhist + size_t(index) * BT; *bytes = BT * 4; return WAM_OK;
+    case WAM_FIELD_X_INIT: *p = st->xb0; *bytes = BT * 4; return WAM_OK;
+    case WAM_FIELD_OBS: *p = st->obs; *bytes = size_t(st->B) * c->No * c->d * 4; return WAM_OK;
+    case WAM_FIELD_RR_P:
+    case WAM_FIELD_RR_R:
+      if (st->pa == nullptr) return fail(c, WAM_ERR_BAD_STATE, "RR is off for this context");
+      *p = field == WAM_FIELD_RR_P ? st->pa : st->ra;
+      *bytes = size_t(st->B) * c->N * c->d * 4;
+      return WAM_OK;
+    default: return fail(c, WAM_ERR_INVALID_ARG, "unknown field");
+  }
+}
+
+}  // namespace
+
+// =========================================================================================
+// Public C ABI
+// =========================================================================================
+extern "C" {
+
+size_t wam_weight_count(const wam_config* cfg) {
+  std::string why;
+  if (validate_cfg(cfg, why) == WAM_ERR_INVALID_ARG) return 0;
+  return weight_count(cfg);
+}
+
+int wam_create(const wam_config* cfg, const float* weights, size_t n_weights, void* stream, wam_ctx** out) {
+  if (out == nullptr) return WAM_ERR_INVALID_ARG;
+  *out = nullptr;
+  wam_ctx* c = new (std::nothrow) wam_ctx();
+  if (c == nullptr) return WAM_ERR_OOM;
+  std::memset(c->ring_ev, 0, sizeof(c->ring_ev));
+  const int r = create_impl(c, cfg, weights, n_weights, stream);
+  if (r != WAM_OK) {
+    std::fprintf(stderr, "wam_create: %s\n", c->err.c_str());
+    destroy_impl(c);
+    delete c;
+    return r;
+  }
+  *out = c;
+  return WAM_OK;
+}
+
+void wam_destroy(wam_ctx* c) {
+  if (c == nullptr) return;
+  destroy_impl(c);
+  delete c;
+}
+
+const char* wam_last_error(const wam_ctx* c) { return c ? c->err.c_str() : "null context"; }
+
+int wam_set_stream(wam_ctx* c, void* stream) {
+  if (c == nullptr) return WAM_ERR_INVALID_ARG;
+  c->stream = static_cast<cudaStream_t>(stream);
+  return WAM_OK;
+}
+
+int wam_state_create(wam_ctx* c, int32_t batch, wam_state** out) {
+  if (c == nullptr || out == nullptr) return WAM_ERR_INVALID_ARG;
+  *out = nullptr;
+  if (batch < 1 || batch > c->Bmax) return fail(c, WAM_ERR_INVALID_ARG, "batch outside [1, batch_max]");
+  wam_state* st = new (std::nothrow) wam_state();
+  if (st == nullptr) return fail(c, WAM_ERR_OOM, "host allocation failed");
+  st->ctx = c;
+  st->B = batch;
+  const size_t BT = size_t(batch) * c->T;
+  auto cleanup = [&](int r) {
+    for (void* p : st->allocs) cudaFree(p);
+    delete st;
+    return r;
+  };
+  int r;
+  if ((r = dalloc(c, st->allocs, &st->x, BT)) != WAM_OK) return cleanup(r);
+  if ((r = dalloc(c, st->allocs, &st->xhist, BT * (c->K + 1))) != WAM_OK) return cleanup(r);
+  if ((r = dalloc(c, st->allocs, &st->vhist, BT * c->K)) != WAM_OK) return cleanup(r);
+  if ((r = dalloc(c, st->allocs, &st->xb0, BT)) != WAM_OK) return cleanup(r);
+  if ((r = dalloc(c, st->allocs, &st->obs, size_t(batch) * c->No * c->d)) != WAM_OK) return cleanup(r);
+  if ((r = dalloc(c, st->allocs, &st->obs_emb, size_t(batch) * c->No * c->d)) != WAM_OK) return cleanup(r);
+  if (rr_enabled(c)) {
+    if ((r = dalloc(c, st->allocs, &st->pa, size_t(batch) * c->N * c->d)) != WAM_OK) return cleanup(r);
+    if ((r = dalloc(c, st->allocs, &st->ra, size_t(batch) * c->N * c->d)) != WAM_OK) return cleanup(r);
+  }
+  cudaError_t e = cudaSuccess;
+  e = e == cudaSuccess ? cudaMemsetAsync(st->xhist, 0, BT * (c->K + 1) * 4, c->stream) : e;
+  e = e == cudaSuccess ? cudaMemsetAsync(st->vhist, 0, BT * c->K * 4, c->stream) : e;
+  if (st->pa) {
+    e = e == cudaSuccess ? cudaMemsetAsync(st->pa, 0, size_t(batch) * c->N * c->d * 4, c->stream) : e;
+    e = e == cudaSuccess ? cudaMemsetAsync(st->ra, 0, size_t(batch) * c->N * c->d * 4, c->stream) : e;
+  }
+  if (e != cudaSuccess) return cleanup(fail_cuda(c, "state init", e));
+  st->meta.assign(batch, EpisodeMeta());
+  *out = st;
+  return WAM_OK;
+}
+
+void wam_state_destroy(wam_state* st) {
+  if (st == nullptr) return;
+  if (st->ctx) cudaStreamSynchronize(st->ctx->stream);
+  for (void* p : st->allocs) cudaFree(p);
+  delete st;
+}
+
+int wam_adapt_state(wam_ctx* c, wam_state* st, const float* new_obs, const int32_t* executed_shift,
+                    const int32_t* entry_stage, const float* fresh_noise, int32_t* status_out) {
+  if (c == nullptr || st == nullptr || st->ctx != c) return WAM_ERR_INVALID_ARG;
+  if (new_obs == nullptr) return fail(c, WAM_ERR_INVALID_ARG, "new_obs is required");
+  const int B = st->B;
+  const wam_config& g = c->cfg;
+  std::vector<AdaptItem> ad(B);
+  std::vector<int32_t> status(B, 0);
+  std::vector<EpisodeMeta> meta = st->meta;  // committed only on success
+  std::vector<int> rebind;                   // episodes needing the consistency score
+  bool need_eps = false, any_tr = false;
+  wam_stats dstats;
+  std::memset(&dstats, 0, sizeof(dstats));
+  for (int b = 0; b < B; ++b) {
+    AdaptItem& a = ad[b];
+    std::memset(&a, 0, sizeof(a));
+    EpisodeMeta& m = meta[b];
+    const int shift = executed_shift ? executed_shift[b] : 0;
+    const int entry = entry_stage ? entry_stage[b] : g.tr_entry_stage;
+    if (shift < 0) return fail(c, WAM_ERR_INVALID_ARG, "executed_shift must be >= 0");
+    if (entry == WAM_ENTRY_COLD) {
+      a.op = kAdaptCold;
+      a.bind_obs = 1;
+      need_eps = true;
+      m = EpisodeMeta();
+      m.stage = 0;
+      status[b] = WAM_ADAPT_COLD_INIT;
+    } else if (m.finished) {
+      const int b0 = entry;
+      const int r = g.tr_retain_stage < 0 ? b0 : g.tr_retain_stage;
+      if (b0 < 0 || b0 >= c->K) return fail(c, WAM_ERR_INVALID_ARG, "entry stage outside [0, K)");
+      if (r < m.hist_from || r >= c->K) return fail(c, WAM_ERR_BAD_STATE, "retained stage not produced by the last replan");
+      a.op = kAdaptTR;
+      a.shift = shift;
+      a.r = r;
+      a.sigma_r = c->sigma[r];
+      a.sigma_b0 = c->sigma[b0];
+      a.bind_obs = 1;
+      need_eps = true;
+      any_tr = true;
+      m.stage = b0;
+      m.b0 = b0;
+      m.hist_from = b0;
+      m.finished = 0;
+      m.since_bind = 0;
+      m.path = kPathPrefix;
+      m.path_steps = 0;
+      dstats.n_noninitial++;
+      status[b] = m.kappa >= g.or_kappa_max ? WAM_ADAPT_TR_INIT_NO_PREFIX : WAM_ADAPT_TR_INIT;
+    } else if (m.stage < 0) {
+      return fail(c, WAM_ERR_BAD_STATE, "episode has no state yet (start it cold)");
+    } else {
+      if (shift != 0) return fail(c, WAM_ERR_BAD_STATE, "rebinding an in-flight replan takes no shift");
+      a.bind_obs = 1;
+      if (m.since_bind == 0) {
+        m.kappa = 0;
+        m.path = kPathRefresh;
+        m.path_steps = 0;
+        status[b] = WAM_ADAPT_REFRESH;
+      } else {
+        rebind.push_back(b);
+      }
+    }
+  }
+  if (need_eps && fresh_noise == nullptr) return fail(c, WAM_ERR_INVALID_ARG, "fresh_noise is required for remapping / cold starts");
+  const size_t obs_elems = size_t(c->No) * c->d;
+  CK(cudaMemcpyAsync(c->d_obs_new, new_obs, sizeof(float) * obs_elems * B, cudaMemcpyDefault, c->stream));
+  if (need_eps) CK(cudaMemcpyAsync(c->d_eps, fresh_noise, sizeof(float) * size_t(B) * c->T, cudaMemcpyDefault, c->stream));
+  if (!rebind.empty()) {
+    // Eq. 4: weighted RMS of the per-component normalised RMSE between the bound (predicted)
+    // condition and the new (real) one; partial sums on the device, combined here in float64.
+    const int M = g.or_n_components;
+    const int nch = or_num_chunks(int64_t(c->No / M) * c->d);
+    float inv_delta[4] = {1.f, 1.f, 1.f, 1.f};
+    for (int m = 0; m < M; ++m) inv_delta[m] = 1.0f / g.or_deltas[m];
+    {
+      Span sp(c, WAM_KCLASS_ADAPT, 0.0, 8.0 * B * obs_elems);
+      CK(or_score_partial(st->obs, c->d_obs_new, B, int64_t(obs_elems), M, inv_delta, nch, c->d_part, c->stream));
+    }
+    std::vector<double> part(size_t(B) * M * nch);
+    TRY(readback(c, part.data(), c->d_part, sizeof(double) * part.size()));
+    const double comp = double(c->No / M) * c->d;
+    for (int b : rebind) {
+      double num = 0.0, den = 0.0;
+      for (int m = 0; m < M; ++m) {
+        double s = 0.0;
+        for (int k = 0; k < nch; ++k) s += part[(size_t(b) * M + m) * nch + k];
+        const double e2 = s / comp;  // e_m^2
+        num += g.or_weights[m] * e2;
+        den += g.or_weights[m];
+      }
+      const double S = std::sqrt(num / den);
+      EpisodeMeta& m = meta[b];
+      dstats.n_start++;
+      if (S < g.or_tau && m.kappa < g.or_kappa_max) {
+        m.kappa++;
+        m.since_bind = 0;
+        dstats.n_bind++;
+        status[b] = WAM_ADAPT_REBIND_ACCEPT;
+      } else {
+        ad[b].op = kAdaptRestart;
+        m.stage = m.b0;
+        m.kappa = 0;
+        m.since_bind = 0;
+        m.path = kPathRefresh;
+        m.path_steps = 0;
+        status[b] = WAM_ADAPT_REBIND_RESTART;
+      }
+    }
+  }
+  TRY(upload(c, c->d_adapt, ad.data(), sizeof(AdaptItem) * B));
+  const int64_t stage_stride = int64_t(B) * c->T;
+  const int nch = tr_num_chunks(c->T, c->V);
+  if (any_tr) {
+    Span sp(c, WAM_KCLASS_ADAPT, 0.0, 8.0 * B * c->T);
+    CK(tr_rms_partial(c->d_adapt, st->xhist, stage_stride, c->K, B, c->T, c->V, nch, c->d_part, c->stream));
+  }
+  {
+    Span sp(c, WAM_KCLASS_ADAPT, 0.0, 16.0 * B * c->T + 8.0 * B * obs_elems);
+    CK(adapt_apply(c->d_adapt, c->d_part, nch, st->x, st->xb0, st->xhist, stage_stride, c->K, c->d_eps, c->d_obs_new,
+                   st->obs, B, c->T, c->V, c->Na, c->ad, int64_t(obs_elems), g.tr_normalize, g.tr_video_mode, c->stream));
+  }
+  st->meta = meta;
+  c->stats.n_noninitial += dstats.n_noninitial;
+  c->stats.n_start += dstats.n_start;
+  c->stats.n_bind += dstats.n_bind;
+  if (status_out) std::memcpy(status_out, status.data(), sizeof(int32_t) * B);
+  return WAM_OK;
+}
+
+int wam_continue(wam_ctx* c, wam_state* st, const int32_t* n_steps, float* actions_out, float* video_out) {
+  if (c == nullptr || st == nullptr || st->ctx != c || n_steps == nullptr) return WAM_ERR_INVALID_ARG;
+  std::vector<int> n(st->B);
+  for (int b = 0; b < st->B; ++b) {
+    n[b] = n_steps[b];
+    const EpisodeMeta& m = st->meta[b];
+    if (n[b] < 0) return fail(c, WAM_ERR_INVALID_ARG, "n_steps must be >= 0");
+    if (n[b] == 0) continue;
+    if (m.stage < 0 || m.finished) return fail(c, WAM_ERR_BAD_STATE, "episode is not adapted (finished or never started)");
+    if (m.stage + n[b] > c->K) return fail(c, WAM_ERR_INVALID_ARG, "stage + n_steps exceeds K");
+  }
+  TRY(run_steps(c, st, n));
+  bool host_out = false;
+  TRY(copy_out(c, st, actions_out, video_out, host_out));
+  if (host_out) TRY(sync_check(c));
+  return WAM_OK;
+}
+
+int wam_sample_cold(wam_ctx* c, wam_state* st, const float* obs, const float* noise, int32_t n_steps, float* actions_out) {
+  if (c == nullptr || st == nullptr || st->ctx != c || obs == nullptr || noise == nullptr) return WAM_ERR_INVALID_ARG;
+  if (n_steps < 1 || n_steps > c->K) return fail(c, WAM_ERR_INVALID_ARG, "n_steps outside [1, K]");
+  std::vector<int32_t> entry(st->B, WAM_ENTRY_COLD);
+  TRY(wam_adapt_state(c, st, obs, nullptr, entry.data(), noise, nullptr));
+  std::vector<int32_t> n(st->B, n_steps);
+  return wam_continue(c, st, n.data(), actions_out, nullptr);
+}
+
+int wam_get_stats(wam_ctx* c, wam_stats* out) {
+  if (c == nullptr || out == nullptr) return WAM_ERR_INVALID_ARG;
+  *out = c->stats;
+  return WAM_OK;
+}
+
+int wam_reset_stats(wam_ctx* c) {
+  if (c == nullptr) return WAM_ERR_INVALID_ARG;
+  std::memset(&c->stats, 0, sizeof(c->stats));
+  return WAM_OK;
+}
+
+int wam_state_log(const wam_state* st, wam_step_record* out, int32_t capacity, int32_t* n_out) {
+  if (st == nullptr || n_out == nullptr || (capacity > 0 && out == nullptr)) return WAM_ERR_INVALID_ARG;
+  const int n = std::min<int>(capacity, static_cast<int>(st->log.size()));
+  if (n > 0) std::memcpy(out, st->log.data(), sizeof(wam_step_record) * n);
+  *n_out = static_cast<int32_t>(st->log.size());
+  return WAM_OK;
+}
+
+int wam_state_read(wam_ctx* c, const wam_state* st, int32_t field, int32_t index, void* out, size_t n_bytes) {
+  if (c == nullptr || st == nullptr || out == nullptr || st->ctx != c) return WAM_ERR_INVALID_ARG;
+  if (field == WAM_FIELD_META) {
+    const size_t need = size_t(st->B) * 8 * sizeof(int32_t);
+    if (n_bytes != need) return fail(c, WAM_ERR_INVALID_ARG, "META needs B*8 int32");
+    int32_t* o = static_cast<int32_t*>(out);
+    for (int b = 0; b < st->B; ++b) {
+      const EpisodeMeta& m = st->meta[b];
+      const int32_t v[8] = {m.stage, m.hist_from, m.b0, m.kappa, m.finished, m.since_bind, m.path, m.rr_valid};
+      std::memcpy(o + 8 * b, v, sizeof(v));
+    }
+    return WAM_OK;
+  }
+  void* p = nullptr;
+  size_t bytes = 0;
+  TRY(field_ptr(c, st, field, index, &p, &bytes));
+  if (n_bytes != bytes) return fail(c, WAM_ERR_INVALID_ARG, "n_bytes does not match the field size");
+  CK(cudaMemcpyAsync(out, p, bytes, cudaMemcpyDefault, c->stream));
+  if (!is_device_ptr(out)) TRY(sync_check(c));
+  return WAM_OK;
+}
+
+int wam_state_write(wam_ctx* c, wam_state* st, int32_t field, int32_t index, const void* in, size_t n_bytes) {
+  if (c == nullptr || st == nullptr || in == nullptr || st->ctx != c) return WAM_ERR_INVALID_ARG;
+  if (field == WAM_FIELD_META) {
+    const size_t need = size_t(st->B) * 8 * sizeof(int32_t);
+    if (n_bytes != need) return fail(c, WAM_ERR_INVALID_ARG, "META needs B*8 int32");
+    const int32_t* v = static_cast<const int32_t*>(in);
+    for (int b = 0; b < st->B; ++b) {
+      const int32_t* e = v + 8 * b;
+      if (e[0] < -1 || e[0] > c->K || e[1] < 0 || e[1] > c->K || e[2] < 0 || e[2] >= c->K || e[3] < 0 || e[6] < 0 || e[6] > 2)
+        return fail(c, WAM_ERR_INVALID_ARG, "META values out of range");
+    }
+    for (int b = 0; b < st->B; ++b) {
+      const int32_t* e = v + 8 * b;
+      EpisodeMeta& m = st->meta[b];
+      m.stage = e[0];
+      m.hist_from = e[1];
+      m.b0 = e[2];
+      m.kappa = e[3];
+      m.finished = e[4];
+      m.since_bind = e[5];
+      m.path = e[6];
+      m.rr_valid = e[7];
+      m.path_steps = 0;
+    }
+    return WAM_OK;
+  }
+  void* p = nullptr;
+  size_t bytes = 0;
+  TRY(field_ptr(c, st, field, index, &p, &bytes));
+  if (n_bytes != bytes) return fail(c, WAM_ERR_INVALID_ARG, "n_bytes does not match the field size");
+  CK(cudaMemcpyAsync(p, in, bytes, cudaMemcpyDefault, c->stream));
+  if (!is_device_ptr(in)) CK(cudaStreamSynchronize(c->stream));
+  return WAM_OK;
+}
+
+int wam_sync(wam_ctx* c) {
+  if (c == nullptr) return WAM_ERR_INVALID_ARG;
+  return sync_check(c);
+}
+
+int wam_profile_enable(wam_ctx* c, int32_t enable) {
+  if (c == nullptr) return WAM_ERR_INVALID_ARG;
+  CK(cudaStreamSynchronize(c->stream));
+  c->spans.clear();
+  c->evnext = 0;
+  c->prof_on = enable != 0;
+  return WAM_OK;
+}
+
+int wam_profile_read(wam_ctx* c, wam_kclass_timing* out) {
+  if (c == nullptr || out == nullptr) return WAM_ERR_INVALID_ARG;
+  CK(cudaStreamSynchronize(c->stream));
+  for (int k = 0; k < WAM_KCLASS_COUNT; ++k) out[k] = wam_kclass_timing{0, 0.0, 0.0, 0.0};
+  for (const ProfSpan& s : c->spans) {
+    float ms = 0.0f;
+    CK(cudaEventElapsedTime(&ms, s.a, s.b));
+    wam_kclass_timing& t = out[s.kclass];
+    t.launches++;
+    t.ms += ms;
+    t.flops += s.flops;
+    t.bytes += s.bytes;
+  }
+  return WAM_OK;
+}
+
+}  // extern "C"

@@ -26,3 +26,27 @@ def micro_config(**overrides):
 @pytest.fixture
 def micro():
     return micro_config
+
+
+def pytest_collection_modifyitems(config, items):
+    """GPU tests need a CUDA device; on a machine without one they are skipped, never faked."""
+    try:
+        import torch
+        has_gpu = torch.cuda.is_available()
+    except Exception:
+        has_gpu = False
+    if has_gpu:
+        return
+    skip = pytest.mark.skip(reason="no CUDA device")
+    for item in items:
+        if "gpu" in item.keywords:
+            item.add_marker(skip)
+
+
+@pytest.fixture(scope="session")
+def wamlib():
+    """The built CUDA library (built in-tree if stale)."""
+    from paper_2609_34608_gb300 import _build
+    from paper_2609_34608_gb300 import wam as W
+    _build.build()
+    return W.lib()

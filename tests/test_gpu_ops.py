@@ -1,0 +1,143 @@
+"""Kernel-level parity on the GPU: each hot-path kernel, called through the C ABI
+(include/wam_ops.h), against the oracle's arithmetic on the same bf16-representable inputs."""
+import numpy as np
+import pytest
+import torch
+
+from oracle import wam_oracle as O
+from paper_2609_34608_gb300 import wam as W
+
+pytestmark = pytest.mark.gpu
+
+
+def _bf16(a):
+    return torch.from_numpy(np.asarray(a, dtype=np.float32)).to(torch.bfloat16)
+
+
+def _f64(t):
+    return t.to(torch.float64).cpu().numpy()
+
+
+GEMM_SHAPES = [
+    (1, 128, 64), (100, 384, 128), (128, 128, 64), (129, 256, 192),
+    (1296, 2304, 768),     # QKV of the 12-block d768 model, one episode
+    (300, 768, 3072),      # MLP down-projection width
+    (2500, 1024, 1024),
+    (4914, 3456, 1152),    # QKV of the 28-block d1152 model, one episode
+    (20000, 1024, 1024),   # enough tiles for the 256-wide variant
+]
+
+
+@pytest.mark.parametrize("M,N,K", GEMM_SHAPES)
+@pytest.mark.parametrize("epi", [W.EPI_BF16, W.EPI_GELU_BF16, W.EPI_RESID_F32, W.EPI_F32])
+def test_gemm_tcgen05_matches_reference(wamlib, M, N, K, epi):
+    rng = np.random.default_rng(M * 7 + N * 3 + K + epi)
+    A = _bf16(rng.standard_normal((M, K)))
+    Wt = _bf16(rng.standard_normal((N, K)) * 0.05)
+    bias = torch.from_numpy((rng.standard_normal(N) * 0.1).astype(np.float32))
+    acc = _f64(A) @ _f64(Wt).T + bias.double().numpy()
+    dev = torch.device("cuda")
+    Ad, Wd, bd = A.to(dev), Wt.to(dev), bias.to(dev)
+    rpi = 37
+    if epi in (W.EPI_BF16, W.EPI_GELU_BF16):
+        C = torch.full((M, N), float("nan"), dtype=torch.bfloat16, device=dev)
+        expect = O.gelu_tanh(acc) if epi == W.EPI_GELU_BF16 else acc
+        W.op_gemm_bf16(Ad, Wd, bd, C, M, N, K, epi)
+        torch.cuda.synchronize()
+        err = np.max(np.abs(_f64(C) - expect))
+        assert err <= 8e-3 * np.max(np.abs(expect)) + 1e-3
+    elif epi == W.EPI_F32:
+        C = torch.full((M, N), float("nan"), dtype=torch.float32, device=dev)
+        W.op_gemm_bf16(Ad, Wd, bd, C, M, N, K, epi)
+        torch.cuda.synchronize()
+        assert np.max(np.abs(_f64(C) - acc)) <= 1e-4 * np.max(np.abs(acc))
+    else:
+        items = (M + rpi - 1) // rpi
+        gate = torch.from_numpy(rng.standard_normal((items, N + 4)).astype(np.float32))
+        h0 = torch.from_numpy(rng.standard_normal((M, N)).astype(np.float32))
+        C = h0.to(dev)
+        W.op_gemm_bf16(Ad, Wd, bd, C, M, N, K, epi, gate=gate.to(dev), gate_stride=N + 4, rows_per_item=rpi)
+        torch.cuda.synchronize()
+        g = gate.double().numpy()[np.arange(M) // rpi, :N]
+        expect = h0.double().numpy() + g * acc
+        assert np.max(np.abs(_f64(C) - expect)) <= 1e-4 * np.max(np.abs(expect))
+
+
+def test_gemm_rejects_unsupported_shapes(wamlib):
+    dev = torch.device("cuda")
+    A = torch.zeros((4, 96), dtype=torch.bfloat16, device=dev)
+    Wt = torch.zeros((128, 96), dtype=torch.bfloat16, device=dev)
+    C = torch.zeros((4, 128), dtype=torch.bfloat16, device=dev)
+    with pytest.raises(W.WamError):
+        W.op_gemm_bf16(A, Wt, None, C, 4, 128, 96, W.EPI_BF16)
+
+
+@pytest.mark.parametrize("M,N,K", [(1, 64, 16), (77, 130, 45), (300, 512, 128)])
+def test_gemm_f32_matches_reference(wamlib, M, N, K):
+    rng = np.random.default_rng(M + N + K)
+    A = rng.standard_normal((M, K)).astype(np.float32)
+    Wt = rng.standard_normal((N, K)).astype(np.float32)
+    b = rng.standard_normal(N).astype(np.float32)
+    dev = torch.device("cuda")
+    C = torch.empty((M, N), dtype=torch.float32, device=dev)
+    W.op_gemm_f32(torch.from_numpy(A).to(dev), torch.from_numpy(Wt).to(dev), torch.from_numpy(b).to(dev), C,
+                  M, N, K, W.EPI_F32)
+    torch.cuda.synchronize()
+    ref = A.astype(np.float64) @ Wt.astype(np.float64).T + b
+    assert np.max(np.abs(C.cpu().numpy() - ref)) <= 1e-5 * np.max(np.abs(ref)) * np.sqrt(K)
+
+
+ATTN_CASES = [
+    (1, 1, 2, 64), (1, 56, 2, 64), (2, 64, 2, 64), (1, 100, 3, 64), (2, 1296, 2, 64),
+    (1, 65, 2, 72), (1, 257, 2, 72), (1, 4914, 1, 72),
+]
+
+
+@pytest.mark.parametrize("B,N,H,dh", ATTN_CASES)
+def test_attention_bf16_matches_oracle(wamlib, B, N, H, dh):
+    rng = np.random.default_rng(B * 1000 + N + H + dh)
+    d = H * dh
+    qkv = _bf16(rng.standard_normal((B * N, 3 * d)))
+    dev = torch.device("cuda")
+    out = torch.full((B * N, d), float("nan"), dtype=torch.bfloat16, device=dev)
+    W.op_attention(qkv.to(dev), out, B, N, d, H, "bf16")
+    torch.cuda.synchronize()
+    q64 = _f64(qkv)
+    got = _f64(out)
+    for b in range(B):
+        blk = q64[b * N:(b + 1) * N]
+        ref = O.attention(blk[:, :d], blk[:, d:2 * d], blk[:, 2 * d:], H)
+        assert np.max(np.abs(got[b * N:(b + 1) * N] - ref)) <= 2e-2
+
+
+def test_attention_f32_matches_oracle(wamlib):
+    rng = np.random.default_rng(9)
+    B, N, H, dh = 2, 56, 4, 32
+    d = H * dh
+    qkv = rng.standard_normal((B * N, 3 * d)).astype(np.float32)
+    dev = torch.device("cuda")
+    out = torch.empty((B * N, d), dtype=torch.float32, device=dev)
+    W.op_attention(torch.from_numpy(qkv).to(dev), out, B, N, d, H, "fp32")
+    torch.cuda.synchronize()
+    got = out.cpu().numpy()
+    for b in range(B):
+        blk = qkv[b * N:(b + 1) * N].astype(np.float64)
+        ref = O.attention(blk[:, :d], blk[:, d:2 * d], blk[:, 2 * d:], H)
+        assert np.max(np.abs(got[b * N:(b + 1) * N] - ref)) <= 2e-5
+
+
+@pytest.mark.parametrize("prec,d", [("bf16", 768), ("fp32", 128), ("bf16", 1152)])
+def test_ln_modulate_matches_oracle(wamlib, prec, d):
+    rng = np.random.default_rng(d)
+    M, rpi = 300, 100
+    h = (rng.standard_normal((M, d)) * 3 + 0.5).astype(np.float32)
+    mods = (rng.standard_normal((M // rpi, 2 * d)) * 0.3).astype(np.float32)
+    dev = torch.device("cuda")
+    md = torch.from_numpy(mods).to(dev)
+    out = torch.empty((M, d), dtype=torch.bfloat16 if prec == "bf16" else torch.float32, device=dev)
+    W.op_ln_modulate(torch.from_numpy(h).to(dev), md.data_ptr(), md.data_ptr() + 4 * d, 2 * d, out, M, d, rpi, prec)
+    torch.cuda.synchronize()
+    item = np.arange(M) // rpi
+    ref = O.layer_norm(h.astype(np.float64)) * (1 + mods[item, d:]) + mods[item, :d]
+    tol = 1e-2 if prec == "bf16" else 2e-5
+    assert np.max(np.abs(_f64(out) - ref)) <= tol * np.max(np.abs(ref))
