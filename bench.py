@@ -1,0 +1,369 @@
+"""Benchmark of the WAMachine hot path on GB300.
+
+One timed step = one closed-loop control step on the 12-block d=768 DiT (1296 joint tokens,
+10 native Euler steps, batch 1): Trajectory Remapping of the finished replan (executed shift 8
+of 16 actions), an anticipatory prefix of 1 step under the predicted observation, Observation
+Rebinding against the real observation (Eq. 4), and the remaining 2 steps with Residual
+Rescaling, ending in one action chunk.  The first replan of the episode is a cold 10-step
+sample (warm-up).  Synthetic inputs: weights N(0, 0.02) seed 0; observations follow
+o' = 0.9 o + sqrt(0.19) N(0,1) with the prediction 0.9 o; fresh noise seed 1000+step.
+
+Printed JSON line: `value` = action chunks/s with every input already resident in HBM;
+`latency_ms` = per-control-step p50/p99 and the observation-to-action part (rebinding + the
+steps after it); `cold` = a native cold 10-step sample; `e2e` = the same control loop through
+the C ABI with pinned host buffers (host<->device copies inside the timed region);
+`roofline` = the dominant kernel class (tcgen05 GEMM) against the measured bf16 peak;
+`cpu_baseline` = the float64 CPU oracle on the host cores for one control step.
+
+Usage: python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+Multi-GPU (torchrun): one replica per rank, no collective on the data path (the work is
+independent episodes); the timed region is bracketed by barriers and the slowest rank counts.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import math
+import multiprocessing as mp
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "action chunks/sec & p50 control-step latency at 1 GB300; tensor-pipe % of peak"
+WORKLOAD = "closed_loop"
+
+
+def _peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(path):
+        with open(path) as f:
+            p = json.load(f)
+        return dict(hbm=p["hbm_gbs"], bf16=p["bf16_tflops"], bf16_sus=p["bf16_tflops_sustained"],
+                    source="measured")
+    return dict(hbm=6800.0, bf16=1900.0, bf16_sus=1700.0, source="fallback")
+
+
+def _workload_config(cfg: dict) -> dict:
+    return {
+        "workload": "closed-loop control step (TR shift 8 + 1 anticipatory step + OR + 2 steps with RR) "
+                    "of the 12-block d768 12-head bf16 DiT, 256 obs + 1024 video + 16x7 action tokens, "
+                    "10 native Euler steps, batch 1",
+        "n_layers": cfg["n_layers"], "d_model": cfg["d_model"], "tokens": cfg["n_obs"] + cfg["n_video"] + cfg["n_action"],
+        "batch": 1, "steps_native": cfg["n_steps"], "warm_steps": cfg["n_steps"] - cfg["tr_entry_stage"],
+        "rr_boundaries": [cfg["rr_q"], cfg["rr_s"], cfg["rr_e"]],
+        "l2": "inputs larger than L2: 255 MB of bf16 weights are streamed by every denoising step",
+    }
+
+
+# ------------------------------------------------------------------------------ clocks
+class ClockSampler:
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.proc = None
+        self.path = tempfile.mktemp(suffix=".csv")
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--id={gpu_index}", f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
+                 "-lms", "200"], stdout=open(self.path, "w"), stderr=subprocess.DEVNULL)
+        except Exception:
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except Exception:
+            self.proc.kill()
+        sm, mx, reasons = [], 0.0, set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        with open(self.path) as f:
+            for line in f:
+                parts = [p.strip() for p in line.split(",")]
+                if len(parts) < 9:
+                    continue
+                try:
+                    sm.append(float(parts[1]))
+                    mx = max(mx, float(parts[2]))
+                except ValueError:
+                    continue
+                for n, v in zip(names, parts[5:9]):
+                    if v.lower().startswith("active"):
+                        reasons.add(n)
+        os.unlink(self.path)
+        if not sm:
+            return None
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": mx, "reasons": sorted(reasons), "samples": len(sm)}
+
+
+# ------------------------------------------------------------------------------ CPU oracle
+def _oracle_control_step_worker(q, cfg, seed, n_steps):
+    """Time the float64 oracle on one warm control step (a bounded sample of the workload)."""
+    from oracle import wam_oracle as O
+    from paper_2609_34608_gb300 import inputs as I
+
+    Wd = I.make_weights(cfg)
+    ocfg = O.OracleConfig.from_dict(cfg)
+    K = cfg["n_steps"]
+    b0 = cfg["tr_entry_stage"]
+    ep = O.OracleEpisode(Wd, ocfg)
+    proc = I.ObsProcess(cfg, 1, seed=seed)
+    rng = np.random.default_rng(seed)
+    T = ocfg.traj_len
+    # a finished previous replan (its stage-K and stage-r latents) to remap from
+    ep.obs = proc.obs[0].astype(np.float64)
+    ep.hist = {K: rng.standard_normal(T), b0: rng.standard_normal(T)}
+    ep.hist_from, ep.stage, ep.finished = b0, K, True
+    times = []
+    for t in range(n_steps):
+        pred, real = proc.predicted()[0], proc.step()[0]
+        eps = I.make_fresh_eps(cfg, 1, t)[0]
+        t0 = time.perf_counter()
+        if ep.adapt(pred, cfg["shift"], eps) == O.ADAPT_TR_INIT:
+            ep.advance(cfg.get("prefix_steps", 1))
+        ep.adapt(real, 0, None)
+        ep.advance(K - ep.stage)
+        times.append(time.perf_counter() - t0)
+    q.put(times)
+
+
+def run_oracle_steps(cfg, n_steps, seed=0):
+    ctx = mp.get_context("spawn")
+    q = ctx.Queue()
+    ncpu = os.cpu_count() or 1
+    os.environ.setdefault("OPENBLAS_NUM_THREADS", str(ncpu))
+    os.environ.setdefault("OMP_NUM_THREADS", str(ncpu))
+    p = ctx.Process(target=_oracle_control_step_worker, args=(q, cfg, seed, n_steps))
+    p.start()
+    times = q.get()
+    p.join()
+    return times, int(os.environ["OPENBLAS_NUM_THREADS"])
+
+
+# ------------------------------------------------------------------------------ reference arm
+def main_reference(args):
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return 0
+    from paper_2609_34608_gb300 import inputs as I
+
+    cfg = I.get_config(WORKLOAD)
+    times, cores = run_oracle_steps(cfg, args.warmup + args.steps)
+    timed = times[args.warmup:]
+    total = sum(timed)
+    value = len(timed) / total
+    sample = "one full warm control step per timed step (3 denoising forwards + TR + OR), float64 oracle"
+    line = {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": "chunks/s", "n_gpus": args.gpus,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1000 * total / len(timed),
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "config": _workload_config(cfg),
+        "cpu_baseline": {"value": value, "unit": "chunks/s", "cores": cores, "kind": "oracle", "sample": sample},
+        "e2e": {"value": value, "unit": "chunks/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line))
+    return 0
+
+
+# ------------------------------------------------------------------------------ our arm
+def main_ours(args):
+    import torch
+
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    dist = None
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("gloo")
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+
+    # The CPU baseline process is spawned before any GPU work.
+    cpu_times, cpu_cores = (None, None)
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        from paper_2609_34608_gb300 import inputs as I0
+        cpu_times, cpu_cores = run_oracle_steps(I0.get_config(WORKLOAD), 2)
+
+    from paper_2609_34608_gb300 import _build
+    from paper_2609_34608_gb300 import inputs as I
+    from paper_2609_34608_gb300 import wam as W
+
+    _build.build()
+    cfg = I.get_config(WORKLOAD)
+    K, b0, shift = cfg["n_steps"], cfg["tr_entry_stage"], cfg["shift"]
+    stream = torch.cuda.Stream(dev)
+    flat = torch.from_numpy(I.flatten_weights(I.make_weights(cfg))).to(dev)
+    ctx = W.Context(cfg, flat, stream=stream.cuda_stream)
+    del flat
+    n_total = args.warmup + args.steps
+    proc = I.ObsProcess(cfg, 1, seed=rank)
+    first_obs = proc.obs.copy()
+    host = []
+    for t in range(n_total + 1):
+        pred = proc.predicted()
+        real = proc.step()
+        host.append((pred, real, I.make_fresh_eps(cfg, 1, t)))
+    with torch.cuda.stream(stream):
+        dev_in = [tuple(torch.from_numpy(a).to(dev) for a in h) for h in host]
+        pin_in = [tuple(torch.from_numpy(a).pin_memory() for a in h) for h in host]
+        act_dev = torch.zeros((1, cfg["n_action"], cfg["action_dim"]), device=dev)
+        act_host = torch.zeros((1, cfg["n_action"], cfg["action_dim"])).pin_memory()
+        noise = torch.from_numpy(I.make_noise(cfg, 1)).to(dev)
+        obs0 = torch.from_numpy(first_obs).to(dev)
+
+    def control_step(inp, act, ev=None):
+        pred, real, eps = inp
+        s1 = ctx.adapt(st, pred, shift=shift, fresh_noise=eps)[0]
+        if s1 == W.ADAPT_TR_INIT:
+            ctx.continue_(st, 1)
+        if ev is not None:
+            ev.record(stream)
+        s2 = ctx.adapt(st, real)[0]
+        ctx.continue_(st, K - (b0 + 1 if s2 == W.ADAPT_REBIND_ACCEPT else b0), act)
+        return s1, s2
+
+    def barrier():
+        torch.cuda.synchronize(dev)
+        if dist is not None:
+            dist.barrier()
+
+    # ---- device-resident inputs -------------------------------------------------------
+    st = ctx.state(1)
+    with torch.cuda.stream(stream):
+        ctx.sample_cold(st, obs0, noise, K, act_dev)
+        for t in range(args.warmup):
+            control_step(dev_in[t], act_dev)
+    ctx.reset_stats()
+    ev_s = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps + 1)]
+    ev_m = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+    clocks = ClockSampler(local)
+    barrier()
+    with torch.cuda.stream(stream):
+        ev_s[0].record(stream)
+        for i in range(args.steps):
+            control_step(dev_in[args.warmup + i], act_dev, ev_m[i])
+            ev_s[i + 1].record(stream)
+    barrier()
+    clk = clocks.stop()
+    stats = ctx.stats()
+    total_ms = ev_s[0].elapsed_time(ev_s[-1])
+    step_ms = [ev_s[i].elapsed_time(ev_s[i + 1]) for i in range(args.steps)]
+    o2a_ms = [ev_m[i].elapsed_time(ev_s[i + 1]) for i in range(args.steps)]
+    if dist is not None:
+        t = torch.tensor([total_ms], dtype=torch.float64)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        total_ms = float(t[0])
+
+    # ---- end to end: pinned host inputs and outputs through the C ABI -----------------
+    st_e = ctx.state(1)
+    with torch.cuda.stream(stream):
+        ctx.sample_cold(st_e, obs0, noise, K, act_dev)
+        st, st_keep = st_e, st
+        for t in range(min(args.warmup, 3)):
+            control_step(pin_in[t], act_host)
+    barrier()
+    e0 = time.perf_counter()
+    ev_e0, ev_e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    with torch.cuda.stream(stream):
+        ev_e0.record(stream)
+        for i in range(args.steps):
+            control_step(pin_in[args.warmup + i], act_host)
+        ev_e1.record(stream)
+    barrier()
+    e2e_wall = time.perf_counter() - e0
+    e2e_ms = ev_e0.elapsed_time(ev_e1)
+    st = st_keep
+    h2d = sum(a.numel() * 4 for a in pin_in[0])
+    d2h = act_host.numel() * 4
+
+    # ---- native cold 10-step sample for comparison -----------------------------------
+    st_c = ctx.state(1)
+    cold_ms = []
+    with torch.cuda.stream(stream):
+        for i in range(max(3, min(10, args.steps))):
+            a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            a.record(stream)
+            ctx.sample_cold(st_c, obs0, noise, K, act_dev)
+            b.record(stream)
+            cold_ms.append((a, b))
+    torch.cuda.synchronize(dev)
+    cold_ms = [a.elapsed_time(b) for a, b in cold_ms][1:]
+
+    # ---- kernel-class timing (CUDA events on the library's stream) --------------------
+    st = st_keep
+    ctx.profile_enable(True)
+    nprof = min(args.steps, 20)
+    with torch.cuda.stream(stream):
+        for i in range(nprof):
+            control_step(dev_in[args.warmup + i], act_dev)
+    prof = ctx.profile_read()
+    ctx.profile_enable(False)
+
+    if rank != 0:
+        return 0
+    peaks = _peaks()
+    g = prof["gemm"]
+    gemm_tflops = g["flops"] / (g["ms"] * 1e-3) / 1e12 if g["ms"] > 0 else 0.0
+    tot_prof = sum(v["ms"] for v in prof.values())
+    value = args.steps * world / (total_ms * 1e-3)
+    line = {
+        "metric": METRIC, "value": value, "unit": "chunks/s", "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": total_ms / args.steps, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+        "config": _workload_config(cfg),
+        "latency_ms": {"p50": float(np.percentile(step_ms, 50)), "p99": float(np.percentile(step_ms, 99)),
+                       "o2a_p50": float(np.percentile(o2a_ms, 50)), "o2a_p99": float(np.percentile(o2a_ms, 99))},
+        "cold": {"ms_p50": float(np.percentile(cold_ms, 50)), "chunks_per_s": 1000.0 / float(np.percentile(cold_ms, 50)),
+                 "what": "native cold 10-step sample of the same model, RR active after the first step"},
+        "reuse": {"r_rr": stats["n_reuse"] / max(1, stats["n_attempt"]), "f_skip": stats["b_skip"] / max(1, stats["b_dense"]),
+                  "r_or": stats["n_bind"] / max(1, stats["n_start"]), "coverage": stats["n_bind"] / max(1, stats["n_noninitial"])},
+        "roofline": {"bound": "tensor", "kernel": "tcgen05 GEMM (QKV / out / MLP projections)",
+                     "achieved": gemm_tflops, "peak": peaks["bf16_sus"], "unit": "TFLOP/s",
+                     "frac": gemm_tflops / peaks["bf16_sus"], "traffic": None,
+                     "peak_source": f"{peaks['source']} sustained bf16"},
+        "kernel_share": {k: (v["ms"] / tot_prof if tot_prof else 0.0) for k, v in prof.items()},
+        "kernel_ms_per_step": {k: v["ms"] / nprof for k, v in prof.items()},
+        "gpu_launches": int(stats["n_kernel_launches"]),
+        "e2e": {"value": args.steps * world / (e2e_ms * 1e-3), "unit": "chunks/s", "h2d_bytes_per_step": int(h2d),
+                "d2h_bytes_per_step": int(d2h), "wall_s": e2e_wall},
+        "clocks": clk,
+    }
+    if cpu_times:
+        ct = cpu_times[-1]
+        line["cpu_baseline"] = {"value": 1.0 / ct, "unit": "chunks/s", "cores": cpu_cores, "kind": "oracle",
+                                "sample": "one warm control step (TR + 1 prefix step + OR + 2 steps, RR), float64 "
+                                          "oracle; best-effort second of two runs"}
+    print(json.dumps(line))
+    return 0
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=50)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+    if args.warmup < 3:
+        raise SystemExit("--warmup must be >= 3")
+    if args.impl == "reference":
+        return main_reference(args)
+    return main_ours(args)
+
+
+if __name__ == "__main__":
+    sys.exit(main())
