@@ -60,6 +60,28 @@ int wam_op_ln_modulate(const float* h, const float* shift, const float* scale,
 
 const char* wam_op_last_error(void);
 
+/*
+ * Trajectory Remapping of `batch` finished trajectories that allocates no device memory, for
+ * callers that cannot allocate: controllers whose control loop forbids allocation after
+ * start-up (bounded step latency), or hosts that own all device memory.  The paper has no
+ * counterpart; this is the same computation as the remap inside wam_adapt_state (Eqs. 1-2 with
+ * the Eq. 12 normaliser when normalize != 0) with one executed shift and one (sigma_r,
+ * sigma_b0) pair for every episode.
+ *   x_bar, x_r, eps, out: [batch, T] float32 device buffers, T = n_video*video_dim +
+ *   n_action*action_dim; eps may be NULL when shift == 0 and video_mode == 0.
+ *   video_mode 0 remaps video without a shift, 1 fills it with sigma_b0 * eps.
+ * Scratch: a fixed 64 KiB array inside the library (8192 float64 partial sums) holds the RMS
+ * partial sums; batch * 2 * ceil(max(n_video*video_dim, n_action*action_dim) / 2048) must not
+ * exceed 8192, else WAM_ERR_UNSUPPORTED.  Every call shares the array and leaves its contents
+ * behind; calls that overlap on the GPU race on it and must be serialised by the caller.  The
+ * first call on each device looks up the array's address; make it before any stream capture.
+ * Errors: WAM_ERR_INVALID_ARG, WAM_ERR_UNSUPPORTED, WAM_ERR_CUDA (message: wam_op_last_error).
+ */
+int wam_tr_remap_static(const float* x_bar, const float* x_r, const float* eps, float* out,
+                        int32_t batch, int32_t n_video, int32_t video_dim, int32_t n_action,
+                        int32_t action_dim, int32_t shift, double sigma_r, double sigma_b0,
+                        int32_t normalize, int32_t video_mode, void* stream);
+
 #ifdef __cplusplus
 }
 #endif

@@ -20,7 +20,8 @@ INCLUDE = os.path.join(ROOT, "include")
 BUILD_DIR = os.path.join(HERE, "_build")
 LIB_PATH = os.path.join(HERE, "libwam_gb300.so")
 
-SOURCES = ["wam_api.cu", "ops.cu", "gemm_tc.cu", "gemm_simt.cu", "attention.cu", "elementwise.cu"]
+SOURCES = ["wam_api.cu", "ops.cu", "gemm_tc.cu", "gemm_simt.cu", "attention.cu", "elementwise.cu",
+           "tr_static.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ARCH + ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "-I", INCLUDE,
                 "--expt-relaxed-constexpr"]

@@ -45,6 +45,10 @@ int check_gemm_args(const void* A, const void* Wt, void* C, int M, int N, int K,
 
 }  // namespace
 
+namespace wam {
+void set_op_error(const std::string& msg) { g_op_err = msg; }
+}  // namespace wam
+
 extern "C" {
 
 const char* wam_op_last_error(void) { return g_op_err.c_str(); }

@@ -1,0 +1,176 @@
+// Trajectory Remapping for callers that cannot allocate device memory.
+//
+// Robot controllers often run their control loop under a no-allocation rule: everything is
+// allocated at start-up so that each control step has bounded latency, and some embed this
+// library inside a host runtime that owns all device memory and gives it none.  Such callers
+// cannot create a context (which allocates its scratch with cudaMalloc), so this entry point
+// remaps a batch of finished trajectories using only the caller's buffers and a fixed array
+// compiled into the library for the float64 partial sums of the direction's RMS.
+//
+// The array holds kStaticPartials doubles (64 KiB) and exists on every GPU that loads the
+// library until the process exits.  All calls share it and it keeps the last call's contents;
+// every slot a call reads is written by the same call first, so nothing needs clearing, but
+// two calls that overlap on the GPU (different streams, or different host threads) race on it
+// and must be serialised by the caller.  The first call on a device looks up the array's
+// device address (cudaGetSymbolAddress, with that device current); make that first call before
+// any stream capture begins.
+#include <mutex>
+#include <string>
+
+#include "common.cuh"
+#include "wam.h"
+#include "wam_ops.h"
+
+namespace wam {
+void set_op_error(const std::string& msg);  // ops.cu
+
+namespace {
+
+constexpr int kStaticChunk = 2048;     // trajectory values per reduction block
+constexpr int kStaticPartials = 8192;  // float64 partial sums: 64 KiB
+constexpr int kMaxDevices = 64;
+
+static __device__ __align__(256) double g_tr_partials[kStaticPartials];
+
+std::mutex g_mu;
+double* g_partials_ptr[kMaxDevices] = {};
+
+WAM_DEV double block_sum(double v, double* red) {
+  v = warp_sum_d(v);
+  if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = v;
+  __syncthreads();
+  double s = 0.0;
+  if (threadIdx.x == 0)
+    for (int w = 0; w < (blockDim.x >> 5); ++w) s += red[w];
+  return s;
+}
+
+// Sum over one chunk of one branch of ((x^r - x_bar) / sigma_r)^2 (Eq. 1 before N).
+__global__ void __launch_bounds__(256) tr_static_partial_kernel(const float* __restrict__ x_bar,
+                                                                const float* __restrict__ x_r,
+                                                                int T, int V, double sigma_r,
+                                                                int nch, double* __restrict__ partial) {
+  __shared__ double red[8];
+  const int b = blockIdx.z, br = blockIdx.y, ch = blockIdx.x;
+  const int beg = br == 0 ? 0 : V;
+  const int len = br == 0 ? V : T - V;
+  const int64_t bo = static_cast<int64_t>(b) * T + beg;
+  const int end = min(len, (ch + 1) * kStaticChunk);
+  double s = 0.0;
+  for (int i = ch * kStaticChunk + threadIdx.x; i < end; i += blockDim.x) {
+    const double u = (static_cast<double>(x_r[bo + i]) - static_cast<double>(x_bar[bo + i])) / sigma_r;
+    s += u * u;
+  }
+  s = block_sum(s, red);
+  if (threadIdx.x == 0) partial[(static_cast<int64_t>(b) * 2 + br) * nch + ch] = s;
+}
+
+// Remapped init (Eq. 2) with the unit-RMS direction (Eq. 12), the action shift and the
+// fresh-noise fill sigma_b0 * eps of uncovered slots.
+__global__ void __launch_bounds__(256) tr_static_apply_kernel(
+    const float* __restrict__ x_bar, const float* __restrict__ x_r, const float* __restrict__ eps,
+    float* __restrict__ out, int T, int V, int Na, int ad, int shift, double sigma_r,
+    double sigma_b0, int normalize, int video_mode, int nch, const double* __restrict__ partial) {
+  __shared__ double rms[2];
+  __shared__ int zero[2];
+  const int b = blockIdx.y;
+  if (threadIdx.x < 2) {
+    double s = 0.0;
+    for (int c = 0; c < nch; ++c) s += partial[(static_cast<int64_t>(b) * 2 + threadIdx.x) * nch + c];
+    const double ms = s / (threadIdx.x == 0 ? V : T - V);
+    rms[threadIdx.x] = normalize ? sqrt(ms) : 1.0;
+    zero[threadIdx.x] = normalize && !(ms > 0.0);
+  }
+  __syncthreads();
+  const int64_t bo = static_cast<int64_t>(b) * T;
+  for (int j = blockIdx.x * blockDim.x + threadIdx.x; j < T; j += gridDim.x * blockDim.x) {
+    int src = -1, br = 0;
+    if (j < V) {
+      if (video_mode == 0) src = j;
+    } else {
+      br = 1;
+      const int ja = j - V;
+      const int row = ja / ad, col = ja - row * ad;
+      if (row + shift < Na) src = V + (row + shift) * ad + col;
+    }
+    float val;
+    if (src >= 0) {
+      const double u = (static_cast<double>(x_r[bo + src]) - static_cast<double>(x_bar[bo + src])) / sigma_r;
+      const double dir = zero[br] ? 0.0 : u / rms[br];
+      val = static_cast<float>(static_cast<double>(x_bar[bo + src]) + sigma_b0 * dir);
+    } else {
+      val = static_cast<float>(sigma_b0 * static_cast<double>(eps[bo + j]));
+    }
+    out[bo + j] = val;
+  }
+}
+
+// Device address of the partial-sum array on the current device, looked up once per device.
+int partials_on_current_device(double** out) {
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) {
+    set_op_error(std::string("cudaGetDevice: ") + cudaGetErrorString(e));
+    return WAM_ERR_CUDA;
+  }
+  if (dev < 0 || dev >= kMaxDevices) {
+    set_op_error("device index beyond the 64 devices this entry point tracks");
+    return WAM_ERR_UNSUPPORTED;
+  }
+  std::lock_guard<std::mutex> lock(g_mu);
+  if (g_partials_ptr[dev] == nullptr) {
+    void* p = nullptr;
+    e = cudaGetSymbolAddress(&p, g_tr_partials);
+    if (e != cudaSuccess || p == nullptr) {
+      set_op_error(std::string("cudaGetSymbolAddress of the static partial sums: ") + cudaGetErrorString(e));
+      return WAM_ERR_CUDA;
+    }
+    g_partials_ptr[dev] = static_cast<double*>(p);
+  }
+  *out = g_partials_ptr[dev];
+  return WAM_OK;
+}
+
+}  // namespace
+}  // namespace wam
+
+extern "C" int wam_tr_remap_static(const float* x_bar, const float* x_r, const float* eps, float* out,
+                                   int32_t batch, int32_t n_video, int32_t video_dim, int32_t n_action,
+                                   int32_t action_dim, int32_t shift, double sigma_r, double sigma_b0,
+                                   int32_t normalize, int32_t video_mode, void* stream) {
+  using namespace wam;
+  if (x_bar == nullptr || x_r == nullptr || out == nullptr || batch < 1 || n_video < 1 || video_dim < 1 ||
+      n_action < 1 || action_dim < 1 || shift < 0 || !(sigma_r > 0.0) || !(sigma_b0 >= 0.0) ||
+      (video_mode != 0 && video_mode != 1)) {
+    set_op_error("invalid argument: null buffer, non-positive size, negative shift or sigma_r <= 0");
+    return WAM_ERR_INVALID_ARG;
+  }
+  const int V = n_video * video_dim;
+  const int T = V + n_action * action_dim;
+  if (eps == nullptr && (video_mode == 1 || shift > 0)) {
+    set_op_error("eps is required when any slot receives fresh noise");
+    return WAM_ERR_INVALID_ARG;
+  }
+  const int nv = (V + kStaticChunk - 1) / kStaticChunk;
+  const int na = (T - V + kStaticChunk - 1) / kStaticChunk;
+  const int nch = nv > na ? nv : na;
+  if (static_cast<int64_t>(batch) * 2 * nch > kStaticPartials) {
+    set_op_error("batch * 2 * ceil(max(video, action values) / 2048) exceeds the 8192 static partial sums");
+    return WAM_ERR_UNSUPPORTED;
+  }
+  double* partials = nullptr;
+  const int r = partials_on_current_device(&partials);
+  if (r != WAM_OK) return r;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  tr_static_partial_kernel<<<dim3(nch, 2, batch), 256, 0, s>>>(x_bar, x_r, T, V, sigma_r, nch, partials);
+  const int blocks = (T + 255) / 256 < 64 ? (T + 255) / 256 : 64;
+  tr_static_apply_kernel<<<dim3(blocks, batch), 256, 0, s>>>(x_bar, x_r, eps, out, T, V, n_action, action_dim,
+                                                            shift, sigma_r, sigma_b0, normalize, video_mode, nch,
+                                                            partials);
+  const cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) {
+    set_op_error(std::string("static-scratch remap launch: ") + cudaGetErrorString(e));
+    return WAM_ERR_CUDA;
+  }
+  return WAM_OK;
+}

@@ -128,6 +128,8 @@ def lib() -> ctypes.CDLL:
         "wam_op_attention": (ctypes.c_int, [_vp, _vp, _i32, _i32, _i32, _i32, _i32, _vp]),
         "wam_op_ln_modulate": (ctypes.c_int, [_vp, _vp, _vp, ctypes.c_int64, _vp, _i32, _i32, _i32, _i32, _vp]),
         "wam_op_last_error": (ctypes.c_char_p, []),
+        "wam_tr_remap_static": (ctypes.c_int, [_vp, _vp, _vp, _vp, _i32, _i32, _i32, _i32, _i32, _i32,
+                                               ctypes.c_double, ctypes.c_double, _i32, _i32, _vp]),
     }
     for name, (res, args) in sig.items():
         fn = getattr(L, name)
@@ -329,3 +331,11 @@ def op_attention(qkv, out, B, N, d, n_heads, precision="bf16", stream=None):
 def op_ln_modulate(h, shift, scale, mod_stride, out, M, d, rows_per_item, precision="bf16", stream=None):
     _op_check(lib().wam_op_ln_modulate(ptr(h), ptr(shift), ptr(scale), mod_stride, ptr(out), M, d,
                                        rows_per_item, PREC[precision], stream))
+
+
+def tr_remap_static(x_bar, x_r, eps, out, batch, n_video, video_dim, n_action, action_dim, shift,
+                    sigma_r, sigma_b0, normalize=1, video_mode=0, stream=None):
+    """Trajectory Remapping without any device allocation (see include/wam_ops.h)."""
+    _op_check(lib().wam_tr_remap_static(ptr(x_bar), ptr(x_r), ptr(eps), ptr(out), batch, n_video, video_dim,
+                                        n_action, action_dim, shift, float(sigma_r), float(sigma_b0),
+                                        normalize, video_mode, stream))
