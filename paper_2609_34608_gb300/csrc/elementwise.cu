@@ -30,84 +30,110 @@ WAM_DEV double block_sum_d(double v, double* red) {
 }
 
 // ---------------------------------------------------------------- conditioning GEMV
-template <typename TW>
-WAM_DEV float2 load_w2(const TW* W, int64_t idx);
-template <>
-WAM_DEV float2 load_w2<float>(const float* W, int64_t idx) {
-  return *reinterpret_cast<const float2*>(W + idx);
-}
-template <>
-WAM_DEV float2 load_w2<bf16>(const bf16* W, int64_t idx) {
-  return __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(W + idx));
-}
+// out = x . W for a few items (the episodes of a step) and a [K, Nout] weight.  The input row of
+// each item is formed while staging: the timestep features of the item's sigma, or
+// act(sum over `in_splits` partial rows + in_bias).  A block owns CPB output columns (CPT per
+// lane, 16-byte weight loads) and one K slice; its 8 warps split the slice and combine in
+// shared memory.  With `splits` > 1 every block writes a partial row per K slice (no bias),
+// which the next stage reduces in a fixed order; with one split the bias is added here.
+template <typename TW> struct WVec;
+template <> struct WVec<bf16> {
+  static constexpr int kCPT = 8;
+  static WAM_DEV void load(const bf16* W, int64_t idx, float (&w)[8]) {
+    const uint4 u = __ldg(reinterpret_cast<const uint4*>(W + idx));
+    const __nv_bfloat162* h = reinterpret_cast<const __nv_bfloat162*>(&u);
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      const float2 f = __bfloat1622float2(h[i]);
+      w[2 * i] = f.x;
+      w[2 * i + 1] = f.y;
+    }
+  }
+};
+template <> struct WVec<float> {
+  static constexpr int kCPT = 4;
+  static WAM_DEV void load(const float* W, int64_t idx, float (&w)[4]) {
+    const float4 f = __ldg(reinterpret_cast<const float4*>(W + idx));
+    w[0] = f.x;
+    w[1] = f.y;
+    w[2] = f.z;
+    w[3] = f.w;
+  }
+};
 
-// out[b, n] = post(sum_k pre(x[b, k]) W[k, n] + bias[n]).  64 output columns per block
-// (2 per lane), the 8 warps split K and combine through shared memory; inputs are staged
-// 8 items at a time so each weight row is read once per group of items.
-template <typename TW, int PRE, int POST>
-__global__ void __launch_bounds__(256) cond_gemv_kernel(const float* __restrict__ x,
-                                                        const StepItem* __restrict__ items,
-                                                        const TW* __restrict__ W,
-                                                        const float* __restrict__ bias,
-                                                        float* __restrict__ out, int Bw, int K,
-                                                        int Nout) {
-  constexpr int kB = 8;
-  extern __shared__ float sx[];  // [kB][K]
-  __shared__ float red[8][kB][64];
+template <typename TW, int KB>
+__global__ void __launch_bounds__(256) cond_gemv_kernel(const float* __restrict__ in_part, int in_splits,
+                                                        const float* __restrict__ in_bias, int in_act,
+                                                        int features, const StepItem* __restrict__ items,
+                                                        const TW* __restrict__ W, int K, int Nout, int Bw,
+                                                        int kslice, float* __restrict__ out,
+                                                        const float* __restrict__ out_bias) {
+  constexpr int CPT = WVec<TW>::kCPT;
+  constexpr int CPB = 32 * CPT;
+  extern __shared__ float smem[];
+  float* sx = smem;                       // [KB][kslice]
+  float* red = smem + KB * kslice;        // [8][KB][CPB]
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int n = blockIdx.x * 64 + lane * 2;
-  const int kper = (K + 7) / 8;
-  const int k0 = warp * kper;
-  const int k1 = min(K, k0 + kper);
-  for (int b0 = 0; b0 < Bw; b0 += kB) {
-    const int nb = min(kB, Bw - b0);
-    for (int i = threadIdx.x; i < nb * K; i += 256) {
-      const int bi = i / K, k = i % K;
-      float v;
-      if constexpr (PRE == kPreFeatures) {
-        // cos / sin of 1000 sigma 10000^(-j/half), argument formed in float64
-        const int half = K / 2;
-        const int j = k < half ? k : k - half;
-        const double f = exp(-log(10000.0) * static_cast<double>(j) / half);
-        const double a = 1000.0 * items[b0 + bi].sigma * f;
-        v = static_cast<float>(k < half ? cos(a) : sin(a));
-      } else {
-        v = x[static_cast<int64_t>(b0 + bi) * K + k];
-        if constexpr (PRE == kPreSilu) v = silu_f(v);
+  const int k_beg = blockIdx.y * kslice;
+  const int k_len = max(0, min(K, k_beg + kslice) - k_beg);
+  const int col0 = blockIdx.x * CPB + lane * CPT;
+  const int kw = (k_len + 7) / 8;
+  const int kw0 = warp * kw, kw1 = min(k_len, kw0 + kw);
+  const int64_t part_stride = static_cast<int64_t>(Bw) * K;
+  for (int b0 = 0; b0 < Bw; b0 += KB) {
+    const int nb = min(KB, Bw - b0);
+    for (int i = threadIdx.x; i < KB * k_len; i += 256) {
+      const int bi = i / k_len, kk = i - bi * k_len, k = k_beg + kk;
+      float v = 0.0f;
+      if (bi < nb) {
+        if (features) {
+          // cos / sin of 1000 sigma 10000^(-j/half), argument formed in float64
+          const int half = K / 2;
+          const int j = k < half ? k : k - half;
+          const double f = exp(-log(10000.0) * static_cast<double>(j) / half);
+          const double a = 1000.0 * items[b0 + bi].sigma * f;
+          v = static_cast<float>(k < half ? cos(a) : sin(a));
+        } else {
+          float acc = in_bias != nullptr ? in_bias[k] : 0.0f;
+          for (int sp = 0; sp < in_splits; ++sp) acc += in_part[sp * part_stride + static_cast<int64_t>(b0 + bi) * K + k];
+          v = in_act ? silu_f(acc) : acc;
+        }
       }
-      sx[bi * K + k] = v;
+      sx[bi * kslice + kk] = v;
     }
     __syncthreads();
-    float acc[kB][2];
+    float acc[KB][CPT];
 #pragma unroll
-    for (int bi = 0; bi < kB; ++bi) acc[bi][0] = acc[bi][1] = 0.0f;
-    if (n < Nout) {
-      for (int k = k0; k < k1; ++k) {
-        const float2 w = load_w2<TW>(W, static_cast<int64_t>(k) * Nout + n);
+    for (int bi = 0; bi < KB; ++bi)
 #pragma unroll
-        for (int bi = 0; bi < kB; ++bi) {
-          const float xv = sx[bi * K + k];
-          acc[bi][0] = fmaf(xv, w.x, acc[bi][0]);
-          acc[bi][1] = fmaf(xv, w.y, acc[bi][1]);
+      for (int c = 0; c < CPT; ++c) acc[bi][c] = 0.0f;
+    if (col0 < Nout) {
+#pragma unroll 4
+      for (int kk = kw0; kk < kw1; ++kk) {
+        float w[CPT];
+        WVec<TW>::load(W, static_cast<int64_t>(k_beg + kk) * Nout + col0, w);
+#pragma unroll
+        for (int bi = 0; bi < KB; ++bi) {
+          const float xv = sx[bi * kslice + kk];
+#pragma unroll
+          for (int c = 0; c < CPT; ++c) acc[bi][c] = fmaf(xv, w[c], acc[bi][c]);
         }
       }
     }
 #pragma unroll
-    for (int bi = 0; bi < kB; ++bi) {
-      red[warp][bi][lane * 2] = acc[bi][0];
-      red[warp][bi][lane * 2 + 1] = acc[bi][1];
-    }
-    __syncthreads();
-    for (int i = threadIdx.x; i < nb * 64; i += 256) {
-      const int bi = i / 64, c = i % 64;
-      const int col = blockIdx.x * 64 + c;
-      if (col < Nout) {
-        float s = 0.0f;
+    for (int bi = 0; bi < KB; ++bi)
 #pragma unroll
-        for (int w = 0; w < 8; ++w) s += red[w][bi][c];
-        s += bias[col];
-        if constexpr (POST == 1) s = silu_f(s);
-        out[static_cast<int64_t>(b0 + bi) * Nout + col] = s;
+      for (int c = 0; c < CPT; ++c) red[(warp * KB + bi) * CPB + lane * CPT + c] = acc[bi][c];
+    __syncthreads();
+    for (int i = threadIdx.x; i < nb * CPB; i += 256) {
+      const int bi = i / CPB, cc = i - bi * CPB;
+      const int col = blockIdx.x * CPB + cc;
+      if (col < Nout) {
+        float sum = 0.0f;
+#pragma unroll
+        for (int w = 0; w < 8; ++w) sum += red[(w * KB + bi) * CPB + cc];
+        if (out_bias != nullptr) sum += out_bias[col];
+        out[static_cast<int64_t>(blockIdx.y) * Bw * Nout + static_cast<int64_t>(b0 + bi) * Nout + col] = sum;
       }
     }
     __syncthreads();
@@ -250,7 +276,9 @@ __global__ void __launch_bounds__(256) final_euler_kernel(
   const float* scale = shift + d;
   const bool video = r < Nv;
   const int od = video ? vd : ad;
-  const float* Wo = video ? vout_w : aout_w;
+  // Output heads are stored with rows padded to 16 floats: each of this lane's y values meets a
+  // 64-byte weight row (four float4 loads) and contributes to all 16 outputs.
+  const float4* Wo = reinterpret_cast<const float4*>(video ? vout_w : aout_w);
   float acc[16];
 #pragma unroll
   for (int j = 0; j < 16; ++j) acc[j] = 0.0f;
@@ -265,20 +293,29 @@ __global__ void __launch_bounds__(256) final_euler_kernel(
                         fmaf((v[i].w - mean) * rstd, 1.0f + sc.w, sh.w)};
 #pragma unroll
     for (int e = 0; e < 4; ++e) {
-      const float* wr = Wo + static_cast<int64_t>(c + e) * od;
 #pragma unroll
-      for (int j = 0; j < 16; ++j)
-        if (j < od) acc[j] = fmaf(y[e], wr[j], acc[j]);
+      for (int q = 0; q < 4; ++q) {
+        const float4 wv = __ldg(Wo + (c + e) * 4 + q);
+        acc[4 * q + 0] = fmaf(y[e], wv.x, acc[4 * q + 0]);
+        acc[4 * q + 1] = fmaf(y[e], wv.y, acc[4 * q + 1]);
+        acc[4 * q + 2] = fmaf(y[e], wv.z, acc[4 * q + 2]);
+        acc[4 * q + 3] = fmaf(y[e], wv.w, acc[4 * q + 3]);
+      }
     }
   }
-  float mine = 0.0f;
+  // Reduce-scatter the 16 partial outputs over the warp: after the halving steps lane l holds
+  // output (l & 15) summed over its half-warp; the last exchange adds the other half.
 #pragma unroll
-  for (int j = 0; j < 16; ++j) {
-    if (j < od) {
-      const float s = warp_sum(acc[j]);
-      if (lane == j) mine = s;
+  for (int sft = 8; sft >= 1; sft >>= 1) {
+    const bool upper = (lane & sft) != 0;
+#pragma unroll
+    for (int j = 0; j < sft; ++j) {
+      const float send = upper ? acc[j] : acc[j + sft];
+      const float keep = upper ? acc[j + sft] : acc[j];
+      acc[j] = keep + __shfl_xor_sync(0xffffffffu, send, sft);
     }
   }
+  const float mine = acc[0] + __shfl_xor_sync(0xffffffffu, acc[0], 16);
   if (lane < od) {
     const float vel = mine + (video ? vout_b : aout_b)[lane];
     const int64_t idx = static_cast<int64_t>(it.ep) * T +
@@ -445,19 +482,25 @@ __global__ void __launch_bounds__(256) rr_probe_kernel(const float* __restrict__
   }
 }
 
-// alpha (Eq. 7), cosine and relative fit (Eq. 8) per (item, branch).
+// alpha (Eq. 7), cosine and relative fit (Eq. 8) per (item, branch): one warp per pair, the
+// partial sums combined lane-strided then by a fixed shuffle tree (deterministic order).
 __global__ void rr_gate_kernel(const double* __restrict__ partial, int Bw, int nch, int64_t n0,
                                int64_t n1, double amin, double amax, double eps, double gcos,
                                double gfit, RRGate* __restrict__ out) {
-  const int i = blockIdx.x * blockDim.x + threadIdx.x;
+  const int i = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+  const int lane = threadIdx.x & 31;
   if (i >= Bw * 2) return;
   const double* p = partial + static_cast<int64_t>(i) * nch * 3;
   double sia = 0.0, saa = 0.0, sii = 0.0;
-  for (int c = 0; c < nch; ++c) {
+  for (int c = lane; c < nch; c += 32) {
     sia += p[3 * c];
     saa += p[3 * c + 1];
     sii += p[3 * c + 2];
   }
+  sia = warp_sum_d(sia);
+  saa = warp_sum_d(saa);
+  sii = warp_sum_d(sii);
+  if (lane != 0) return;
   const double n = static_cast<double>((i & 1) ? n1 : n0);
   double alpha = (sia / n) / fmax(saa / n, eps);
   alpha = fmin(fmax(alpha, amin), amax);
@@ -561,41 +604,38 @@ __global__ void copy2d_kernel(const float* __restrict__ in, int64_t spitch, TO* 
   }
 }
 
-template <typename TW, int PRE, int POST>
-cudaError_t gemv_launch(const float* x, const StepItem* items, const TW* W, const float* bias,
-                        float* out, int Bw, int K, int Nout, cudaStream_t s) {
-  const size_t smem = static_cast<size_t>(8) * K * sizeof(float);
-  static bool attr = false;
-  if (!attr) {
-    cudaError_t e = cudaFuncSetAttribute(cond_gemv_kernel<TW, PRE, POST>,
-                                         cudaFuncAttributeMaxDynamicSharedMemorySize, 8 * 4096 * 4);
-    if (e != cudaSuccess) return e;
-    attr = true;
-  }
-  cond_gemv_kernel<TW, PRE, POST><<<(Nout + 63) / 64, 256, smem, s>>>(x, items, W, bias, out, Bw, K, Nout);
+template <typename TW, int KB>
+cudaError_t gemv_launch(const CondGemv& g, cudaStream_t s) {
+  constexpr int CPB = 32 * WVec<TW>::kCPT;
+  const int kslice = (g.K + g.splits - 1) / g.splits;
+  const size_t smem = sizeof(float) * (static_cast<size_t>(KB) * kslice + 8 * KB * CPB);
+  if (smem > 200 * 1024) return cudaErrorInvalidValue;
+  cudaError_t e = cudaFuncSetAttribute(cond_gemv_kernel<TW, KB>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       static_cast<int>(smem));
+  if (e != cudaSuccess) return e;
+  dim3 grid((g.Nout + CPB - 1) / CPB, g.splits);
+  cond_gemv_kernel<TW, KB><<<grid, 256, smem, s>>>(g.in_part, g.in_splits, g.in_bias, g.in_act, g.features,
+                                                   g.items, static_cast<const TW*>(g.W), g.K, g.Nout, g.Bw,
+                                                   kslice, g.out, g.out_bias);
   return cudaGetLastError();
 }
 
 template <typename TW>
-cudaError_t gemv_pre_post(const float* x, const StepItem* items, const TW* W, const float* bias,
-                          float* out, int Bw, int K, int Nout, int pre, int post, cudaStream_t s) {
-  if (pre == kPreFeatures && post == 1) return gemv_launch<TW, kPreFeatures, 1>(x, items, W, bias, out, Bw, K, Nout, s);
-  if (pre == kPreNone && post == 0) return gemv_launch<TW, kPreNone, 0>(x, items, W, bias, out, Bw, K, Nout, s);
-  if (pre == kPreSilu && post == 0) return gemv_launch<TW, kPreSilu, 0>(x, items, W, bias, out, Bw, K, Nout, s);
-  return cudaErrorInvalidValue;
+cudaError_t gemv_items(const CondGemv& g, cudaStream_t s) {
+  if (g.Bw == 1) return gemv_launch<TW, 1>(g, s);
+  if (g.Bw == 2) return gemv_launch<TW, 2>(g, s);
+  if (g.Bw <= 4) return gemv_launch<TW, 4>(g, s);
+  return gemv_launch<TW, 8>(g, s);
 }
 
 unsigned row_blocks(int64_t rows) { return static_cast<unsigned>((rows + kRowWarps - 1) / kRowWarps); }
 
 }  // namespace
 
-cudaError_t cond_gemv(const float* x, const StepItem* items, const void* W, bool w_bf16,
-                      const float* bias, float* out, int Bw, int K, int Nout, int pre, int post,
-                      cudaStream_t s) {
-  if (Bw <= 0) return cudaSuccess;
-  if (K > 4096 || (Nout & 1)) return cudaErrorInvalidValue;
-  return w_bf16 ? gemv_pre_post<bf16>(x, items, static_cast<const bf16*>(W), bias, out, Bw, K, Nout, pre, post, s)
-                : gemv_pre_post<float>(x, items, static_cast<const float*>(W), bias, out, Bw, K, Nout, pre, post, s);
+cudaError_t cond_gemv(const CondGemv& g, cudaStream_t s) {
+  if (g.Bw <= 0) return cudaSuccess;
+  if (g.Nout % (g.w_bf16 ? 8 : 4) != 0 || g.splits < 1) return cudaErrorInvalidValue;
+  return g.w_bf16 ? gemv_items<bf16>(g, s) : gemv_items<float>(g, s);
 }
 
 cudaError_t embed_tokens(float* h, float* xhist, int64_t stage_stride, const StepItem* items,
@@ -645,7 +685,7 @@ cudaError_t final_euler(const float* h, const StepItem* items, const float* mods
                         float* xhist, float* vhist, int64_t stage_stride, int T, int Bw, int No,
                         int Nv, int vd, int Na, int ad, int d, cudaStream_t s) {
   if (Bw <= 0) return cudaSuccess;
-  if (d % 128 != 0 || vd > 16 || ad > 16) return cudaErrorInvalidValue;
+  if (d % 128 != 0 || vd > 16 || ad > 16) return cudaErrorInvalidValue;  // heads padded to 16
   const unsigned grid = row_blocks(static_cast<int64_t>(Bw) * (Nv + Na));
 #define WAM_FE_CASE(NV)                                                                       \
   case NV:                                                                                    \
@@ -718,8 +758,8 @@ cudaError_t rr_gate(const double* partial, int Bw, int nch, int64_t n0, int64_t 
                     double amax, double eps, double gcos, double gfit, RRGate* out,
                     cudaStream_t s) {
   if (Bw <= 0) return cudaSuccess;
-  rr_gate_kernel<<<(Bw * 2 + 63) / 64, 64, 0, s>>>(partial, Bw, nch, n0, n1, amin, amax, eps,
-                                                   gcos, gfit, out);
+  rr_gate_kernel<<<(Bw * 2 * 32 + 127) / 128, 128, 0, s>>>(partial, Bw, nch, n0, n1, amin, amax, eps,
+                                                           gcos, gfit, out);
   return cudaGetLastError();
 }
 

@@ -43,10 +43,23 @@ constexpr int kTrChunk = 2048;     // elements per TR reduction block
 constexpr int kProbeChunk = 8192;  // elements per RR probe block
 constexpr int kOrChunk = 8192;     // elements per OR score block
 
-cudaError_t cond_gemv(const float* x, const StepItem* items, const void* W, bool w_bf16,
-                      const float* bias, float* out, int Bw, int K, int Nout, int pre, int post,
-                      cudaStream_t s);
-enum GemvPre { kPreNone = 0, kPreSilu = 1, kPreFeatures = 2 };
+// One conditioning GEMV: out[split][b][n] = sum over the split's K slice of x[b][k] W[k][n]
+// (+ out_bias[n] when splits == 1), x[b][k] = timestep features of items[b].sigma when
+// `features`, else act(in_bias[k] + sum over in_splits partial rows of in_part).
+struct CondGemv {
+  const float* in_part;
+  int in_splits;
+  const float* in_bias;
+  int in_act;     // 1: SiLU
+  int features;   // 1: sinusoidal timestep features (K of them)
+  const StepItem* items;
+  const void* W;  // [K, Nout]
+  bool w_bf16;
+  int K, Nout, Bw, splits;
+  float* out;
+  const float* out_bias;
+};
+cudaError_t cond_gemv(const CondGemv& g, cudaStream_t s);
 
 cudaError_t embed_tokens(float* h, float* xhist, int64_t stage_stride, const StepItem* items,
                          const float* x, int T, const float* obs_emb, const float* vid_w,

@@ -23,6 +23,8 @@ namespace {
 constexpr int kRingSlots = 64;
 constexpr size_t kSlotBytes = 16384;
 constexpr int kMaxBatch = 256;
+constexpr int kT1Splits = 8;  // K splits of the two conditioning-MLP GEMVs
+constexpr int kT2Splits = 8;
 
 struct LayerW {
   void* qkv_wt = nullptr;
@@ -346,18 +348,23 @@ int run_steps(wam_ctx* c, wam_state* st, const std::vector<int>& n) {
     }
     const int Bw = static_cast<int>(items.size());
     TRY(upload(c, c->d_items, items.data(), sizeof(StepItem) * Bw));
-    // conditioning: features -> SiLU(W1) -> W2 -> SiLU -> every layer's modulation
+    // conditioning: features -> W1 (split K) -> SiLU -> W2 (split K) -> SiLU -> every layer's
+    // modulation; each stage reduces the previous stage's K-split partial rows in a fixed order
     {
       Span sp(c, WAM_KCLASS_COND, 2.0 * Bw * 256 * d, 4.0 * 256 * d);
-      CK(cond_gemv(nullptr, c->d_items, c->t_w1, false, c->t_b1, c->t1, Bw, 256, d, kPreFeatures, 1, c->stream));
+      const CondGemv g{nullptr, 0, nullptr, 0, 1, c->d_items, c->t_w1, false, 256, d, Bw, kT1Splits, c->t1, nullptr};
+      CK(cond_gemv(g, c->stream));
     }
     {
       Span sp(c, WAM_KCLASS_COND, 2.0 * Bw * d * d, 4.0 * d * d);
-      CK(cond_gemv(c->t1, c->d_items, c->t_w2, false, c->t_b2, c->cvec, Bw, d, d, kPreNone, 0, c->stream));
+      const CondGemv g{c->t1, kT1Splits, c->t_b1, 1, 0, c->d_items, c->t_w2, false, d, d, Bw, kT2Splits, c->cvec, nullptr};
+      CK(cond_gemv(g, c->stream));
     }
     {
       Span sp(c, WAM_KCLASS_COND, 2.0 * Bw * d * c->mod_n, (c->bf16 ? 2.0 : 4.0) * d * c->mod_n);
-      CK(cond_gemv(c->cvec, c->d_items, c->mod_w, c->bf16, c->mod_b, c->mods, Bw, d, static_cast<int>(c->mod_n), kPreSilu, 0, c->stream));
+      const CondGemv g{c->cvec, kT2Splits, c->t_b2, 1, 0, c->d_items, c->mod_w, c->bf16, d, static_cast<int>(c->mod_n),
+                       Bw, 1, c->mods, c->mod_b};
+      CK(cond_gemv(g, c->stream));
     }
     {
       Span sp(c, WAM_KCLASS_NORM, 0.0, 4.0 * Bw * double(N) * d * 2.0);
@@ -590,10 +597,18 @@ int build_weights(wam_ctx* c, const float* src) {
   }
   CK(copy_cast_2d(take(size_t(d) * 2 * d), 2 * d, static_cast<uint8_t*>(c->mod_w) + size_t(L) * 6 * d * wel, b16, c->mod_n, d, 2 * d, c->stream));
   CK(cudaMemcpyAsync(c->mod_b + size_t(L) * 6 * d, take(2 * d), sizeof(float) * 2 * d, cudaMemcpyDeviceToDevice, c->stream));
-  TRY(dvec(&c->vout_w, take(size_t(d) * c->vd), size_t(d) * c->vd));
-  TRY(dvec(&c->vout_b, take(c->vd), c->vd));
-  TRY(dvec(&c->aout_w, take(size_t(d) * c->ad), size_t(d) * c->ad));
-  TRY(dvec(&c->aout_b, take(c->ad), c->ad));
+  // output heads padded to 16 columns (zeros beyond video_dim / action_dim): 64-byte rows
+  auto head = [&](float** w, float** bvec, int od) -> int {
+    TRY(dalloc(c, c->allocs, w, size_t(d) * 16));
+    TRY(dalloc(c, c->allocs, bvec, 16));
+    CK(cudaMemsetAsync(*w, 0, sizeof(float) * d * 16, c->stream));
+    CK(cudaMemsetAsync(*bvec, 0, sizeof(float) * 16, c->stream));
+    CK(copy_cast_2d(take(size_t(d) * od), od, *w, false, 16, d, od, c->stream));
+    CK(cudaMemcpyAsync(*bvec, take(od), sizeof(float) * od, cudaMemcpyDeviceToDevice, c->stream));
+    return WAM_OK;
+  };
+  TRY(head(&c->vout_w, &c->vout_b, c->vd));
+  TRY(head(&c->aout_w, &c->aout_b, c->ad));
   if (off != weight_count(&c->cfg)) return fail(c, WAM_ERR_INVALID_ARG, "internal weight layout mismatch");
   return WAM_OK;
 }
@@ -681,8 +696,8 @@ int create_impl(wam_ctx* c, const wam_config* cfg, const float* weights, size_t 
   c->att = att;
   c->u = u;
   c->obs_lp = olp;
-  TRY(dalloc(c, c->allocs, &c->t1, size_t(c->Bmax) * c->d));
-  TRY(dalloc(c, c->allocs, &c->cvec, size_t(c->Bmax) * c->d));
+  TRY(dalloc(c, c->allocs, &c->t1, size_t(kT1Splits) * c->Bmax * c->d));
+  TRY(dalloc(c, c->allocs, &c->cvec, size_t(kT2Splits) * c->Bmax * c->d));
   TRY(dalloc(c, c->allocs, &c->mods, size_t(c->Bmax) * c->mod_n));
   TRY(dalloc(c, c->allocs, &c->d_items, c->Bmax));
   TRY(dalloc(c, c->allocs, &c->d_map, c->Bmax));
