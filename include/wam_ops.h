@@ -45,7 +45,7 @@ int wam_op_gemm_f32(const float* A, const float* Wt, const float* bias, float* C
  *   qkv [B*N, 3d] (q | k | v column blocks, head h owns columns h*dh .. h*dh+dh-1 of each),
  *   out [B*N, d].  softmax(q k^T / sqrt(dh)) v, no mask.
  * precision WAM_PREC_BF16: bf16 in / out, fp32 accumulation, head dim 64 or 72.
- * precision WAM_PREC_FP32: float32 in / out, head dim <= 128 and a multiple of 32... any dh <= 128.
+ * precision WAM_PREC_FP32: float32 in / out, any head dim <= 128.
  */
 int wam_op_attention(const void* qkv, void* out, int32_t B, int32_t N, int32_t d,
                      int32_t n_heads, int32_t precision, void* stream);
@@ -57,6 +57,25 @@ int wam_op_attention(const void* qkv, void* out, int32_t B, int32_t N, int32_t d
 int wam_op_ln_modulate(const float* h, const float* shift, const float* scale,
                        int64_t mod_stride, void* out, int32_t M, int32_t d,
                        int32_t rows_per_item, int32_t precision, void* stream);
+
+/*
+ * QKV projection for the tensor-core attention: qkv = A Wt^T + bias with A [M, d], Wt [3d, d]
+ * (bf16, K-major), written as bf16 q | k columns into qkv [M, 3d] and with the v columns
+ * transposed per item and head into vt [(M / rows_per_item) * d, vt_ld]: element (token n of
+ * item i, head h, channel c) at row i*d + h*64 + c, column n.  vt_ld >= rows_per_item, a
+ * multiple of 8; columns rows_per_item..vt_ld-1 are never written (keep them zero).  The v
+ * columns of qkv are left untouched.
+ */
+int wam_op_gemm_qkv_vt(const void* A, const void* Wt, const float* bias, void* qkv, void* vt,
+                       int32_t M, int32_t d, int32_t rows_per_item, int32_t vt_ld, void* stream);
+
+/*
+ * Full bidirectional attention on tcgen05 (head dim 64): q and k from qkv [B*N, 3d] (bf16),
+ * v from vt as written by wam_op_gemm_qkv_vt with vt_ld = N rounded up to a multiple of 8,
+ * out [B*N, d] bf16.  softmax(q k^T / 8) v per item and head, no mask.
+ */
+int wam_op_attention_tc(const void* qkv, const void* vt, void* out, int32_t B, int32_t N,
+                        int32_t d, int32_t n_heads, void* stream);
 
 const char* wam_op_last_error(void);
 

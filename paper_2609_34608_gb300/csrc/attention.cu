@@ -85,6 +85,8 @@ __global__ void __launch_bounds__(128) attn_bf16_kernel(const bf16* __restrict__
   const int warp = tid >> 5;
   const int lane = tid & 31;
   const int q0 = blockIdx.x * C::kBQ;
+  pdl_wait();
+  pdl_launch_dependents();
   const int h = blockIdx.y;
   const int b = blockIdx.z;
   const int64_t ld = 3 * static_cast<int64_t>(d);
@@ -250,6 +252,8 @@ __global__ void __launch_bounds__(128) attn_bf16_kernel(const bf16* __restrict__
 __global__ void __launch_bounds__(256) attn_f32_kernel(const float* __restrict__ qkv,
                                                        float* __restrict__ out, int B, int N,
                                                        int d, int H, float scale) {
+  pdl_wait();
+  pdl_launch_dependents();
   const int64_t gw = (static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x) >> 5;
   const int lane = threadIdx.x & 31;
   if (gw >= static_cast<int64_t>(B) * H * N) return;
@@ -310,8 +314,7 @@ cudaError_t launch_bf16(const bf16* qkv, bf16* out, int B, int N, int d, int H, 
   }
   dim3 grid((N + C::kBQ - 1) / C::kBQ, H, B);
   const float scale_log2 = 1.4426950408889634f / sqrtf(static_cast<float>(DH));
-  attn_bf16_kernel<DH><<<grid, 128, C::kSmem, s>>>(qkv, out, N, d, scale_log2);
-  return cudaGetLastError();
+  return launch_pdl(attn_bf16_kernel<DH>, grid, dim3(128), C::kSmem, s, qkv, out, N, d, scale_log2);
 }
 
 }  // namespace
@@ -334,9 +337,8 @@ cudaError_t attention_f32(const float* qkv, float* out, int B, int N, int d, int
   if (d / H > 128) return cudaErrorInvalidValue;
   const int64_t warps = static_cast<int64_t>(B) * H * N;
   const int64_t blocks = (warps * 32 + 255) / 256;
-  attn_f32_kernel<<<static_cast<unsigned>(blocks), 256, 0, s>>>(qkv, out, B, N, d, H,
-                                                                 1.0f / sqrtf(static_cast<float>(d / H)));
-  return cudaGetLastError();
+  return launch_pdl(attn_f32_kernel, dim3(static_cast<unsigned>(blocks)), dim3(256), 0, s, qkv, out, B, N, d, H,
+                    1.0f / sqrtf(static_cast<float>(d / H)));
 }
 
 }  // namespace wam

@@ -24,6 +24,29 @@ WAM_DEV uint64_t globaltimer_ns() {
   return t;
 }
 
+// Programmatic dependent launch: every hot-path kernel is launched so that the next kernel in
+// the stream may be scheduled while it runs.  A kernel calls pdl_wait() before it touches data
+// written by earlier work in the stream (the wait returns once that work has completed and its
+// memory is visible), and pdl_launch_dependents() to let the next kernel start its prologue.
+WAM_DEV void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+WAM_DEV void pdl_launch_dependents() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
+
+template <typename... KArgs, typename... Args>
+inline cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem,
+                              cudaStream_t s, Args... args) {
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kernel, static_cast<KArgs>(args)...);
+}
+
 WAM_DEV float warp_sum(float v) {
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
@@ -65,7 +88,7 @@ template <> struct Act<bf16> {
 };
 
 // ---- GEMM epilogue description (shared by the tensor-core and SIMT GEMMs) ---------------
-enum EpiMode { kEpiBf16 = 0, kEpiGeluBf16 = 1, kEpiResidF32 = 2, kEpiF32 = 3 };
+enum EpiMode { kEpiBf16 = 0, kEpiGeluBf16 = 1, kEpiResidF32 = 2, kEpiF32 = 3, kEpiQkvVt = 4 };
 
 struct EpiArgs {
   const float* bias;     // [N] or null
@@ -74,6 +97,8 @@ struct EpiArgs {
   int64_t gate_stride;   // floats between gate rows of consecutive items
   int rows_per_item;     // rows of one item (tokens of one episode)
   const int* item_map;   // nullable: gate row of local item i = item_map[i]
+  bf16* vt;              // QKV_VT: V^T destination [items * heads * 64, vt_ld]
+  int vt_ld;             // QKV_VT: padded token count (row length of V^T)
 };
 
 // ---- internal interfaces -----------------------------------------------------------------
@@ -92,5 +117,12 @@ cudaError_t attention_bf16(const bf16* qkv, bf16* out, int B, int N, int d, int 
 cudaError_t attention_f32(const float* qkv, float* out, int B, int N, int d, int H,
                           cudaStream_t s);
 bool attention_bf16_supported(int head_dim);
+// tcgen05 attention (attention_tc.cu), head dim 64: Q / K read from the qkv buffer through
+// tm_qk (box 64 x 128), V^T [items*heads*64, vt_ld] through tm_vt (box 64 x 64).
+cudaError_t attention_tc(const CUtensorMap& tm_qk, const CUtensorMap& tm_vt, bf16* out, int B, int N, int d,
+                         int H, int* dev_err, cudaStream_t s);
+int attention_tc_vt_ld(int N);
+int tc_encode_bf16_box(CUtensorMap* map, const void* base, uint64_t rows, uint64_t cols, uint64_t ld,
+                       uint32_t box_cols, uint32_t box_rows);
 
 }  // namespace wam

@@ -68,6 +68,8 @@ __global__ void __launch_bounds__(256) cond_gemv_kernel(const float* __restrict_
                                                         const TW* __restrict__ W, int K, int Nout, int Bw,
                                                         int kslice, float* __restrict__ out,
                                                         const float* __restrict__ out_bias) {
+  pdl_wait();
+  pdl_launch_dependents();
   constexpr int CPT = WVec<TW>::kCPT;
   constexpr int CPB = 32 * CPT;
   extern __shared__ float smem[];
@@ -148,6 +150,8 @@ __global__ void __launch_bounds__(256) embed_kernel(
     const float* __restrict__ vid_b, const float* __restrict__ act_w,
     const float* __restrict__ act_b, const float* __restrict__ pos, int Bw, int No, int Nv,
     int vd, int Na, int ad, int d) {
+  pdl_wait();
+  pdl_launch_dependents();
   const int N = No + Nv + Na;
   const int64_t gw = static_cast<int64_t>(blockIdx.x) * kRowWarps + (threadIdx.x >> 5);
   const int lane = threadIdx.x & 31;
@@ -220,6 +224,8 @@ __global__ void __launch_bounds__(256) ln_mod_kernel(const float* __restrict__ h
                                                      const int* __restrict__ item_map,
                                                      TO* __restrict__ out, int M, int d,
                                                      int rows_per_item) {
+  pdl_wait();
+  pdl_launch_dependents();
   const int64_t row = static_cast<int64_t>(blockIdx.x) * kRowWarps + (threadIdx.x >> 5);
   const int lane = threadIdx.x & 31;
   if (row >= M) return;
@@ -259,6 +265,8 @@ __global__ void __launch_bounds__(256) final_euler_kernel(
     const float* __restrict__ aout_w, const float* __restrict__ aout_b, float* __restrict__ x,
     float* __restrict__ xhist, float* __restrict__ vhist, int64_t stage_stride, int T, int Bw,
     int No, int Nv, int vd, int Na, int ad, int d) {
+  pdl_wait();
+  pdl_launch_dependents();
   const int rows = Nv + Na;
   const int64_t gw = static_cast<int64_t>(blockIdx.x) * kRowWarps + (threadIdx.x >> 5);
   const int lane = threadIdx.x & 31;
@@ -335,6 +343,8 @@ __global__ void __launch_bounds__(256) tr_rms_partial_kernel(const AdaptItem* __
                                                              int64_t stage_stride, int K, int T,
                                                              int V, int nch,
                                                              double* __restrict__ partial) {
+  pdl_wait();
+  pdl_launch_dependents();
   __shared__ double red[8];
   const int b = blockIdx.z, br = blockIdx.y, ch = blockIdx.x;
   const AdaptItem it = items[b];
@@ -363,6 +373,8 @@ __global__ void __launch_bounds__(256) adapt_apply_kernel(
     int64_t stage_stride, int K, const float* __restrict__ eps,
     const float* __restrict__ obs_new, float* __restrict__ obs, int T, int V, int Na, int ad,
     int64_t obs_elems, int normalize, int video_mode, int traj_blocks) {
+  pdl_wait();
+  pdl_launch_dependents();
   __shared__ double rms[2];
   __shared__ int zero[2];
   const int b = blockIdx.y;
@@ -428,6 +440,8 @@ __global__ void __launch_bounds__(256) or_partial_kernel(const float* __restrict
                                                          int64_t obs_elems, int M,
                                                          float4 inv_delta, int nch,
                                                          double* __restrict__ partial) {
+  pdl_wait();
+  pdl_launch_dependents();
   __shared__ double red[8];
   const int b = blockIdx.z, m = blockIdx.y, ch = blockIdx.x;
   const int64_t comp = obs_elems / M;
@@ -451,6 +465,8 @@ __global__ void __launch_bounds__(256) rr_probe_kernel(const float* __restrict__
                                                        const StepItem* __restrict__ items,
                                                        int N, int d, int split_row, int nch,
                                                        double* __restrict__ partial) {
+  pdl_wait();
+  pdl_launch_dependents();
   __shared__ double red[8];
   const int w = blockIdx.z, br = blockIdx.y, ch = blockIdx.x;
   const int ep = items[w].ep;
@@ -487,6 +503,8 @@ __global__ void __launch_bounds__(256) rr_probe_kernel(const float* __restrict__
 __global__ void rr_gate_kernel(const double* __restrict__ partial, int Bw, int nch, int64_t n0,
                                int64_t n1, double amin, double amax, double eps, double gcos,
                                double gfit, RRGate* __restrict__ out) {
+  pdl_wait();
+  pdl_launch_dependents();
   const int i = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
   const int lane = threadIdx.x & 31;
   if (i >= Bw * 2) return;
@@ -529,6 +547,8 @@ __global__ void __launch_bounds__(256) rr_apply_kernel(float* __restrict__ h,
                                                        const StepItem* __restrict__ items,
                                                        const RRApply* __restrict__ ap, int N,
                                                        int d, int split_row) {
+  pdl_wait();
+  pdl_launch_dependents();
   const int w = blockIdx.y;
   const RRApply a = ap[w];
   if (a.mode == kRRNone) return;
@@ -564,6 +584,8 @@ __global__ void __launch_bounds__(256) rr_apply_kernel(float* __restrict__ h,
 
 // ---------------------------------------------------------------- preparation
 __global__ void cast_kernel(const float* __restrict__ in, bf16* __restrict__ out, int64_t n) {
+  pdl_wait();
+  pdl_launch_dependents();
   for (int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; i < n;
        i += static_cast<int64_t>(gridDim.x) * blockDim.x)
     out[i] = __float2bfloat16(in[i]);
@@ -614,7 +636,7 @@ cudaError_t gemv_launch(const CondGemv& g, cudaStream_t s) {
                                        static_cast<int>(smem));
   if (e != cudaSuccess) return e;
   dim3 grid((g.Nout + CPB - 1) / CPB, g.splits);
-  cond_gemv_kernel<TW, KB><<<grid, 256, smem, s>>>(g.in_part, g.in_splits, g.in_bias, g.in_act, g.features,
+  launch_pdl(cond_gemv_kernel<TW, KB>, dim3(grid), dim3(256), smem, s, g.in_part, g.in_splits, g.in_bias, g.in_act, g.features,
                                                    g.items, static_cast<const TW*>(g.W), g.K, g.Nout, g.Bw,
                                                    kslice, g.out, g.out_bias);
   return cudaGetLastError();
@@ -645,7 +667,7 @@ cudaError_t embed_tokens(float* h, float* xhist, int64_t stage_stride, const Ste
                          cudaStream_t s) {
   if (Bw <= 0) return cudaSuccess;
   const int64_t rows = static_cast<int64_t>(Bw) * (No + Nv + Na);
-  embed_kernel<<<row_blocks(rows), 32 * kRowWarps, 0, s>>>(h, xhist, stage_stride, items, x, T,
+  launch_pdl(embed_kernel, dim3(row_blocks(rows)), dim3(32 * kRowWarps), 0, s, h, xhist, stage_stride, items, x, T,
                                                            obs_emb, vid_w, vid_b, act_w, act_b,
                                                            pos, Bw, No, Nv, vd, Na, ad, d);
   return cudaGetLastError();
@@ -663,11 +685,11 @@ cudaError_t ln_modulate(const float* h, float* hcopy, const float* mods, int64_t
 #define WAM_LN_CASE(NV)                                                                            \
   case NV:                                                                                         \
     if (out_bf16)                                                                                  \
-      ln_mod_kernel<NV, bf16><<<grid, 256, 0, s>>>(h, hcopy, mods, mod_stride, shift_off,          \
+      launch_pdl(ln_mod_kernel<NV, bf16>, dim3(grid), dim3(256), 0, s, h, hcopy, mods, mod_stride, shift_off,          \
                                                    scale_off, item_map, static_cast<bf16*>(out), M, \
                                                    d, rows_per_item);                              \
     else                                                                                           \
-      ln_mod_kernel<NV, float><<<grid, 256, 0, s>>>(h, hcopy, mods, mod_stride, shift_off,         \
+      launch_pdl(ln_mod_kernel<NV, float>, dim3(grid), dim3(256), 0, s, h, hcopy, mods, mod_stride, shift_off,         \
                                                     scale_off, item_map, static_cast<float*>(out), \
                                                     M, d, rows_per_item);                          \
     break;
@@ -689,7 +711,7 @@ cudaError_t final_euler(const float* h, const StepItem* items, const float* mods
   const unsigned grid = row_blocks(static_cast<int64_t>(Bw) * (Nv + Na));
 #define WAM_FE_CASE(NV)                                                                       \
   case NV:                                                                                    \
-    final_euler_kernel<NV><<<grid, 256, 0, s>>>(h, items, mods, mod_stride, fin_off, vout_w,  \
+    launch_pdl(final_euler_kernel<NV>, dim3(grid), dim3(256), 0, s, h, items, mods, mod_stride, fin_off, vout_w,  \
                                                 vout_b, aout_w, aout_b, x, xhist, vhist,      \
                                                 stage_stride, T, Bw, No, Nv, vd, Na, ad, d); \
     break;
@@ -710,7 +732,7 @@ int tr_num_chunks(int T, int V) {
 cudaError_t tr_rms_partial(const AdaptItem* items, const float* xhist, int64_t stage_stride,
                            int K, int B, int T, int V, int nch, double* partial, cudaStream_t s) {
   dim3 grid(nch, 2, B);
-  tr_rms_partial_kernel<<<grid, 256, 0, s>>>(items, xhist, stage_stride, K, T, V, nch, partial);
+  launch_pdl(tr_rms_partial_kernel, dim3(grid), dim3(256), 0, s, items, xhist, stage_stride, K, T, V, nch, partial);
   return cudaGetLastError();
 }
 
@@ -722,7 +744,7 @@ cudaError_t adapt_apply(const AdaptItem* items, const double* partial, int nch, 
   const int traj_blocks = (T + 255) / 256 < 64 ? (T + 255) / 256 : 64;
   const int obs_blocks = static_cast<int>((obs_elems + 255) / 256 < 64 ? (obs_elems + 255) / 256 : 64);
   dim3 grid(traj_blocks + obs_blocks, B);
-  adapt_apply_kernel<<<grid, 256, 0, s>>>(items, partial, nch, x, xb0, xhist, stage_stride, K,
+  launch_pdl(adapt_apply_kernel, dim3(grid), dim3(256), 0, s, items, partial, nch, x, xb0, xhist, stage_stride, K,
                                           eps, obs_new, obs, T, V, Na, ad, obs_elems, normalize,
                                           video_mode, traj_blocks);
   return cudaGetLastError();
@@ -737,7 +759,7 @@ cudaError_t or_score_partial(const float* pred, const float* real, int B, int64_
                              cudaStream_t s) {
   dim3 grid(nch, M, B);
   const float4 idl = make_float4(inv_delta4[0], inv_delta4[1], inv_delta4[2], inv_delta4[3]);
-  or_partial_kernel<<<grid, 256, 0, s>>>(pred, real, obs_elems, M, idl, nch, partial);
+  launch_pdl(or_partial_kernel, dim3(grid), dim3(256), 0, s, pred, real, obs_elems, M, idl, nch, partial);
   return cudaGetLastError();
 }
 
@@ -750,7 +772,7 @@ cudaError_t rr_probe_partial(const float* h, const float* hq, const float* pa,
                              double* partial, cudaStream_t s) {
   if (Bw <= 0) return cudaSuccess;
   dim3 grid(nch, 2, Bw);
-  rr_probe_kernel<<<grid, 256, 0, s>>>(h, hq, pa, items, N, d, split_row, nch, partial);
+  launch_pdl(rr_probe_kernel, dim3(grid), dim3(256), 0, s, h, hq, pa, items, N, d, split_row, nch, partial);
   return cudaGetLastError();
 }
 
@@ -758,7 +780,7 @@ cudaError_t rr_gate(const double* partial, int Bw, int nch, int64_t n0, int64_t 
                     double amax, double eps, double gcos, double gfit, RRGate* out,
                     cudaStream_t s) {
   if (Bw <= 0) return cudaSuccess;
-  rr_gate_kernel<<<(Bw * 2 * 32 + 127) / 128, 128, 0, s>>>(partial, Bw, nch, n0, n1, amin, amax, eps,
+  launch_pdl(rr_gate_kernel, dim3((Bw * 2 * 32 + 127) / 128), dim3(128), 0, s, partial, Bw, nch, n0, n1, amin, amax, eps,
                                                            gcos, gfit, out);
   return cudaGetLastError();
 }
@@ -770,7 +792,7 @@ cudaError_t rr_apply(float* h, const float* hm, const float* hq, float* pa, floa
   const int64_t n4 = static_cast<int64_t>(N) * d / 4;
   const int bx = static_cast<int>((n4 + 255) / 256 < 1024 ? (n4 + 255) / 256 : 1024);
   dim3 grid(bx, Bw);
-  rr_apply_kernel<<<grid, 256, 0, s>>>(h, hm, hq, pa, ra, items, ap, N, d, split_row);
+  launch_pdl(rr_apply_kernel, dim3(grid), dim3(256), 0, s, h, hm, hq, pa, ra, items, ap, N, d, split_row);
   return cudaGetLastError();
 }
 

@@ -31,6 +31,8 @@ __global__ void __launch_bounds__(256) simt_gemm_kernel(const float* __restrict_
                                                         int K, EpiArgs e) {
   __shared__ float As[kKc][kT + 4];
   __shared__ float Bs[kKc][kT + 4];
+  pdl_wait();
+  pdl_launch_dependents();
   const int tx = threadIdx.x & 15;
   const int ty = threadIdx.x >> 4;
   const int m0 = blockIdx.y * kT;
@@ -82,13 +84,12 @@ cudaError_t simt_gemm(const float* A, const float* Wt, int M, int N, int K, int 
   if (M <= 0) return cudaSuccess;
   dim3 grid((N + kT - 1) / kT, (M + kT - 1) / kT);
   switch (epi) {
-    case kEpiBf16: simt_gemm_kernel<kEpiBf16><<<grid, 256, 0, s>>>(A, Wt, M, N, K, e); break;
-    case kEpiGeluBf16: simt_gemm_kernel<kEpiGeluBf16><<<grid, 256, 0, s>>>(A, Wt, M, N, K, e); break;
-    case kEpiResidF32: simt_gemm_kernel<kEpiResidF32><<<grid, 256, 0, s>>>(A, Wt, M, N, K, e); break;
-    case kEpiF32: simt_gemm_kernel<kEpiF32><<<grid, 256, 0, s>>>(A, Wt, M, N, K, e); break;
+    case kEpiBf16: return launch_pdl(simt_gemm_kernel<kEpiBf16>, grid, dim3(256), 0, s, A, Wt, M, N, K, e);
+    case kEpiGeluBf16: return launch_pdl(simt_gemm_kernel<kEpiGeluBf16>, grid, dim3(256), 0, s, A, Wt, M, N, K, e);
+    case kEpiResidF32: return launch_pdl(simt_gemm_kernel<kEpiResidF32>, grid, dim3(256), 0, s, A, Wt, M, N, K, e);
+    case kEpiF32: return launch_pdl(simt_gemm_kernel<kEpiF32>, grid, dim3(256), 0, s, A, Wt, M, N, K, e);
     default: return cudaErrorInvalidValue;
   }
-  return cudaGetLastError();
 }
 
 }  // namespace wam

@@ -16,6 +16,7 @@
 #include <mutex>
 
 #include "common.cuh"
+#include "tcgen05.cuh"
 
 namespace wam {
 namespace {
@@ -35,112 +36,6 @@ struct TileCfg {
   static constexpr int kBarrierBytes = 256;
   static constexpr int kSmemBytes = kStages * kStageBytes + kBarrierBytes + 1024;
 };
-
-WAM_DEV uint32_t smem_u32(const void* p) {
-  return static_cast<uint32_t>(__cvta_generic_to_shared(p));
-}
-
-WAM_DEV void mbar_init(uint32_t bar, uint32_t count) {
-  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(count) : "memory");
-}
-WAM_DEV void mbar_expect_tx(uint32_t bar, uint32_t bytes) {
-  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(bytes)
-               : "memory");
-}
-WAM_DEV void mbar_arrive(uint32_t bar) {
-  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
-}
-WAM_DEV bool mbar_try_wait(uint32_t bar, uint32_t parity) {
-  uint32_t ok;
-  asm volatile(
-      "{\n\t.reg .pred p;\n\t"
-      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
-      "selp.u32 %0, 1, 0, p;\n\t}"
-      : "=r"(ok)
-      : "r"(bar), "r"(parity)
-      : "memory");
-  return ok != 0;
-}
-
-// Bounded wait: true when the phase completed; false on abort (flag raised by another role
-// or by this wait's own time limit).
-WAM_DEV bool mbar_wait(uint32_t bar, uint32_t parity, volatile int* abort_flag, int* dev_err) {
-  if (mbar_try_wait(bar, parity)) return true;
-  const uint64_t t0 = globaltimer_ns();
-  for (uint32_t i = 1;; ++i) {
-    if (mbar_try_wait(bar, parity)) return true;
-    if ((i & 63u) == 0) {
-      if (*abort_flag) return false;
-      if (globaltimer_ns() - t0 > kWaitLimitNs) {
-        *abort_flag = 1;
-        if (dev_err != nullptr) atomicOr(dev_err, kDevErrTimeout);
-        return false;
-      }
-    }
-  }
-}
-
-WAM_DEV void tma_load_2d(uint32_t dst, const CUtensorMap* map, int x, int y, uint32_t bar) {
-  asm volatile(
-      "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes"
-      " [%0], [%1, {%2, %3}], [%4];" ::"r"(dst),
-      "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(bar)
-      : "memory");
-}
-
-WAM_DEV void tc_fence_before() { asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory"); }
-WAM_DEV void tc_fence_after() { asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory"); }
-
-// Shared-memory matrix descriptor for a K-major operand tile written by TMA with the 128-byte
-// swizzle: rows of 128 bytes, 8-row core groups 1024 bytes apart (stride byte offset), the
-// leading byte offset unused for this layout, descriptor version 1, swizzle mode 2 (128 B).
-WAM_DEV uint64_t sw128_desc(uint32_t saddr) {
-  uint64_t d = 0;
-  d |= static_cast<uint64_t>((saddr & 0x3FFFFu) >> 4);
-  d |= static_cast<uint64_t>(16u >> 4) << 16;
-  d |= static_cast<uint64_t>(1024u >> 4) << 32;
-  d |= static_cast<uint64_t>(1) << 46;
-  d |= static_cast<uint64_t>(2) << 61;
-  return d;
-}
-
-// Instruction descriptor of kind::f16: fp32 accumulator, bf16 A and B, both K-major,
-// N >> 3 at bit 17, M >> 4 at bit 24.
-template <int BN>
-WAM_DEV uint32_t idesc_bf16() {
-  return (1u << 4) | (1u << 7) | (1u << 10) | (static_cast<uint32_t>(BN >> 3) << 17) |
-         (static_cast<uint32_t>(kBM >> 4) << 24);
-}
-
-WAM_DEV void umma_bf16(uint32_t d_tmem, uint64_t a, uint64_t b, uint32_t idesc, uint32_t acc) {
-  asm volatile(
-      "{\n\t.reg .pred p;\n\t"
-      "setp.ne.b32 p, %4, 0;\n\t"
-      "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
-      "l"(a), "l"(b), "r"(idesc), "r"(acc)
-      : "memory");
-}
-
-WAM_DEV void umma_commit(uint32_t bar) {
-  asm volatile(
-      "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(bar)
-      : "memory");
-}
-
-WAM_DEV void tmem_ld32(uint32_t taddr, uint32_t (&r)[32]) {
-  asm volatile(
-      "tcgen05.ld.sync.aligned.32x32b.x32.b32 "
-      "{%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,"
-      "%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];"
-      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
-        "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]),
-        "=r"(r[13]), "=r"(r[14]), "=r"(r[15]), "=r"(r[16]), "=r"(r[17]), "=r"(r[18]),
-        "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]), "=r"(r[24]),
-        "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]),
-        "=r"(r[31])
-      : "r"(taddr));
-  asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
-}
 
 // Fused accumulator read-back for one row segment of 32 columns.
 template <int EPI>
@@ -177,6 +72,34 @@ WAM_DEV void epilogue32(const EpiArgs& e, int N, int row, int col0, const uint32
       u.z = *reinterpret_cast<uint32_t*>(&p2);
       u.w = *reinterpret_cast<uint32_t*>(&p3);
       dst[j] = u;
+    }
+  } else if constexpr (EPI == kEpiQkvVt) {
+    // q | k columns as bf16 rows; v columns transposed per (item, head) into V^T so that the
+    // attention's P.V product reads a K-major operand.  Lanes hold consecutive tokens, so each
+    // of the 32 stores of a warp writes 64 contiguous bytes.
+    const int d = N / 3;
+    if (col0 < 2 * d) {
+      uint4* dst = reinterpret_cast<uint4*>(static_cast<bf16*>(e.C) + static_cast<int64_t>(row) * N + col0);
+#pragma unroll
+      for (int j = 0; j < 4; ++j) {
+        uint4 u;
+        __nv_bfloat162 p0 = __floats2bfloat162_rn(v[8 * j + 0], v[8 * j + 1]);
+        __nv_bfloat162 p1 = __floats2bfloat162_rn(v[8 * j + 2], v[8 * j + 3]);
+        __nv_bfloat162 p2 = __floats2bfloat162_rn(v[8 * j + 4], v[8 * j + 5]);
+        __nv_bfloat162 p3 = __floats2bfloat162_rn(v[8 * j + 6], v[8 * j + 7]);
+        u.x = *reinterpret_cast<uint32_t*>(&p0);
+        u.y = *reinterpret_cast<uint32_t*>(&p1);
+        u.z = *reinterpret_cast<uint32_t*>(&p2);
+        u.w = *reinterpret_cast<uint32_t*>(&p3);
+        dst[j] = u;
+      }
+    } else {
+      const int cc = col0 - 2 * d;
+      const int item = row / e.rows_per_item;
+      const int n = row - item * e.rows_per_item;
+      bf16* dst = e.vt + (static_cast<int64_t>(item) * d + cc) * e.vt_ld + n;
+#pragma unroll
+      for (int i = 0; i < 32; ++i) dst[static_cast<int64_t>(i) * e.vt_ld] = __float2bfloat16(v[i]);
     }
   } else if constexpr (EPI == kEpiF32) {
     float4* dst = reinterpret_cast<float4*>(static_cast<float*>(e.C) + static_cast<int64_t>(row) * N + col0);
@@ -249,17 +172,31 @@ __global__ void __launch_bounds__(kThreads, 1)
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
+  pdl_launch_dependents();
 
   if (warp == 0 && lane == 0) {
     // ---------------- TMA producer ----------------
     asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmA)) : "memory");
     asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmB)) : "memory");
+    // The weight operand does not depend on earlier kernels: its first stages are requested
+    // before waiting for them, overlapping the previous kernel's tail.
+    const int pre = blockIdx.x < num_tiles ? (num_k < C::kStages ? num_k : C::kStages) : 0;
+    for (int s = 0; s < pre; ++s) {
+      const uint32_t fb = smem_u32(&full[s]);
+      const uint32_t b_dst = smem_u32(tiles + s * C::kStageBytes) + kTileBytesA;
+      mbar_expect_tx(fb, C::kStageBytes);
+#pragma unroll
+      for (int h = 0; h < BN / kBoxRows; ++h)
+        tma_load_2d(b_dst + h * kBoxRows * 128, &tmB, s * kBK, (blockIdx.x / num_m) * BN + h * kBoxRows, fb);
+    }
+    pdl_wait();
     int stage = 0;
     uint32_t phase = 0;
     int issued[C::kStages];
     uint32_t issued_phase[C::kStages];
     for (int s = 0; s < C::kStages; ++s) issued[s] = 0, issued_phase[s] = 0;
     bool ok = true;
+    bool first = true;
     for (int tile = blockIdx.x; ok && tile < num_tiles; tile += gridDim.x) {
       const int mt = tile % num_m;
       const int nt = tile / num_m;
@@ -271,11 +208,13 @@ __global__ void __launch_bounds__(kThreads, 1)
         const uint32_t fb = smem_u32(&full[stage]);
         const uint32_t a_dst = smem_u32(tiles + stage * C::kStageBytes);
         const uint32_t b_dst = a_dst + kTileBytesA;
-        mbar_expect_tx(fb, C::kStageBytes);
-        tma_load_2d(a_dst, &tmA, kb * kBK, mt * kBM, fb);
+        if (!(first && kb < pre)) {
+          mbar_expect_tx(fb, C::kStageBytes);
 #pragma unroll
-        for (int h = 0; h < BN / kBoxRows; ++h)
-          tma_load_2d(b_dst + h * kBoxRows * 128, &tmB, kb * kBK, nt * BN + h * kBoxRows, fb);
+          for (int h = 0; h < BN / kBoxRows; ++h)
+            tma_load_2d(b_dst + h * kBoxRows * 128, &tmB, kb * kBK, nt * BN + h * kBoxRows, fb);
+        }
+        tma_load_2d(a_dst, &tmA, kb * kBK, mt * kBM, fb);
         issued[stage] = 1;
         issued_phase[stage] = phase;
         if (++stage == C::kStages) {
@@ -283,6 +222,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           phase ^= 1u;
         }
       }
+      first = false;
     }
     if (!ok) {
       // Drain: let every copy this thread issued land before the CTA releases its smem.
@@ -296,7 +236,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
   } else if (warp == 1 && lane == 0) {
     // ---------------- MMA issuer ----------------
-    const uint32_t idesc = idesc_bf16<BN>();
+    pdl_wait();
+    const uint32_t idesc = idesc_bf16(kBM, BN);
     int stage = 0;
     uint32_t phase = 0;
     int it = 0;
@@ -343,6 +284,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
   } else if (warp >= 2) {
     // ---------------- epilogue ----------------
+    pdl_wait();
     const int quarter = warp & 3;  // TMEM lanes this warp may access
     int it = 0;
     for (int tile = blockIdx.x; tile < num_tiles; tile += gridDim.x, ++it) {
@@ -408,8 +350,8 @@ cudaError_t launch(const CUtensorMap& ta, const CUtensorMap& tb, int M, int N, i
   }
   const int tiles = ((M + kBM - 1) / kBM) * (N / BN);
   const int grid = tiles < num_sms ? tiles : num_sms;
-  gemm_tc_kernel<BN, EPI><<<grid, kThreads, C::kSmemBytes, s>>>(ta, tb, M, N, K, e, dev_err);
-  return cudaGetLastError();
+  return launch_pdl(gemm_tc_kernel<BN, EPI>, dim3(grid), dim3(kThreads), C::kSmemBytes, s, ta, tb, M, N, K, e,
+                    dev_err);
 }
 
 template <int BN>
@@ -420,11 +362,27 @@ cudaError_t dispatch_epi(const CUtensorMap& ta, const CUtensorMap& tb, int M, in
     case kEpiGeluBf16: return launch<BN, kEpiGeluBf16>(ta, tb, M, N, K, e, num_sms, dev_err, s);
     case kEpiResidF32: return launch<BN, kEpiResidF32>(ta, tb, M, N, K, e, num_sms, dev_err, s);
     case kEpiF32: return launch<BN, kEpiF32>(ta, tb, M, N, K, e, num_sms, dev_err, s);
+    case kEpiQkvVt: return launch<BN, kEpiQkvVt>(ta, tb, M, N, K, e, num_sms, dev_err, s);
     default: return cudaErrorInvalidValue;
   }
 }
 
 }  // namespace
+
+int tc_encode_bf16_box(CUtensorMap* map, const void* base, uint64_t rows, uint64_t cols, uint64_t ld,
+                       uint32_t box_cols, uint32_t box_rows) {
+  PFN_cuTensorMapEncodeTiled_v12000 fn = encode_fn();
+  if (fn == nullptr) return -1;
+  if ((reinterpret_cast<uintptr_t>(base) & 15u) != 0 || (ld * 2) % 16 != 0) return -2;
+  cuuint64_t dims[2] = {cols, rows};
+  cuuint64_t strides[1] = {ld * 2};
+  cuuint32_t box[2] = {box_cols, box_rows};
+  cuuint32_t estr[2] = {1, 1};
+  CUresult r = fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box, estr,
+                  CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                  CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS ? 0 : -3;
+}
 
 int tc_encode_kmajor_bf16(CUtensorMap* map, const void* base, uint64_t rows, uint64_t K) {
   PFN_cuTensorMapEncodeTiled_v12000 fn = encode_fn();

@@ -31,6 +31,8 @@ EpiArgs make_epi(const float* bias, void* C, const float* gate, int64_t gstride,
   e.gate_stride = gstride;
   e.rows_per_item = rpi > 0 ? rpi : 1;
   e.item_map = nullptr;
+  e.vt = nullptr;
+  e.vt_ld = 0;
   return e;
 }
 
@@ -117,6 +119,46 @@ int wam_op_ln_modulate(const float* h, const float* shift, const float* scale, i
   cudaError_t e = ln_modulate(h, nullptr, base, mod_stride, shift_off, scale_off, nullptr, out,
                               precision == WAM_PREC_BF16, M, d, rows_per_item, static_cast<cudaStream_t>(stream));
   return e == cudaSuccess ? WAM_OK : op_cuda("LN-modulate launch", e);
+}
+
+int wam_op_gemm_qkv_vt(const void* A, const void* Wt, const float* bias, void* qkv, void* vt, int32_t M,
+                       int32_t d, int32_t rows_per_item, int32_t vt_ld, void* stream) {
+  const int N = 3 * d, K = d;
+  int r = check_gemm_args(A, Wt, qkv, M, N, K, WAM_EPI_BF16, nullptr, rows_per_item);
+  if (r != WAM_OK) return r;
+  if (vt == nullptr || rows_per_item <= 0 || vt_ld < rows_per_item || vt_ld % 8 != 0 || d % 64 != 0 || d % 128 != 0)
+    return op_fail(WAM_ERR_INVALID_ARG, "bad V^T arguments");
+  if (!aligned16(A) || !aligned16(Wt) || !aligned16(qkv) || (bias && !aligned16(bias)))
+    return op_fail(WAM_ERR_INVALID_ARG, "operands must be 16-byte aligned");
+  int dev = 0, sms = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e == cudaSuccess) e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  if (e != cudaSuccess) return op_cuda("device query", e);
+  CUtensorMap ta, tb;
+  if (tc_encode_kmajor_bf16(&ta, A, static_cast<uint64_t>(M > 0 ? M : 1), K) != 0 ||
+      tc_encode_kmajor_bf16(&tb, Wt, N, K) != 0)
+    return op_fail(WAM_ERR_CUDA, "cuTensorMapEncodeTiled failed");
+  EpiArgs ep = make_epi(bias, qkv, nullptr, 0, rows_per_item);
+  ep.vt = static_cast<bf16*>(vt);
+  ep.vt_ld = vt_ld;
+  e = tc_gemm(ta, tb, M, N, K, kEpiQkvVt, ep, sms, nullptr, static_cast<cudaStream_t>(stream));
+  return e == cudaSuccess ? WAM_OK : op_cuda("tcgen05 QKV GEMM launch", e);
+}
+
+int wam_op_attention_tc(const void* qkv, const void* vt, void* out, int32_t B, int32_t N, int32_t d,
+                        int32_t n_heads, void* stream) {
+  if (qkv == nullptr || vt == nullptr || out == nullptr || B < 0 || N < 0 || n_heads <= 0 || d != 64 * n_heads)
+    return op_fail(WAM_ERR_INVALID_ARG, "tcgen05 attention needs head dim 64");
+  if (!aligned16(qkv) || !aligned16(vt) || !aligned16(out)) return op_fail(WAM_ERR_INVALID_ARG, "16-byte alignment required");
+  if (B == 0 || N == 0) return WAM_OK;
+  const int vt_ld = attention_tc_vt_ld(N);
+  CUtensorMap tq, tv;
+  if (tc_encode_bf16_box(&tq, qkv, static_cast<uint64_t>(B) * N, 3 * d, 3 * d, 64, 128) != 0 ||
+      tc_encode_bf16_box(&tv, vt, static_cast<uint64_t>(B) * d, vt_ld, vt_ld, 64, 64) != 0)
+    return op_fail(WAM_ERR_CUDA, "cuTensorMapEncodeTiled failed");
+  cudaError_t e = attention_tc(tq, tv, static_cast<bf16*>(out), B, N, d, n_heads, nullptr,
+                               static_cast<cudaStream_t>(stream));
+  return e == cudaSuccess ? WAM_OK : op_cuda("tcgen05 attention launch", e);
 }
 
 }  // extern "C"

@@ -84,6 +84,11 @@ struct wam_ctx {
   float *h = nullptr, *hq = nullptr, *hm = nullptr;
   void *xln = nullptr, *qkv = nullptr, *att = nullptr, *u = nullptr, *obs_lp = nullptr;
   CUtensorMap tm_xln, tm_att, tm_u, tm_obs_lp;
+  // tensor-core attention (head dim 64): V^T per (episode, head) and the TMA maps it reads
+  bool tc_attn = false;
+  void* vt = nullptr;
+  int vt_ld = 0;
+  CUtensorMap tm_qk, tm_vt;
   float *t1 = nullptr, *cvec = nullptr, *mods = nullptr;
   StepItem* d_items = nullptr;
   int* d_map = nullptr;
@@ -260,6 +265,8 @@ EpiArgs epi_args(const float* bias, void* C, const float* gate, int64_t gstride,
   e.gate_stride = gstride;
   e.rows_per_item = rpi;
   e.item_map = map;
+  e.vt = nullptr;
+  e.vt_ld = 0;
   return e;
 }
 
@@ -276,12 +283,20 @@ int run_layer(wam_ctx* c, int l, float* hb, int Bw, const int* map, float* hcopy
   const int base = l * 6 * d;
   LayerW& w = c->layers[l];
   TRY(ln_mod(c, hb, hcopy, base, base + d, map, M));
-  TRY(gemm(c, &c->tm_xln, c->xln, &w.tm_qkv, w.qkv_wt, M, 3 * d, d, kEpiBf16,
-           epi_args(w.qkv_b, c->qkv, nullptr, 0, c->N, nullptr)));
+  {
+    EpiArgs eq = epi_args(w.qkv_b, c->qkv, nullptr, 0, c->N, nullptr);
+    if (c->tc_attn) {
+      eq.vt = static_cast<bf16*>(c->vt);
+      eq.vt_ld = c->vt_ld;
+    }
+    TRY(gemm(c, &c->tm_xln, c->xln, &w.tm_qkv, w.qkv_wt, M, 3 * d, d, c->tc_attn ? kEpiQkvVt : kEpiBf16, eq));
+  }
   {
     const double el = c->bf16 ? 2.0 : 4.0;
     Span sp(c, WAM_KCLASS_ATTN, 4.0 * Bw * double(c->N) * c->N * d, el * 4.0 * M * d);
-    if (c->bf16)
+    if (c->tc_attn)
+      CK(attention_tc(c->tm_qk, c->tm_vt, static_cast<bf16*>(c->att), Bw, c->N, d, c->H, c->d_err, c->stream));
+    else if (c->bf16)
       CK(attention_bf16(static_cast<const bf16*>(c->qkv), static_cast<bf16*>(c->att), Bw, c->N, d, c->H, c->stream));
     else
       CK(attention_f32(static_cast<const float*>(c->qkv), static_cast<float*>(c->att), Bw, c->N, d, c->H, c->stream));
@@ -721,6 +736,17 @@ int create_impl(wam_ctx* c, const wam_config* cfg, const float* weights, size_t 
     TRY(encode(c, &c->tm_u, c->u, rows, c->dff));
     TRY(encode(c, &c->tm_obs_lp, c->obs_lp, size_t(c->Bmax) * c->No, c->d));
     TRY(encode(c, &c->tm_obs_w, c->obs_wt, c->d, c->d));
+    c->tc_attn = c->d / c->H == 64;
+    if (c->tc_attn) {
+      c->vt_ld = attention_tc_vt_ld(c->N);
+      uint8_t* vt = nullptr;
+      TRY(dalloc(c, c->allocs, &vt, size_t(c->Bmax) * c->d * c->vt_ld * 2));
+      CK(cudaMemsetAsync(vt, 0, size_t(c->Bmax) * c->d * c->vt_ld * 2, c->stream));
+      c->vt = vt;
+      if (tc_encode_bf16_box(&c->tm_qk, c->qkv, rows, 3 * c->d, 3 * c->d, 64, 128) != 0 ||
+          tc_encode_bf16_box(&c->tm_vt, c->vt, size_t(c->Bmax) * c->d, c->vt_ld, c->vt_ld, 64, 64) != 0)
+        return fail(c, WAM_ERR_CUDA, "cuTensorMapEncodeTiled failed for the attention operands");
+    }
     for (LayerW& w : c->layers) {
       TRY(encode(c, &w.tm_qkv, w.qkv_wt, 3 * c->d, c->d));
       TRY(encode(c, &w.tm_out, w.out_wt, c->d, c->d));

@@ -128,6 +128,8 @@ def lib() -> ctypes.CDLL:
         "wam_op_attention": (ctypes.c_int, [_vp, _vp, _i32, _i32, _i32, _i32, _i32, _vp]),
         "wam_op_ln_modulate": (ctypes.c_int, [_vp, _vp, _vp, ctypes.c_int64, _vp, _i32, _i32, _i32, _i32, _vp]),
         "wam_op_last_error": (ctypes.c_char_p, []),
+        "wam_op_gemm_qkv_vt": (ctypes.c_int, [_vp, _vp, _vp, _vp, _vp, _i32, _i32, _i32, _i32, _vp]),
+        "wam_op_attention_tc": (ctypes.c_int, [_vp, _vp, _vp, _i32, _i32, _i32, _i32, _vp]),
         "wam_tr_remap_static": (ctypes.c_int, [_vp, _vp, _vp, _vp, _i32, _i32, _i32, _i32, _i32, _i32,
                                                ctypes.c_double, ctypes.c_double, _i32, _i32, _vp]),
     }
@@ -326,6 +328,15 @@ def op_gemm_f32(A, Wt, bias, C, M, N, K, epilogue, gate=None, gate_stride=0, row
 
 def op_attention(qkv, out, B, N, d, n_heads, precision="bf16", stream=None):
     _op_check(lib().wam_op_attention(ptr(qkv), ptr(out), B, N, d, n_heads, PREC[precision], stream))
+
+
+def op_gemm_qkv_vt(A, Wt, bias, qkv, vt, M, d, rows_per_item, vt_ld, stream=None):
+    _op_check(lib().wam_op_gemm_qkv_vt(ptr(A), ptr(Wt), ptr(bias), ptr(qkv), ptr(vt), M, d, rows_per_item, vt_ld,
+                                       stream))
+
+
+def op_attention_tc(qkv, vt, out, B, N, d, n_heads, stream=None):
+    _op_check(lib().wam_op_attention_tc(ptr(qkv), ptr(vt), ptr(out), B, N, d, n_heads, stream))
 
 
 def op_ln_modulate(h, shift, scale, mod_stride, out, M, d, rows_per_item, precision="bf16", stream=None):

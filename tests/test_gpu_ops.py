@@ -141,3 +141,35 @@ def test_ln_modulate_matches_oracle(wamlib, prec, d):
     ref = O.layer_norm(h.astype(np.float64)) * (1 + mods[item, d:]) + mods[item, :d]
     tol = 1e-2 if prec == "bf16" else 2e-5
     assert np.max(np.abs(_f64(out) - ref)) <= tol * np.max(np.abs(ref))
+
+
+TC_ATTN_CASES = [(1, 1, 2), (1, 56, 2), (2, 128, 2), (1, 129, 4), (1, 1296, 12), (2, 300, 2), (1, 2464, 4)]
+
+
+@pytest.mark.parametrize("B,N,H", TC_ATTN_CASES)
+def test_attention_tcgen05_matches_oracle(wamlib, B, N, H):
+    """QKV projection writing V^T, then the tcgen05 attention, against the oracle's attention of
+    the same bf16 q, k, v."""
+    rng = np.random.default_rng(B * 100 + N + H)
+    d = 64 * H
+    dev = torch.device("cuda")
+    x = _bf16(rng.standard_normal((B * N, d)))
+    Wt = _bf16(rng.standard_normal((3 * d, d)) / np.sqrt(d))
+    bias = torch.from_numpy((rng.standard_normal(3 * d) * 0.1).astype(np.float32))
+    vt_ld = (N + 7) // 8 * 8
+    qkv = torch.full((B * N, 3 * d), float("nan"), dtype=torch.bfloat16, device=dev)
+    vt = torch.zeros((B * d, vt_ld), dtype=torch.bfloat16, device=dev)
+    out = torch.full((B * N, d), float("nan"), dtype=torch.bfloat16, device=dev)
+    W.op_gemm_qkv_vt(x.to(dev), Wt.to(dev), bias.to(dev), qkv, vt, B * N, d, N, vt_ld)
+    W.op_attention_tc(qkv, vt, out, B, N, d, H)
+    torch.cuda.synchronize()
+    proj = torch.from_numpy(_f64(x) @ _f64(Wt).T + bias.double().numpy())
+    qk = _f64(qkv)[:, :2 * d]
+    assert np.max(np.abs(qk - proj.numpy()[:, :2 * d])) <= 2e-2 * np.max(np.abs(proj.numpy()))
+    v_from_vt = _f64(vt).reshape(B, H, 64, vt_ld)[..., :N].transpose(0, 3, 1, 2).reshape(B * N, d)
+    assert np.max(np.abs(v_from_vt - proj.numpy()[:, 2 * d:])) <= 2e-2 * np.max(np.abs(proj.numpy()))
+    got = _f64(out)
+    for b in range(B):
+        blk = slice(b * N, (b + 1) * N)
+        ref = O.attention(qk[blk, :d], qk[blk, d:], v_from_vt[blk], H)
+        assert np.max(np.abs(got[blk] - ref)) <= 2e-2
