@@ -104,8 +104,11 @@ struct EpiArgs {
 // ---- internal interfaces -----------------------------------------------------------------
 // tcgen05 GEMM (gemm_tc.cu).  CUtensorMap is the driver's 128-byte opaque descriptor.
 int tc_encode_kmajor_bf16(CUtensorMap* map, const void* base, uint64_t rows, uint64_t K);
-cudaError_t tc_gemm(const CUtensorMap& ta, const CUtensorMap& tb, int M, int N, int K, int epi,
-                    const EpiArgs& e, int num_sms, int* dev_err, cudaStream_t s);
+// Same operand with 64-row boxes: the B map of 64-column output tiles.
+int tc_encode_kmajor_bf16_box64(CUtensorMap* map, const void* base, uint64_t rows, uint64_t K);
+// tb64 (nullable) lets the launcher pick 64-column tiles for narrow projections.
+cudaError_t tc_gemm(const CUtensorMap& ta, const CUtensorMap& tb, const CUtensorMap* tb64, int M, int N, int K,
+                    int epi, const EpiArgs& e, int num_sms, int* dev_err, cudaStream_t s);
 
 // float32 SIMT GEMM (gemm_simt.cu): C = A[M,K] Wt[N,K]^T
 cudaError_t simt_gemm(const float* A, const float* Wt, int M, int N, int K, int epi,

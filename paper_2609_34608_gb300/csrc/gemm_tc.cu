@@ -25,11 +25,12 @@ constexpr int kBM = 128;
 constexpr int kBK = 64;           // 64 bf16 = 128 bytes = one swizzle row
 constexpr int kThreads = 192;
 constexpr int kTileBytesA = kBM * kBK * 2;  // 16 KB
-constexpr int kBoxRows = 128;               // TMA box rows for both operands
+constexpr int kBoxRows = 128;               // TMA box rows of the A operand and wide B tiles
 
 template <int BN>
 struct TileCfg {
-  static constexpr int kStages = (BN == 256) ? 4 : 6;
+  static constexpr int kStages = (BN == 256) ? 4 : (BN == 128 ? 6 : 8);
+  static constexpr int kBoxB = BN < kBoxRows ? BN : kBoxRows;  // rows per B load
   static constexpr int kTileBytesB = BN * kBK * 2;
   static constexpr int kStageBytes = kTileBytesA + kTileBytesB;
   static constexpr int kTmemCols = 2 * BN;
@@ -186,8 +187,8 @@ __global__ void __launch_bounds__(kThreads, 1)
       const uint32_t b_dst = smem_u32(tiles + s * C::kStageBytes) + kTileBytesA;
       mbar_expect_tx(fb, C::kStageBytes);
 #pragma unroll
-      for (int h = 0; h < BN / kBoxRows; ++h)
-        tma_load_2d(b_dst + h * kBoxRows * 128, &tmB, s * kBK, (blockIdx.x / num_m) * BN + h * kBoxRows, fb);
+      for (int h = 0; h < BN / C::kBoxB; ++h)
+        tma_load_2d(b_dst + h * C::kBoxB * 128, &tmB, s * kBK, (blockIdx.x / num_m) * BN + h * C::kBoxB, fb);
     }
     pdl_wait();
     int stage = 0;
@@ -211,8 +212,8 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (!(first && kb < pre)) {
           mbar_expect_tx(fb, C::kStageBytes);
 #pragma unroll
-          for (int h = 0; h < BN / kBoxRows; ++h)
-            tma_load_2d(b_dst + h * kBoxRows * 128, &tmB, kb * kBK, nt * BN + h * kBoxRows, fb);
+          for (int h = 0; h < BN / C::kBoxB; ++h)
+            tma_load_2d(b_dst + h * C::kBoxB * 128, &tmB, kb * kBK, nt * BN + h * C::kBoxB, fb);
         }
         tma_load_2d(a_dst, &tmA, kb * kBK, mt * kBM, fb);
         issued[stage] = 1;
@@ -384,6 +385,10 @@ int tc_encode_bf16_box(CUtensorMap* map, const void* base, uint64_t rows, uint64
   return r == CUDA_SUCCESS ? 0 : -3;
 }
 
+int tc_encode_kmajor_bf16_box64(CUtensorMap* map, const void* base, uint64_t rows, uint64_t K) {
+  return tc_encode_bf16_box(map, base, rows, K, K, kBK, 64);
+}
+
 int tc_encode_kmajor_bf16(CUtensorMap* map, const void* base, uint64_t rows, uint64_t K) {
   PFN_cuTensorMapEncodeTiled_v12000 fn = encode_fn();
   if (fn == nullptr) return -1;
@@ -398,16 +403,24 @@ int tc_encode_kmajor_bf16(CUtensorMap* map, const void* base, uint64_t rows, uin
   return r == CUDA_SUCCESS ? 0 : -3;
 }
 
-cudaError_t tc_gemm(const CUtensorMap& ta, const CUtensorMap& tb, int M, int N, int K, int epi,
-                    const EpiArgs& e, int num_sms, int* dev_err, cudaStream_t s) {
+cudaError_t tc_gemm(const CUtensorMap& ta, const CUtensorMap& tb, const CUtensorMap* tb64, int M, int N, int K,
+                    int epi, const EpiArgs& e, int num_sms, int* dev_err, cudaStream_t s) {
   if (M <= 0) return cudaSuccess;
   if (K % kBK != 0 || N % 128 != 0) return cudaErrorInvalidValue;
-  // Wide tiles only when they still fill every SM; small-M problems keep more CTAs busy
-  // with 128-column tiles.
+  // Tile width: each CTA's operand delivery (about 17 cycles per KB of A + B tile per K block)
+  // bounds these kernels, so pick the width that minimises waves x bytes per K block:
+  // narrow tiles spread a small projection over more SMs, wide ones halve the A re-reads.
   const int m_tiles = (M + kBM - 1) / kBM;
-  const bool wide = (N % 256 == 0) && m_tiles * (N / 256) >= num_sms;
-  return wide ? dispatch_epi<256>(ta, tb, M, N, K, epi, e, num_sms, dev_err, s)
-              : dispatch_epi<128>(ta, tb, M, N, K, epi, e, num_sms, dev_err, s);
+  auto cost = [&](int bn) {
+    const long tiles = static_cast<long>(m_tiles) * (N / bn);
+    return ((tiles + num_sms - 1) / num_sms) * (16 + bn / 8);
+  };
+  int bn = 128;
+  if (N % 256 == 0 && cost(256) <= cost(bn)) bn = 256;
+  if (tb64 != nullptr && cost(64) < cost(bn)) bn = 64;
+  if (bn == 64) return dispatch_epi<64>(ta, *tb64, M, N, K, epi, e, num_sms, dev_err, s);
+  if (bn == 256) return dispatch_epi<256>(ta, tb, M, N, K, epi, e, num_sms, dev_err, s);
+  return dispatch_epi<128>(ta, tb, M, N, K, epi, e, num_sms, dev_err, s);
 }
 
 }  // namespace wam

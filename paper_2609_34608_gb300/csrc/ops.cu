@@ -68,11 +68,11 @@ int wam_op_gemm_bf16(const void* A, const void* Wt, const float* bias, void* C, 
   cudaError_t e = cudaGetDevice(&dev);
   if (e == cudaSuccess) e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
   if (e != cudaSuccess) return op_cuda("device query", e);
-  CUtensorMap ta, tb;
+  CUtensorMap ta, tb, tb64;
   if (tc_encode_kmajor_bf16(&ta, A, static_cast<uint64_t>(M > 0 ? M : 1), K) != 0 ||
-      tc_encode_kmajor_bf16(&tb, Wt, N, K) != 0)
+      tc_encode_kmajor_bf16(&tb, Wt, N, K) != 0 || tc_encode_kmajor_bf16_box64(&tb64, Wt, N, K) != 0)
     return op_fail(WAM_ERR_CUDA, "cuTensorMapEncodeTiled failed");
-  e = tc_gemm(ta, tb, M, N, K, epilogue, make_epi(bias, C, gate, gate_stride, rows_per_item), sms, nullptr,
+  e = tc_gemm(ta, tb, &tb64, M, N, K, epilogue, make_epi(bias, C, gate, gate_stride, rows_per_item), sms, nullptr,
               static_cast<cudaStream_t>(stream));
   return e == cudaSuccess ? WAM_OK : op_cuda("tcgen05 GEMM launch", e);
 }
@@ -141,7 +141,7 @@ int wam_op_gemm_qkv_vt(const void* A, const void* Wt, const float* bias, void* q
   EpiArgs ep = make_epi(bias, qkv, nullptr, 0, rows_per_item);
   ep.vt = static_cast<bf16*>(vt);
   ep.vt_ld = vt_ld;
-  e = tc_gemm(ta, tb, M, N, K, kEpiQkvVt, ep, sms, nullptr, static_cast<cudaStream_t>(stream));
+  e = tc_gemm(ta, tb, nullptr, M, N, K, kEpiQkvVt, ep, sms, nullptr, static_cast<cudaStream_t>(stream));
   return e == cudaSuccess ? WAM_OK : op_cuda("tcgen05 QKV GEMM launch", e);
 }
 

@@ -36,6 +36,7 @@ struct LayerW {
   float* up_b = nullptr;
   float* down_b = nullptr;
   CUtensorMap tm_qkv, tm_out, tm_up, tm_down;
+  CUtensorMap tm_out64, tm_down64;  // 64-row boxes for 64-column output tiles
 };
 
 struct ProfSpan {
@@ -245,12 +246,12 @@ int sync_check(wam_ctx* c) {
 
 // ---------------------------------------------------------------------------------- GEMM
 int gemm(wam_ctx* c, const CUtensorMap* ta, const void* A, const CUtensorMap* tb, const void* Wt,
-         int M, int N, int K, int epi, const EpiArgs& e) {
+         int M, int N, int K, int epi, const EpiArgs& e, const CUtensorMap* tb64 = nullptr) {
   const double out_b = (epi == kEpiResidF32) ? 8.0 : (epi == kEpiF32 ? 4.0 : (c->bf16 ? 2.0 : 4.0));
   const double in_b = c->bf16 ? 2.0 : 4.0;
   Span sp(c, WAM_KCLASS_GEMM, 2.0 * M * N * K, in_b * (double(M) * K + double(N) * K) + out_b * double(M) * N);
   if (c->bf16) {
-    CK(tc_gemm(*ta, *tb, M, N, K, epi, e, c->num_sms, c->d_err, c->stream));
+    CK(tc_gemm(*ta, *tb, tb64, M, N, K, epi, e, c->num_sms, c->d_err, c->stream));
   } else {
     CK(simt_gemm(static_cast<const float*>(A), static_cast<const float*>(Wt), M, N, K, epi, e, c->stream));
   }
@@ -302,12 +303,12 @@ int run_layer(wam_ctx* c, int l, float* hb, int Bw, const int* map, float* hcopy
       CK(attention_f32(static_cast<const float*>(c->qkv), static_cast<float*>(c->att), Bw, c->N, d, c->H, c->stream));
   }
   TRY(gemm(c, &c->tm_att, c->att, &w.tm_out, w.out_wt, M, d, d, kEpiResidF32,
-           epi_args(w.out_b, hb, c->mods + base + 2 * d, c->mod_n, c->N, map)));
+           epi_args(w.out_b, hb, c->mods + base + 2 * d, c->mod_n, c->N, map), &w.tm_out64));
   TRY(ln_mod(c, hb, nullptr, base + 3 * d, base + 4 * d, map, M));
   TRY(gemm(c, &c->tm_xln, c->xln, &w.tm_up, w.up_wt, M, c->dff, d, kEpiGeluBf16,
            epi_args(w.up_b, c->u, nullptr, 0, c->N, nullptr)));
   TRY(gemm(c, &c->tm_u, c->u, &w.tm_down, w.down_wt, M, d, c->dff, kEpiResidF32,
-           epi_args(w.down_b, hb, c->mods + base + 5 * d, c->mod_n, c->N, map)));
+           epi_args(w.down_b, hb, c->mods + base + 5 * d, c->mod_n, c->N, map), &w.tm_down64));
   return WAM_OK;
 }
 
@@ -752,6 +753,9 @@ int create_impl(wam_ctx* c, const wam_config* cfg, const float* weights, size_t 
       TRY(encode(c, &w.tm_out, w.out_wt, c->d, c->d));
       TRY(encode(c, &w.tm_up, w.up_wt, c->dff, c->d));
       TRY(encode(c, &w.tm_down, w.down_wt, c->d, c->dff));
+      if (tc_encode_kmajor_bf16_box64(&w.tm_out64, w.out_wt, c->d, c->d) != 0 ||
+          tc_encode_kmajor_bf16_box64(&w.tm_down64, w.down_wt, c->d, c->dff) != 0)
+        return fail(c, WAM_ERR_CUDA, "cuTensorMapEncodeTiled failed for 64-row weight boxes");
     }
   }
   CK(cudaHostAlloc(reinterpret_cast<void**>(&c->ring), kRingSlots * kSlotBytes, cudaHostAllocDefault));
