@@ -2,13 +2,17 @@
 //
 // One CTA owns 128 queries of one (item, head); TMEM lane r is query r.  Per block of 128 keys:
 //   S = Q K^T    tcgen05.mma M=128 N=128 K=64 into one of two TMEM S buffers (cols 0 / 128)
-//   softmax      warps 4-7, one thread per query row: tcgen05.ld of the S row, online max /
-//                sum in the log2 domain, rescale of the O row in TMEM when the max grew,
-//                P (bf16) written to shared memory in the 128-byte-swizzled K-major layout
+//   softmax      warps 4-11, two threads per query row (64 keys each): tcgen05.ld of the S
+//                half-row, online max / sum in the log2 domain (the pair exchanges its max
+//                through shared memory), P (bf16) written to one of two shared-memory buffers in
+//                the 128-byte-swizzled K-major layout.  O in TMEM is rescaled only when a row's
+//                running max grows by more than 2^8 (otherwise the stale max keeps every P <= 256),
+//                so the softmax rarely waits for the previous block's P.V
 //   O += P V     tcgen05.mma M=128 N=64 K=128 with P from shared memory and V^T (written by the
 //                QKV projection's epilogue) as the K-major B operand; O in TMEM cols 256..319
-// Warp 0 streams Q once and K / V^T tiles through a two-stage TMA ring; warp 1 issues the MMAs,
-// computing S of block j+1 while the softmax works on block j.  Every wait is bounded.
+// Warp 0 streams Q once and K / V^T tiles through four-stage TMA rings (a K tile is released as
+// soon as its S is computed, a V^T tile after its P.V); warp 1 issues the MMAs, computing S of
+// block j+1 while the softmax works on block j.  Every wait is bounded.
 #include "common.cuh"
 #include "tcgen05.cuh"
 
@@ -18,17 +22,20 @@ namespace {
 constexpr int kQ = 128;
 constexpr int kKV = 128;
 constexpr int kDH = 64;
-constexpr int kThreadsAttn = 256;
+constexpr int kThreadsAttn = 384;
+constexpr float kRescaleLog2 = 8.0f;  // lazy-rescale threshold (log2 units)
 constexpr int kQBytes = kQ * kDH * 2;    // 16 KB
 constexpr int kKBytes = kKV * kDH * 2;   // 16 KB
 constexpr int kVBytes = kDH * kKV * 2;   // 16 KB: two 8 KB atom columns (64 keys each)
 constexpr int kPBytes = kQ * kKV * 2;    // 32 KB: two 16 KB atom columns (64 keys each)
 constexpr int kOffQ = 0;
+constexpr int kKVStages = 4;
 constexpr int kOffK = kOffQ + kQBytes;
-constexpr int kOffV = kOffK + 2 * kKBytes;
-constexpr int kOffP = kOffV + 2 * kVBytes;
-constexpr int kOffBar = kOffP + kPBytes;
-constexpr int kSmemAttn = kOffBar + 256 + 1024;
+constexpr int kOffV = kOffK + kKVStages * kKBytes;
+constexpr int kOffP = kOffV + kKVStages * kVBytes;   // two P buffers
+constexpr int kOffX = kOffP + 2 * kPBytes;   // max / sum exchange [2][2][128] floats
+constexpr int kOffBar = kOffX + 2048;
+constexpr int kSmemAttn = kOffBar + 512 + 1024;  // barriers, TMEM slot, abort flag; alignment slack
 constexpr uint32_t kTmemCols = 512;
 constexpr uint32_t kColO = 256;
 
@@ -45,14 +52,18 @@ __global__ void __launch_bounds__(kThreadsAttn, 1)
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint64_t* bars = reinterpret_cast<uint64_t*>(smem + kOffBar);
   uint64_t* q_full = bars + 0;
-  uint64_t* kv_full = bars + 1;   // [2]
-  uint64_t* kv_empty = bars + 3;  // [2]
-  uint64_t* s_full = bars + 5;    // [2]
-  uint64_t* s_empty = bars + 7;   // [2]
-  uint64_t* p_full = bars + 9;
-  uint64_t* o_done = bars + 10;
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 11);
+  uint64_t* k_full = bars + 1;    // [4]
+  uint64_t* k_empty = bars + 5;   // [4]
+  uint64_t* v_full = bars + 9;    // [4]
+  uint64_t* v_empty = bars + 13;  // [4]
+  uint64_t* s_full = bars + 17;   // [2]
+  uint64_t* s_empty = bars + 19;  // [2]
+  uint64_t* p_full = bars + 21;   // [2]
+  uint64_t* pv_done = bars + 23;  // [2]: P.V of the block that used P buffer i finished
+  uint64_t* xpair = bars + 25;    // [4 quarters][2]: the two threads of a row exchanged values
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 33);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+  float* xch = reinterpret_cast<float*>(smem + kOffX);  // [2 buffers][2 halves][128 rows]
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
@@ -64,14 +75,19 @@ __global__ void __launch_bounds__(kThreadsAttn, 1)
 
   if (threadIdx.x == 0) {
     mbar_init(smem_u32(q_full), 1);
-    for (int i = 0; i < 2; ++i) {
-      mbar_init(smem_u32(&kv_full[i]), 1);
-      mbar_init(smem_u32(&kv_empty[i]), 1);
-      mbar_init(smem_u32(&s_full[i]), 1);
-      mbar_init(smem_u32(&s_empty[i]), 128);
+    for (int i = 0; i < kKVStages; ++i) {
+      mbar_init(smem_u32(&k_full[i]), 1);
+      mbar_init(smem_u32(&k_empty[i]), 1);
+      mbar_init(smem_u32(&v_full[i]), 1);
+      mbar_init(smem_u32(&v_empty[i]), 1);
     }
-    mbar_init(smem_u32(p_full), 128);
-    mbar_init(smem_u32(o_done), 1);
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(smem_u32(&s_full[i]), 1);
+      mbar_init(smem_u32(&s_empty[i]), 256);
+      mbar_init(smem_u32(&p_full[i]), 256);
+      mbar_init(smem_u32(&pv_done[i]), 1);
+    }
+    for (int i = 0; i < 8; ++i) mbar_init(smem_u32(&xpair[i]), 64);
     *abort_flag = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
@@ -92,13 +108,17 @@ __global__ void __launch_bounds__(kThreadsAttn, 1)
     tma_load_2d(smem_u32(smem + kOffQ), &tmQK, h * kDH, row_base + q0, smem_u32(q_full));
     const int vt_row = (b * H + h) * kDH;
     for (int j = 0; j < nkv; ++j) {
-      const int s = j & 1;
-      if (!mbar_wait(smem_u32(&kv_empty[s]), ((j >> 1) & 1) ^ 1u, abort_flag, dev_err)) break;
-      const uint32_t fb = smem_u32(&kv_full[s]);
-      mbar_expect_tx(fb, kKBytes + kVBytes);
-      tma_load_2d(smem_u32(smem + kOffK + s * kKBytes), &tmQK, d + h * kDH, row_base + j * kKV, fb);
-      tma_load_2d(smem_u32(smem + kOffV + s * kVBytes), &tmVt, j * kKV, vt_row, fb);
-      tma_load_2d(smem_u32(smem + kOffV + s * kVBytes + kVBytes / 2), &tmVt, j * kKV + 64, vt_row, fb);
+      const int s = j % kKVStages;
+      const uint32_t par = ((j / kKVStages) & 1) ^ 1u;
+      if (!mbar_wait(smem_u32(&k_empty[s]), par, abort_flag, dev_err)) break;
+      const uint32_t kb = smem_u32(&k_full[s]);
+      mbar_expect_tx(kb, kKBytes);
+      tma_load_2d(smem_u32(smem + kOffK + s * kKBytes), &tmQK, d + h * kDH, row_base + j * kKV, kb);
+      if (!mbar_wait(smem_u32(&v_empty[s]), par, abort_flag, dev_err)) break;
+      const uint32_t vb = smem_u32(&v_full[s]);
+      mbar_expect_tx(vb, kVBytes);
+      tma_load_2d(smem_u32(smem + kOffV + s * kVBytes), &tmVt, j * kKV, vt_row, vb);
+      tma_load_2d(smem_u32(smem + kOffV + s * kVBytes + kVBytes / 2), &tmVt, j * kKV + 64, vt_row, vb);
     }
   } else if (warp == 1 && lane == 0) {
     // ---------------- MMA issue ----------------
@@ -106,40 +126,57 @@ __global__ void __launch_bounds__(kThreadsAttn, 1)
     const uint32_t idO = idesc_bf16(kQ, kDH);
     bool ok = mbar_wait(smem_u32(q_full), 0, abort_flag, dev_err);
     const uint32_t sq = smem_u32(smem + kOffQ);
-    const uint32_t sp = smem_u32(smem + kOffP);
     for (int j = 0; ok && j <= nkv; ++j) {
       if (j < nkv) {
         const int s = j & 1;
-        if (!mbar_wait(smem_u32(&kv_full[s]), (j >> 1) & 1, abort_flag, dev_err)) break;
+        const int ks = j % kKVStages;
+        if (!mbar_wait(smem_u32(&k_full[ks]), (j / kKVStages) & 1, abort_flag, dev_err)) break;
         if (!mbar_wait(smem_u32(&s_empty[s]), ((j >> 1) & 1) ^ 1u, abort_flag, dev_err)) break;
         tc_fence_after();
-        const uint32_t sk = smem_u32(smem + kOffK + s * kKBytes);
+        const uint32_t sk = smem_u32(smem + kOffK + ks * kKBytes);
 #pragma unroll
         for (int t = 0; t < kDH / 16; ++t)
           umma_bf16(tmem + s * kKV, sw128_desc(sq + t * 32), sw128_desc(sk + t * 32), idS, t > 0 ? 1u : 0u);
         umma_commit(smem_u32(&s_full[s]));
+        umma_commit(smem_u32(&k_empty[ks]));
       }
       if (j >= 1) {
         const int jj = j - 1;
-        if (!mbar_wait(smem_u32(p_full), jj & 1, abort_flag, dev_err)) break;
+        const int pb = jj & 1;
+        const int vs = jj % kKVStages;
+        if (!mbar_wait(smem_u32(&v_full[vs]), (jj / kKVStages) & 1, abort_flag, dev_err)) break;
+        if (!mbar_wait(smem_u32(&p_full[pb]), (jj >> 1) & 1, abort_flag, dev_err)) break;
         tc_fence_after();
-        const uint32_t sv = smem_u32(smem + kOffV + (jj & 1) * kVBytes);
+        const uint32_t sp = smem_u32(smem + kOffP + pb * kPBytes);
+        const uint32_t sv = smem_u32(smem + kOffV + vs * kVBytes);
 #pragma unroll
         for (int t = 0; t < kKV / 16; ++t) {
           const uint32_t a = sp + (t >> 2) * (kPBytes / 2) + (t & 3) * 32;
           const uint32_t bb = sv + (t >> 2) * (kVBytes / 2) + (t & 3) * 32;
           umma_bf16(tmem + kColO, sw128_desc(a), sw128_desc(bb), idO, (jj > 0 || t > 0) ? 1u : 0u);
         }
-        umma_commit(smem_u32(o_done));
-        umma_commit(smem_u32(&kv_empty[jj & 1]));
+        umma_commit(smem_u32(&pv_done[pb]));
+        umma_commit(smem_u32(&v_empty[vs]));
       }
     }
   } else if (warp >= 4) {
-    // ---------------- softmax: one query row per thread ----------------
+    // ---------------- softmax: two threads per query row ----------------
     const int quarter = warp & 3;
+    const int half = (warp - 4) >> 2;         // keys [64 half, 64 half + 64), O cols [32 half, +32)
     const int r = quarter * 32 + lane;
     const uint32_t lane_addr = tmem + (static_cast<uint32_t>(quarter * 32) << 16);
-    uint8_t* prow = smem + kOffP + r * 128;
+    // Exchange with the partner thread of the same row (the other warp of this quarter) through
+    // a double-buffered slot guarded by an mbarrier of the 64 threads of the two warps; use u
+    // of the exchange goes to buffer u & 1 and completes phase u >> 1 of its barrier.
+    auto exchange = [&](int u, float v, float& partner) -> bool {
+      float* slot = xch + (u & 1) * 2 * kQ;
+      slot[half * kQ + r] = v;
+      const uint32_t bar = smem_u32(&xpair[quarter * 2 + (u & 1)]);
+      mbar_arrive(bar);
+      if (!mbar_wait(bar, (u >> 1) & 1, abort_flag, dev_err)) return false;
+      partner = slot[(half ^ 1) * kQ + r];
+      return true;
+    };
     float m = -1e30f, l = 0.0f;
     bool ok = true;
     for (int j = 0; j < nkv; ++j) {
@@ -149,78 +186,94 @@ __global__ void __launch_bounds__(kThreadsAttn, 1)
         break;
       }
       tc_fence_after();
-      float p[kKV];
+      float p[64];
 #pragma unroll
-      for (int c = 0; c < kKV / 32; ++c) {
+      for (int c = 0; c < 2; ++c) {
         uint32_t v[32];
-        tmem_ld32(lane_addr + s * kKV + c * 32, v);
+        tmem_ld32(lane_addr + s * kKV + half * 64 + c * 32, v);
 #pragma unroll
         for (int i = 0; i < 32; ++i) p[c * 32 + i] = __uint_as_float(v[i]);
       }
       tc_fence_before();
       mbar_arrive(smem_u32(&s_empty[s]));
-      const int kv0 = j * kKV;
-      if (kv0 + kKV > N) {
+      const int kv0 = j * kKV + half * 64;
+      if (kv0 + 64 > N) {
 #pragma unroll
-        for (int i = 0; i < kKV; ++i)
+        for (int i = 0; i < 64; ++i)
           if (kv0 + i >= N) p[i] = -1e30f;
       }
-      float mx = p[0];
+      float mx8[8];
 #pragma unroll
-      for (int i = 1; i < kKV; ++i) mx = fmaxf(mx, p[i]);
-      const float m_new = fmaxf(m, mx * scale_log2);
-      float rs = 0.0f;
+      for (int k = 0; k < 8; ++k) mx8[k] = p[k];
 #pragma unroll
-      for (int i = 0; i < kKV; ++i) {
-        p[i] = ex2(fmaf(p[i], scale_log2, -m_new));
-        rs += p[i];
+      for (int i = 8; i < 64; ++i) mx8[i & 7] = fmaxf(mx8[i & 7], p[i]);
+      float mx = fmaxf(fmaxf(fmaxf(mx8[0], mx8[1]), fmaxf(mx8[2], mx8[3])),
+                       fmaxf(fmaxf(mx8[4], mx8[5]), fmaxf(mx8[6], mx8[7])));
+      float mx_partner;
+      if (!exchange(j, mx, mx_partner)) {
+        ok = false;
+        break;
       }
-      const float corr = ex2(m - m_new);
-      l = l * corr + rs;
-      m = m_new;
-      if (j > 0) {
-        // P.V of the previous block must be complete: O is then stable and P's buffer free.
-        if (!warp_wait(smem_u32(o_done), (j - 1) & 1, abort_flag, dev_err)) {
+      mx = fmaxf(mx, mx_partner);
+      const float cand = mx * scale_log2;
+      // Lazy rescale: keep the stale max unless the new one exceeds it by more than 2^8.
+      const bool grow = j == 0 || cand > m + kRescaleLog2;
+      const float m_use = grow ? fmaxf(m, cand) : m;
+      const float corr = grow ? ex2(m - m_use) : 1.0f;
+      float rs8[8];
+#pragma unroll
+      for (int k = 0; k < 8; ++k) rs8[k] = 0.0f;
+#pragma unroll
+      for (int i = 0; i < 64; ++i) {
+        p[i] = ex2(fmaf(p[i], scale_log2, -m_use));
+        rs8[i & 7] += p[i];
+      }
+      l = l * corr + (((rs8[0] + rs8[1]) + (rs8[2] + rs8[3])) + ((rs8[4] + rs8[5]) + (rs8[6] + rs8[7])));
+      m = m_use;
+      if (j > 0 && __any_sync(0xffffffffu, corr != 1.0f)) {
+        // Rescale this thread's 32 O columns once every earlier P.V has landed.
+        if (!warp_wait(smem_u32(&pv_done[(j - 1) & 1]), ((j - 1) >> 1) & 1, abort_flag, dev_err)) {
           ok = false;
           break;
         }
         tc_fence_after();
-        if (__any_sync(0xffffffffu, corr != 1.0f)) {
+        uint32_t v[32];
+        tmem_ld32(lane_addr + kColO + half * 32, v);
 #pragma unroll
-          for (int c = 0; c < kDH / 32; ++c) {
-            uint32_t v[32];
-            tmem_ld32(lane_addr + kColO + c * 32, v);
-#pragma unroll
-            for (int i = 0; i < 32; ++i) v[i] = __float_as_uint(__uint_as_float(v[i]) * corr);
-            tmem_st32(lane_addr + kColO + c * 32, v);
-          }
-        }
+        for (int i = 0; i < 32; ++i) v[i] = __float_as_uint(__uint_as_float(v[i]) * corr);
+        tmem_st32(lane_addr + kColO + half * 32, v);
       }
-      // P row -> shared memory: 16 chunks of 8 bf16; chunk c of atom column c/8 lands at
-      // 16-byte slot (c%8) xor (r%8) of the row (128-byte swizzle).
+      // P buffer j&1 is free once the P.V of block j-2 finished.
+      const int pb = j & 1;
+      if (j >= 2 && !warp_wait(smem_u32(&pv_done[pb]), ((j - 2) >> 1) & 1, abort_flag, dev_err)) {
+        ok = false;
+        break;
+      }
+      // 8 chunks of 8 bf16 into atom column `half`; chunk c lands at slot c xor (r % 8).
+      uint8_t* prow = smem + kOffP + pb * kPBytes + half * (kPBytes / 2) + r * 128;
 #pragma unroll
-      for (int c = 0; c < kKV / 8; ++c) {
+      for (int c = 0; c < 8; ++c) {
         uint4 u;
         u.x = pack_bf16x2(p[8 * c + 0], p[8 * c + 1]);
         u.y = pack_bf16x2(p[8 * c + 2], p[8 * c + 3]);
         u.z = pack_bf16x2(p[8 * c + 4], p[8 * c + 5]);
         u.w = pack_bf16x2(p[8 * c + 6], p[8 * c + 7]);
-        *reinterpret_cast<uint4*>(prow + (c >> 3) * (kPBytes / 2) + (((c & 7) ^ (r & 7)) << 4)) = u;
+        *reinterpret_cast<uint4*>(prow + ((c ^ (r & 7)) << 4)) = u;
       }
       asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
       tc_fence_before();
-      mbar_arrive(smem_u32(p_full));
+      mbar_arrive(smem_u32(&p_full[pb]));
     }
-    if (ok && warp_wait(smem_u32(o_done), (nkv - 1) & 1, abort_flag, dev_err)) {
-      tc_fence_after();
-      const float inv = 1.0f / l;
-      const int q = q0 + r;
-      uint4* dst = reinterpret_cast<uint4*>(out + static_cast<int64_t>(row_base + q) * d + h * kDH);
-#pragma unroll
-      for (int c = 0; c < kDH / 32; ++c) {
+    float l_partner = 0.0f;
+    if (ok && exchange(nkv, l, l_partner)) {
+      const float inv = 1.0f / (l + l_partner);
+      if (warp_wait(smem_u32(&pv_done[(nkv - 1) & 1]), ((nkv - 1) >> 1) & 1, abort_flag, dev_err)) {
+        tc_fence_after();
+        const int q = q0 + r;
         uint32_t v[32];
-        tmem_ld32(lane_addr + kColO + c * 32, v);
+        tmem_ld32(lane_addr + kColO + half * 32, v);
         if (q < N) {
+          uint4* dst = reinterpret_cast<uint4*>(out + static_cast<int64_t>(row_base + q) * d + h * kDH + half * 32);
 #pragma unroll
           for (int k = 0; k < 4; ++k) {
             uint4 u;
@@ -228,7 +281,7 @@ __global__ void __launch_bounds__(kThreadsAttn, 1)
             u.y = pack_bf16x2(__uint_as_float(v[8 * k + 2]) * inv, __uint_as_float(v[8 * k + 3]) * inv);
             u.z = pack_bf16x2(__uint_as_float(v[8 * k + 4]) * inv, __uint_as_float(v[8 * k + 5]) * inv);
             u.w = pack_bf16x2(__uint_as_float(v[8 * k + 6]) * inv, __uint_as_float(v[8 * k + 7]) * inv);
-            dst[c * 4 + k] = u;
+            dst[k] = u;
           }
         }
       }
