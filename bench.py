@@ -312,6 +312,11 @@ def main_ours(args):
     prof = ctx.profile_read()
     ctx.profile_enable(False)
 
+    serving = None
+    if not args.no_serving:
+        ctx.close()
+        serving = run_serving(dev, stream)
+
     if rank != 0:
         return 0
     peaks = _peaks()
@@ -341,6 +346,10 @@ def main_ours(args):
                 "d2h_bytes_per_step": int(d2h), "wall_s": e2e_wall},
         "clocks": clk,
     }
+    if serving is not None:
+        for k in ("gemm", "attn"):
+            serving[k + "_frac"] = serving[k + "_tflops"] / peaks["bf16_sus"]
+        line["serving"] = serving
     if cpu_times:
         ct = cpu_times[-1]
         line["cpu_baseline"] = {"value": 1.0 / ct, "unit": "chunks/s", "cores": cpu_cores, "kind": "oracle",
@@ -350,6 +359,63 @@ def main_ours(args):
     return 0
 
 
+def run_serving(dev, stream, warm_batches=2, batches=3):
+    """Batched serving: 32 independent episodes per batch on the 24-block d1024 DiT (2464 tokens);
+    each batch mixes 16 fresh episodes (cold, 10 steps) and 16 warm continuations (TR shift 16,
+    2 of 10 steps), run as one state so every step batches the active episodes."""
+    import torch
+
+    from paper_2609_34608_gb300 import inputs as I
+    from paper_2609_34608_gb300 import wam as W
+
+    cfg = I.get_config("serving")
+    B, K = cfg["batch"], cfg["n_steps"]
+    flat = torch.from_numpy(I.flatten_weights(I.make_weights(cfg))).to(dev)
+    ctx = W.Context(cfg, flat, stream=stream.cuda_stream)
+    del flat
+    half = B // 2
+    entry = np.array([W.ENTRY_COLD] * half + [K - 2] * half, np.int32)
+    shift = np.array([0] * half + [16] * half, np.int32)
+    n_steps = np.array([K] * half + [2] * half, np.int32)
+    with torch.cuda.stream(stream):
+        obs = [torch.from_numpy(I.make_obs(cfg, B, seed=100 + i)).to(dev) for i in range(warm_batches + batches + 1)]
+        eps = [torch.from_numpy(I.make_fresh_eps(cfg, B, i)).to(dev) for i in range(warm_batches + batches + 1)]
+        act = torch.zeros((B, cfg["n_action"], cfg["action_dim"]), device=dev)
+        st = ctx.state(B)
+        ctx.sample_cold(st, obs[0], eps[0], K, act)
+
+    def batch(i):
+        ctx.adapt(st, obs[i], shift=shift, entry=entry, fresh_noise=eps[i])
+        ctx.continue_(st, n_steps, act)
+
+    with torch.cuda.stream(stream):
+        for i in range(warm_batches):
+            batch(1 + i)
+    torch.cuda.synchronize(dev)
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    with torch.cuda.stream(stream):
+        e0.record(stream)
+        for i in range(batches):
+            batch(1 + warm_batches + i)
+        e1.record(stream)
+    torch.cuda.synchronize(dev)
+    ms = e0.elapsed_time(e1) / batches
+    ctx.profile_enable(True)
+    with torch.cuda.stream(stream):
+        batch(1)
+    prof = ctx.profile_read()
+    ctx.close()
+    tf = lambda k: prof[k]["flops"] / (prof[k]["ms"] * 1e-3) / 1e12 if prof[k]["ms"] > 0 else 0.0
+    tot = sum(v["ms"] for v in prof.values())
+    return {
+        "workload": "24-block d1024 16-head bf16 DiT, 384 obs + 2048 video + 32x7 action tokens; batch of 32 "
+                    "episodes: 16 cold (10 steps) + 16 warm (TR shift 16, 2 of 10 steps) per batch",
+        "chunks_per_s": B / (ms * 1e-3), "ms_per_batch": ms, "batches": batches,
+        "gemm_tflops": tf("gemm"), "attn_tflops": tf("attn"),
+        "kernel_share": {k: (v["ms"] / tot if tot else 0.0) for k, v in prof.items()},
+    }
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -357,6 +423,7 @@ def main():
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-serving", action="store_true", help="skip the batched serving section")
     args = ap.parse_args()
     if args.warmup < 3:
         raise SystemExit("--warmup must be >= 3")

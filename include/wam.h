@@ -166,7 +166,8 @@ void wam_destroy(wam_ctx* ctx);
 const char* wam_last_error(const wam_ctx* ctx);
 int wam_set_stream(wam_ctx* ctx, void* stream);
 
-/* Per-episode replan / denoising / layer state for `batch` episodes (1..batch_max). */
+/* Per-episode replan / denoising / layer state for `batch` episodes (1..batch_max).
+ * A state belongs to its context: destroy every state before destroying the context. */
 int wam_state_create(wam_ctx* ctx, int32_t batch, wam_state** out);
 void wam_state_destroy(wam_state* st);
 

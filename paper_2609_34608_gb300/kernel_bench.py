@@ -1,0 +1,75 @@
+"""Single-kernel timing through the C ABI (include/wam_ops.h), for kernel tuning and ncu captures.
+
+    python -m paper_2609_34608_gb300.kernel_bench gemm M N K [--iters I]
+    python -m paper_2609_34608_gb300.kernel_bench attn B N H [--iters I] [--impl tc|mma]
+
+Each invocation builds the library if needed, warms up, then times `iters` back-to-back launches
+with CUDA events on the current stream and prints one JSON line (microseconds per launch and
+algorithmic TFLOP/s: 2MNK for the GEMM, 4 B N^2 d for attention).
+"""
+from __future__ import annotations
+
+import argparse
+import json
+
+import torch
+
+from . import _build
+from . import wam as W
+
+
+def _time(fn, iters: int) -> float:
+    for _ in range(3):
+        fn()
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record()
+    for _ in range(iters):
+        fn()
+    e1.record()
+    torch.cuda.synchronize()
+    return e0.elapsed_time(e1) * 1000.0 / iters
+
+
+def bench_gemm(M: int, N: int, K: int, iters: int) -> dict:
+    dev = torch.device("cuda")
+    A = torch.randn(M, K, device=dev).to(torch.bfloat16)
+    Wt = (torch.randn(N, K, device=dev) * 0.05).to(torch.bfloat16)
+    C = torch.empty(M, N, device=dev, dtype=torch.bfloat16)
+    b = torch.zeros(N, device=dev)
+    us = _time(lambda: W.op_gemm_bf16(A, Wt, b, C, M, N, K, W.EPI_BF16), iters)
+    return {"kernel": "gemm_tc", "M": M, "N": N, "K": K, "us": us, "tflops": 2.0 * M * N * K / us / 1e6}
+
+
+def bench_attn(B: int, N: int, H: int, iters: int, impl: str) -> dict:
+    dev = torch.device("cuda")
+    d = 64 * H
+    qkv = torch.randn(B * N, 3 * d, device=dev).to(torch.bfloat16)
+    out = torch.empty(B * N, d, device=dev, dtype=torch.bfloat16)
+    if impl == "tc":
+        vt_ld = (N + 7) // 8 * 8
+        vt = torch.randn(B * d, vt_ld, device=dev).to(torch.bfloat16)
+        fn = lambda: W.op_attention_tc(qkv, vt, out, B, N, d, H)
+    else:
+        fn = lambda: W.op_attention(qkv, out, B, N, d, H, "bf16")
+    us = _time(fn, iters)
+    return {"kernel": f"attention_{impl}", "B": B, "N": N, "H": H, "us": us,
+            "tflops": 4.0 * B * N * N * d / us / 1e6}
+
+
+def main() -> None:
+    ap = argparse.ArgumentParser()
+    ap.add_argument("kind", choices=["gemm", "attn"])
+    ap.add_argument("dims", type=int, nargs=3)
+    ap.add_argument("--iters", type=int, default=20)
+    ap.add_argument("--impl", choices=["tc", "mma"], default="tc")
+    a = ap.parse_args()
+    _build.build()
+    if a.kind == "gemm":
+        print(json.dumps(bench_gemm(*a.dims, a.iters)))
+    else:
+        print(json.dumps(bench_attn(*a.dims, a.iters, a.impl)))
+
+
+if __name__ == "__main__":
+    main()

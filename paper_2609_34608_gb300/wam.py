@@ -9,6 +9,7 @@ from __future__ import annotations
 import ctypes
 import os
 import re
+import weakref
 
 import numpy as np
 
@@ -190,6 +191,7 @@ class State:
         h = _vp()
         ctx._check(lib().wam_state_create(ctx.handle, batch, ctypes.byref(h)))
         self.handle = h
+        ctx._states.add(self)
 
     def close(self):
         if self.handle:
@@ -217,13 +219,17 @@ class Context:
         if code != WAM_OK:
             raise WamError(code, "wam_create failed (see stderr)")
         self.handle = h
+        self._states = weakref.WeakSet()
 
     def _check(self, code: int):
         if code != WAM_OK:
             raise WamError(code, lib().wam_last_error(self.handle).decode())
 
     def close(self):
+        """Destroy every live state of this context, then the context itself."""
         if getattr(self, "handle", None):
+            for st in list(getattr(self, "_states", ())):
+                st.close()
             lib().wam_destroy(self.handle)
             self.handle = _vp()
 
