@@ -143,7 +143,8 @@ def test_ln_modulate_matches_oracle(wamlib, prec, d):
     assert np.max(np.abs(_f64(out) - ref)) <= tol * np.max(np.abs(ref))
 
 
-TC_ATTN_CASES = [(1, 1, 2), (1, 56, 2), (2, 128, 2), (1, 129, 4), (1, 1296, 12), (2, 300, 2), (1, 2464, 4)]
+TC_ATTN_CASES = [(1, 1, 2), (1, 56, 2), (2, 128, 2), (1, 129, 4), (1, 1296, 12), (2, 300, 2), (1, 2464, 4),
+                 (2, 2464, 16), (8, 600, 8), (20, 130, 8)]
 
 
 @pytest.mark.parametrize("B,N,H", TC_ATTN_CASES)
