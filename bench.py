@@ -51,6 +51,23 @@ def _peaks():
     return dict(hbm=6800.0, bf16=1900.0, bf16_sus=1700.0, source="fallback")
 
 
+def _gemm_traffic():
+    """DRAM bytes per GEMM launch from the committed ncu summary, if the kernel source is
+    unchanged since those counters were taken (else None)."""
+    import hashlib
+    import re
+    summ = os.path.join(ROOT, "profiles", "gemm_tc_closed_loop.md")
+    src = os.path.join(ROOT, "paper_2609_34608_gb300", "csrc", "gemm_tc.cu")
+    try:
+        text = open(summ).read()
+        tb = int(re.search(r"traffic_bytes_per_launch: (\d+)", text).group(1))
+        sha = re.search(r"kernel_source_sha1_prefix: ([0-9a-f]+)", text).group(1)
+        cur = hashlib.sha1(open(src, "rb").read()).hexdigest()
+    except (OSError, AttributeError, ValueError):
+        return None
+    return tb if cur.startswith(sha) else None
+
+
 def _workload_config(cfg: dict) -> dict:
     return {
         "workload": "closed-loop control step (TR shift 8 + 1 anticipatory step + OR + 2 steps with RR) "
@@ -337,7 +354,8 @@ def main_ours(args):
                   "r_or": stats["n_bind"] / max(1, stats["n_start"]), "coverage": stats["n_bind"] / max(1, stats["n_noninitial"])},
         "roofline": {"bound": "tensor", "kernel": "tcgen05 GEMM (QKV / out / MLP projections)",
                      "achieved": gemm_tflops, "peak": peaks["bf16_sus"], "unit": "TFLOP/s",
-                     "frac": gemm_tflops / peaks["bf16_sus"], "traffic": None,
+                     "frac": gemm_tflops / peaks["bf16_sus"], "traffic": _gemm_traffic(),
+                     "algorithmic_bytes_per_launch": g["bytes"] / max(1, g["launches"]),
                      "peak_source": f"{peaks['source']} sustained bf16"},
         "kernel_share": {k: (v["ms"] / tot_prof if tot_prof else 0.0) for k, v in prof.items()},
         "kernel_ms_per_step": {k: v["ms"] / nprof for k, v in prof.items()},
