@@ -51,6 +51,29 @@ def _peaks():
     return dict(hbm=6800.0, bf16=1900.0, bf16_sus=1700.0, source="fallback")
 
 
+TENSOR_CLASSES = ("gemm", "attn")
+
+
+def kernel_table(prof: dict, units: int, peaks: dict) -> dict:
+    """Per kernel class: time per unit, share, and achieved rate against the measured peak
+    (TFLOP/s for the tensor-core classes, GB/s of algorithmic bytes for the HBM-bound ones)."""
+    tot = sum(v["ms"] for v in prof.values())
+    out = {}
+    for k, v in prof.items():
+        if v["launches"] == 0:
+            continue
+        row = {"ms_per_unit": v["ms"] / units, "share": v["ms"] / tot if tot else 0.0, "launches": v["launches"]}
+        if v["ms"] > 0:
+            if k in TENSOR_CLASSES:
+                row["tflops"] = v["flops"] / (v["ms"] * 1e-3) / 1e12
+                row["frac"] = row["tflops"] / peaks["bf16_sus"]
+            else:
+                row["gbs"] = v["bytes"] / (v["ms"] * 1e-3) / 1e9
+                row["frac"] = row["gbs"] / peaks["hbm"]
+        out[k] = row
+    return out
+
+
 def _gemm_traffic():
     """DRAM bytes per GEMM launch from the committed ncu summary, if the kernel source is
     unchanged since those counters were taken (else None)."""
@@ -329,17 +352,17 @@ def main_ours(args):
     prof = ctx.profile_read()
     ctx.profile_enable(False)
 
-    serving = None
+    serving = serving_rr = None
     if not args.no_serving:
         ctx.close()
-        serving = run_serving(dev, stream)
+        serving = run_serving(dev, stream, _peaks())
+        serving_rr = run_serving(dev, stream, _peaks(), relax_gate=True)
 
     if rank != 0:
         return 0
     peaks = _peaks()
     g = prof["gemm"]
     gemm_tflops = g["flops"] / (g["ms"] * 1e-3) / 1e12 if g["ms"] > 0 else 0.0
-    tot_prof = sum(v["ms"] for v in prof.values())
     value = args.steps * world / (total_ms * 1e-3)
     line = {
         "metric": METRIC, "value": value, "unit": "chunks/s", "n_gpus": world, "steps": args.steps,
@@ -357,17 +380,15 @@ def main_ours(args):
                      "frac": gemm_tflops / peaks["bf16_sus"], "traffic": _gemm_traffic(),
                      "algorithmic_bytes_per_launch": g["bytes"] / max(1, g["launches"]),
                      "peak_source": f"{peaks['source']} sustained bf16"},
-        "kernel_share": {k: (v["ms"] / tot_prof if tot_prof else 0.0) for k, v in prof.items()},
-        "kernel_ms_per_step": {k: v["ms"] / nprof for k, v in prof.items()},
+        "kernels": kernel_table(prof, nprof, peaks),
         "gpu_launches": int(stats["n_kernel_launches"]),
         "e2e": {"value": args.steps * world / (e2e_ms * 1e-3), "unit": "chunks/s", "h2d_bytes_per_step": int(h2d),
                 "d2h_bytes_per_step": int(d2h), "wall_s": e2e_wall},
         "clocks": clk,
     }
     if serving is not None:
-        for k in ("gemm", "attn"):
-            serving[k + "_frac"] = serving[k + "_tflops"] / peaks["bf16_sus"]
         line["serving"] = serving
+        line["serving_rr_accept"] = serving_rr
     if cpu_times:
         ct = cpu_times[-1]
         line["cpu_baseline"] = {"value": 1.0 / ct, "unit": "chunks/s", "cores": cpu_cores, "kind": "oracle",
@@ -377,16 +398,19 @@ def main_ours(args):
     return 0
 
 
-def run_serving(dev, stream, warm_batches=2, batches=3):
+def run_serving(dev, stream, peaks, warm_batches=2, batches=3, relax_gate=False):
     """Batched serving: 32 independent episodes per batch on the 24-block d1024 DiT (2464 tokens);
     each batch mixes 16 fresh episodes (cold, 10 steps) and 16 warm continuations (TR shift 16,
-    2 of 10 steps), run as one state so every step batches the active episodes."""
+    2 of 10 steps), run as one state so every step batches the active episodes.  With
+    `relax_gate` the RR thresholds let every check pass (the injection path and the layer skip
+    at scale; not the acceptance rate of any trained model)."""
     import torch
 
     from paper_2609_34608_gb300 import inputs as I
     from paper_2609_34608_gb300 import wam as W
 
-    cfg = I.get_config("serving")
+    over = dict(rr_gamma_cos=-1.0, rr_gamma_fit=1e30) if relax_gate else {}
+    cfg = I.get_config("serving", **over)
     B, K = cfg["batch"], cfg["n_steps"]
     flat = torch.from_numpy(I.flatten_weights(I.make_weights(cfg))).to(dev)
     ctx = W.Context(cfg, flat, stream=stream.cuda_stream)
@@ -418,20 +442,27 @@ def run_serving(dev, stream, warm_batches=2, batches=3):
         e1.record(stream)
     torch.cuda.synchronize(dev)
     ms = e0.elapsed_time(e1) / batches
+    ctx.reset_stats()
     ctx.profile_enable(True)
     with torch.cuda.stream(stream):
         batch(1)
     prof = ctx.profile_read()
+    stats = ctx.stats()
     ctx.close()
-    tf = lambda k: prof[k]["flops"] / (prof[k]["ms"] * 1e-3) / 1e12 if prof[k]["ms"] > 0 else 0.0
-    tot = sum(v["ms"] for v in prof.values())
-    return {
+    kt = kernel_table(prof, 1, peaks)
+    res = {
         "workload": "24-block d1024 16-head bf16 DiT, 384 obs + 2048 video + 32x7 action tokens; batch of 32 "
                     "episodes: 16 cold (10 steps) + 16 warm (TR shift 16, 2 of 10 steps) per batch",
         "chunks_per_s": B / (ms * 1e-3), "ms_per_batch": ms, "batches": batches,
-        "gemm_tflops": tf("gemm"), "attn_tflops": tf("attn"),
-        "kernel_share": {k: (v["ms"] / tot if tot else 0.0) for k, v in prof.items()},
+        "gemm_tflops": kt["gemm"]["tflops"], "attn_tflops": kt["attn"]["tflops"],
+        "gemm_frac": kt["gemm"]["frac"], "attn_frac": kt["attn"]["frac"],
+        "kernels_per_batch": kt,
+        "reuse": {"r_rr": stats["n_reuse"] / max(1, stats["n_attempt"]),
+                  "f_skip": stats["b_skip"] / max(1, stats["b_dense"])},
     }
+    if relax_gate:
+        res["workload"] += "; RR gate thresholds relaxed so every check passes"
+    return res
 
 
 def main():

@@ -237,12 +237,16 @@ int wam_state_write(wam_ctx* ctx, wam_state* st, int32_t field, int32_t index, c
 int wam_sync(wam_ctx* ctx);
 
 /* Kernel-class timing spans recorded with CUDA events on the context's stream. */
-#define WAM_KCLASS_GEMM 0
-#define WAM_KCLASS_ATTN 1
-#define WAM_KCLASS_NORM 2      /* LN-modulate, embed, final+Euler */
+#define WAM_KCLASS_GEMM 0      /* tcgen05 / SIMT projections */
+#define WAM_KCLASS_ATTN 1      /* attention */
+#define WAM_KCLASS_NORM 2      /* LN-modulate */
 #define WAM_KCLASS_COND 3      /* conditioning GEMVs */
-#define WAM_KCLASS_ADAPT 4     /* TR / OR / RR kernels */
-#define WAM_KCLASS_COUNT 5
+#define WAM_KCLASS_ADAPT 4     /* TR remap / OR score / bind (wam_adapt_state) */
+#define WAM_KCLASS_EMBED 5     /* token embedding, observation cast */
+#define WAM_KCLASS_FINAL 6     /* final layer + Euler update */
+#define WAM_KCLASS_RR_PROBE 7  /* RR probe reductions and gate */
+#define WAM_KCLASS_RR_APPLY 8  /* RR gather, injection / refresh */
+#define WAM_KCLASS_COUNT 9
 typedef struct wam_kclass_timing {
   int64_t launches;
   double ms;          /* summed event-measured duration */

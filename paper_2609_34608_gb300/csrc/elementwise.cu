@@ -257,62 +257,31 @@ __global__ void __launch_bounds__(256) ln_mod_kernel(const float* __restrict__ h
 }
 
 // ---------------------------------------------------------------- final layer + Euler
+// Modulated LN of a token row, the output head (16 columns; the zero-padded [d, 16] video and
+// action heads are staged once per block in shared memory, transposed to [16, d] so a lane's
+// float4 reads are consecutive across the warp), the Euler update of that token's trajectory
+// values and their retention.  Work unit: up to two consecutive token rows of the same head of
+// one item, processed by one warp so each weight element read from shared memory serves both.
 template <int NV4>
-__global__ void __launch_bounds__(256) final_euler_kernel(
-    const float* __restrict__ h, const StepItem* __restrict__ items,
-    const float* __restrict__ mods, int64_t mod_stride, int fin_off,
-    const float* __restrict__ vout_w, const float* __restrict__ vout_b,
-    const float* __restrict__ aout_w, const float* __restrict__ aout_b, float* __restrict__ x,
-    float* __restrict__ xhist, float* __restrict__ vhist, int64_t stage_stride, int T, int Bw,
-    int No, int Nv, int vd, int Na, int ad, int d) {
-  pdl_wait();
-  pdl_launch_dependents();
-  const int rows = Nv + Na;
-  const int64_t gw = static_cast<int64_t>(blockIdx.x) * kRowWarps + (threadIdx.x >> 5);
-  const int lane = threadIdx.x & 31;
-  if (gw >= static_cast<int64_t>(Bw) * rows) return;
-  const int w = static_cast<int>(gw / rows), r = static_cast<int>(gw % rows);
-  const StepItem it = items[w];
-  const int N = No + Nv + Na;
-  const float4* hr = reinterpret_cast<const float4*>(h + (static_cast<int64_t>(w) * N + No + r) * d);
-  float4 v[NV4];
+WAM_DEV void ln_mod_row(const float* __restrict__ hrow, const float* shift, const float* scale, int d,
+                        int lane, float4 (&y)[NV4]) {
+  const float4* hr = reinterpret_cast<const float4*>(hrow);
 #pragma unroll
-  for (int i = 0; i < NV4; ++i) v[i] = hr[lane + 32 * i];
+  for (int i = 0; i < NV4; ++i) y[i] = hr[lane + 32 * i];
   float mean, rstd;
-  row_stats<NV4>(v, d, mean, rstd);
-  const float* shift = mods + w * mod_stride + fin_off;
-  const float* scale = shift + d;
-  const bool video = r < Nv;
-  const int od = video ? vd : ad;
-  // Output heads are stored with rows padded to 16 floats: each of this lane's y values meets a
-  // 64-byte weight row (four float4 loads) and contributes to all 16 outputs.
-  const float4* Wo = reinterpret_cast<const float4*>(video ? vout_w : aout_w);
-  float acc[16];
-#pragma unroll
-  for (int j = 0; j < 16; ++j) acc[j] = 0.0f;
+  row_stats<NV4>(y, d, mean, rstd);
 #pragma unroll
   for (int i = 0; i < NV4; ++i) {
     const int c = (lane + 32 * i) * 4;
     const float4 sh = *reinterpret_cast<const float4*>(shift + c);
     const float4 sc = *reinterpret_cast<const float4*>(scale + c);
-    const float y[4] = {fmaf((v[i].x - mean) * rstd, 1.0f + sc.x, sh.x),
-                        fmaf((v[i].y - mean) * rstd, 1.0f + sc.y, sh.y),
-                        fmaf((v[i].z - mean) * rstd, 1.0f + sc.z, sh.z),
-                        fmaf((v[i].w - mean) * rstd, 1.0f + sc.w, sh.w)};
-#pragma unroll
-    for (int e = 0; e < 4; ++e) {
-#pragma unroll
-      for (int q = 0; q < 4; ++q) {
-        const float4 wv = __ldg(Wo + (c + e) * 4 + q);
-        acc[4 * q + 0] = fmaf(y[e], wv.x, acc[4 * q + 0]);
-        acc[4 * q + 1] = fmaf(y[e], wv.y, acc[4 * q + 1]);
-        acc[4 * q + 2] = fmaf(y[e], wv.z, acc[4 * q + 2]);
-        acc[4 * q + 3] = fmaf(y[e], wv.w, acc[4 * q + 3]);
-      }
-    }
+    y[i] = make_float4(fmaf((y[i].x - mean) * rstd, 1.0f + sc.x, sh.x), fmaf((y[i].y - mean) * rstd, 1.0f + sc.y, sh.y),
+                       fmaf((y[i].z - mean) * rstd, 1.0f + sc.z, sh.z), fmaf((y[i].w - mean) * rstd, 1.0f + sc.w, sh.w));
   }
-  // Reduce-scatter the 16 partial outputs over the warp: after the halving steps lane l holds
-  // output (l & 15) summed over its half-warp; the last exchange adds the other half.
+}
+
+// Reduce-scatter 16 partial outputs over the warp: lane l ends with output (l & 15).
+WAM_DEV float reduce_scatter16(float (&acc)[16], int lane) {
 #pragma unroll
   for (int sft = 8; sft >= 1; sft >>= 1) {
     const bool upper = (lane & sft) != 0;
@@ -323,17 +292,80 @@ __global__ void __launch_bounds__(256) final_euler_kernel(
       acc[j] = keep + __shfl_xor_sync(0xffffffffu, send, sft);
     }
   }
-  const float mine = acc[0] + __shfl_xor_sync(0xffffffffu, acc[0], 16);
-  if (lane < od) {
-    const float vel = mine + (video ? vout_b : aout_b)[lane];
-    const int64_t idx = static_cast<int64_t>(it.ep) * T +
-                        (video ? static_cast<int64_t>(r) * vd
-                               : static_cast<int64_t>(Nv) * vd + static_cast<int64_t>(r - Nv) * ad) +
-                        lane;
-    const float xn = static_cast<float>(static_cast<double>(x[idx]) + it.dsigma * static_cast<double>(vel));
-    x[idx] = xn;
-    xhist[static_cast<int64_t>(it.stage + 1) * stage_stride + idx] = xn;
-    vhist[static_cast<int64_t>(it.stage) * stage_stride + idx] = vel;
+  return acc[0] + __shfl_xor_sync(0xffffffffu, acc[0], 16);
+}
+
+template <int NV4>
+__global__ void __launch_bounds__(256) final_euler_kernel(
+    const float* __restrict__ h, const StepItem* __restrict__ items,
+    const float* __restrict__ mods, int64_t mod_stride, int fin_off,
+    const float* __restrict__ vout_w, const float* __restrict__ vout_b,
+    const float* __restrict__ aout_w, const float* __restrict__ aout_b, float* __restrict__ x,
+    float* __restrict__ xhist, float* __restrict__ vhist, int64_t stage_stride, int T, int Bw,
+    int No, int Nv, int vd, int Na, int ad, int d) {
+  extern __shared__ float swt[];  // [2 heads][16 outputs][d]
+  pdl_wait();
+  pdl_launch_dependents();
+  const int lane = threadIdx.x & 31;
+  // Coalesced float4 reads of the [d, 16] heads, transposed into shared memory.
+  for (int i = threadIdx.x; i < 2 * 4 * d; i += blockDim.x) {
+    const int head = i / (4 * d), k = i - head * 4 * d, c = k >> 2, q = k & 3;
+    const float4 w = reinterpret_cast<const float4*>(head == 0 ? vout_w : aout_w)[k];
+    float* dst = swt + head * 16 * d + (4 * q) * d + c;
+    dst[0] = w.x;
+    dst[d] = w.y;
+    dst[2 * d] = w.z;
+    dst[3 * d] = w.w;
+  }
+  __syncthreads();
+  const int N = No + Nv + Na;
+  const int gv = (Nv + 1) / 2, ga = (Na + 1) / 2, groups = gv + ga;
+  const int64_t total = static_cast<int64_t>(Bw) * groups;
+  for (int64_t g = static_cast<int64_t>(blockIdx.x) * kRowWarps + (threadIdx.x >> 5); g < total;
+       g += static_cast<int64_t>(gridDim.x) * kRowWarps) {
+    const int w = static_cast<int>(g / groups), gi = static_cast<int>(g % groups);
+    const bool video = gi < gv;
+    const int r0 = video ? 2 * gi : Nv + 2 * (gi - gv);  // row among the item's video + action rows
+    const int nrows = video ? min(2, Nv - 2 * gi) : min(2, Na - 2 * (gi - gv));
+    const StepItem it = items[w];
+    const float* shift = mods + w * mod_stride + fin_off;
+    const float* scale = shift + d;
+    float4 y0[NV4], y1[NV4];
+    ln_mod_row<NV4>(h + (static_cast<int64_t>(w) * N + No + r0) * d, shift, scale, d, lane, y0);
+    if (nrows == 2) ln_mod_row<NV4>(h + (static_cast<int64_t>(w) * N + No + r0 + 1) * d, shift, scale, d, lane, y1);
+    const float* Wt = swt + (video ? 0 : 16 * d);
+    float acc0[16], acc1[16];
+#pragma unroll
+    for (int j = 0; j < 16; ++j) acc0[j] = acc1[j] = 0.0f;
+#pragma unroll
+    for (int i = 0; i < NV4; ++i) {
+      const int c = (lane + 32 * i) * 4;
+#pragma unroll
+      for (int j = 0; j < 16; ++j) {
+        const float4 wv = *reinterpret_cast<const float4*>(Wt + j * d + c);
+        acc0[j] = fmaf(y0[i].x, wv.x, fmaf(y0[i].y, wv.y, fmaf(y0[i].z, wv.z, fmaf(y0[i].w, wv.w, acc0[j]))));
+        if (nrows == 2)
+          acc1[j] = fmaf(y1[i].x, wv.x, fmaf(y1[i].y, wv.y, fmaf(y1[i].z, wv.z, fmaf(y1[i].w, wv.w, acc1[j]))));
+      }
+    }
+    const float out0 = reduce_scatter16(acc0, lane);
+    const float out1 = reduce_scatter16(acc1, lane);
+    const int od = video ? vd : ad;
+    const float bias = lane < od ? (video ? vout_b : aout_b)[lane] : 0.0f;
+    for (int rr = 0; rr < nrows; ++rr) {
+      if (lane < od) {
+        const int r = r0 + rr;
+        const float vel = (rr == 0 ? out0 : out1) + bias;
+        const int64_t idx = static_cast<int64_t>(it.ep) * T +
+                            (video ? static_cast<int64_t>(r) * vd
+                                   : static_cast<int64_t>(Nv) * vd + static_cast<int64_t>(r - Nv) * ad) +
+                            lane;
+        const float xn = static_cast<float>(static_cast<double>(x[idx]) + it.dsigma * static_cast<double>(vel));
+        x[idx] = xn;
+        xhist[static_cast<int64_t>(it.stage + 1) * stage_stride + idx] = xn;
+        vhist[static_cast<int64_t>(it.stage) * stage_stride + idx] = vel;
+      }
+    }
   }
 }
 
@@ -582,6 +614,19 @@ __global__ void __launch_bounds__(256) rr_apply_kernel(float* __restrict__ h,
   }
 }
 
+// Copy the items that must run the middle layers into the compact middle-layer buffer.
+__global__ void __launch_bounds__(256) rr_gather_kernel(float* __restrict__ hm, const float* __restrict__ h,
+                                                        const int* __restrict__ map, int64_t item4) {
+  pdl_wait();
+  pdl_launch_dependents();
+  const int c = blockIdx.y;
+  const float4* src = reinterpret_cast<const float4*>(h) + static_cast<int64_t>(map[c]) * item4;
+  float4* dst = reinterpret_cast<float4*>(hm) + static_cast<int64_t>(c) * item4;
+  for (int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; i < item4;
+       i += static_cast<int64_t>(gridDim.x) * blockDim.x)
+    dst[i] = src[i];
+}
+
 // ---------------------------------------------------------------- preparation
 __global__ void cast_kernel(const float* __restrict__ in, bf16* __restrict__ out, int64_t n) {
   pdl_wait();
@@ -708,13 +753,33 @@ cudaError_t final_euler(const float* h, const StepItem* items, const float* mods
                         int Nv, int vd, int Na, int ad, int d, cudaStream_t s) {
   if (Bw <= 0) return cudaSuccess;
   if (d % 128 != 0 || vd > 16 || ad > 16) return cudaErrorInvalidValue;  // heads padded to 16
-  const unsigned grid = row_blocks(static_cast<int64_t>(Bw) * (Nv + Na));
+  // One block per SM (or fewer), each staging both output heads once; warps stride over the
+  // row pairs.
+  static int num_sms = 0;
+  if (num_sms == 0) {
+    int dev = 0;
+    cudaGetDevice(&dev);
+    cudaDeviceGetAttribute(&num_sms, cudaDevAttrMultiProcessorCount, dev);
+  }
+  const int64_t units = static_cast<int64_t>(Bw) * ((Nv + 1) / 2 + (Na + 1) / 2);
+  const int64_t want = (units + kRowWarps - 1) / kRowWarps;
+  const unsigned grid = static_cast<unsigned>(want < 2 * num_sms ? want : 2 * num_sms);
+  const size_t smem = static_cast<size_t>(2) * d * 16 * sizeof(float);
 #define WAM_FE_CASE(NV)                                                                       \
-  case NV:                                                                                    \
-    launch_pdl(final_euler_kernel<NV>, dim3(grid), dim3(256), 0, s, h, items, mods, mod_stride, fin_off, vout_w,  \
+  case NV: {                                                                                  \
+    static int smem_set = 0;                                                                  \
+    if (smem_set < static_cast<int>(smem)) {                                                  \
+      cudaError_t e = cudaFuncSetAttribute(final_euler_kernel<NV>,                           \
+                                           cudaFuncAttributeMaxDynamicSharedMemorySize,       \
+                                           static_cast<int>(smem));                           \
+      if (e != cudaSuccess) return e;                                                         \
+      smem_set = static_cast<int>(smem);                                                      \
+    }                                                                                         \
+    launch_pdl(final_euler_kernel<NV>, dim3(grid), dim3(256), smem, s, h, items, mods, mod_stride, fin_off, vout_w,  \
                                                 vout_b, aout_w, aout_b, x, xhist, vhist,      \
                                                 stage_stride, T, Bw, No, Nv, vd, Na, ad, d); \
-    break;
+    break;                                                                                    \
+  }
   switch (d / 128) {
     WAM_NV4_CASES(WAM_FE_CASE)
     default: return cudaErrorInvalidValue;
@@ -793,6 +858,14 @@ cudaError_t rr_apply(float* h, const float* hm, const float* hq, float* pa, floa
   const int bx = static_cast<int>((n4 + 255) / 256 < 1024 ? (n4 + 255) / 256 : 1024);
   dim3 grid(bx, Bw);
   launch_pdl(rr_apply_kernel, dim3(grid), dim3(256), 0, s, h, hm, hq, pa, ra, items, ap, N, d, split_row);
+  return cudaGetLastError();
+}
+
+cudaError_t rr_gather(float* hm, const float* h, const int* map, int nmid, int64_t item_elems, cudaStream_t s) {
+  if (nmid <= 0) return cudaSuccess;
+  const int64_t item4 = item_elems / 4;
+  const int bx = static_cast<int>((item4 + 255) / 256 < 512 ? (item4 + 255) / 256 : 512);
+  launch_pdl(rr_gather_kernel, dim3(bx, nmid), dim3(256), 0, s, hm, h, map, item4);
   return cudaGetLastError();
 }
 

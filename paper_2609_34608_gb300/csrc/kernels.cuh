@@ -98,6 +98,8 @@ cudaError_t rr_probe_partial(const float* h, const float* hq, const float* pa,
 cudaError_t rr_gate(const double* partial, int Bw, int nch, int64_t n0, int64_t n1, double amin,
                     double amax, double eps, double gcos, double gfit, RRGate* out,
                     cudaStream_t s);
+// hm[c] = h[map[c]] for the nmid items that run the middle layers (rows of N*d floats)
+cudaError_t rr_gather(float* hm, const float* h, const int* map, int nmid, int64_t item_elems, cudaStream_t s);
 cudaError_t rr_apply(float* h, const float* hm, const float* hq, float* pa, float* ra,
                      const StepItem* items, const RRApply* ap, int Bw, int N, int d,
                      int split_row, cudaStream_t s);

@@ -316,7 +316,7 @@ int obs_embed(wam_ctx* c, wam_state* st) {
   const int M = st->B * c->No;
   if (c->bf16) {
     {
-      Span sp(c, WAM_KCLASS_NORM, 0.0, 6.0 * M * c->d);
+      Span sp(c, WAM_KCLASS_EMBED, 0.0, 6.0 * M * c->d);
       CK(cast_f32_bf16(st->obs, static_cast<bf16*>(c->obs_lp), int64_t(M) * c->d, c->stream));
     }
     TRY(gemm(c, &c->tm_obs_lp, c->obs_lp, &c->tm_obs_w, c->obs_wt, M, c->d, c->d, kEpiF32,
@@ -383,7 +383,7 @@ int run_steps(wam_ctx* c, wam_state* st, const std::vector<int>& n) {
       CK(cond_gemv(g, c->stream));
     }
     {
-      Span sp(c, WAM_KCLASS_NORM, 0.0, 4.0 * Bw * double(N) * d * 2.0);
+      Span sp(c, WAM_KCLASS_EMBED, 0.0, 4.0 * Bw * double(N) * d * 2.0);
       CK(embed_tokens(c->h, st->xhist, stage_stride, c->d_items, st->x, c->T, st->obs_emb, c->vid_w, c->vid_b,
                       c->act_w, c->act_b, c->pos, Bw, c->No, c->Nv, c->vd, c->Na, c->ad, d, c->stream));
     }
@@ -413,11 +413,11 @@ int run_steps(wam_ctx* c, wam_state* st, const std::vector<int>& n) {
       if (any_gate) {
         const int nch = rr_num_chunks(int64_t(std::max(split_row, N - split_row)) * d);
         {
-          Span sp(c, WAM_KCLASS_ADAPT, 0.0, 12.0 * Bw * double(N) * d);
+          Span sp(c, WAM_KCLASS_RR_PROBE, 0.0, 12.0 * Bw * double(N) * d);
           CK(rr_probe_partial(c->h, c->hq, st->pa, c->d_items, Bw, N, d, split_row, nch, c->d_part, c->stream));
         }
         {
-          Span sp(c, WAM_KCLASS_ADAPT);
+          Span sp(c, WAM_KCLASS_RR_PROBE);
           CK(rr_gate(c->d_part, Bw, nch, int64_t(split_row) * d, int64_t(N - split_row) * d, c->cfg.rr_alpha_min,
                      c->cfg.rr_alpha_max, c->cfg.rr_eps, c->cfg.rr_gamma_cos, c->cfg.rr_gamma_fit, c->d_gate, c->stream));
         }
@@ -441,21 +441,26 @@ int run_steps(wam_ctx* c, wam_state* st, const std::vector<int>& n) {
       }
       const int nmid = static_cast<int>(midmap.size());
       if (nmid > 0) {
-        for (int j = 0; j < nmid; ++j)
-          CK(cudaMemcpyAsync(c->hm + int64_t(j) * N * d, c->h + int64_t(midmap[j]) * N * d,
-                             sizeof(float) * N * d, cudaMemcpyDeviceToDevice, c->stream));
         TRY(upload(c, c->d_map, midmap.data(), sizeof(int) * nmid));
+        {
+          Span sp(c, WAM_KCLASS_RR_APPLY, 0.0, 8.0 * nmid * double(N) * d);
+          CK(rr_gather(c->hm, c->h, c->d_map, nmid, int64_t(N) * d, c->stream));
+        }
         for (int l = s; l < e; ++l) TRY(run_layer(c, l, c->hm, nmid, c->d_map, nullptr));
       }
       TRY(upload(c, c->d_rrapply, ap.data(), sizeof(RRApply) * Bw));
       {
-        Span sp(c, WAM_KCLASS_ADAPT, 0.0, 16.0 * Bw * double(N) * d);
+        // algorithmic bytes per element: inject 12 (h, R_a in; h out), refresh 24 (h_s, h_e, h_q
+        // in; R_a, p_a, h out), copy-back 8
+        double per = 0.0;
+        for (int w = 0; w < Bw; ++w) per += ap[w].mode == kRRInject ? 12.0 : (ap[w].mode == kRRRefresh ? 24.0 : 8.0);
+        Span sp(c, WAM_KCLASS_RR_APPLY, 0.0, per * double(N) * d);
         CK(rr_apply(c->h, c->hm, c->hq, st->pa, st->ra, c->d_items, c->d_rrapply, Bw, N, d, split_row, c->stream));
       }
       for (int l = e; l < L; ++l) TRY(run_layer(c, l, c->h, Bw, nullptr, nullptr));
     }
     {
-      Span sp(c, WAM_KCLASS_NORM, 2.0 * Bw * double(c->Nv * c->vd + c->Na * c->ad) * d,
+      Span sp(c, WAM_KCLASS_FINAL, 2.0 * Bw * double(c->Nv * c->vd + c->Na * c->ad) * d,
               4.0 * Bw * double(c->Nv + c->Na) * d + 16.0 * Bw * c->T);
       CK(final_euler(c->h, c->d_items, c->mods, c->mod_n, 6 * L * d, c->vout_w, c->vout_b, c->aout_w, c->aout_b,
                      st->x, st->xhist, st->vhist, stage_stride, c->T, Bw, c->No, c->Nv, c->vd, c->Na, c->ad, d,

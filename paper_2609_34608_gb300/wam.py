@@ -24,7 +24,7 @@ ADAPT_TR_INIT, ADAPT_TR_INIT_NO_PREFIX, ADAPT_COLD_INIT = 1, 2, 3
 ADAPT_REBIND_ACCEPT, ADAPT_REBIND_RESTART, ADAPT_REFRESH = 4, 5, 6
 FIELD_X, FIELD_X_STAGE, FIELD_V_STEP, FIELD_X_INIT, FIELD_OBS, FIELD_RR_P, FIELD_RR_R, FIELD_META = range(8)
 EPI_BF16, EPI_GELU_BF16, EPI_RESID_F32, EPI_F32 = 0, 1, 2, 3
-KCLASSES = ["gemm", "attn", "norm", "cond", "adapt"]
+KCLASSES = ["gemm", "attn", "norm", "cond", "adapt", "embed", "final", "rr_probe", "rr_apply"]
 
 
 class WamError(RuntimeError):
