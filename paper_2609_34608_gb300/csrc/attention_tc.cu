@@ -2,14 +2,16 @@
 //
 // One CTA owns 128 queries of one (item, head); TMEM lane r is query r.  Per block of 128 keys:
 //   S = Q K^T    tcgen05.mma M=128 N=128 K=64 into one of two TMEM S buffers (cols 0 / 128)
-//   softmax      warps 4-11, two threads per query row (64 keys each): tcgen05.ld of the S
-//                half-row, online max / sum in the log2 domain (the pair exchanges its max
-//                through shared memory), P (bf16) written to one of two shared-memory buffers in
-//                the 128-byte-swizzled K-major layout.  O in TMEM is rescaled only when a row's
-//                running max grows by more than 2^8 (otherwise the stale max keeps every P <= 256),
-//                so the softmax rarely waits for the previous block's P.V
-//   O += P V     tcgen05.mma M=128 N=64 K=128 with P from shared memory and V^T (written by the
-//                QKV projection's epilogue) as the K-major B operand; O in TMEM cols 256..319
+//   softmax      warps 4-11, two threads per query row, each an independent online-softmax
+//                stream over its half (64 keys) of every block: tcgen05.ld of the S half-row,
+//                running max / sum in the log2 domain, P (bf16) written to one of two
+//                shared-memory buffers in the 128-byte-swizzled K-major layout.  Each half
+//                accumulates into its own O in TMEM, rescaled only when its running max grows by
+//                more than 2^8 (the stale max keeps every P <= 256); the two streams are merged
+//                once, at the end, so the halves never wait on each other per block
+//   O_h += P_h V_h  tcgen05.mma M=128 N=64 K=64 per half with P from shared memory and V^T
+//                (written by the QKV projection's epilogue) as the K-major B operand;
+//                O_0 in TMEM cols 256..319, O_1 in cols 320..383
 // Warp 0 streams Q once and K / V^T tiles through four-stage TMA rings (a K tile is released as
 // soon as its S is computed, a V^T tile after its P.V); warp 1 issues the MMAs, computing S of
 // block j+1 while the softmax works on block j.  Every wait is bounded.
@@ -37,7 +39,7 @@ constexpr int kOffX = kOffP + 2 * kPBytes;   // max / sum exchange [2][2][128] f
 constexpr int kOffBar = kOffX + 2048;
 constexpr int kSmemAttn = kOffBar + 512 + 1024;  // barriers, TMEM slot, abort flag; alignment slack
 constexpr uint32_t kTmemCols = 512;
-constexpr uint32_t kColO = 256;
+constexpr uint32_t kColO = 256;  // O_0 at 256..319, O_1 at 320..383
 
 WAM_DEV float ex2(float x) {
   float y;
@@ -151,9 +153,11 @@ __global__ void __launch_bounds__(kThreadsAttn, 1)
         const uint32_t sv = smem_u32(smem + kOffV + vs * kVBytes);
 #pragma unroll
         for (int t = 0; t < kKV / 16; ++t) {
+          // keys 16t..16t+15 belong to half t/4: its own O accumulator
           const uint32_t a = sp + (t >> 2) * (kPBytes / 2) + (t & 3) * 32;
           const uint32_t bb = sv + (t >> 2) * (kVBytes / 2) + (t & 3) * 32;
-          umma_bf16(tmem + kColO, sw128_desc(a), sw128_desc(bb), idO, (jj > 0 || t > 0) ? 1u : 0u);
+          umma_bf16(tmem + kColO + (t >> 2) * kDH, sw128_desc(a), sw128_desc(bb), idO,
+                    (jj > 0 || (t & 3) > 0) ? 1u : 0u);
         }
         umma_commit(smem_u32(&pv_done[pb]));
         umma_commit(smem_u32(&v_empty[vs]));
@@ -167,7 +171,8 @@ __global__ void __launch_bounds__(kThreadsAttn, 1)
     const uint32_t lane_addr = tmem + (static_cast<uint32_t>(quarter * 32) << 16);
     // Exchange with the partner thread of the same row (the other warp of this quarter) through
     // a double-buffered slot guarded by an mbarrier of the 64 threads of the two warps; use u
-    // of the exchange goes to buffer u & 1 and completes phase u >> 1 of its barrier.
+    // of the exchange goes to buffer u & 1 and completes phase u >> 1 of its barrier (used
+    // twice, to merge the two half streams at the end).
     auto exchange = [&](int u, float v, float& partner) -> bool {
       float* slot = xch + (u & 1) * 2 * kQ;
       slot[half * kQ + r] = v;
@@ -177,7 +182,9 @@ __global__ void __launch_bounds__(kThreadsAttn, 1)
       partner = slot[(half ^ 1) * kQ + r];
       return true;
     };
-    float m = -1e30f, l = 0.0f;
+    // The running max starts at a finite floor far above the mask value (-1e30 before scaling),
+    // so a half whose keys are all masked (N <= 64) keeps P = 0 and l = 0.
+    float m = -1e20f, l = 0.0f;
     bool ok = true;
     for (int j = 0; j < nkv; ++j) {
       const int s = j & 1;
@@ -207,14 +214,8 @@ __global__ void __launch_bounds__(kThreadsAttn, 1)
       for (int k = 0; k < 8; ++k) mx8[k] = p[k];
 #pragma unroll
       for (int i = 8; i < 64; ++i) mx8[i & 7] = fmaxf(mx8[i & 7], p[i]);
-      float mx = fmaxf(fmaxf(fmaxf(mx8[0], mx8[1]), fmaxf(mx8[2], mx8[3])),
-                       fmaxf(fmaxf(mx8[4], mx8[5]), fmaxf(mx8[6], mx8[7])));
-      float mx_partner;
-      if (!exchange(j, mx, mx_partner)) {
-        ok = false;
-        break;
-      }
-      mx = fmaxf(mx, mx_partner);
+      const float mx = fmaxf(fmaxf(fmaxf(mx8[0], mx8[1]), fmaxf(mx8[2], mx8[3])),
+                             fmaxf(fmaxf(mx8[4], mx8[5]), fmaxf(mx8[6], mx8[7])));
       const float cand = mx * scale_log2;
       // Lazy rescale: keep the stale max unless the new one exceeds it by more than 2^8.
       const bool grow = j == 0 || cand > m + kRescaleLog2;
@@ -237,11 +238,14 @@ __global__ void __launch_bounds__(kThreadsAttn, 1)
           break;
         }
         tc_fence_after();
-        uint32_t v[32];
-        tmem_ld32(lane_addr + kColO + half * 32, v);
 #pragma unroll
-        for (int i = 0; i < 32; ++i) v[i] = __float_as_uint(__uint_as_float(v[i]) * corr);
-        tmem_st32(lane_addr + kColO + half * 32, v);
+        for (int c = 0; c < kDH / 32; ++c) {
+          uint32_t v[32];
+          tmem_ld32(lane_addr + kColO + half * kDH + c * 32, v);
+#pragma unroll
+          for (int i = 0; i < 32; ++i) v[i] = __float_as_uint(__uint_as_float(v[i]) * corr);
+          tmem_st32(lane_addr + kColO + half * kDH + c * 32, v);
+        }
       }
       // P buffer j&1 is free once the P.V of block j-2 finished.
       const int pb = j & 1;
@@ -264,23 +268,33 @@ __global__ void __launch_bounds__(kThreadsAttn, 1)
       tc_fence_before();
       mbar_arrive(smem_u32(&p_full[pb]));
     }
-    float l_partner = 0.0f;
-    if (ok && exchange(nkv, l, l_partner)) {
-      const float inv = 1.0f / (l + l_partner);
+    // Merge the two half streams: O = sum_h O_h 2^(m_h - M), l = sum_h l_h 2^(m_h - M).
+    float m_partner = 0.0f, l_partner = 0.0f;
+    if (ok && exchange(0, m, m_partner) && exchange(1, l, l_partner)) {
+      const float M = fmaxf(m, m_partner);
+      const float f_own = ex2(m - M), f_par = ex2(m_partner - M);
+      const float inv = 1.0f / (l * f_own + l_partner * f_par);
+      const float w0 = (half == 0 ? f_own : f_par) * inv;   // weight of O_0
+      const float w1 = (half == 0 ? f_par : f_own) * inv;   // weight of O_1
       if (warp_wait(smem_u32(&pv_done[(nkv - 1) & 1]), ((nkv - 1) >> 1) & 1, abort_flag, dev_err)) {
         tc_fence_after();
         const int q = q0 + r;
-        uint32_t v[32];
-        tmem_ld32(lane_addr + kColO + half * 32, v);
+        uint32_t v0[32], v1[32];
+        tmem_ld32(lane_addr + kColO + half * 32, v0);        // O_0, this thread's 32 columns
+        tmem_ld32(lane_addr + kColO + kDH + half * 32, v1);  // O_1, same columns
         if (q < N) {
           uint4* dst = reinterpret_cast<uint4*>(out + static_cast<int64_t>(row_base + q) * d + h * kDH + half * 32);
 #pragma unroll
           for (int k = 0; k < 4; ++k) {
+            float o[8];
+#pragma unroll
+            for (int e = 0; e < 8; ++e)
+              o[e] = fmaf(__uint_as_float(v0[8 * k + e]), w0, __uint_as_float(v1[8 * k + e]) * w1);
             uint4 u;
-            u.x = pack_bf16x2(__uint_as_float(v[8 * k + 0]) * inv, __uint_as_float(v[8 * k + 1]) * inv);
-            u.y = pack_bf16x2(__uint_as_float(v[8 * k + 2]) * inv, __uint_as_float(v[8 * k + 3]) * inv);
-            u.z = pack_bf16x2(__uint_as_float(v[8 * k + 4]) * inv, __uint_as_float(v[8 * k + 5]) * inv);
-            u.w = pack_bf16x2(__uint_as_float(v[8 * k + 6]) * inv, __uint_as_float(v[8 * k + 7]) * inv);
+            u.x = pack_bf16x2(o[0], o[1]);
+            u.y = pack_bf16x2(o[2], o[3]);
+            u.z = pack_bf16x2(o[4], o[5]);
+            u.w = pack_bf16x2(o[6], o[7]);
             dst[k] = u;
           }
         }
