@@ -4,17 +4,22 @@
 //   S = Q K^T    tcgen05.mma M=128 N=128 K=64 into one of two TMEM S buffers (cols 0 / 128)
 //   softmax      warps 4-11, two threads per query row, each an independent online-softmax
 //                stream over its half (64 keys) of every block: tcgen05.ld of the S half-row,
-//                running max / sum in the log2 domain, P (bf16) written to one of two
-//                shared-memory buffers in the 128-byte-swizzled K-major layout.  Each half
+//                running max / sum in the log2 domain, P (bf16 pairs) stored with tcgen05.st
+//                into one of two TMEM P buffers (row r in lane r, keys 2c, 2c+1 in column c).
+//                Each half
 //                accumulates into its own O in TMEM, rescaled only when its running max grows by
 //                more than 2^8 (the stale max keeps every P <= 256); the two streams are merged
 //                once, at the end, so the halves never wait on each other per block
-//   O_h += P_h V_h  tcgen05.mma M=128 N=64 K=64 per half with P from shared memory and V^T
-//                (written by the QKV projection's epilogue) as the K-major B operand;
-//                O_0 in TMEM cols 256..319, O_1 in cols 320..383
-// Warp 0 streams Q once and K / V^T tiles through four-stage TMA rings (a K tile is released as
-// soon as its S is computed, a V^T tile after its P.V); warp 1 issues the MMAs, computing S of
-// block j+1 while the softmax works on block j.  Every wait is bounded.
+//   O_h += P_h V_h  tcgen05.mma M=128 N=64 K=64 per half with the A operand P read from TMEM
+//                and V^T (written by the QKV projection's epilogue) as the K-major B operand
+//                from shared memory; O_0 in TMEM cols 256..319, O_1 in cols 320..383, P buffers
+//                in cols 384..447 and 448..511.  Keeping P out of shared memory leaves the
+//                shared-memory port to the TMA fills and the Q / K / V^T operand reads
+// Warp 0 streams Q once and K / V^T tiles through a four-stage TMA ring (one barrier per stage
+// for both tiles; a stage is released when the P.V of its block finished).  Warp 1 issues
+// S = Q K^T and warp 2 issues P.V, each from one thread, so the S of block j+1 is computed while
+// the P.V of block j-1 runs and neither waits behind the other's barriers.  Softmax arrivals are
+// one per warp.  Every wait is bounded.
 #include "common.cuh"
 #include "tcgen05.cuh"
 
@@ -29,17 +34,19 @@ constexpr float kRescaleLog2 = 8.0f;  // lazy-rescale threshold (log2 units)
 constexpr int kQBytes = kQ * kDH * 2;    // 16 KB
 constexpr int kKBytes = kKV * kDH * 2;   // 16 KB
 constexpr int kVBytes = kDH * kKV * 2;   // 16 KB: two 8 KB atom columns (64 keys each)
-constexpr int kPBytes = kQ * kKV * 2;    // 32 KB: two 16 KB atom columns (64 keys each)
 constexpr int kOffQ = 0;
 constexpr int kKVStages = 4;
 constexpr int kOffK = kOffQ + kQBytes;
 constexpr int kOffV = kOffK + kKVStages * kKBytes;
-constexpr int kOffP = kOffV + kKVStages * kVBytes;   // two P buffers
-constexpr int kOffX = kOffP + 2 * kPBytes;   // max / sum exchange [2][2][128] floats
+constexpr int kOffX = kOffV + kKVStages * kVBytes;   // max / sum exchange [2][2][128] floats
 constexpr int kOffBar = kOffX + 2048;
+constexpr int kNumBars = 1 + 2 * kKVStages + 6 + 8;
 constexpr int kSmemAttn = kOffBar + 512 + 1024;  // barriers, TMEM slot, abort flag; alignment slack
+static_assert(kNumBars * 8 + 8 <= 512, "barrier block exceeds its reservation");
 constexpr uint32_t kTmemCols = 512;
 constexpr uint32_t kColO = 256;  // O_0 at 256..319, O_1 at 320..383
+constexpr uint32_t kColP = 384;  // P buffers at 384..447 and 448..511 (bf16 pairs)
+constexpr int kSoftmaxWarps = 8;
 
 WAM_DEV float ex2(float x) {
   float y;
@@ -54,16 +61,13 @@ __global__ void __launch_bounds__(kThreadsAttn, 1)
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint64_t* bars = reinterpret_cast<uint64_t*>(smem + kOffBar);
   uint64_t* q_full = bars + 0;
-  uint64_t* k_full = bars + 1;    // [4]
-  uint64_t* k_empty = bars + 5;   // [4]
-  uint64_t* v_full = bars + 9;    // [4]
-  uint64_t* v_empty = bars + 13;  // [4]
-  uint64_t* s_full = bars + 17;   // [2]
-  uint64_t* s_empty = bars + 19;  // [2]
-  uint64_t* p_full = bars + 21;   // [2]
-  uint64_t* pv_done = bars + 23;  // [2]: P.V of the block that used P buffer i finished
-  uint64_t* xpair = bars + 25;    // [4 quarters][2]: the two threads of a row exchanged values
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 33);
+  uint64_t* kv_full = bars + 1;                   // [kKVStages]: K and V^T tiles of the stage landed
+  uint64_t* kv_empty = kv_full + kKVStages;       // [kKVStages]: P.V of the stage's block finished
+  uint64_t* s_full = kv_empty + kKVStages;        // [2]
+  uint64_t* s_empty = s_full + 2;                 // [2]
+  uint64_t* p_full = s_empty + 2;                 // [2]
+  uint64_t* xpair = p_full + 2;                   // [4 quarters][2]: the two threads of a row exchanged values
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(xpair + 8);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
   float* xch = reinterpret_cast<float*>(smem + kOffX);  // [2 buffers][2 halves][128 rows]
 
@@ -78,16 +82,13 @@ __global__ void __launch_bounds__(kThreadsAttn, 1)
   if (threadIdx.x == 0) {
     mbar_init(smem_u32(q_full), 1);
     for (int i = 0; i < kKVStages; ++i) {
-      mbar_init(smem_u32(&k_full[i]), 1);
-      mbar_init(smem_u32(&k_empty[i]), 1);
-      mbar_init(smem_u32(&v_full[i]), 1);
-      mbar_init(smem_u32(&v_empty[i]), 1);
+      mbar_init(smem_u32(&kv_full[i]), 1);
+      mbar_init(smem_u32(&kv_empty[i]), 1);
     }
     for (int i = 0; i < 2; ++i) {
       mbar_init(smem_u32(&s_full[i]), 1);
-      mbar_init(smem_u32(&s_empty[i]), 256);
-      mbar_init(smem_u32(&p_full[i]), 256);
-      mbar_init(smem_u32(&pv_done[i]), 1);
+      mbar_init(smem_u32(&s_empty[i]), kSoftmaxWarps);   // one arrival per softmax warp
+      mbar_init(smem_u32(&p_full[i]), kSoftmaxWarps);
     }
     for (int i = 0; i < 8; ++i) mbar_init(smem_u32(&xpair[i]), 64);
     *abort_flag = 0;
@@ -111,57 +112,53 @@ __global__ void __launch_bounds__(kThreadsAttn, 1)
     const int vt_row = (b * H + h) * kDH;
     for (int j = 0; j < nkv; ++j) {
       const int s = j % kKVStages;
-      const uint32_t par = ((j / kKVStages) & 1) ^ 1u;
-      if (!mbar_wait(smem_u32(&k_empty[s]), par, abort_flag, dev_err)) break;
-      const uint32_t kb = smem_u32(&k_full[s]);
-      mbar_expect_tx(kb, kKBytes);
-      tma_load_2d(smem_u32(smem + kOffK + s * kKBytes), &tmQK, d + h * kDH, row_base + j * kKV, kb);
-      if (!mbar_wait(smem_u32(&v_empty[s]), par, abort_flag, dev_err)) break;
-      const uint32_t vb = smem_u32(&v_full[s]);
-      mbar_expect_tx(vb, kVBytes);
-      tma_load_2d(smem_u32(smem + kOffV + s * kVBytes), &tmVt, j * kKV, vt_row, vb);
-      tma_load_2d(smem_u32(smem + kOffV + s * kVBytes + kVBytes / 2), &tmVt, j * kKV + 64, vt_row, vb);
+      if (!mbar_wait(smem_u32(&kv_empty[s]), ((j / kKVStages) & 1) ^ 1u, abort_flag, dev_err)) break;
+      const uint32_t fb = smem_u32(&kv_full[s]);
+      mbar_expect_tx(fb, kKBytes + kVBytes);
+      tma_load_2d(smem_u32(smem + kOffK + s * kKBytes), &tmQK, d + h * kDH, row_base + j * kKV, fb);
+      tma_load_2d(smem_u32(smem + kOffV + s * kVBytes), &tmVt, j * kKV, vt_row, fb);
+      tma_load_2d(smem_u32(smem + kOffV + s * kVBytes + kVBytes / 2), &tmVt, j * kKV + 64, vt_row, fb);
     }
   } else if (warp == 1 && lane == 0) {
-    // ---------------- MMA issue ----------------
+    // ---------------- S = Q K^T issue ----------------
+    // A second thread issues P.V: tcgen05.commit tracks the MMAs of the issuing thread only, so
+    // the two streams complete independently and neither waits behind the other's barriers.
     const uint32_t idS = idesc_bf16(kQ, kKV);
-    const uint32_t idO = idesc_bf16(kQ, kDH);
     bool ok = mbar_wait(smem_u32(q_full), 0, abort_flag, dev_err);
     const uint32_t sq = smem_u32(smem + kOffQ);
-    for (int j = 0; ok && j <= nkv; ++j) {
-      if (j < nkv) {
-        const int s = j & 1;
-        const int ks = j % kKVStages;
-        if (!mbar_wait(smem_u32(&k_full[ks]), (j / kKVStages) & 1, abort_flag, dev_err)) break;
-        if (!mbar_wait(smem_u32(&s_empty[s]), ((j >> 1) & 1) ^ 1u, abort_flag, dev_err)) break;
-        tc_fence_after();
-        const uint32_t sk = smem_u32(smem + kOffK + ks * kKBytes);
+    for (int j = 0; ok && j < nkv; ++j) {
+      const int s = j & 1;
+      const int ks = j % kKVStages;
+      if (!mbar_wait(smem_u32(&kv_full[ks]), (j / kKVStages) & 1, abort_flag, dev_err)) break;
+      if (!mbar_wait(smem_u32(&s_empty[s]), ((j >> 1) & 1) ^ 1u, abort_flag, dev_err)) break;
+      tc_fence_after();
+      const uint32_t sk = smem_u32(smem + kOffK + ks * kKBytes);
 #pragma unroll
-        for (int t = 0; t < kDH / 16; ++t)
-          umma_bf16(tmem + s * kKV, sw128_desc(sq + t * 32), sw128_desc(sk + t * 32), idS, t > 0 ? 1u : 0u);
-        umma_commit(smem_u32(&s_full[s]));
-        umma_commit(smem_u32(&k_empty[ks]));
-      }
-      if (j >= 1) {
-        const int jj = j - 1;
-        const int pb = jj & 1;
-        const int vs = jj % kKVStages;
-        if (!mbar_wait(smem_u32(&v_full[vs]), (jj / kKVStages) & 1, abort_flag, dev_err)) break;
-        if (!mbar_wait(smem_u32(&p_full[pb]), (jj >> 1) & 1, abort_flag, dev_err)) break;
-        tc_fence_after();
-        const uint32_t sp = smem_u32(smem + kOffP + pb * kPBytes);
-        const uint32_t sv = smem_u32(smem + kOffV + vs * kVBytes);
+      for (int t = 0; t < kDH / 16; ++t)
+        umma_bf16(tmem + s * kKV, sw128_desc(sq + t * 32), sw128_desc(sk + t * 32), idS, t > 0 ? 1u : 0u);
+      umma_commit(smem_u32(&s_full[s]));
+    }
+  } else if (warp == 2 && lane == 0) {
+    // ---------------- O_h += P_h V_h issue ----------------
+    // kv_empty[stage] completes when the P.V of the stage's block finished: it releases the K and
+    // V^T tiles to the producer and tells the softmax that the P buffer and O are free.
+    const uint32_t idO = idesc_bf16(kQ, kDH);
+    for (int j = 0; j < nkv; ++j) {
+      const int pb = j & 1;
+      const int vs = j % kKVStages;
+      if (!mbar_wait(smem_u32(&p_full[pb]), (j >> 1) & 1, abort_flag, dev_err)) break;
+      if (!mbar_wait(smem_u32(&kv_full[vs]), (j / kKVStages) & 1, abort_flag, dev_err)) break;
+      tc_fence_after();
+      const uint32_t tp = tmem + kColP + pb * 64;
+      const uint32_t sv = smem_u32(smem + kOffV + vs * kVBytes);
 #pragma unroll
-        for (int t = 0; t < kKV / 16; ++t) {
-          // keys 16t..16t+15 belong to half t/4: its own O accumulator
-          const uint32_t a = sp + (t >> 2) * (kPBytes / 2) + (t & 3) * 32;
-          const uint32_t bb = sv + (t >> 2) * (kVBytes / 2) + (t & 3) * 32;
-          umma_bf16(tmem + kColO + (t >> 2) * kDH, sw128_desc(a), sw128_desc(bb), idO,
-                    (jj > 0 || (t & 3) > 0) ? 1u : 0u);
-        }
-        umma_commit(smem_u32(&pv_done[pb]));
-        umma_commit(smem_u32(&v_empty[vs]));
+      for (int t = 0; t < kKV / 16; ++t) {
+        // keys 16t..16t+15 (P columns 8t..8t+7) belong to half t/4: its own O accumulator
+        const uint32_t bb = sv + (t >> 2) * (kVBytes / 2) + (t & 3) * 32;
+        umma_bf16_ta(tmem + kColO + (t >> 2) * kDH, tp + t * 8, sw128_desc(bb), idO,
+                     (j > 0 || (t & 3) > 0) ? 1u : 0u);
       }
+      umma_commit(smem_u32(&kv_empty[vs]));
     }
   } else if (warp >= 4) {
     // ---------------- softmax: two threads per query row ----------------
@@ -202,7 +199,8 @@ __global__ void __launch_bounds__(kThreadsAttn, 1)
         for (int i = 0; i < 32; ++i) p[c * 32 + i] = __uint_as_float(v[i]);
       }
       tc_fence_before();
-      mbar_arrive(smem_u32(&s_empty[s]));
+      __syncwarp();
+      if (lane == 0) mbar_arrive(smem_u32(&s_empty[s]));
       const int kv0 = j * kKV + half * 64;
       if (kv0 + 64 > N) {
 #pragma unroll
@@ -233,7 +231,7 @@ __global__ void __launch_bounds__(kThreadsAttn, 1)
       m = m_use;
       if (j > 0 && __any_sync(0xffffffffu, corr != 1.0f)) {
         // Rescale this thread's 32 O columns once every earlier P.V has landed.
-        if (!warp_wait(smem_u32(&pv_done[(j - 1) & 1]), ((j - 1) >> 1) & 1, abort_flag, dev_err)) {
+        if (!warp_wait(smem_u32(&kv_empty[(j - 1) % kKVStages]), ((j - 1) / kKVStages) & 1, abort_flag, dev_err)) {
           ok = false;
           break;
         }
@@ -249,24 +247,18 @@ __global__ void __launch_bounds__(kThreadsAttn, 1)
       }
       // P buffer j&1 is free once the P.V of block j-2 finished.
       const int pb = j & 1;
-      if (j >= 2 && !warp_wait(smem_u32(&pv_done[pb]), ((j - 2) >> 1) & 1, abort_flag, dev_err)) {
+      if (j >= 2 && !warp_wait(smem_u32(&kv_empty[(j - 2) % kKVStages]), ((j - 2) / kKVStages) & 1, abort_flag, dev_err)) {
         ok = false;
         break;
       }
-      // 8 chunks of 8 bf16 into atom column `half`; chunk c lands at slot c xor (r % 8).
-      uint8_t* prow = smem + kOffP + pb * kPBytes + half * (kPBytes / 2) + r * 128;
+      // 32 bf16 pairs into columns [32 half, 32 half + 32) of P buffer pb, row r in lane r.
+      uint32_t pk[32];
 #pragma unroll
-      for (int c = 0; c < 8; ++c) {
-        uint4 u;
-        u.x = pack_bf16x2(p[8 * c + 0], p[8 * c + 1]);
-        u.y = pack_bf16x2(p[8 * c + 2], p[8 * c + 3]);
-        u.z = pack_bf16x2(p[8 * c + 4], p[8 * c + 5]);
-        u.w = pack_bf16x2(p[8 * c + 6], p[8 * c + 7]);
-        *reinterpret_cast<uint4*>(prow + ((c ^ (r & 7)) << 4)) = u;
-      }
-      asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+      for (int c = 0; c < 32; ++c) pk[c] = pack_bf16x2(p[2 * c], p[2 * c + 1]);
+      tmem_st32(lane_addr + kColP + pb * 64 + half * 32, pk);
       tc_fence_before();
-      mbar_arrive(smem_u32(&p_full[pb]));
+      __syncwarp();
+      if (lane == 0) mbar_arrive(smem_u32(&p_full[pb]));
     }
     // Merge the two half streams: O = sum_h O_h 2^(m_h - M), l = sum_h l_h 2^(m_h - M).
     float m_partner = 0.0f, l_partner = 0.0f;
@@ -276,7 +268,7 @@ __global__ void __launch_bounds__(kThreadsAttn, 1)
       const float inv = 1.0f / (l * f_own + l_partner * f_par);
       const float w0 = (half == 0 ? f_own : f_par) * inv;   // weight of O_0
       const float w1 = (half == 0 ? f_par : f_own) * inv;   // weight of O_1
-      if (warp_wait(smem_u32(&pv_done[(nkv - 1) & 1]), ((nkv - 1) >> 1) & 1, abort_flag, dev_err)) {
+      if (warp_wait(smem_u32(&kv_empty[(nkv - 1) % kKVStages]), ((nkv - 1) / kKVStages) & 1, abort_flag, dev_err)) {
         tc_fence_after();
         const int q = q0 + r;
         uint32_t v0[32], v1[32];
