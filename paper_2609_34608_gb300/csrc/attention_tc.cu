@@ -1,25 +1,23 @@
 // Full bidirectional attention on the fifth-generation tensor cores (head dim 64).
 //
 // One CTA owns 128 queries of one (item, head); TMEM lane r is query r.  Per block of 128 keys:
-//   S = Q K^T    tcgen05.mma M=128 N=128 K=64 into one of two TMEM S buffers (cols 0 / 128)
+//   S = Q K^T    tcgen05.mma M=128 N=128 K=64 into one of three TMEM S buffers (cols 0/128/256)
 //   softmax      warps 4-11, two threads per query row, each an independent online-softmax
-//                stream over its half (64 keys) of every block: tcgen05.ld of the S half-row,
-//                running max / sum in the log2 domain, P (bf16 pairs) stored with tcgen05.st
-//                into one of two TMEM P buffers (row r in lane r, keys 2c, 2c+1 in column c).
-//                Each half
-//                accumulates into its own O in TMEM, rescaled only when its running max grows by
-//                more than 2^8 (the stale max keeps every P <= 256); the two streams are merged
+//                stream over its half (64 keys) of every block: tcgen05.ld of its S half-row,
+//                running max / sum in the log2 domain, then P (bf16 pairs) stored with tcgen05.st
+//                over the first 32 columns of the same half-row, so P needs no TMEM of its own.
+//                Each half accumulates into its own O, rescaled only when its running max grows
+//                by more than 2^8 (the stale max keeps every P <= 256); the two streams are merged
 //                once, at the end, so the halves never wait on each other per block
 //   O_h += P_h V_h  tcgen05.mma M=128 N=64 K=64 per half with the A operand P read from TMEM
 //                and V^T (written by the QKV projection's epilogue) as the K-major B operand
-//                from shared memory; O_0 in TMEM cols 256..319, O_1 in cols 320..383, P buffers
-//                in cols 384..447 and 448..511.  Keeping P out of shared memory leaves the
-//                shared-memory port to the TMA fills and the Q / K / V^T operand reads
-// Warp 0 streams Q once and K / V^T tiles through a four-stage TMA ring (one barrier per stage
+//                from shared memory; O_0 in TMEM cols 384..447, O_1 in cols 448..511
+// Warp 0 streams Q once and K / V^T tiles through a six-stage TMA ring (one barrier per stage
 // for both tiles; a stage is released when the P.V of its block finished).  Warp 1 issues
-// S = Q K^T and warp 2 issues P.V, each from one thread, so the S of block j+1 is computed while
-// the P.V of block j-1 runs and neither waits behind the other's barriers.  Softmax arrivals are
-// one per warp.  Every wait is bounded.
+// S = Q K^T and warp 2 issues P.V, each from one thread: tcgen05.commit tracks the MMAs of the
+// issuing thread only, so the two streams complete independently.  An S buffer is reused once
+// the P.V that read its P finished, so S runs up to two blocks ahead of the softmax.  Softmax
+// arrivals are one per warp.  Every wait is bounded.
 #include "common.cuh"
 #include "tcgen05.cuh"
 
@@ -35,17 +33,17 @@ constexpr int kQBytes = kQ * kDH * 2;    // 16 KB
 constexpr int kKBytes = kKV * kDH * 2;   // 16 KB
 constexpr int kVBytes = kDH * kKV * 2;   // 16 KB: two 8 KB atom columns (64 keys each)
 constexpr int kOffQ = 0;
-constexpr int kKVStages = 4;
+constexpr int kKVStages = 6;
+constexpr int kSBuf = 3;  // TMEM S buffers (each also holds its block's P)
 constexpr int kOffK = kOffQ + kQBytes;
 constexpr int kOffV = kOffK + kKVStages * kKBytes;
 constexpr int kOffX = kOffV + kKVStages * kVBytes;   // max / sum exchange [2][2][128] floats
 constexpr int kOffBar = kOffX + 2048;
-constexpr int kNumBars = 1 + 2 * kKVStages + 6 + 8;
+constexpr int kNumBars = 1 + 2 * kKVStages + 3 * kSBuf + 8;
 constexpr int kSmemAttn = kOffBar + 512 + 1024;  // barriers, TMEM slot, abort flag; alignment slack
 static_assert(kNumBars * 8 + 8 <= 512, "barrier block exceeds its reservation");
 constexpr uint32_t kTmemCols = 512;
-constexpr uint32_t kColO = 256;  // O_0 at 256..319, O_1 at 320..383
-constexpr uint32_t kColP = 384;  // P buffers at 384..447 and 448..511 (bf16 pairs)
+constexpr uint32_t kColO = 384;  // O_0 at 384..447, O_1 at 448..511
 constexpr int kSoftmaxWarps = 8;
 
 WAM_DEV float ex2(float x) {
@@ -63,10 +61,10 @@ __global__ void __launch_bounds__(kThreadsAttn, 1)
   uint64_t* q_full = bars + 0;
   uint64_t* kv_full = bars + 1;                   // [kKVStages]: K and V^T tiles of the stage landed
   uint64_t* kv_empty = kv_full + kKVStages;       // [kKVStages]: P.V of the stage's block finished
-  uint64_t* s_full = kv_empty + kKVStages;        // [2]
-  uint64_t* s_empty = s_full + 2;                 // [2]
-  uint64_t* p_full = s_empty + 2;                 // [2]
-  uint64_t* xpair = p_full + 2;                   // [4 quarters][2]: the two threads of a row exchanged values
+  uint64_t* s_full = kv_empty + kKVStages;        // [kSBuf]: S of the buffer's block computed
+  uint64_t* s_free = s_full + kSBuf;              // [kSBuf]: P.V that read the buffer's P finished
+  uint64_t* p_full = s_free + kSBuf;              // [kSBuf]: P of the buffer's block stored
+  uint64_t* xpair = p_full + kSBuf;               // [4 quarters][2]: the two threads of a row exchanged values
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(xpair + 8);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
   float* xch = reinterpret_cast<float*>(smem + kOffX);  // [2 buffers][2 halves][128 rows]
@@ -85,10 +83,10 @@ __global__ void __launch_bounds__(kThreadsAttn, 1)
       mbar_init(smem_u32(&kv_full[i]), 1);
       mbar_init(smem_u32(&kv_empty[i]), 1);
     }
-    for (int i = 0; i < 2; ++i) {
+    for (int i = 0; i < kSBuf; ++i) {
       mbar_init(smem_u32(&s_full[i]), 1);
-      mbar_init(smem_u32(&s_empty[i]), kSoftmaxWarps);   // one arrival per softmax warp
-      mbar_init(smem_u32(&p_full[i]), kSoftmaxWarps);
+      mbar_init(smem_u32(&s_free[i]), 1);
+      mbar_init(smem_u32(&p_full[i]), kSoftmaxWarps);   // one arrival per softmax warp
     }
     for (int i = 0; i < 8; ++i) mbar_init(smem_u32(&xpair[i]), 64);
     *abort_flag = 0;
@@ -127,10 +125,10 @@ __global__ void __launch_bounds__(kThreadsAttn, 1)
     bool ok = mbar_wait(smem_u32(q_full), 0, abort_flag, dev_err);
     const uint32_t sq = smem_u32(smem + kOffQ);
     for (int j = 0; ok && j < nkv; ++j) {
-      const int s = j & 1;
+      const int s = j % kSBuf;
       const int ks = j % kKVStages;
       if (!mbar_wait(smem_u32(&kv_full[ks]), (j / kKVStages) & 1, abort_flag, dev_err)) break;
-      if (!mbar_wait(smem_u32(&s_empty[s]), ((j >> 1) & 1) ^ 1u, abort_flag, dev_err)) break;
+      if (!mbar_wait(smem_u32(&s_free[s]), ((j / kSBuf) & 1) ^ 1u, abort_flag, dev_err)) break;
       tc_fence_after();
       const uint32_t sk = smem_u32(smem + kOffK + ks * kKBytes);
 #pragma unroll
@@ -141,23 +139,26 @@ __global__ void __launch_bounds__(kThreadsAttn, 1)
   } else if (warp == 2 && lane == 0) {
     // ---------------- O_h += P_h V_h issue ----------------
     // kv_empty[stage] completes when the P.V of the stage's block finished: it releases the K and
-    // V^T tiles to the producer and tells the softmax that the P buffer and O are free.
+    // V^T tiles to the producer and tells the softmax that O is up to date; s_free[buffer] hands
+    // the S buffer (and the P inside it) back to the S thread.
     const uint32_t idO = idesc_bf16(kQ, kDH);
     for (int j = 0; j < nkv; ++j) {
-      const int pb = j & 1;
+      const int sb = j % kSBuf;
       const int vs = j % kKVStages;
-      if (!mbar_wait(smem_u32(&p_full[pb]), (j >> 1) & 1, abort_flag, dev_err)) break;
+      if (!mbar_wait(smem_u32(&p_full[sb]), (j / kSBuf) & 1, abort_flag, dev_err)) break;
       if (!mbar_wait(smem_u32(&kv_full[vs]), (j / kKVStages) & 1, abort_flag, dev_err)) break;
       tc_fence_after();
-      const uint32_t tp = tmem + kColP + pb * 64;
+      const uint32_t tp = tmem + sb * kKV;
       const uint32_t sv = smem_u32(smem + kOffV + vs * kVBytes);
 #pragma unroll
       for (int t = 0; t < kKV / 16; ++t) {
-        // keys 16t..16t+15 (P columns 8t..8t+7) belong to half t/4: its own O accumulator
+        // keys 16t..16t+15 belong to half h = t/4, whose P sits in columns 64h .. 64h+31 of the
+        // buffer (eight columns per 16 keys); each half has its own O accumulator
         const uint32_t bb = sv + (t >> 2) * (kVBytes / 2) + (t & 3) * 32;
-        umma_bf16_ta(tmem + kColO + (t >> 2) * kDH, tp + t * 8, sw128_desc(bb), idO,
+        umma_bf16_ta(tmem + kColO + (t >> 2) * kDH, tp + (t >> 2) * 64 + (t & 3) * 8, sw128_desc(bb), idO,
                      (j > 0 || (t & 3) > 0) ? 1u : 0u);
       }
+      umma_commit(smem_u32(&s_free[sb]));
       umma_commit(smem_u32(&kv_empty[vs]));
     }
   } else if (warp >= 4) {
@@ -184,8 +185,8 @@ __global__ void __launch_bounds__(kThreadsAttn, 1)
     float m = -1e20f, l = 0.0f;
     bool ok = true;
     for (int j = 0; j < nkv; ++j) {
-      const int s = j & 1;
-      if (!warp_wait(smem_u32(&s_full[s]), (j >> 1) & 1, abort_flag, dev_err)) {
+      const int s = j % kSBuf;
+      if (!warp_wait(smem_u32(&s_full[s]), (j / kSBuf) & 1, abort_flag, dev_err)) {
         ok = false;
         break;
       }
@@ -198,9 +199,6 @@ __global__ void __launch_bounds__(kThreadsAttn, 1)
 #pragma unroll
         for (int i = 0; i < 32; ++i) p[c * 32 + i] = __uint_as_float(v[i]);
       }
-      tc_fence_before();
-      __syncwarp();
-      if (lane == 0) mbar_arrive(smem_u32(&s_empty[s]));
       const int kv0 = j * kKV + half * 64;
       if (kv0 + 64 > N) {
 #pragma unroll
@@ -245,20 +243,14 @@ __global__ void __launch_bounds__(kThreadsAttn, 1)
           tmem_st32(lane_addr + kColO + half * kDH + c * 32, v);
         }
       }
-      // P buffer j&1 is free once the P.V of block j-2 finished.
-      const int pb = j & 1;
-      if (j >= 2 && !warp_wait(smem_u32(&kv_empty[(j - 2) % kKVStages]), ((j - 2) / kKVStages) & 1, abort_flag, dev_err)) {
-        ok = false;
-        break;
-      }
-      // 32 bf16 pairs into columns [32 half, 32 half + 32) of P buffer pb, row r in lane r.
+      // 32 bf16 pairs over the first 32 columns of this thread's S half-row (already read).
       uint32_t pk[32];
 #pragma unroll
       for (int c = 0; c < 32; ++c) pk[c] = pack_bf16x2(p[2 * c], p[2 * c + 1]);
-      tmem_st32(lane_addr + kColP + pb * 64 + half * 32, pk);
+      tmem_st32(lane_addr + s * kKV + half * 64, pk);
       tc_fence_before();
       __syncwarp();
-      if (lane == 0) mbar_arrive(smem_u32(&p_full[pb]));
+      if (lane == 0) mbar_arrive(smem_u32(&p_full[s]));
     }
     // Merge the two half streams: O = sum_h O_h 2^(m_h - M), l = sum_h l_h 2^(m_h - M).
     float m_partner = 0.0f, l_partner = 0.0f;
