@@ -14,10 +14,10 @@
 //                from shared memory; O_0 in TMEM cols 384..447, O_1 in cols 448..511
 // Warp 0 streams Q once and K / V^T tiles through a six-stage TMA ring (one barrier per stage
 // for both tiles; a stage is released when the P.V of its block finished).  Warp 1 issues
-// S = Q K^T and warp 2 issues P.V, each from one thread: tcgen05.commit tracks the MMAs of the
-// issuing thread only, so the two streams complete independently.  An S buffer is reused once
-// the P.V that read its P finished, so S runs up to two blocks ahead of the softmax.  Softmax
-// arrivals are one per warp.  Every wait is bounded.
+// S = Q K^T, warps 2 and 3 issue the P.V of the two halves, each from one thread:
+// tcgen05.commit tracks the MMAs of the issuing thread only, so the streams complete
+// independently.  An S buffer is reused once both P.V that read its P finished, so S runs up to
+// two blocks ahead of the softmax.  Softmax arrivals are one per warp.  Every wait is bounded.
 #include "common.cuh"
 #include "tcgen05.cuh"
 
@@ -81,11 +81,11 @@ __global__ void __launch_bounds__(kThreadsAttn, 1)
     mbar_init(smem_u32(q_full), 1);
     for (int i = 0; i < kKVStages; ++i) {
       mbar_init(smem_u32(&kv_full[i]), 1);
-      mbar_init(smem_u32(&kv_empty[i]), 1);
+      mbar_init(smem_u32(&kv_empty[i]), 2);   // one commit from each P.V thread
     }
     for (int i = 0; i < kSBuf; ++i) {
       mbar_init(smem_u32(&s_full[i]), 1);
-      mbar_init(smem_u32(&s_free[i]), 1);
+      mbar_init(smem_u32(&s_free[i]), 2);
       mbar_init(smem_u32(&p_full[i]), kSoftmaxWarps);   // one arrival per softmax warp
     }
     for (int i = 0; i < 8; ++i) mbar_init(smem_u32(&xpair[i]), 64);
@@ -136,11 +136,13 @@ __global__ void __launch_bounds__(kThreadsAttn, 1)
         umma_bf16(tmem + s * kKV, sw128_desc(sq + t * 32), sw128_desc(sk + t * 32), idS, t > 0 ? 1u : 0u);
       umma_commit(smem_u32(&s_full[s]));
     }
-  } else if (warp == 2 && lane == 0) {
-    // ---------------- O_h += P_h V_h issue ----------------
-    // kv_empty[stage] completes when the P.V of the stage's block finished: it releases the K and
-    // V^T tiles to the producer and tells the softmax that O is up to date; s_free[buffer] hands
-    // the S buffer (and the P inside it) back to the S thread.
+  } else if ((warp == 2 || warp == 3) && lane == 0) {
+    // ---------------- O_h += P_h V_h issue, h = warp - 2 ----------------
+    // Each half's four MMAs come from their own thread.  kv_empty[stage] completes (two commits)
+    // when both halves of the stage's block finished: it releases the K and V^T tiles to the
+    // producer and tells the softmax that O is up to date; s_free[buffer] hands the S buffer (and
+    // the P inside it) back to the S thread.
+    const int hv = warp - 2;
     const uint32_t idO = idesc_bf16(kQ, kDH);
     for (int j = 0; j < nkv; ++j) {
       const int sb = j % kSBuf;
@@ -148,16 +150,13 @@ __global__ void __launch_bounds__(kThreadsAttn, 1)
       if (!mbar_wait(smem_u32(&p_full[sb]), (j / kSBuf) & 1, abort_flag, dev_err)) break;
       if (!mbar_wait(smem_u32(&kv_full[vs]), (j / kKVStages) & 1, abort_flag, dev_err)) break;
       tc_fence_after();
-      const uint32_t tp = tmem + sb * kKV;
-      const uint32_t sv = smem_u32(smem + kOffV + vs * kVBytes);
+      // keys 64 hv + 16t .. +15: P in columns 64 hv + 8t .. +7 of the buffer, V^T in atom column hv
+      const uint32_t tp = tmem + sb * kKV + hv * 64;
+      const uint32_t sv = smem_u32(smem + kOffV + vs * kVBytes) + hv * (kVBytes / 2);
 #pragma unroll
-      for (int t = 0; t < kKV / 16; ++t) {
-        // keys 16t..16t+15 belong to half h = t/4, whose P sits in columns 64h .. 64h+31 of the
-        // buffer (eight columns per 16 keys); each half has its own O accumulator
-        const uint32_t bb = sv + (t >> 2) * (kVBytes / 2) + (t & 3) * 32;
-        umma_bf16_ta(tmem + kColO + (t >> 2) * kDH, tp + (t >> 2) * 64 + (t & 3) * 8, sw128_desc(bb), idO,
-                     (j > 0 || (t & 3) > 0) ? 1u : 0u);
-      }
+      for (int t = 0; t < 4; ++t)
+        umma_bf16_ta(tmem + kColO + hv * kDH, tp + t * 8, sw128_desc(sv + t * 32), idO,
+                     (j > 0 || t > 0) ? 1u : 0u);
       umma_commit(smem_u32(&s_free[sb]));
       umma_commit(smem_u32(&kv_empty[vs]));
     }
