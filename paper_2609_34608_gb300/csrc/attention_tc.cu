@@ -52,6 +52,12 @@ WAM_DEV float ex2(float x) {
   return y;
 }
 
+WAM_DEV float max3(float a, float b, float c) {
+  float y;
+  asm("max.f32 %0, %1, %2, %3;" : "=f"(y) : "f"(a), "f"(b), "f"(c));
+  return y;
+}
+
 __global__ void __launch_bounds__(kThreadsAttn, 1)
     attn_tc_kernel(const __grid_constant__ CUtensorMap tmQK, const __grid_constant__ CUtensorMap tmVt,
                    bf16* __restrict__ out, int N, int d, int H, float scale_log2, int* dev_err) {
@@ -119,8 +125,8 @@ __global__ void __launch_bounds__(kThreadsAttn, 1)
     }
   } else if (warp == 1 && lane == 0) {
     // ---------------- S = Q K^T issue ----------------
-    // A second thread issues P.V: tcgen05.commit tracks the MMAs of the issuing thread only, so
-    // the two streams complete independently and neither waits behind the other's barriers.
+    // Warps 2 and 3 issue P.V: tcgen05.commit tracks the MMAs of the issuing thread only, so
+    // the streams complete independently and none waits behind another's barriers.
     const uint32_t idS = idesc_bf16(kQ, kKV);
     bool ok = mbar_wait(smem_u32(q_full), 0, abort_flag, dev_err);
     const uint32_t sq = smem_u32(smem + kOffQ);
@@ -204,27 +210,37 @@ __global__ void __launch_bounds__(kThreadsAttn, 1)
         for (int i = 0; i < 64; ++i)
           if (kv0 + i >= N) p[i] = -1e30f;
       }
-      float mx8[8];
+      // Row max with three-input max (four independent chains), then the exponentials with
+      // packed f32x2 FMA / add: the softmax warps share their SM sub-partitions with the MMA
+      // issuing threads, so fewer instructions here means faster MMA issue there.
+      float mx4[4] = {p[0], p[1], p[2], p[3]};
 #pragma unroll
-      for (int k = 0; k < 8; ++k) mx8[k] = p[k];
+      for (int i = 4; i < 64; i += 8) {
 #pragma unroll
-      for (int i = 8; i < 64; ++i) mx8[i & 7] = fmaxf(mx8[i & 7], p[i]);
-      const float mx = fmaxf(fmaxf(fmaxf(mx8[0], mx8[1]), fmaxf(mx8[2], mx8[3])),
-                             fmaxf(fmaxf(mx8[4], mx8[5]), fmaxf(mx8[6], mx8[7])));
+        for (int k = 0; k < 4; ++k) mx4[k] = max3(mx4[k], p[i + 2 * k], p[i + 2 * k + 1]);
+      }
+      const float mx = max3(mx4[0], mx4[1], fmaxf(mx4[2], mx4[3]));
       const float cand = mx * scale_log2;
       // Lazy rescale: keep the stale max unless the new one exceeds it by more than 2^8.
       const bool grow = j == 0 || cand > m + kRescaleLog2;
       const float m_use = grow ? fmaxf(m, cand) : m;
       const float corr = grow ? ex2(m - m_use) : 1.0f;
-      float rs8[8];
+      const float2 sc2 = make_float2(scale_log2, scale_log2);
+      const float2 nm2 = make_float2(-m_use, -m_use);
+      float2 rs2[4];
 #pragma unroll
-      for (int k = 0; k < 8; ++k) rs8[k] = 0.0f;
+      for (int k = 0; k < 4; ++k) rs2[k] = make_float2(0.0f, 0.0f);
 #pragma unroll
-      for (int i = 0; i < 64; ++i) {
-        p[i] = ex2(fmaf(p[i], scale_log2, -m_use));
-        rs8[i & 7] += p[i];
+      for (int c = 0; c < 32; ++c) {
+        float2 x = __ffma2_rn(make_float2(p[2 * c], p[2 * c + 1]), sc2, nm2);
+        x.x = ex2(x.x);
+        x.y = ex2(x.y);
+        p[2 * c] = x.x;
+        p[2 * c + 1] = x.y;
+        rs2[c & 3] = __fadd2_rn(rs2[c & 3], x);
       }
-      l = l * corr + (((rs8[0] + rs8[1]) + (rs8[2] + rs8[3])) + ((rs8[4] + rs8[5]) + (rs8[6] + rs8[7])));
+      const float2 rs = __fadd2_rn(__fadd2_rn(rs2[0], rs2[1]), __fadd2_rn(rs2[2], rs2[3]));
+      l = l * corr + (rs.x + rs.y);
       m = m_use;
       if (j > 0 && __any_sync(0xffffffffu, corr != 1.0f)) {
         // Rescale this thread's 32 O columns once every earlier P.V has landed.
