@@ -14,10 +14,12 @@
 //                from shared memory; O_0 in TMEM cols 384..447, O_1 in cols 448..511
 // Warp 0 streams Q once and K / V^T tiles through a six-stage TMA ring (one barrier per stage
 // for both tiles; a stage is released when the P.V of its block finished).  Warp 1 issues
-// S = Q K^T, warps 2 and 3 issue the P.V of the two halves, each from one thread:
-// tcgen05.commit tracks the MMAs of the issuing thread only, so the streams complete
-// independently.  An S buffer is reused once both P.V that read its P finished, so S runs up to
-// two blocks ahead of the softmax.  Softmax arrivals are one per warp.  Every wait is bounded.
+// S = Q K^T, warps 2 and 3 issue the P.V of the two halves; each of these warps waits as a
+// whole and issues its MMAs and their commit from one elected lane (warp-uniform operands keep
+// the issue fast next to the busy softmax warps).  tcgen05.commit tracks the MMAs of the
+// issuing thread only, so the streams complete independently.  An S buffer is reused once both
+// P.V that read its P finished, so S runs up to two blocks ahead of the softmax.  Softmax
+// arrivals are one per warp.  Every wait is bounded.
 #include "common.cuh"
 #include "tcgen05.cuh"
 
@@ -123,27 +125,30 @@ __global__ void __launch_bounds__(kThreadsAttn, 1)
       tma_load_2d(smem_u32(smem + kOffV + s * kVBytes), &tmVt, j * kKV, vt_row, fb);
       tma_load_2d(smem_u32(smem + kOffV + s * kVBytes + kVBytes / 2), &tmVt, j * kKV + 64, vt_row, fb);
     }
-  } else if (warp == 1 && lane == 0) {
-    // ---------------- S = Q K^T issue ----------------
+  } else if (warp == 1) {
+    // ---------------- S = Q K^T issue (whole warp waits, one elected lane issues) ----------------
     // Warps 2 and 3 issue P.V: tcgen05.commit tracks the MMAs of the issuing thread only, so
     // the streams complete independently and none waits behind another's barriers.
     const uint32_t idS = idesc_bf16(kQ, kKV);
-    bool ok = mbar_wait(smem_u32(q_full), 0, abort_flag, dev_err);
+    bool ok = warp_all_wait(smem_u32(q_full), 0, abort_flag, dev_err);
     const uint32_t sq = smem_u32(smem + kOffQ);
     for (int j = 0; ok && j < nkv; ++j) {
       const int s = j % kSBuf;
       const int ks = j % kKVStages;
-      if (!mbar_wait(smem_u32(&kv_full[ks]), (j / kKVStages) & 1, abort_flag, dev_err)) break;
-      if (!mbar_wait(smem_u32(&s_free[s]), ((j / kSBuf) & 1) ^ 1u, abort_flag, dev_err)) break;
+      if (!warp_all_wait(smem_u32(&kv_full[ks]), (j / kKVStages) & 1, abort_flag, dev_err)) break;
+      if (!warp_all_wait(smem_u32(&s_free[s]), ((j / kSBuf) & 1) ^ 1u, abort_flag, dev_err)) break;
       tc_fence_after();
       const uint32_t sk = smem_u32(smem + kOffK + ks * kKBytes);
+      if (elect_one()) {
 #pragma unroll
-      for (int t = 0; t < kDH / 16; ++t)
-        umma_bf16(tmem + s * kKV, sw128_desc(sq + t * 32), sw128_desc(sk + t * 32), idS, t > 0 ? 1u : 0u);
-      umma_commit(smem_u32(&s_full[s]));
+        for (int t = 0; t < kDH / 16; ++t)
+          umma_bf16(tmem + s * kKV, sw128_desc(sq + t * 32), sw128_desc(sk + t * 32), idS, t > 0 ? 1u : 0u);
+        umma_commit(smem_u32(&s_full[s]));   // same lane as the MMAs it tracks
+      }
+      __syncwarp();
     }
-  } else if ((warp == 2 || warp == 3) && lane == 0) {
-    // ---------------- O_h += P_h V_h issue, h = warp - 2 ----------------
+  } else if (warp == 2 || warp == 3) {
+    // ---------------- O_h += P_h V_h issue, h = warp - 2 (as for S) ----------------
     // Each half's four MMAs come from their own thread.  kv_empty[stage] completes (two commits)
     // when both halves of the stage's block finished: it releases the K and V^T tiles to the
     // producer and tells the softmax that O is up to date; s_free[buffer] hands the S buffer (and
@@ -153,18 +158,21 @@ __global__ void __launch_bounds__(kThreadsAttn, 1)
     for (int j = 0; j < nkv; ++j) {
       const int sb = j % kSBuf;
       const int vs = j % kKVStages;
-      if (!mbar_wait(smem_u32(&p_full[sb]), (j / kSBuf) & 1, abort_flag, dev_err)) break;
-      if (!mbar_wait(smem_u32(&kv_full[vs]), (j / kKVStages) & 1, abort_flag, dev_err)) break;
+      if (!warp_all_wait(smem_u32(&p_full[sb]), (j / kSBuf) & 1, abort_flag, dev_err)) break;
+      if (!warp_all_wait(smem_u32(&kv_full[vs]), (j / kKVStages) & 1, abort_flag, dev_err)) break;
       tc_fence_after();
       // keys 64 hv + 16t .. +15: P in columns 64 hv + 8t .. +7 of the buffer, V^T in atom column hv
       const uint32_t tp = tmem + sb * kKV + hv * 64;
       const uint32_t sv = smem_u32(smem + kOffV + vs * kVBytes) + hv * (kVBytes / 2);
+      if (elect_one()) {
 #pragma unroll
-      for (int t = 0; t < 4; ++t)
-        umma_bf16_ta(tmem + kColO + hv * kDH, tp + t * 8, sw128_desc(sv + t * 32), idO,
-                     (j > 0 || t > 0) ? 1u : 0u);
-      umma_commit(smem_u32(&s_free[sb]));
-      umma_commit(smem_u32(&kv_empty[vs]));
+        for (int t = 0; t < 4; ++t)
+          umma_bf16_ta(tmem + kColO + hv * kDH, tp + t * 8, sw128_desc(sv + t * 32), idO,
+                       (j > 0 || t > 0) ? 1u : 0u);
+        umma_commit(smem_u32(&s_free[sb]));   // same lane as the MMAs they track
+        umma_commit(smem_u32(&kv_empty[vs]));
+      }
+      __syncwarp();
     }
   } else if (warp >= 4) {
     // ---------------- softmax: two threads per query row ----------------

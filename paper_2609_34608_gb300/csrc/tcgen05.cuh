@@ -155,6 +155,23 @@ WAM_DEV void tmem_dealloc(uint32_t taddr, uint32_t ncols) {
                : "memory");
 }
 
+// True in exactly one lane of the (fully active) warp.
+WAM_DEV bool elect_one() {
+  uint32_t e;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "elect.sync _|p, 0xffffffff;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(e));
+  return e != 0;
+}
+
+// Every lane of the warp polls the mbarrier (one shared-memory request per poll for the warp);
+// the warp agrees on the outcome, so an abort leaves it converged.
+WAM_DEV bool warp_all_wait(uint32_t bar, uint32_t parity, volatile int* abort_flag, int* dev_err) {
+  return __all_sync(0xffffffffu, mbar_wait(bar, parity, abort_flag, dev_err));
+}
+
 // One lane waits on an mbarrier phase and the warp proceeds together (for warp-collective
 // tcgen05.ld / tcgen05.st that follow).  Returns false on abort.
 WAM_DEV bool warp_wait(uint32_t bar, uint32_t parity, volatile int* abort_flag, int* dev_err) {
