@@ -35,6 +35,28 @@ int wam_op_gemm_bf16(const void* A, const void* Wt, const float* bias, void* C, 
                      int32_t N, int32_t K, int32_t epilogue, const float* gate,
                      int64_t gate_stride, int32_t rows_per_item, void* stream);
 
+/*
+ * The same GEMM with an explicit plan, for tuning and for tests that cover every kernel variant.
+ *   tile_n     output tile width: 64, 128 or 256 (0 = the library's choice, as wam_op_gemm_bf16,
+ *              with K splitting allowed when a workspace is given)
+ *   k_splits   number of K ranges per output tile (0 or 1 = none, up to 4); a split tile's units
+ *              publish fp32 partials to `workspace` and the last unit to finish sums them in range
+ *              order, so results do not depend on timing.  Needs: the K stages (K / 128 for
+ *              64- / 128-wide tiles when K % 128 == 0, else K / 64) divisible by k_splits, and all
+ *              tiles x k_splits units in one wave (at most the SM count).
+ *   workspace  device buffer of wam_op_gemm_workspace_bytes() bytes, 16-byte aligned, zero-filled
+ *              before its first use (every call leaves it reusable); NULL = no splitting.  Calls
+ *              sharing a workspace must be ordered (same stream).
+ * Returns WAM_ERR_UNSUPPORTED when the plan does not fit the shape.
+ */
+int wam_op_gemm_bf16_plan(const void* A, const void* Wt, const float* bias, void* C, int32_t M,
+                          int32_t N, int32_t K, int32_t epilogue, const float* gate,
+                          int64_t gate_stride, int32_t rows_per_item, int32_t tile_n,
+                          int32_t k_splits, void* workspace, size_t workspace_bytes, void* stream);
+
+/* Bytes of the split-K workspace of wam_op_gemm_bf16_plan on the current device. */
+size_t wam_op_gemm_workspace_bytes(void);
+
 /* Same contraction in float32 SIMT (the library's fp32 precision mode). */
 int wam_op_gemm_f32(const float* A, const float* Wt, const float* bias, float* C, int32_t M,
                     int32_t N, int32_t K, int32_t epilogue, const float* gate,

@@ -103,12 +103,32 @@ struct EpiArgs {
 
 // ---- internal interfaces -----------------------------------------------------------------
 // tcgen05 GEMM (gemm_tc.cu).  CUtensorMap is the driver's 128-byte opaque descriptor.
-int tc_encode_kmajor_bf16(CUtensorMap* map, const void* base, uint64_t rows, uint64_t K);
-// Same operand with 64-row boxes: the B map of 64-column output tiles.
-int tc_encode_kmajor_bf16_box64(CUtensorMap* map, const void* base, uint64_t rows, uint64_t K);
-// tb64 (nullable) lets the launcher pick 64-column tiles for narrow projections.
-cudaError_t tc_gemm(const CUtensorMap& ta, const CUtensorMap& tb, const CUtensorMap* tb64, int M, int N, int K,
-                    int epi, const EpiArgs& e, int num_sms, int* dev_err, cudaStream_t s);
+// Tensor maps of one K-major bf16 GEMM operand [rows][K] for every tile shape the GEMM may pick:
+// boxes of 128 rows (the A operand and 128- / 256-wide B tiles) and of 64 rows (64-wide B tiles),
+// one or two 64-column K-atoms deep (two only when K % 128 == 0).
+struct GemmOperand {
+  CUtensorMap r128_k1, r128_k2, r64_k1, r64_k2;
+  bool k2;    // two-atom maps encoded
+  bool r64;   // 64-row maps encoded
+};
+int tc_encode_gemm_operand(GemmOperand* op, const void* base, uint64_t rows, uint64_t K, bool rows64);
+// Output tile width (64 / 128 / 256) and number of K ranges per tile; {0, 0} = choose.
+struct GemmPlan {
+  int bn;
+  int splits;
+};
+// Device scratch of split-K: fp32 partial tiles, then one int ticket counter per output tile.
+// The counters must be zero before the first use; every GEMM leaves them zero.
+struct SplitWorkspace {
+  float* ws;
+  int* counters;
+  size_t ws_bytes;
+};
+size_t tc_gemm_workspace_bytes(int num_sms);
+GemmPlan tc_gemm_plan(int M, int N, int K, bool has64, bool can_split, int num_sms);
+// ws == nullptr: no K split.  plan.bn == 0: chosen by tc_gemm_plan.
+cudaError_t tc_gemm(const GemmOperand& a, const GemmOperand& b, int M, int N, int K, int epi, const EpiArgs& e,
+                    int num_sms, int* dev_err, cudaStream_t s, const SplitWorkspace* ws, GemmPlan plan);
 
 // float32 SIMT GEMM (gemm_simt.cu): C = A[M,K] Wt[N,K]^T
 cudaError_t simt_gemm(const float* A, const float* Wt, int M, int N, int K, int epi,

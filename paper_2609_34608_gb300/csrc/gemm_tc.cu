@@ -3,12 +3,25 @@
 // C[M,N] = A[M,K] . Wt[N,K]^T with bf16 operands and an fp32 accumulator held in TMEM, and the
 // block's elementwise tail fused into the accumulator read-back (bias, GELU, adaLN-gated
 // residual).  Persistent, warp-specialised CTAs:
-//   warp 0      TMA producer: 128x64 A and BNx64 B tiles, 128-byte swizzle, STAGES-deep ring
-//   warp 1      MMA issuer: one thread issues tcgen05.mma (M=128, N=BN, K=16) and commits
+//   warp 0      TMA producer: a stage holds KA K-atoms (64 bf16 = one 128-byte swizzle row each)
+//               of the 128-row A tile and the BN-row B tile, each operand fetched by 3-D boxes
+//               {64, rows, KA}; with KA = 2 one request moves 32 KB.  The single producer
+//               thread's round trip per stage (barrier wait, expect-tx, copy issue) rather than
+//               bandwidth bounds small projections, so fewer, larger requests are faster
+//   warp 1      MMA issuer: one thread issues tcgen05.mma (M=128, N=BN for one-atom stages, else
+//               N=min(BN,128), K=16) and commits
 //               smem-slot / accumulator-ready mbarriers; also owns the TMEM allocation
 //   warps 2..5  epilogue: tcgen05.ld 32x32b per TMEM lane quarter, fused tail, 16-byte stores
 // The accumulator is double buffered in TMEM (2 x BN columns) so the epilogue of one tile
-// overlaps the main loop of the next.  Every mbarrier wait is bounded (%globaltimer); on
+// overlaps the main loop of the next.
+//
+// K split: a projection with too few output tiles to fill the GPU is cut into `splits` work units
+// per tile, each over a contiguous range of K.  A unit's epilogue stores its fp32 partial tile to
+// a workspace and takes a ticket from the tile's counter; the unit that takes the last ticket
+// (no CTA ever waits for another) fetches all partials into its (now idle) stage buffers with
+// bulk asynchronous copies, sums them in split order, which makes the result independent of
+// which unit finishes last, applies the fused tail and resets the counter.  Splitting is only
+// planned in one wave (one unit per CTA) and when the partials fit the stage buffers.  Every mbarrier wait is bounded (%globaltimer); on
 // timeout the CTA raises an abort flag, sets the context's device error word, drains what it
 // issued and frees TMEM before returning.
 #include <cudaTypedefs.h>
@@ -27,15 +40,21 @@ constexpr int kThreads = 192;
 constexpr int kTileBytesA = kBM * kBK * 2;  // 16 KB
 constexpr int kBoxRows = 128;               // TMA box rows of the A operand and wide B tiles
 
-template <int BN>
+template <int BN, int KA>
 struct TileCfg {
-  static constexpr int kStages = (BN == 256) ? 4 : (BN == 128 ? 6 : 8);
-  static constexpr int kBoxB = BN < kBoxRows ? BN : kBoxRows;  // rows per B load
-  static constexpr int kTileBytesB = BN * kBK * 2;
-  static constexpr int kStageBytes = kTileBytesA + kTileBytesB;
+  static constexpr int kBoxB = BN < kBoxRows ? BN : kBoxRows;  // rows per B request
+  // One atom per stage: the B boxes lie back to back, so one MMA spans all BN columns.  Two atoms:
+  // each box holds both atoms of its rows ([atom][rows]), so each box gets its own MMA.
+  static constexpr int kMmaN = KA == 1 ? BN : kBoxB;
+  static constexpr int kBytesA = KA * kTileBytesA;              // [KA atoms][128 rows][128 B]
+  static constexpr int kBoxBytesB = KA * kBoxB * kBK * 2;       // [KA atoms][kBoxB rows][128 B]
+  static constexpr int kStageBytes = kBytesA + (BN / kBoxB) * kBoxBytesB;
+  static constexpr int kStages = (192 * 1024) / kStageBytes;    // 2 .. 8
   static constexpr int kTmemCols = 2 * BN;
   static constexpr int kBarrierBytes = 256;
   static constexpr int kSmemBytes = kStages * kStageBytes + kBarrierBytes + 1024;
+  static_assert(kStages >= 2 && kStages <= 8, "stage count");
+  static_assert((2 * kStages + 7) * 8 + 12 <= kBarrierBytes, "barrier block");
 };
 
 // Fused accumulator read-back for one row segment of 32 columns.
@@ -124,11 +143,17 @@ WAM_DEV void epilogue32(const EpiArgs& e, int N, int row, int col0, const uint32
   }
 }
 
-template <int BN, int EPI>
+struct SplitArgs {
+  int splits;       // K ranges per output tile (1 = no split)
+  float* ws;        // [tiles][splits][BN / 4][kBM][4] fp32 partials
+  int* counters;    // [tiles] tickets, zero between launches
+};
+
+template <int BN, int EPI, int KA>
 __global__ void __launch_bounds__(kThreads, 1)
     gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
-                   int M, int N, int K, EpiArgs e, int* dev_err) {
-  using C = TileCfg<BN>;
+                   int M, int N, int K, EpiArgs e, SplitArgs sp, int* dev_err) {
+  using C = TileCfg<BN, KA>;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint8_t* tiles = smem;
@@ -138,15 +163,32 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint64_t* tfull = bars + 2 * C::kStages;
   uint64_t* tempty = tfull + 2;
   uint64_t* drain = tempty + 2;
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain + 1);
+  uint64_t* epbar = drain + 1;   // the 128 epilogue threads, once per split-K hand-off
+  uint64_t* rbar = epbar + 1;    // bulk copies of a tile's partials landed
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(rbar + 1);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+  volatile int* last_flag = abort_flag + 1;
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
   const int num_m = (M + kBM - 1) / kBM;
   const int num_n = N / BN;
-  const int num_tiles = num_m * num_n;
-  const int num_k = K / kBK;
+  const int num_mn = num_m * num_n;
+  const int splits = sp.splits;
+  const int num_units = num_mn * splits;
+  const int num_k = K / (kBK * KA) / splits;   // stages per work unit
+  // unit u: output tile mn = u % num_mn (m fastest), K range u / num_mn
+  auto unit_mt = [&](int u) { return (u % num_mn) % num_m; };
+  auto unit_nt = [&](int u) { return (u % num_mn) / num_m; };
+  auto unit_kb0 = [&](int u) { return (u / num_mn) * num_k; };
+  // K-atoms [atom, atom + KA) of rows [row, row + box): one 2-D box {64, rows} for one atom, one
+  // 3-D box {64, rows, 2} for two
+  auto load_k = [&](uint32_t dst, const CUtensorMap* map, int row, int atom, uint32_t bar) {
+    if constexpr (KA == 1)
+      tma_load_2d(dst, map, atom * kBK, row, bar);
+    else
+      tma_load_3d(dst, map, 0, row, atom, bar);
+  };
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < C::kStages; ++s) {
@@ -158,6 +200,8 @@ __global__ void __launch_bounds__(kThreads, 1)
       mbar_init(smem_u32(&tempty[a]), 128);
     }
     mbar_init(smem_u32(drain), 1);
+    mbar_init(smem_u32(epbar), 128);
+    mbar_init(smem_u32(rbar), 1);
     *abort_flag = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
@@ -181,14 +225,15 @@ __global__ void __launch_bounds__(kThreads, 1)
     asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmB)) : "memory");
     // The weight operand does not depend on earlier kernels: its first stages are requested
     // before waiting for them, overlapping the previous kernel's tail.
-    const int pre = blockIdx.x < num_tiles ? (num_k < C::kStages ? num_k : C::kStages) : 0;
+    const int u0 = blockIdx.x;
+    const int pre = u0 < num_units ? (num_k < C::kStages ? num_k : C::kStages) : 0;
     for (int s = 0; s < pre; ++s) {
       const uint32_t fb = smem_u32(&full[s]);
-      const uint32_t b_dst = smem_u32(tiles + s * C::kStageBytes) + kTileBytesA;
+      const uint32_t b_dst = smem_u32(tiles + s * C::kStageBytes) + C::kBytesA;
       mbar_expect_tx(fb, C::kStageBytes);
 #pragma unroll
       for (int h = 0; h < BN / C::kBoxB; ++h)
-        tma_load_2d(b_dst + h * C::kBoxB * 128, &tmB, s * kBK, (blockIdx.x / num_m) * BN + h * C::kBoxB, fb);
+        load_k(b_dst + h * C::kBoxBytesB, &tmB, unit_nt(u0) * BN + h * C::kBoxB, (unit_kb0(u0) + s) * KA, fb);
     }
     pdl_wait();
     int stage = 0;
@@ -198,9 +243,10 @@ __global__ void __launch_bounds__(kThreads, 1)
     for (int s = 0; s < C::kStages; ++s) issued[s] = 0, issued_phase[s] = 0;
     bool ok = true;
     bool first = true;
-    for (int tile = blockIdx.x; ok && tile < num_tiles; tile += gridDim.x) {
-      const int mt = tile % num_m;
-      const int nt = tile / num_m;
+    for (int unit = blockIdx.x; ok && unit < num_units; unit += gridDim.x) {
+      const int mt = unit_mt(unit);
+      const int nt = unit_nt(unit);
+      const int kb0 = unit_kb0(unit);
       for (int kb = 0; kb < num_k; ++kb) {
         if (!mbar_wait(smem_u32(&empty[stage]), phase ^ 1u, abort_flag, dev_err)) {
           ok = false;
@@ -208,14 +254,14 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         const uint32_t fb = smem_u32(&full[stage]);
         const uint32_t a_dst = smem_u32(tiles + stage * C::kStageBytes);
-        const uint32_t b_dst = a_dst + kTileBytesA;
+        const uint32_t b_dst = a_dst + C::kBytesA;
         if (!(first && kb < pre)) {
           mbar_expect_tx(fb, C::kStageBytes);
 #pragma unroll
           for (int h = 0; h < BN / C::kBoxB; ++h)
-            tma_load_2d(b_dst + h * C::kBoxB * 128, &tmB, kb * kBK, nt * BN + h * C::kBoxB, fb);
+            load_k(b_dst + h * C::kBoxBytesB, &tmB, nt * BN + h * C::kBoxB, (kb0 + kb) * KA, fb);
         }
-        tma_load_2d(a_dst, &tmA, kb * kBK, mt * kBM, fb);
+        load_k(a_dst, &tmA, mt * kBM, (kb0 + kb) * KA, fb);
         issued[stage] = 1;
         issued_phase[stage] = phase;
         if (++stage == C::kStages) {
@@ -238,13 +284,13 @@ __global__ void __launch_bounds__(kThreads, 1)
   } else if (warp == 1 && lane == 0) {
     // ---------------- MMA issuer ----------------
     pdl_wait();
-    const uint32_t idesc = idesc_bf16(kBM, BN);
+    const uint32_t idesc = idesc_bf16(kBM, C::kMmaN);
     int stage = 0;
     uint32_t phase = 0;
     int it = 0;
     bool ok = true;
     bool issued_any = false;
-    for (int tile = blockIdx.x; ok && tile < num_tiles; tile += gridDim.x, ++it) {
+    for (int unit = blockIdx.x; ok && unit < num_units; unit += gridDim.x, ++it) {
       const int acc = it & 1;
       const uint32_t acc_phase = (it >> 1) & 1;
       if (!mbar_wait(smem_u32(&tempty[acc]), acc_phase ^ 1u, abort_flag, dev_err)) {
@@ -260,11 +306,17 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         tc_fence_after();
         const uint32_t a0 = smem_u32(tiles + stage * C::kStageBytes);
-        const uint32_t b0 = a0 + kTileBytesA;
+        const uint32_t b0 = a0 + C::kBytesA;
 #pragma unroll
-        for (int k = 0; k < kBK / 16; ++k) {
-          umma_bf16(d_tmem, sw128_desc(a0 + k * 32), sw128_desc(b0 + k * 32), idesc,
-                    (kb | k) != 0 ? 1u : 0u);
+        for (int a = 0; a < KA; ++a) {
+#pragma unroll
+          for (int k = 0; k < kBK / 16; ++k) {
+#pragma unroll
+            for (int h = 0; h < BN / C::kMmaN; ++h)
+              umma_bf16(d_tmem + h * C::kMmaN, sw128_desc(a0 + a * kTileBytesA + k * 32),
+                        sw128_desc(b0 + h * C::kBoxBytesB + a * C::kBoxB * 128 + k * 32), idesc,
+                        (kb | a | k) != 0 ? 1u : 0u);
+          }
         }
         issued_any = true;
         umma_commit(smem_u32(&empty[stage]));
@@ -288,7 +340,17 @@ __global__ void __launch_bounds__(kThreads, 1)
     pdl_wait();
     const int quarter = warp & 3;  // TMEM lanes this warp may access
     int it = 0;
-    for (int tile = blockIdx.x; tile < num_tiles; tile += gridDim.x, ++it) {
+    uint32_t ep_phase = 0;
+    uint32_t rb_phase = 0;
+    // All 128 epilogue threads meet on an mbarrier (bounded wait, unlike a named barrier).
+    auto ep_sync = [&]() -> bool {
+      mbar_arrive(smem_u32(epbar));
+      const bool r = mbar_wait(smem_u32(epbar), ep_phase, abort_flag, dev_err);
+      ep_phase ^= 1u;
+      return r;
+    };
+    const int r_local = quarter * 32 + lane;   // tile row of this thread
+    for (int unit = blockIdx.x; unit < num_units; unit += gridDim.x, ++it) {
       const int acc = it & 1;
       const uint32_t acc_phase = (it >> 1) & 1;
       // One lane waits; the warp then proceeds together (tcgen05.ld is warp-collective).
@@ -298,18 +360,84 @@ __global__ void __launch_bounds__(kThreads, 1)
       __syncwarp();
       if (!ok) break;
       tc_fence_after();
-      const int mt = tile % num_m;
-      const int nt = tile / num_m;
-      const int row = mt * kBM + quarter * 32 + lane;
+      const int mt = unit_mt(unit);
+      const int nt = unit_nt(unit);
+      const int row = mt * kBM + r_local;
       const uint32_t taddr = tmem_base + (static_cast<uint32_t>(quarter * 32) << 16) + acc * BN;
+      if (splits == 1) {
+#pragma unroll 1
+        for (int c = 0; c < BN / 32; ++c) {
+          uint32_t r[32];
+          tmem_ld32(taddr + c * 32, r);
+          if (row < M) epilogue32<EPI>(e, N, row, nt * BN + c * 32, r);
+        }
+        tc_fence_before();
+        mbar_arrive(smem_u32(&tempty[acc]));
+        continue;
+      }
+      // ---- K split: publish this unit's partial, then the last unit of the tile finishes it ----
+      const int mn = unit % num_mn;
+      const int ks = unit / num_mn;
+      float4* part = reinterpret_cast<float4*>(sp.ws) + (static_cast<size_t>(mn) * splits + ks) * (kBM * BN / 4);
 #pragma unroll 1
       for (int c = 0; c < BN / 32; ++c) {
         uint32_t r[32];
         tmem_ld32(taddr + c * 32, r);
-        if (row < M) epilogue32<EPI>(e, N, row, nt * BN + c * 32, r);
+#pragma unroll
+        for (int j = 0; j < 8; ++j)   // [BN/4][kBM][4]: a warp's 32 rows of one column quad are contiguous
+          __stcg(part + (c * 8 + j) * kBM + r_local,
+                 make_float4(__uint_as_float(r[4 * j]), __uint_as_float(r[4 * j + 1]),
+                             __uint_as_float(r[4 * j + 2]), __uint_as_float(r[4 * j + 3])));
       }
       tc_fence_before();
       mbar_arrive(smem_u32(&tempty[acc]));
+      __threadfence();
+      if (!ep_sync()) break;
+      if (threadIdx.x == 64) *last_flag = (atomicAdd(sp.counters + mn, 1) == splits - 1) ? 1 : 0;
+      if (!ep_sync()) break;
+      if (*last_flag == 0) continue;
+      // Last unit of the tile: bulk-copy every partial ([splits][BN/4][kBM][4] fp32, contiguous in
+      // the workspace) into the stage buffers, which this CTA's finished main loop left idle.
+      const uint32_t bytes = static_cast<uint32_t>(splits) * kBM * BN * 4;
+      if (threadIdx.x == 64) {
+        __threadfence();
+        sp.counters[mn] = 0;   // every unit of the tile has taken its ticket
+        asm volatile("fence.proxy.async.global;" ::: "memory");   // partials written by other CTAs
+        const uint8_t* src = reinterpret_cast<const uint8_t*>(sp.ws) + static_cast<size_t>(mn) * bytes;
+        mbar_expect_tx(smem_u32(rbar), bytes);
+        for (uint32_t off = 0; off < bytes; off += 32768u) {
+          const uint32_t n = bytes - off < 32768u ? bytes - off : 32768u;
+          asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];"
+                       ::"r"(smem_u32(tiles) + off), "l"(src + off), "r"(n), "r"(smem_u32(rbar))
+                       : "memory");
+        }
+      }
+      if (!mbar_wait(smem_u32(rbar), rb_phase, abort_flag, dev_err)) break;
+      rb_phase ^= 1u;
+      const float4* parts = reinterpret_cast<const float4*>(tiles);
+#pragma unroll 1
+      for (int c = 0; c < BN / 32; ++c) {
+        float v[32];
+#pragma unroll
+        for (int j = 0; j < 8; ++j) {
+          float4 a = parts[(c * 8 + j) * kBM + r_local];
+          for (int q = 1; q < splits; ++q) {
+            const float4 b = parts[(q * (BN / 4) + c * 8 + j) * kBM + r_local];
+            a.x += b.x;
+            a.y += b.y;
+            a.z += b.z;
+            a.w += b.w;
+          }
+          v[4 * j] = a.x;
+          v[4 * j + 1] = a.y;
+          v[4 * j + 2] = a.z;
+          v[4 * j + 3] = a.w;
+        }
+        uint32_t r[32];
+#pragma unroll
+        for (int i = 0; i < 32; ++i) r[i] = __float_as_uint(v[i]);
+        if (row < M) epilogue32<EPI>(e, N, row, nt * BN + c * 32, r);
+      }
     }
   }
 
@@ -338,37 +466,151 @@ PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
   return fn;
 }
 
-template <int BN, int EPI>
+template <int BN, int EPI, int KA>
 cudaError_t launch(const CUtensorMap& ta, const CUtensorMap& tb, int M, int N, int K,
-                   const EpiArgs& e, int num_sms, int* dev_err, cudaStream_t s) {
-  using C = TileCfg<BN>;
+                   const EpiArgs& e, const SplitArgs& sp, int num_sms, int* dev_err, cudaStream_t s) {
+  using C = TileCfg<BN, KA>;
   static bool attr_set = false;
   if (!attr_set) {
-    cudaError_t err = cudaFuncSetAttribute(gemm_tc_kernel<BN, EPI>,
+    cudaError_t err = cudaFuncSetAttribute(gemm_tc_kernel<BN, EPI, KA>,
                                            cudaFuncAttributeMaxDynamicSharedMemorySize, C::kSmemBytes);
     if (err != cudaSuccess) return err;
     attr_set = true;
   }
-  const int tiles = ((M + kBM - 1) / kBM) * (N / BN);
-  const int grid = tiles < num_sms ? tiles : num_sms;
-  return launch_pdl(gemm_tc_kernel<BN, EPI>, dim3(grid), dim3(kThreads), C::kSmemBytes, s, ta, tb, M, N, K, e,
-                    dev_err);
+  const int units = ((M + kBM - 1) / kBM) * (N / BN) * sp.splits;
+  const int grid = units < num_sms ? units : num_sms;
+  return launch_pdl(gemm_tc_kernel<BN, EPI, KA>, dim3(grid), dim3(kThreads), C::kSmemBytes, s, ta, tb, M, N,
+                    K, e, sp, dev_err);
 }
 
-template <int BN>
-cudaError_t dispatch_epi(const CUtensorMap& ta, const CUtensorMap& tb, int M, int N, int K,
-                         int epi, const EpiArgs& e, int num_sms, int* dev_err, cudaStream_t s) {
+template <int BN, int KA>
+cudaError_t dispatch_epi(const CUtensorMap& ta, const CUtensorMap& tb, int M, int N, int K, int epi,
+                         const EpiArgs& e, const SplitArgs& sp, int num_sms, int* dev_err, cudaStream_t s) {
   switch (epi) {
-    case kEpiBf16: return launch<BN, kEpiBf16>(ta, tb, M, N, K, e, num_sms, dev_err, s);
-    case kEpiGeluBf16: return launch<BN, kEpiGeluBf16>(ta, tb, M, N, K, e, num_sms, dev_err, s);
-    case kEpiResidF32: return launch<BN, kEpiResidF32>(ta, tb, M, N, K, e, num_sms, dev_err, s);
-    case kEpiF32: return launch<BN, kEpiF32>(ta, tb, M, N, K, e, num_sms, dev_err, s);
-    case kEpiQkvVt: return launch<BN, kEpiQkvVt>(ta, tb, M, N, K, e, num_sms, dev_err, s);
+    case kEpiBf16: return launch<BN, kEpiBf16, KA>(ta, tb, M, N, K, e, sp, num_sms, dev_err, s);
+    case kEpiGeluBf16: return launch<BN, kEpiGeluBf16, KA>(ta, tb, M, N, K, e, sp, num_sms, dev_err, s);
+    case kEpiResidF32: return launch<BN, kEpiResidF32, KA>(ta, tb, M, N, K, e, sp, num_sms, dev_err, s);
+    case kEpiF32: return launch<BN, kEpiF32, KA>(ta, tb, M, N, K, e, sp, num_sms, dev_err, s);
+    case kEpiQkvVt: return launch<BN, kEpiQkvVt, KA>(ta, tb, M, N, K, e, sp, num_sms, dev_err, s);
     default: return cudaErrorInvalidValue;
   }
 }
 
+// Measured time of one pipeline stage of a CTA's main loop (cycles) for each tile shape: the
+// single MMA-issuing thread and the operand round trip, not the tensor rate, set these for the
+// tile sizes used here.  `ka` K-atoms of 64 per stage.
+long stage_cycles(int bn, int ka) {
+  if (bn == 64) return ka == 2 ? 860 : 700;
+  if (bn == 128) return ka == 2 ? 760 : 480;
+  return 620;  // 256 columns, one atom per stage
+}
+
+int pick_ka(int bn, int K) { return (bn <= 128 && K % (2 * kBK) == 0) ? 2 : 1; }
+
+// Bytes of stage buffers of a tile shape: the most partials the last unit of a split tile can
+// gather (splits x 128 x bn fp32).
+long split_capacity(int bn, int ka) {
+  if (bn == 64) return ka == 2 ? TileCfg<64, 2>::kStages * TileCfg<64, 2>::kStageBytes
+                               : TileCfg<64, 1>::kStages * TileCfg<64, 1>::kStageBytes;
+  if (bn == 128) return ka == 2 ? TileCfg<128, 2>::kStages * TileCfg<128, 2>::kStageBytes
+                                : TileCfg<128, 1>::kStages * TileCfg<128, 1>::kStageBytes;
+  return TileCfg<256, 1>::kStages * TileCfg<256, 1>::kStageBytes;
+}
+
 }  // namespace
+
+// Maps of one K-major bf16 operand [rows][K]: for one-atom boxes the plain 2-D {K, rows} with box
+// {64, box_rows}; for two-atom boxes {64 (one swizzle row), rows, K/64} with the atom dimension
+// 128 bytes apart and box {64, box_rows, 2}.
+static int encode_kmajor_3d(CUtensorMap* map, const void* base, uint64_t rows, uint64_t K, uint32_t box_rows,
+                            uint32_t ka) {
+  PFN_cuTensorMapEncodeTiled_v12000 fn = encode_fn();
+  if (fn == nullptr) return -1;
+  if ((reinterpret_cast<uintptr_t>(base) & 15u) != 0 || K % kBK != 0) return -2;
+  if (ka == 1) return tc_encode_bf16_box(map, base, rows, K, K, static_cast<uint32_t>(kBK), box_rows);
+  cuuint64_t dims[3] = {static_cast<cuuint64_t>(kBK), rows, K / kBK};
+  cuuint64_t strides[2] = {K * 2, static_cast<cuuint64_t>(kBK) * 2};
+  cuuint32_t box[3] = {static_cast<cuuint32_t>(kBK), box_rows, ka};
+  cuuint32_t estr[3] = {1, 1, 1};
+  CUresult r = fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(base), dims, strides, box, estr,
+                  CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                  CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS ? 0 : -3;
+}
+
+int tc_encode_gemm_operand(GemmOperand* op, const void* base, uint64_t rows, uint64_t K, bool rows64) {
+  op->k2 = K % (2 * kBK) == 0;
+  op->r64 = rows64;
+  int r = encode_kmajor_3d(&op->r128_k1, base, rows, K, kBoxRows, 1);
+  if (r == 0 && op->k2) r = encode_kmajor_3d(&op->r128_k2, base, rows, K, kBoxRows, 2);
+  if (r == 0 && rows64) r = encode_kmajor_3d(&op->r64_k1, base, rows, K, 64, 1);
+  if (r == 0 && rows64 && op->k2) r = encode_kmajor_3d(&op->r64_k2, base, rows, K, 64, 2);
+  return r;
+}
+
+size_t tc_gemm_workspace_bytes(int num_sms) {
+  // Splitting is only planned when all units fit in one wave: at most num_sms partial tiles of
+  // 128 x 256 fp32, plus one counter per output tile.
+  return static_cast<size_t>(num_sms) * kBM * 256 * sizeof(float) + static_cast<size_t>(num_sms) * sizeof(int);
+}
+
+GemmPlan tc_gemm_plan(int M, int N, int K, bool has64, bool can_split, int num_sms) {
+  GemmPlan best{128, 1};
+  if (M <= 0) return best;
+  const long m_tiles = (M + kBM - 1) / kBM;
+  long best_cost = -1;
+  const int bns[3] = {64, 128, 256};
+  for (int bn : bns) {
+    if (N % bn != 0 || (bn == 64 && !has64)) continue;
+    const int ka = pick_ka(bn, K);
+    const int stages = K / (kBK * ka);
+    for (int sp = 1; sp <= 4; ++sp) {
+      if (sp > 1 && (!can_split || stages % sp != 0)) continue;
+      const long units = m_tiles * (N / bn) * sp;
+      if (sp > 1 && (units > num_sms || static_cast<long>(sp) * kBM * bn * 4 > split_capacity(bn, ka))) continue;
+      const long waves = (units + num_sms - 1) / num_sms;
+      // per unit: fill + epilogue, then the main loop; a split adds the partial hand-off
+      const long cost = waves * (2500 + (bn / 64) * 300 + (stages / sp) * stage_cycles(bn, ka)) +
+                        (sp > 1 ? 900 + 300 * sp : 0);
+      if (best_cost < 0 || cost < best_cost) {
+        best_cost = cost;
+        best = GemmPlan{bn, sp};
+      }
+    }
+  }
+  return best;
+}
+
+cudaError_t tc_gemm(const GemmOperand& a, const GemmOperand& b, int M, int N, int K, int epi, const EpiArgs& e,
+                    int num_sms, int* dev_err, cudaStream_t s, const SplitWorkspace* ws, GemmPlan plan) {
+  if (M <= 0) return cudaSuccess;
+  if (K % kBK != 0 || N % 128 != 0) return cudaErrorInvalidValue;
+  if (plan.bn == 0) plan = tc_gemm_plan(M, N, K, b.r64, ws != nullptr && ws->ws != nullptr, num_sms);
+  const int bn = plan.bn;
+  if ((bn != 64 && bn != 128 && bn != 256) || N % bn != 0 || (bn == 64 && !b.r64)) return cudaErrorInvalidValue;
+  const int ka = pick_ka(bn, K);
+  if (ka == 2 && !(a.k2 && b.k2)) return cudaErrorInvalidValue;
+  SplitArgs sp{plan.splits < 1 ? 1 : plan.splits, nullptr, nullptr};
+  if (sp.splits > 1) {
+    const long units = static_cast<long>((M + kBM - 1) / kBM) * (N / bn) * sp.splits;
+    if (ws == nullptr || ws->ws == nullptr || (K / (kBK * ka)) % sp.splits != 0 || units > num_sms ||
+        static_cast<size_t>(units) * kBM * bn * sizeof(float) > ws->ws_bytes ||
+        static_cast<long>(sp.splits) * kBM * bn * 4 > split_capacity(bn, ka))
+      return cudaErrorInvalidValue;
+    sp.ws = ws->ws;
+    sp.counters = ws->counters;
+  }
+  const CUtensorMap& ta = ka == 2 ? a.r128_k2 : a.r128_k1;
+  if (bn == 64) {
+    const CUtensorMap& tb = ka == 2 ? b.r64_k2 : b.r64_k1;
+    return ka == 2 ? dispatch_epi<64, 2>(ta, tb, M, N, K, epi, e, sp, num_sms, dev_err, s)
+                   : dispatch_epi<64, 1>(ta, tb, M, N, K, epi, e, sp, num_sms, dev_err, s);
+  }
+  if (bn == 256) return dispatch_epi<256, 1>(ta, b.r128_k1, M, N, K, epi, e, sp, num_sms, dev_err, s);
+  const CUtensorMap& tb = ka == 2 ? b.r128_k2 : b.r128_k1;
+  return ka == 2 ? dispatch_epi<128, 2>(ta, tb, M, N, K, epi, e, sp, num_sms, dev_err, s)
+                 : dispatch_epi<128, 1>(ta, tb, M, N, K, epi, e, sp, num_sms, dev_err, s);
+}
 
 int tc_encode_bf16_box(CUtensorMap* map, const void* base, uint64_t rows, uint64_t cols, uint64_t ld,
                        uint32_t box_cols, uint32_t box_rows) {
@@ -383,44 +625,6 @@ int tc_encode_bf16_box(CUtensorMap* map, const void* base, uint64_t rows, uint64
                   CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
                   CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
   return r == CUDA_SUCCESS ? 0 : -3;
-}
-
-int tc_encode_kmajor_bf16_box64(CUtensorMap* map, const void* base, uint64_t rows, uint64_t K) {
-  return tc_encode_bf16_box(map, base, rows, K, K, kBK, 64);
-}
-
-int tc_encode_kmajor_bf16(CUtensorMap* map, const void* base, uint64_t rows, uint64_t K) {
-  PFN_cuTensorMapEncodeTiled_v12000 fn = encode_fn();
-  if (fn == nullptr) return -1;
-  if ((reinterpret_cast<uintptr_t>(base) & 15u) != 0 || (K * 2) % 16 != 0) return -2;
-  cuuint64_t dims[2] = {K, rows};
-  cuuint64_t strides[1] = {K * 2};
-  cuuint32_t box[2] = {static_cast<cuuint32_t>(kBK), static_cast<cuuint32_t>(kBoxRows)};
-  cuuint32_t estr[2] = {1, 1};
-  CUresult r = fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides,
-                  box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
-                  CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
-  return r == CUDA_SUCCESS ? 0 : -3;
-}
-
-cudaError_t tc_gemm(const CUtensorMap& ta, const CUtensorMap& tb, const CUtensorMap* tb64, int M, int N, int K,
-                    int epi, const EpiArgs& e, int num_sms, int* dev_err, cudaStream_t s) {
-  if (M <= 0) return cudaSuccess;
-  if (K % kBK != 0 || N % 128 != 0) return cudaErrorInvalidValue;
-  // Tile width: each CTA's operand delivery (about 17 cycles per KB of A + B tile per K block)
-  // bounds these kernels, so pick the width that minimises waves x bytes per K block:
-  // narrow tiles spread a small projection over more SMs, wide ones halve the A re-reads.
-  const int m_tiles = (M + kBM - 1) / kBM;
-  auto cost = [&](int bn) {
-    const long tiles = static_cast<long>(m_tiles) * (N / bn);
-    return ((tiles + num_sms - 1) / num_sms) * (16 + bn / 8);
-  };
-  int bn = 128;
-  if (N % 256 == 0 && cost(256) <= cost(bn)) bn = 256;
-  if (tb64 != nullptr && cost(64) < cost(bn)) bn = 64;
-  if (bn == 64) return dispatch_epi<64>(ta, *tb64, M, N, K, epi, e, num_sms, dev_err, s);
-  if (bn == 256) return dispatch_epi<256>(ta, tb, M, N, K, epi, e, num_sms, dev_err, s);
-  return dispatch_epi<128>(ta, tb, M, N, K, epi, e, num_sms, dev_err, s);
 }
 
 }  // namespace wam

@@ -1,5 +1,5 @@
 // Kernel-level entry points (wam_ops.h): single hot-path kernels on caller-owned device
-// buffers, for parity tests and kernel benchmarks.  They allocate nothing.
+// buffers, for parity tests and kernel benchmarks.  They allocate no device memory.
 #include <string>
 
 #include "kernels.cuh"
@@ -58,22 +58,55 @@ const char* wam_op_last_error(void) { return g_op_err.c_str(); }
 int wam_op_gemm_bf16(const void* A, const void* Wt, const float* bias, void* C, int32_t M, int32_t N,
                      int32_t K, int32_t epilogue, const float* gate, int64_t gate_stride,
                      int32_t rows_per_item, void* stream) {
+  return wam_op_gemm_bf16_plan(A, Wt, bias, C, M, N, K, epilogue, gate, gate_stride, rows_per_item, 0, 0, nullptr, 0,
+                               stream);
+}
+
+size_t wam_op_gemm_workspace_bytes(void) {
+  int dev = 0, sms = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
+    return 0;
+  return tc_gemm_workspace_bytes(sms);
+}
+
+int wam_op_gemm_bf16_plan(const void* A, const void* Wt, const float* bias, void* C, int32_t M, int32_t N,
+                          int32_t K, int32_t epilogue, const float* gate, int64_t gate_stride,
+                          int32_t rows_per_item, int32_t tile_n, int32_t k_splits, void* workspace,
+                          size_t workspace_bytes, void* stream) {
   int r = check_gemm_args(A, Wt, C, M, N, K, epilogue, gate, rows_per_item);
   if (r != WAM_OK) return r;
   if (K % 64 != 0 || N % 128 != 0) return op_fail(WAM_ERR_UNSUPPORTED, "needs K % 64 == 0 and N % 128 == 0");
   if (!aligned16(A) || !aligned16(Wt) || !aligned16(C) || (bias && !aligned16(bias)) || (gate && !aligned16(gate)) ||
       (gate && gate_stride % 4 != 0))
     return op_fail(WAM_ERR_INVALID_ARG, "operands must be 16-byte aligned");
+  if (tile_n != 0 && tile_n != 64 && tile_n != 128 && tile_n != 256)
+    return op_fail(WAM_ERR_INVALID_ARG, "tile_n must be 0, 64, 128 or 256");
+  if (k_splits < 0 || k_splits > 4) return op_fail(WAM_ERR_INVALID_ARG, "k_splits must be 0 .. 4");
   int dev = 0, sms = 0;
   cudaError_t e = cudaGetDevice(&dev);
   if (e == cudaSuccess) e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
   if (e != cudaSuccess) return op_cuda("device query", e);
-  CUtensorMap ta, tb, tb64;
-  if (tc_encode_kmajor_bf16(&ta, A, static_cast<uint64_t>(M > 0 ? M : 1), K) != 0 ||
-      tc_encode_kmajor_bf16(&tb, Wt, N, K) != 0 || tc_encode_kmajor_bf16_box64(&tb64, Wt, N, K) != 0)
+  const size_t need = tc_gemm_workspace_bytes(sms);
+  if (workspace != nullptr && (workspace_bytes < need || !aligned16(workspace)))
+    return op_fail(WAM_ERR_INVALID_ARG, "workspace smaller than wam_op_gemm_workspace_bytes() or unaligned");
+  GemmOperand ta, tb;
+  if (tc_encode_gemm_operand(&ta, A, static_cast<uint64_t>(M > 0 ? M : 1), K, false) != 0 ||
+      tc_encode_gemm_operand(&tb, Wt, N, K, true) != 0)
     return op_fail(WAM_ERR_CUDA, "cuTensorMapEncodeTiled failed");
-  e = tc_gemm(ta, tb, &tb64, M, N, K, epilogue, make_epi(bias, C, gate, gate_stride, rows_per_item), sms, nullptr,
-              static_cast<cudaStream_t>(stream));
+  SplitWorkspace ws{nullptr, nullptr, 0};
+  if (workspace != nullptr) {
+    const size_t counters_bytes = static_cast<size_t>(sms) * sizeof(int);
+    ws = SplitWorkspace{static_cast<float*>(workspace),
+                        reinterpret_cast<int*>(static_cast<uint8_t*>(workspace) + need - counters_bytes),
+                        need - counters_bytes};
+  }
+  const GemmPlan plan{tile_n, tile_n == 0 ? 0 : (k_splits < 1 ? 1 : k_splits)};
+  if (plan.bn == 0 && k_splits > 1) return op_fail(WAM_ERR_INVALID_ARG, "k_splits needs an explicit tile_n");
+  e = tc_gemm(ta, tb, M, N, K, epilogue, make_epi(bias, C, gate, gate_stride, rows_per_item), sms, nullptr,
+              static_cast<cudaStream_t>(stream), workspace != nullptr ? &ws : nullptr, plan);
+  if (e == cudaErrorInvalidValue)
+    return op_fail(WAM_ERR_UNSUPPORTED, "tile width / K split not possible for this shape (K ranges must divide "
+                                        "the K stages, all units must fit one wave, a split needs a workspace)");
   return e == cudaSuccess ? WAM_OK : op_cuda("tcgen05 GEMM launch", e);
 }
 
@@ -134,14 +167,15 @@ int wam_op_gemm_qkv_vt(const void* A, const void* Wt, const float* bias, void* q
   cudaError_t e = cudaGetDevice(&dev);
   if (e == cudaSuccess) e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
   if (e != cudaSuccess) return op_cuda("device query", e);
-  CUtensorMap ta, tb;
-  if (tc_encode_kmajor_bf16(&ta, A, static_cast<uint64_t>(M > 0 ? M : 1), K) != 0 ||
-      tc_encode_kmajor_bf16(&tb, Wt, N, K) != 0)
+  GemmOperand ta, tb;
+  if (tc_encode_gemm_operand(&ta, A, static_cast<uint64_t>(M > 0 ? M : 1), K, false) != 0 ||
+      tc_encode_gemm_operand(&tb, Wt, N, K, false) != 0)
     return op_fail(WAM_ERR_CUDA, "cuTensorMapEncodeTiled failed");
   EpiArgs ep = make_epi(bias, qkv, nullptr, 0, rows_per_item);
   ep.vt = static_cast<bf16*>(vt);
   ep.vt_ld = vt_ld;
-  e = tc_gemm(ta, tb, nullptr, M, N, K, kEpiQkvVt, ep, sms, nullptr, static_cast<cudaStream_t>(stream));
+  e = tc_gemm(ta, tb, M, N, K, kEpiQkvVt, ep, sms, nullptr, static_cast<cudaStream_t>(stream), nullptr,
+              GemmPlan{0, 0});
   return e == cudaSuccess ? WAM_OK : op_cuda("tcgen05 QKV GEMM launch", e);
 }
 

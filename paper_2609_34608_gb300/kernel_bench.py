@@ -3,9 +3,9 @@
     python -m paper_2609_34608_gb300.kernel_bench gemm M N K [--iters I]
     python -m paper_2609_34608_gb300.kernel_bench attn B N H [--iters I] [--impl tc|mma]
 
-Each invocation builds the library if needed, warms up, then times `iters` back-to-back launches
-with CUDA events on the current stream and prints one JSON line (microseconds per launch and
-algorithmic TFLOP/s: 2MNK for the GEMM, 4 B N^2 d for attention).
+Each invocation builds the library if needed, warms up, captures `iters` back-to-back launches in
+a CUDA graph, times a replay with CUDA events and prints one JSON line (microseconds per launch
+and algorithmic TFLOP/s: 2MNK for the GEMM, 4 B N^2 d for attention).
 """
 from __future__ import annotations
 
@@ -19,13 +19,25 @@ from . import wam as W
 
 
 def _time(fn, iters: int) -> float:
-    for _ in range(3):
-        fn()
+    """Microseconds per call of fn(stream): `iters` calls captured in one CUDA graph and replayed,
+    so the host-side work of each op call (tensor-map encoding) is not in the measurement."""
+    side = torch.cuda.Stream()
+    side.wait_stream(torch.cuda.current_stream())
+    with torch.cuda.stream(side):
+        for _ in range(3):
+            fn(side.cuda_stream)
+    torch.cuda.current_stream().wait_stream(side)
+    torch.cuda.synchronize()
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g):
+        s = torch.cuda.current_stream().cuda_stream
+        for _ in range(iters):
+            fn(s)
+    g.replay()
     torch.cuda.synchronize()
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     e0.record()
-    for _ in range(iters):
-        fn()
+    g.replay()
     e1.record()
     torch.cuda.synchronize()
     return e0.elapsed_time(e1) * 1000.0 / iters
@@ -37,7 +49,7 @@ def bench_gemm(M: int, N: int, K: int, iters: int) -> dict:
     Wt = (torch.randn(N, K, device=dev) * 0.05).to(torch.bfloat16)
     C = torch.empty(M, N, device=dev, dtype=torch.bfloat16)
     b = torch.zeros(N, device=dev)
-    us = _time(lambda: W.op_gemm_bf16(A, Wt, b, C, M, N, K, W.EPI_BF16), iters)
+    us = _time(lambda st: W.op_gemm_bf16(A, Wt, b, C, M, N, K, W.EPI_BF16, stream=st), iters)
     return {"kernel": "gemm_tc", "M": M, "N": N, "K": K, "us": us, "tflops": 2.0 * M * N * K / us / 1e6}
 
 
@@ -49,9 +61,9 @@ def bench_attn(B: int, N: int, H: int, iters: int, impl: str) -> dict:
     if impl == "tc":
         vt_ld = (N + 7) // 8 * 8
         vt = torch.randn(B * d, vt_ld, device=dev).to(torch.bfloat16)
-        fn = lambda: W.op_attention_tc(qkv, vt, out, B, N, d, H)
+        fn = lambda st: W.op_attention_tc(qkv, vt, out, B, N, d, H, stream=st)
     else:
-        fn = lambda: W.op_attention(qkv, out, B, N, d, H, "bf16")
+        fn = lambda st: W.op_attention(qkv, out, B, N, d, H, "bf16", stream=st)
     us = _time(fn, iters)
     return {"kernel": f"attention_{impl}", "B": B, "N": N, "H": H, "us": us,
             "tflops": 4.0 * B * N * N * d / us / 1e6}

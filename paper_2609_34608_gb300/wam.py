@@ -126,6 +126,9 @@ def lib() -> ctypes.CDLL:
         "wam_profile_read": (ctypes.c_int, [_vp, _vp]),
         "wam_op_gemm_bf16": (ctypes.c_int, [_vp, _vp, _vp, _vp, _i32, _i32, _i32, _i32, _vp, ctypes.c_int64, _i32, _vp]),
         "wam_op_gemm_f32": (ctypes.c_int, [_vp, _vp, _vp, _vp, _i32, _i32, _i32, _i32, _vp, ctypes.c_int64, _i32, _vp]),
+        "wam_op_gemm_bf16_plan": (ctypes.c_int, [_vp, _vp, _vp, _vp, _i32, _i32, _i32, _i32, _vp, ctypes.c_int64, _i32,
+                                                 _i32, _i32, _vp, ctypes.c_size_t, _vp]),
+        "wam_op_gemm_workspace_bytes": (ctypes.c_size_t, []),
         "wam_op_attention": (ctypes.c_int, [_vp, _vp, _i32, _i32, _i32, _i32, _i32, _vp]),
         "wam_op_ln_modulate": (ctypes.c_int, [_vp, _vp, _vp, ctypes.c_int64, _vp, _i32, _i32, _i32, _i32, _vp]),
         "wam_op_last_error": (ctypes.c_char_p, []),
@@ -325,6 +328,20 @@ def _op_check(code: int):
 def op_gemm_bf16(A, Wt, bias, C, M, N, K, epilogue, gate=None, gate_stride=0, rows_per_item=1, stream=None):
     _op_check(lib().wam_op_gemm_bf16(ptr(A), ptr(Wt), ptr(bias), ptr(C), M, N, K, epilogue, ptr(gate),
                                      gate_stride, rows_per_item, stream))
+
+
+def op_gemm_bf16_plan(A, Wt, bias, C, M, N, K, epilogue, tile_n, k_splits, workspace=None, gate=None,
+                      gate_stride=0, rows_per_item=1, stream=None):
+    """wam_op_gemm_bf16 with an explicit output tile width and K split (workspace: a zero-filled
+    device buffer of gemm_workspace_bytes() bytes, needed when k_splits > 1)."""
+    nbytes = 0 if workspace is None else workspace.numel() * workspace.element_size()
+    _op_check(lib().wam_op_gemm_bf16_plan(ptr(A), ptr(Wt), ptr(bias), ptr(C), M, N, K, epilogue, ptr(gate),
+                                          gate_stride, rows_per_item, tile_n, k_splits, ptr(workspace), nbytes,
+                                          stream))
+
+
+def gemm_workspace_bytes():
+    return int(lib().wam_op_gemm_workspace_bytes())
 
 
 def op_gemm_f32(A, Wt, bias, C, M, N, K, epilogue, gate=None, gate_stride=0, rows_per_item=1, stream=None):

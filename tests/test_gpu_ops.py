@@ -28,9 +28,9 @@ GEMM_SHAPES = [
 ]
 
 
-@pytest.mark.parametrize("M,N,K", GEMM_SHAPES)
-@pytest.mark.parametrize("epi", [W.EPI_BF16, W.EPI_GELU_BF16, W.EPI_RESID_F32, W.EPI_F32])
-def test_gemm_tcgen05_matches_reference(wamlib, M, N, K, epi):
+def _check_gemm(M, N, K, epi, run):
+    """Run `run(A, Wt, bias, C, gate, rows_per_item)` on seeded bf16 operands and compare with the
+    float64 product plus the epilogue's tail."""
     rng = np.random.default_rng(M * 7 + N * 3 + K + epi)
     A = _bf16(rng.standard_normal((M, K)))
     Wt = _bf16(rng.standard_normal((N, K)) * 0.05)
@@ -42,13 +42,13 @@ def test_gemm_tcgen05_matches_reference(wamlib, M, N, K, epi):
     if epi in (W.EPI_BF16, W.EPI_GELU_BF16):
         C = torch.full((M, N), float("nan"), dtype=torch.bfloat16, device=dev)
         expect = O.gelu_tanh(acc) if epi == W.EPI_GELU_BF16 else acc
-        W.op_gemm_bf16(Ad, Wd, bd, C, M, N, K, epi)
+        run(Ad, Wd, bd, C, None, rpi)
         torch.cuda.synchronize()
         err = np.max(np.abs(_f64(C) - expect))
         assert err <= 8e-3 * np.max(np.abs(expect)) + 1e-3
     elif epi == W.EPI_F32:
         C = torch.full((M, N), float("nan"), dtype=torch.float32, device=dev)
-        W.op_gemm_bf16(Ad, Wd, bd, C, M, N, K, epi)
+        run(Ad, Wd, bd, C, None, rpi)
         torch.cuda.synchronize()
         assert np.max(np.abs(_f64(C) - acc)) <= 1e-4 * np.max(np.abs(acc))
     else:
@@ -56,11 +56,81 @@ def test_gemm_tcgen05_matches_reference(wamlib, M, N, K, epi):
         gate = torch.from_numpy(rng.standard_normal((items, N + 4)).astype(np.float32))
         h0 = torch.from_numpy(rng.standard_normal((M, N)).astype(np.float32))
         C = h0.to(dev)
-        W.op_gemm_bf16(Ad, Wd, bd, C, M, N, K, epi, gate=gate.to(dev), gate_stride=N + 4, rows_per_item=rpi)
+        run(Ad, Wd, bd, C, gate.to(dev), rpi)
         torch.cuda.synchronize()
         g = gate.double().numpy()[np.arange(M) // rpi, :N]
         expect = h0.double().numpy() + g * acc
         assert np.max(np.abs(_f64(C) - expect)) <= 1e-4 * np.max(np.abs(expect))
+    return C
+
+
+@pytest.mark.parametrize("M,N,K", GEMM_SHAPES)
+@pytest.mark.parametrize("epi", [W.EPI_BF16, W.EPI_GELU_BF16, W.EPI_RESID_F32, W.EPI_F32])
+def test_gemm_tcgen05_matches_reference(wamlib, M, N, K, epi):
+    def run(A, Wt, b, C, gate, rpi):
+        W.op_gemm_bf16(A, Wt, b, C, M, N, K, epi, gate=gate, gate_stride=N + 4, rows_per_item=rpi)
+    _check_gemm(M, N, K, epi, run)
+
+
+# (M, N, K, tile width, K ranges): every kernel variant the planner can choose, incl. K splits.
+PLAN_CASES = [
+    (1392, 768, 3072, 128, 2),   # MLP down-projection of the 12-block d768 model, one episode
+    (1392, 768, 768, 128, 2),    # its attention out-projection
+    (1392, 768, 3072, 64, 1),
+    (300, 768, 3072, 64, 4),
+    (129, 256, 192, 128, 3),     # K = 192: one-atom stages, three ranges, ragged M
+    (1392, 3072, 768, 256, 1),
+    (200, 512, 768, 128, 3),     # three ranges: the partials fill the stage buffers exactly
+    (1, 128, 256, 128, 2),       # a single row, two ranges of one stage each
+]
+
+
+@pytest.mark.parametrize("M,N,K,tile_n,k_splits", PLAN_CASES)
+@pytest.mark.parametrize("epi", [W.EPI_BF16, W.EPI_GELU_BF16, W.EPI_RESID_F32, W.EPI_F32])
+def test_gemm_plans_match_reference(wamlib, M, N, K, tile_n, k_splits, epi):
+    ws = torch.zeros(W.gemm_workspace_bytes(), dtype=torch.uint8, device="cuda")
+
+    def run(A, Wt, b, C, gate, rpi):
+        W.op_gemm_bf16_plan(A, Wt, b, C, M, N, K, epi, tile_n, k_splits, workspace=ws, gate=gate,
+                            gate_stride=N + 4, rows_per_item=rpi)
+    _check_gemm(M, N, K, epi, run)
+    # the ticket counters are back at zero for the next call
+    n_sms = torch.cuda.get_device_properties(0).multi_processor_count
+    assert int(ws[ws.numel() - 4 * n_sms:].count_nonzero()) == 0
+
+
+def test_gemm_split_is_deterministic(wamlib):
+    """A K-split result does not depend on which unit finished last: repeated runs agree bit for bit."""
+    M, N, K = 1392, 768, 3072
+    rng = np.random.default_rng(5)
+    dev = torch.device("cuda")
+    A = _bf16(rng.standard_normal((M, K))).to(dev)
+    Wt = _bf16(rng.standard_normal((N, K)) * 0.05).to(dev)
+    ws = torch.zeros(W.gemm_workspace_bytes(), dtype=torch.uint8, device=dev)
+    outs = []
+    for _ in range(3):
+        C = torch.empty((M, N), dtype=torch.float32, device=dev)
+        W.op_gemm_bf16_plan(A, Wt, None, C, M, N, K, W.EPI_F32, 128, 2, workspace=ws)
+        outs.append(C.cpu())
+    assert all(torch.equal(outs[0], o) for o in outs[1:])
+
+
+def test_gemm_plan_rejections(wamlib):
+    dev = torch.device("cuda")
+    A = torch.zeros((1392, 768), dtype=torch.bfloat16, device=dev)
+    Wt = torch.zeros((768, 768), dtype=torch.bfloat16, device=dev)
+    C = torch.zeros((1392, 768), dtype=torch.float32, device=dev)
+    ws = torch.zeros(W.gemm_workspace_bytes(), dtype=torch.uint8, device=dev)
+    with pytest.raises(W.WamError):   # a split without a workspace
+        W.op_gemm_bf16_plan(A, Wt, None, C, 1392, 768, 768, W.EPI_F32, 128, 2)
+    with pytest.raises(W.WamError):   # 6 K stages do not split in 4
+        W.op_gemm_bf16_plan(A, Wt, None, C, 1392, 768, 768, W.EPI_F32, 128, 4, workspace=ws)
+    with pytest.raises(W.WamError):   # 11 x 12 x 2 units exceed one wave
+        W.op_gemm_bf16_plan(A, Wt, None, C, 1392, 768, 768, W.EPI_F32, 64, 2, workspace=ws)
+    with pytest.raises(W.WamError):   # no such tile width
+        W.op_gemm_bf16_plan(A, Wt, None, C, 1392, 768, 768, W.EPI_F32, 96, 1, workspace=ws)
+    with pytest.raises(W.WamError):   # 256-wide partials of two ranges exceed the stage buffers
+        W.op_gemm_bf16_plan(A[:200], Wt, None, C[:200], 200, 768, 768, W.EPI_F32, 256, 2, workspace=ws)
 
 
 def test_gemm_rejects_unsupported_shapes(wamlib):
