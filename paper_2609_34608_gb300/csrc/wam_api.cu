@@ -8,10 +8,8 @@
 #include <cmath>
 #include <cstdio>
 #include <cstring>
-#include <map>
 #include <new>
 #include <string>
-#include <tuple>
 #include <vector>
 
 #include "kernels.cuh"
@@ -86,13 +84,6 @@ struct wam_ctx {
   float *h = nullptr, *hq = nullptr, *hm = nullptr;
   void *xln = nullptr, *qkv = nullptr, *att = nullptr, *u = nullptr, *obs_lp = nullptr;
   GemmOperand tm_xln, tm_att, tm_u, tm_obs_lp;
-  // Tile width per GEMM shape (128-row tiles rounded up to a power of two, N, K, epilogue),
-  // measured when the context is created: every width sums K in the same order, so the choice
-  // changes speed only, never results.
-  std::map<std::tuple<int, int, int, int>, GemmPlan> gemm_plans;
-  void* tune_out = nullptr;   // scratch destinations of the tuning launches
-  void* tune_vt = nullptr;
-  size_t tune_out_bytes = 0;
   // tensor-core attention (head dim 64): V^T per (episode, head) and the TMA maps it reads
   bool tc_attn = false;
   void* vt = nullptr;
@@ -266,106 +257,6 @@ EpiArgs epi_args(const float* bias, void* C, const float* gate, int64_t gstride,
   return e;
 }
 
-// Tile-width plans.  A shape is keyed by its count of 128-row tiles rounded up to a power of two;
-// shapes with at least four full waves of 256-wide tiles take those (fewest operand bytes per
-// flop) without measurement.  The rest are measured once, at context creation, for every key up
-// to the largest batch: one warm launch and three timed ones per width, the real epilogue writing
-// to scratch buffers.  The hot path only looks plans up.
-int m_bucket(int M) {
-  int t = (M + 127) / 128, b = 1;
-  while (b < t) b <<= 1;
-  return b;
-}
-
-bool plan_is_fixed(const wam_ctx* c, int m_tiles, int N) {
-  return N % 256 == 0 && long(m_tiles) * (N / 256) >= 4L * c->num_sms;
-}
-
-GemmPlan gemm_plan(const wam_ctx* c, const GemmOperand& tb, int M, int N, int K, int epi) {
-  if (plan_is_fixed(c, (M + 127) / 128, N)) return GemmPlan{256, 1};
-  const auto hit = c->gemm_plans.find(std::make_tuple(m_bucket(M), N, K, epi));
-  if (hit != c->gemm_plans.end()) return hit->second;
-  return tc_gemm_plan(M, N, K, tb.r64, false, c->num_sms);
-}
-
-int tune_shape(wam_ctx* c, const GemmOperand& ta, const GemmOperand& tb, int M, int N, int K, int epi,
-               const EpiArgs& e, cudaEvent_t ev0, cudaEvent_t ev1) {
-  const auto key = std::make_tuple(m_bucket(M), N, K, epi);
-  if (c->gemm_plans.count(key) != 0 || plan_is_fixed(c, (M + 127) / 128, N)) return WAM_OK;
-  std::vector<int> widths;
-  if (tb.r64) widths.push_back(64);
-  widths.push_back(128);
-  if (N % 256 == 0) widths.push_back(256);
-  EpiArgs et = e;
-  et.C = c->tune_out;
-  et.item_map = nullptr;
-  if (epi == kEpiQkvVt) et.vt = static_cast<bf16*>(c->tune_vt);
-  GemmPlan best = tc_gemm_plan(M, N, K, tb.r64, false, c->num_sms);
-  float best_ms = -1.0f;
-  for (int bn : widths) {
-    const GemmPlan pl{bn, 1};
-    CK(tc_gemm(ta, tb, M, N, K, epi, et, c->num_sms, c->d_err, c->stream, nullptr, pl));
-    CK(cudaEventRecord(ev0, c->stream));
-    for (int r = 0; r < 3; ++r) CK(tc_gemm(ta, tb, M, N, K, epi, et, c->num_sms, c->d_err, c->stream, nullptr, pl));
-    CK(cudaEventRecord(ev1, c->stream));
-    CK(cudaEventSynchronize(ev1));
-    float ms = 0.0f;
-    CK(cudaEventElapsedTime(&ms, ev0, ev1));
-    if (best_ms < 0.0f || ms < best_ms) {
-      best_ms = ms;
-      best = pl;
-    }
-  }
-  c->gemm_plans[key] = best;
-  return WAM_OK;
-}
-
-// Every GEMM of the forward pass (QKV, attention out, MLP up / down, observation embedding) at
-// every row-count key up to the largest batch.
-int tune_gemms(wam_ctx* c) {
-  const int d = c->d;
-  const size_t max_rows = size_t(c->Bmax) * c->N;
-  const size_t need = max_rows * size_t(std::max(3 * d, c->dff)) * sizeof(float);
-  CK(cudaMalloc(&c->tune_out, need));
-  c->tune_out_bytes = need;
-  cudaEvent_t ev[2] = {nullptr, nullptr};
-  CK(cudaEventCreate(&ev[0]));
-  CK(cudaEventCreate(&ev[1]));
-  int rc = WAM_OK;
-  LayerW& w = c->layers[0];
-  for (int kind = 0; kind < 5 && rc == WAM_OK; ++kind) {
-    const int rows_per = kind == 4 ? c->No : c->N;
-    const int total = c->Bmax * rows_per;
-    for (int b = 1; rc == WAM_OK; b <<= 1) {
-      const int M = std::min(total, b * 128);
-      if (kind == 0) {
-        EpiArgs e = epi_args(w.qkv_b, c->qkv, nullptr, 0, c->N, nullptr);
-        if (c->tc_attn) e.vt_ld = c->vt_ld;
-        rc = tune_shape(c, c->tm_xln, w.tm_qkv, M, 3 * d, d, c->tc_attn ? kEpiQkvVt : kEpiBf16, e, ev[0], ev[1]);
-      } else if (kind == 1) {
-        rc = tune_shape(c, c->tm_att, w.tm_out, M, d, d, kEpiResidF32,
-                        epi_args(w.out_b, c->h, c->mods + 2 * d, c->mod_n, c->N, nullptr), ev[0], ev[1]);
-      } else if (kind == 2) {
-        rc = tune_shape(c, c->tm_xln, w.tm_up, M, c->dff, d, kEpiGeluBf16,
-                        epi_args(w.up_b, c->u, nullptr, 0, c->N, nullptr), ev[0], ev[1]);
-      } else if (kind == 3) {
-        rc = tune_shape(c, c->tm_u, w.tm_down, M, d, c->dff, kEpiResidF32,
-                        epi_args(w.down_b, c->h, c->mods + 5 * d, c->mod_n, c->N, nullptr), ev[0], ev[1]);
-      } else {
-        rc = tune_shape(c, c->tm_obs_lp, c->tm_obs_w, M, d, d, kEpiF32,
-                        epi_args(c->obs_b, c->tune_out, nullptr, 0, c->No, nullptr), ev[0], ev[1]);
-      }
-      if (M == total) break;
-    }
-  }
-  cudaEventDestroy(ev[0]);
-  cudaEventDestroy(ev[1]);
-  CK(cudaFree(c->tune_out));
-  c->tune_out = nullptr;
-  c->tune_out_bytes = 0;
-  return rc;
-}
-
 int gemm(wam_ctx* c, const GemmOperand* ta, const void* A, const GemmOperand* tb, const void* Wt,
          int M, int N, int K, int epi, const EpiArgs& e) {
   const double out_b = (epi == kEpiResidF32) ? 8.0 : (epi == kEpiF32 ? 4.0 : (c->bf16 ? 2.0 : 4.0));
@@ -373,7 +264,7 @@ int gemm(wam_ctx* c, const GemmOperand* ta, const void* A, const GemmOperand* tb
   Span sp(c, WAM_KCLASS_GEMM, 2.0 * M * N * K, in_b * (double(M) * K + double(N) * K) + out_b * double(M) * N);
   if (c->bf16) {
     CK(tc_gemm(*ta, *tb, M, N, K, epi, e, c->num_sms, c->d_err, c->stream, nullptr,
-               gemm_plan(c, *tb, M, N, K, epi)));
+               tc_gemm_plan(M, N, K, tb->r64, false, c->num_sms)));
   } else {
     CK(simt_gemm(static_cast<const float*>(A), static_cast<const float*>(Wt), M, N, K, epi, e, c->stream));
   }
@@ -859,9 +750,6 @@ int create_impl(wam_ctx* c, const wam_config* cfg, const float* weights, size_t 
       TRY(dalloc(c, c->allocs, &vt, size_t(c->Bmax) * c->d * c->vt_ld * 2));
       CK(cudaMemsetAsync(vt, 0, size_t(c->Bmax) * c->d * c->vt_ld * 2, c->stream));
       c->vt = vt;
-      uint8_t* tvt = nullptr;
-      TRY(dalloc(c, c->allocs, &tvt, size_t(c->Bmax) * c->d * c->vt_ld * 2));
-      c->tune_vt = tvt;
       if (tc_encode_bf16_box(&c->tm_qk, c->qkv, rows, 3 * c->d, 3 * c->d, 64, 128) != 0 ||
           tc_encode_bf16_box(&c->tm_vt, c->vt, size_t(c->Bmax) * c->d, c->vt_ld, c->vt_ld, 64, 64) != 0)
         return fail(c, WAM_ERR_CUDA, "cuTensorMapEncodeTiled failed for the attention operands");
@@ -872,7 +760,6 @@ int create_impl(wam_ctx* c, const wam_config* cfg, const float* weights, size_t 
       TRY(encode(c, &w.tm_up, w.up_wt, c->dff, c->d));
       TRY(encode(c, &w.tm_down, w.down_wt, c->d, c->dff, true));
     }
-    TRY(tune_gemms(c));
   }
   CK(cudaHostAlloc(reinterpret_cast<void**>(&c->ring), kRingSlots * kSlotBytes, cudaHostAllocDefault));
   for (int i = 0; i < kRingSlots; ++i) {
@@ -887,7 +774,6 @@ int create_impl(wam_ctx* c, const wam_config* cfg, const float* weights, size_t 
 void destroy_impl(wam_ctx* c) {
   if (!c->allocs.empty()) cudaStreamSynchronize(c->stream);
   for (void* p : c->allocs) cudaFree(p);
-  if (c->tune_out != nullptr) cudaFree(c->tune_out);
   c->allocs.clear();
   if (c->ring) {
     cudaFreeHost(c->ring);
@@ -1246,6 +1132,13 @@ int wam_state_write(wam_ctx* c, wam_state* st, int32_t field, int32_t index, con
 int wam_sync(wam_ctx* c) {
   if (c == nullptr) return WAM_ERR_INVALID_ARG;
   return sync_check(c);
+}
+
+int wam_gemm_tile_width(const wam_ctx* c, int32_t M, int32_t N, int32_t K, int32_t epilogue) {
+  if (c == nullptr || M < 0 || N <= 0 || K <= 0) return WAM_ERR_INVALID_ARG;
+  if (!c->bf16) return WAM_ERR_UNSUPPORTED;
+  const bool r64 = epilogue == kEpiResidF32;   // the projections encoded with 64-row boxes
+  return tc_gemm_plan(M, N, K, r64, false, c->num_sms).bn;
 }
 
 int wam_profile_enable(wam_ctx* c, int32_t enable) {

@@ -129,6 +129,7 @@ def lib() -> ctypes.CDLL:
         "wam_op_gemm_bf16_plan": (ctypes.c_int, [_vp, _vp, _vp, _vp, _i32, _i32, _i32, _i32, _vp, ctypes.c_int64, _i32,
                                                  _i32, _i32, _vp, ctypes.c_size_t, _vp]),
         "wam_op_gemm_workspace_bytes": (ctypes.c_size_t, []),
+        "wam_gemm_tile_width": (ctypes.c_int, [_vp, _i32, _i32, _i32, _i32]),
         "wam_op_attention": (ctypes.c_int, [_vp, _vp, _i32, _i32, _i32, _i32, _i32, _vp]),
         "wam_op_ln_modulate": (ctypes.c_int, [_vp, _vp, _vp, ctypes.c_int64, _vp, _i32, _i32, _i32, _i32, _vp]),
         "wam_op_last_error": (ctypes.c_char_p, []),
@@ -273,6 +274,13 @@ class Context:
 
     def sync(self):
         self._check(lib().wam_sync(self.handle))
+
+    def gemm_tile_width(self, M: int, N: int, K: int, epilogue: int) -> int:
+        """Output tile width the context uses for this GEMM shape (chosen from the shape alone)."""
+        r = lib().wam_gemm_tile_width(self.handle, M, N, K, epilogue)
+        if r < 0:
+            self._check(r)
+        return r
 
     def log(self, st: State) -> list[dict]:
         n = _i32()
