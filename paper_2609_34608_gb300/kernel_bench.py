@@ -2,10 +2,18 @@
 
     python -m paper_2609_34608_gb300.kernel_bench gemm M N K [--iters I]
     python -m paper_2609_34608_gb300.kernel_bench attn B N H [--iters I] [--impl tc|mma]
+    python -m paper_2609_34608_gb300.kernel_bench step CONFIG [--batch B] [--rounds R] [--relax-gate]
 
 Each invocation builds the library if needed, warms up, captures `iters` back-to-back launches in
 a CUDA graph, times a replay with CUDA events and prints one JSON line (microseconds per launch
 and algorithmic TFLOP/s: 2MNK for the GEMM, 4 B N^2 d for attention).
+
+`step` drives a named model configuration (inputs.NAMED_CONFIGS) through the library's public
+calls with seeded synthetic inputs: a cold sample of all episodes, then R warm rounds, each a
+Trajectory Remapping by the configuration's shift with Observation Rebinding to new observations
+and a continuation of two steps (Residual Rescaling active; --relax-gate lets every RR check
+pass, exercising the injection path).  It prints the cold and per-round times; its launches are
+what the elementwise / adaptation profiles capture.
 """
 from __future__ import annotations
 
@@ -69,18 +77,55 @@ def bench_attn(B: int, N: int, H: int, iters: int, impl: str) -> dict:
             "tflops": 4.0 * B * N * N * d / us / 1e6}
 
 
+def bench_step(name: str, batch: int, rounds: int, relax_gate: bool) -> dict:
+    import numpy as np
+
+    from . import inputs as I
+    dev = torch.device("cuda")
+    over = dict(rr_gamma_cos=-1.0, rr_gamma_fit=1e30) if relax_gate else {}
+    cfg = I.get_config(name, batch=batch, **over)
+    K = cfg["n_steps"]
+    stream = torch.cuda.Stream()
+    ctx = W.Context(cfg, I.flatten_weights(I.make_weights(cfg)), stream=stream.cuda_stream)
+    st = ctx.state(batch)
+    shift = np.full(batch, int(cfg["shift"]), np.int32)
+    entry = np.full(batch, K - 2, np.int32)
+    with torch.cuda.stream(stream):
+        obs = [torch.from_numpy(I.make_obs(cfg, batch, seed=100 + i)).to(dev) for i in range(rounds + 1)]
+        eps = [torch.from_numpy(I.make_fresh_eps(cfg, batch, i)).to(dev) for i in range(rounds + 1)]
+        noise = torch.from_numpy(I.make_noise(cfg, batch)).to(dev)
+        e = [torch.cuda.Event(enable_timing=True) for _ in range(rounds + 2)]
+        e[0].record(stream)
+        ctx.sample_cold(st, obs[0], noise, K)
+        e[1].record(stream)
+        for r in range(rounds):
+            ctx.adapt(st, obs[r + 1], shift=shift, entry=entry, fresh_noise=eps[r + 1])
+            ctx.continue_(st, np.full(batch, 2, np.int32))
+            e[r + 2].record(stream)
+    torch.cuda.synchronize()
+    out = {"kind": "step", "config": name, "batch": batch, "cold_ms": e[0].elapsed_time(e[1]),
+           "warm_round_ms": [e[r + 1].elapsed_time(e[r + 2]) for r in range(rounds)], "stats": ctx.stats()}
+    ctx.close()
+    return out
+
+
 def main() -> None:
     ap = argparse.ArgumentParser()
-    ap.add_argument("kind", choices=["gemm", "attn"])
-    ap.add_argument("dims", type=int, nargs=3)
+    ap.add_argument("kind", choices=["gemm", "attn", "step"])
+    ap.add_argument("dims", nargs="+")
     ap.add_argument("--iters", type=int, default=20)
     ap.add_argument("--impl", choices=["tc", "mma"], default="tc")
+    ap.add_argument("--batch", type=int, default=1)
+    ap.add_argument("--rounds", type=int, default=1)
+    ap.add_argument("--relax-gate", action="store_true")
     a = ap.parse_args()
     _build.build()
     if a.kind == "gemm":
-        print(json.dumps(bench_gemm(*a.dims, a.iters)))
+        print(json.dumps(bench_gemm(*map(int, a.dims), a.iters)))
+    elif a.kind == "attn":
+        print(json.dumps(bench_attn(*map(int, a.dims), a.iters, a.impl)))
     else:
-        print(json.dumps(bench_attn(*a.dims, a.iters, a.impl)))
+        print(json.dumps(bench_step(a.dims[0], a.batch, a.rounds, a.relax_gate)))
 
 
 if __name__ == "__main__":
