@@ -92,6 +92,11 @@ struct wam_ctx {
   float *t1 = nullptr, *cvec = nullptr, *mods = nullptr;
   StepItem* d_items = nullptr;
   int* d_map = nullptr;
+  // conditioning once per distinct sigma of a step: those items, their modulation rows, and the
+  // work item -> distinct sigma index used to broadcast the rows
+  StepItem* d_uitems = nullptr;
+  int* d_uidx = nullptr;
+  float* mods_u = nullptr;
   RRApply* d_rrapply = nullptr;
   RRGate* d_gate = nullptr;
   AdaptItem* d_adapt = nullptr;
@@ -346,7 +351,8 @@ int run_steps(wam_ctx* c, wam_state* st, const std::vector<int>& n) {
   int max_n = 0;
   for (int b = 0; b < B; ++b) max_n = std::max(max_n, n[b]);
   st->log.clear();
-  std::vector<StepItem> items;
+  std::vector<StepItem> items, uitems;
+  std::vector<int> uidx;
   std::vector<int> rr_path, gate_ok;
   std::vector<RRGate> gates(2 * B);
   std::vector<RRApply> ap(B);
@@ -365,23 +371,44 @@ int run_steps(wam_ctx* c, wam_state* st, const std::vector<int>& n) {
     }
     const int Bw = static_cast<int>(items.size());
     TRY(upload(c, c->d_items, items.data(), sizeof(StepItem) * Bw));
+    // The conditioning depends on sigma alone, so it is computed once per distinct sigma of the
+    // step (exact equality: equal sigmas give bit-identical modulations) and its rows are then
+    // broadcast to the work items that share it.
+    uitems.clear();
+    uidx.assign(Bw, 0);
+    for (int w = 0; w < Bw; ++w) {
+      int j = 0;
+      while (j < static_cast<int>(uitems.size()) && uitems[j].sigma != items[w].sigma) ++j;
+      if (j == static_cast<int>(uitems.size())) uitems.push_back(items[w]);
+      uidx[w] = j;
+    }
+    const int U = static_cast<int>(uitems.size());
+    const bool share = U < Bw;
+    const StepItem* cond_items = c->d_items;
+    if (share) {
+      TRY(upload(c, c->d_uitems, uitems.data(), sizeof(StepItem) * U));
+      TRY(upload(c, c->d_uidx, uidx.data(), sizeof(int) * Bw));
+      cond_items = c->d_uitems;
+    }
     // conditioning: features -> W1 (split K) -> SiLU -> W2 (split K) -> SiLU -> every layer's
     // modulation; each stage reduces the previous stage's K-split partial rows in a fixed order
     {
-      Span sp(c, WAM_KCLASS_COND, 2.0 * Bw * 256 * d, 4.0 * 256 * d);
-      const CondGemv g{nullptr, 0, nullptr, 0, 1, c->d_items, c->t_w1, false, 256, d, Bw, kT1Splits, c->t1, nullptr};
+      Span sp(c, WAM_KCLASS_COND, 2.0 * U * 256 * d, 4.0 * 256 * d);
+      const CondGemv g{nullptr, 0, nullptr, 0, 1, cond_items, c->t_w1, false, 256, d, U, kT1Splits, c->t1, nullptr};
       CK(cond_gemv(g, c->stream));
     }
     {
-      Span sp(c, WAM_KCLASS_COND, 2.0 * Bw * d * d, 4.0 * d * d);
-      const CondGemv g{c->t1, kT1Splits, c->t_b1, 1, 0, c->d_items, c->t_w2, false, d, d, Bw, kT2Splits, c->cvec, nullptr};
+      Span sp(c, WAM_KCLASS_COND, 2.0 * U * d * d, 4.0 * d * d);
+      const CondGemv g{c->t1, kT1Splits, c->t_b1, 1, 0, cond_items, c->t_w2, false, d, d, U, kT2Splits, c->cvec, nullptr};
       CK(cond_gemv(g, c->stream));
     }
     {
-      Span sp(c, WAM_KCLASS_COND, 2.0 * Bw * d * c->mod_n, (c->bf16 ? 2.0 : 4.0) * d * c->mod_n);
-      const CondGemv g{c->cvec, kT2Splits, c->t_b2, 1, 0, c->d_items, c->mod_w, c->bf16, d, static_cast<int>(c->mod_n),
-                       Bw, 1, c->mods, c->mod_b};
+      Span sp(c, WAM_KCLASS_COND, 2.0 * U * d * c->mod_n,
+              (c->bf16 ? 2.0 : 4.0) * d * c->mod_n + (share ? 8.0 * Bw * c->mod_n : 0.0));
+      const CondGemv g{c->cvec, kT2Splits, c->t_b2, 1, 0, cond_items, c->mod_w, c->bf16, d, static_cast<int>(c->mod_n),
+                       U, 1, share ? c->mods_u : c->mods, c->mod_b};
       CK(cond_gemv(g, c->stream));
+      if (share) CK(rr_gather(c->mods, c->mods_u, c->d_uidx, Bw, c->mod_n, c->stream));
     }
     {
       Span sp(c, WAM_KCLASS_EMBED, 0.0, 4.0 * Bw * double(N) * d * 2.0);
@@ -723,6 +750,9 @@ int create_impl(wam_ctx* c, const wam_config* cfg, const float* weights, size_t 
   TRY(dalloc(c, c->allocs, &c->mods, size_t(c->Bmax) * c->mod_n));
   TRY(dalloc(c, c->allocs, &c->d_items, c->Bmax));
   TRY(dalloc(c, c->allocs, &c->d_map, c->Bmax));
+  TRY(dalloc(c, c->allocs, &c->d_uitems, c->Bmax));
+  TRY(dalloc(c, c->allocs, &c->d_uidx, c->Bmax));
+  TRY(dalloc(c, c->allocs, &c->mods_u, size_t(c->Bmax) * c->mod_n));
   TRY(dalloc(c, c->allocs, &c->d_rrapply, c->Bmax));
   TRY(dalloc(c, c->allocs, &c->d_gate, 2 * c->Bmax));
   TRY(dalloc(c, c->allocs, &c->d_adapt, c->Bmax));
