@@ -131,18 +131,18 @@ __global__ void __launch_bounds__(kThreadsAttn, 1)
     // the streams complete independently and none waits behind another's barriers.
     const uint32_t idS = idesc_bf16(kQ, kKV);
     bool ok = warp_all_wait(smem_u32(q_full), 0, abort_flag, dev_err);
-    const uint32_t sq = smem_u32(smem + kOffQ);
+    const uint64_t dq = sw128_desc(smem_u32(smem + kOffQ));
     for (int j = 0; ok && j < nkv; ++j) {
       const int s = j % kSBuf;
       const int ks = j % kKVStages;
       if (!warp_all_wait(smem_u32(&kv_full[ks]), (j / kKVStages) & 1, abort_flag, dev_err)) break;
       if (!warp_all_wait(smem_u32(&s_free[s]), ((j / kSBuf) & 1) ^ 1u, abort_flag, dev_err)) break;
       tc_fence_after();
-      const uint32_t sk = smem_u32(smem + kOffK + ks * kKBytes);
+      const uint64_t dk = sw128_desc(smem_u32(smem + kOffK + ks * kKBytes));
       if (elect_one()) {
 #pragma unroll
-        for (int t = 0; t < kDH / 16; ++t)
-          umma_bf16(tmem + s * kKV, sw128_desc(sq + t * 32), sw128_desc(sk + t * 32), idS, t > 0 ? 1u : 0u);
+        for (int t = 0; t < kDH / 16; ++t)   // descriptor address field is addr >> 4: +32 B = +2
+          umma_bf16(tmem + s * kKV, dq + 2 * t, dk + 2 * t, idS, t > 0 ? 1u : 0u);
         umma_commit(smem_u32(&s_full[s]));   // same lane as the MMAs it tracks
       }
       __syncwarp();
@@ -163,12 +163,11 @@ __global__ void __launch_bounds__(kThreadsAttn, 1)
       tc_fence_after();
       // keys 64 hv + 16t .. +15: P in columns 64 hv + 8t .. +7 of the buffer, V^T in atom column hv
       const uint32_t tp = tmem + sb * kKV + hv * 64;
-      const uint32_t sv = smem_u32(smem + kOffV + vs * kVBytes) + hv * (kVBytes / 2);
+      const uint64_t dv = sw128_desc(smem_u32(smem + kOffV + vs * kVBytes) + hv * (kVBytes / 2));
       if (elect_one()) {
 #pragma unroll
         for (int t = 0; t < 4; ++t)
-          umma_bf16_ta(tmem + kColO + hv * kDH, tp + t * 8, sw128_desc(sv + t * 32), idO,
-                       (j > 0 || t > 0) ? 1u : 0u);
+          umma_bf16_ta(tmem + kColO + hv * kDH, tp + t * 8, dv + 2 * t, idO, (j > 0 || t > 0) ? 1u : 0u);
         umma_commit(smem_u32(&s_free[sb]));   // same lane as the MMAs they track
         umma_commit(smem_u32(&kv_empty[vs]));
       }

@@ -306,15 +306,17 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         tc_fence_after();
         const uint32_t a0 = smem_u32(tiles + stage * C::kStageBytes);
-        const uint32_t b0 = a0 + C::kBytesA;
+        // One descriptor per operand and stage; the address field holds addr >> 4 and shared
+        // memory stays below 256 KB, so an offset is one add of (offset >> 4).
+        const uint64_t da = sw128_desc(a0), db = sw128_desc(a0 + C::kBytesA);
 #pragma unroll
         for (int a = 0; a < KA; ++a) {
 #pragma unroll
           for (int k = 0; k < kBK / 16; ++k) {
 #pragma unroll
             for (int h = 0; h < BN / C::kMmaN; ++h)
-              umma_bf16(d_tmem + h * C::kMmaN, sw128_desc(a0 + a * kTileBytesA + k * 32),
-                        sw128_desc(b0 + h * C::kBoxBytesB + a * C::kBoxB * 128 + k * 32), idesc,
+              umma_bf16(d_tmem + h * C::kMmaN, da + ((a * kTileBytesA + k * 32) >> 4),
+                        db + ((h * C::kBoxBytesB + a * C::kBoxB * 128 + k * 32) >> 4), idesc,
                         (kb | a | k) != 0 ? 1u : 0u);
           }
         }
