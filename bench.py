@@ -13,7 +13,9 @@ Printed JSON line: `value` = action chunks/s with every input already resident i
 steps after it); `cold` = a native cold 10-step sample; `e2e` = the same control loop through
 the C ABI with pinned host buffers (host<->device copies inside the timed region);
 `roofline` = the dominant kernel class (tcgen05 GEMM) against the measured bf16 peak;
-`cpu_baseline` = the float64 CPU oracle on the host cores for one control step.
+`ablation` = the same control steps with the layer stack launched kernel by kernel instead of
+replayed from CUDA graphs; `cpu_baseline` = the float64 CPU oracle on the host cores for one
+control step.
 
 Usage: python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
 Multi-GPU (torchrun): one replica per rank, no collective on the data path (the work is
@@ -342,6 +344,21 @@ def main_ours(args):
     torch.cuda.synchronize(dev)
     cold_ms = [a.elapsed_time(b) for a, b in cold_ms][1:]
 
+    # ---- ablation: the same control steps with every kernel launched individually ------
+    # (CUDA-graph replay of the layer stack off; the paper's Table 3 "Graph" switch)
+    st = st_keep
+    n_abl = min(args.steps, 50)
+    ctx.set_graph_replay(False)
+    a0, a1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    with torch.cuda.stream(stream):
+        a0.record(stream)
+        for i in range(n_abl):
+            control_step(dev_in[args.warmup + i], act_dev)
+        a1.record(stream)
+    torch.cuda.synchronize(dev)
+    ctx.set_graph_replay(True)
+    abl_ms = a0.elapsed_time(a1) / n_abl
+
     # ---- kernel-class timing (CUDA events on the library's stream) --------------------
     st = st_keep
     ctx.profile_enable(True)
@@ -373,6 +390,8 @@ def main_ours(args):
                        "o2a_p50": float(np.percentile(o2a_ms, 50)), "o2a_p99": float(np.percentile(o2a_ms, 99))},
         "cold": {"ms_p50": float(np.percentile(cold_ms, 50)), "chunks_per_s": 1000.0 / float(np.percentile(cold_ms, 50)),
                  "what": "native cold 10-step sample of the same model, RR active after the first step"},
+        "ablation": {"graph_replay_off": {"chunks_per_s": 1000.0 / abl_ms, "ms_per_step": abl_ms, "steps": n_abl,
+                                          "what": "same control steps, every kernel launched individually"}},
         "reuse": {"r_rr": stats["n_reuse"] / max(1, stats["n_attempt"]), "f_skip": stats["b_skip"] / max(1, stats["b_dense"]),
                   "r_or": stats["n_bind"] / max(1, stats["n_start"]), "coverage": stats["n_bind"] / max(1, stats["n_noninitial"])},
         "roofline": {"bound": "tensor", "kernel": "tcgen05 GEMM (QKV / out / MLP projections)",

@@ -258,6 +258,16 @@ int wam_profile_enable(wam_ctx* ctx, int32_t enable);
 int wam_profile_read(wam_ctx* ctx, wam_kclass_timing* out /* [WAM_KCLASS_COUNT] */);
 
 /*
+ * CUDA-graph replay of the layer stack (default on).  Each contiguous range of DiT layers a step
+ * runs (all layers; or the head, the gathered middle and the tail around Residual Rescaling) is
+ * captured into a CUDA graph the second time the same range, batch width and buffers occur, and
+ * replayed from then on; host decisions (RR gate, OR rule, TR bookkeeping) stay outside the graphs,
+ * as in the paper (§4, App. D).  enable = 0 launches every kernel individually (the ablation).
+ * Results are identical either way.
+ */
+int wam_set_graph_replay(wam_ctx* ctx, int32_t enable);
+
+/*
  * Output tile width (64, 128 or 256 columns) the context's bf16 path uses for the GEMM
  * [M, K] x [K, N] with the given epilogue (WAM_EPI_*, or 4 for the QKV projection that also
  * writes V^T), chosen from the shape alone: 64 while 128-wide tiles cannot fill the SMs, 256 from

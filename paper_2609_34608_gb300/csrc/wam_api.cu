@@ -8,8 +8,10 @@
 #include <cmath>
 #include <cstdio>
 #include <cstring>
+#include <map>
 #include <new>
 #include <string>
+#include <tuple>
 #include <vector>
 
 #include "kernels.cuh"
@@ -94,6 +96,12 @@ struct wam_ctx {
   int* d_map = nullptr;
   // conditioning once per distinct sigma of a step: those items, their modulation rows, and the
   // work item -> distinct sigma index used to broadcast the rows
+  // CUDA graphs of layer ranges: key (first layer, end layer, episodes, stream buffer, item map,
+  // layer that also saves h_q or -1) -> executable graph, captured on a range's second use
+  bool graph_replay = true;
+  bool graphs_ok = true;
+  std::map<std::tuple<int, int, int, const void*, const void*, int>, cudaGraphExec_t> layer_graphs;
+  std::map<std::tuple<int, int, int, const void*, const void*, int>, int> layer_graph_uses;
   StepItem* d_uitems = nullptr;
   int* d_uidx = nullptr;
   float* mods_u = nullptr;
@@ -318,6 +326,49 @@ int run_layer(wam_ctx* c, int l, float* hb, int Bw, const int* map, float* hcopy
   return WAM_OK;
 }
 
+// Layers [l0, l1) of the episodes in hb (item map `map`, or none), saving h_q at layer `hq_layer`
+// (or -1).  The ~7 launches per layer have fixed arguments for a given key, so a range is
+// captured into a CUDA graph on its second use (the first runs eagerly, which also sets every
+// kernel attribute outside capture) and replayed afterwards: one graph launch instead of the
+// per-kernel launch gaps.  Profiling (per-kernel events) and a failed capture run eagerly.
+int run_layers(wam_ctx* c, int l0, int l1, float* hb, int Bw, const int* map, int hq_layer) {
+  if (l0 >= l1) return WAM_OK;
+  auto eager = [&]() -> int {
+    for (int l = l0; l < l1; ++l) TRY(run_layer(c, l, hb, Bw, map, l == hq_layer ? c->hq : nullptr));
+    return WAM_OK;
+  };
+  if (!c->graph_replay || !c->graphs_ok || c->prof_on) return eager();
+  const auto key = std::make_tuple(l0, l1, Bw, static_cast<const void*>(hb), static_cast<const void*>(map), hq_layer);
+  const auto hit = c->layer_graphs.find(key);
+  if (hit != c->layer_graphs.end()) {
+    CK(cudaGraphLaunch(hit->second, c->stream));
+    return WAM_OK;
+  }
+  if (++c->layer_graph_uses[key] < 2) return eager();
+  cudaGraph_t g = nullptr;
+  if (cudaStreamBeginCapture(c->stream, cudaStreamCaptureModeThreadLocal) != cudaSuccess) {
+    cudaGetLastError();
+    c->graphs_ok = false;
+    return eager();
+  }
+  int rc = WAM_OK;
+  for (int l = l0; l < l1 && rc == WAM_OK; ++l) rc = run_layer(c, l, hb, Bw, map, l == hq_layer ? c->hq : nullptr);
+  const cudaError_t ec = cudaStreamEndCapture(c->stream, &g);
+  cudaGraphExec_t ex = nullptr;
+  if (rc == WAM_OK && ec == cudaSuccess && g != nullptr && cudaGraphInstantiate(&ex, g, 0) == cudaSuccess) {
+    cudaGraphDestroy(g);
+    c->layer_graphs[key] = ex;
+    CK(cudaGraphLaunch(ex, c->stream));
+    return WAM_OK;
+  }
+  // Capture not possible here: nothing of it ran; run the range eagerly from now on.
+  if (g != nullptr) cudaGraphDestroy(g);
+  cudaGetLastError();
+  c->err.clear();
+  c->graphs_ok = false;
+  return eager();
+}
+
 int obs_embed(wam_ctx* c, wam_state* st) {
   const int M = st->B * c->No;
   if (c->bf16) {
@@ -435,9 +486,9 @@ int run_steps(wam_ctx* c, wam_state* st, const std::vector<int>& n) {
     }
     std::vector<int> accepted(Bw, 0);
     if (!any_rr) {
-      for (int l = 0; l < L; ++l) TRY(run_layer(c, l, c->h, Bw, nullptr, nullptr));
+      TRY(run_layers(c, 0, L, c->h, Bw, nullptr, -1));
     } else {
-      for (int l = 0; l < s; ++l) TRY(run_layer(c, l, c->h, Bw, nullptr, l == q ? c->hq : nullptr));
+      TRY(run_layers(c, 0, s, c->h, Bw, nullptr, q));
       if (any_gate) {
         const int nch = rr_num_chunks(int64_t(std::max(split_row, N - split_row)) * d);
         {
@@ -474,7 +525,7 @@ int run_steps(wam_ctx* c, wam_state* st, const std::vector<int>& n) {
           Span sp(c, WAM_KCLASS_RR_APPLY, 0.0, 8.0 * nmid * double(N) * d);
           CK(rr_gather(c->hm, c->h, c->d_map, nmid, int64_t(N) * d, c->stream));
         }
-        for (int l = s; l < e; ++l) TRY(run_layer(c, l, c->hm, nmid, c->d_map, nullptr));
+        TRY(run_layers(c, s, e, c->hm, nmid, c->d_map, -1));
       }
       TRY(upload(c, c->d_rrapply, ap.data(), sizeof(RRApply) * Bw));
       {
@@ -485,7 +536,7 @@ int run_steps(wam_ctx* c, wam_state* st, const std::vector<int>& n) {
         Span sp(c, WAM_KCLASS_RR_APPLY, 0.0, per * double(N) * d);
         CK(rr_apply(c->h, c->hm, c->hq, st->pa, st->ra, c->d_items, c->d_rrapply, Bw, N, d, split_row, c->stream));
       }
-      for (int l = e; l < L; ++l) TRY(run_layer(c, l, c->h, Bw, nullptr, nullptr));
+      TRY(run_layers(c, e, L, c->h, Bw, nullptr, -1));
     }
     {
       Span sp(c, WAM_KCLASS_FINAL, 2.0 * Bw * double(c->Nv * c->vd + c->Na * c->ad) * d,
@@ -803,6 +854,8 @@ int create_impl(wam_ctx* c, const wam_config* cfg, const float* weights, size_t 
 
 void destroy_impl(wam_ctx* c) {
   if (!c->allocs.empty()) cudaStreamSynchronize(c->stream);
+  for (auto& kv : c->layer_graphs) cudaGraphExecDestroy(kv.second);
+  c->layer_graphs.clear();
   for (void* p : c->allocs) cudaFree(p);
   c->allocs.clear();
   if (c->ring) {
@@ -1162,6 +1215,12 @@ int wam_state_write(wam_ctx* c, wam_state* st, int32_t field, int32_t index, con
 int wam_sync(wam_ctx* c) {
   if (c == nullptr) return WAM_ERR_INVALID_ARG;
   return sync_check(c);
+}
+
+int wam_set_graph_replay(wam_ctx* c, int32_t enable) {
+  if (c == nullptr) return WAM_ERR_INVALID_ARG;
+  c->graph_replay = enable != 0;
+  return WAM_OK;
 }
 
 int wam_gemm_tile_width(const wam_ctx* c, int32_t M, int32_t N, int32_t K, int32_t epilogue) {

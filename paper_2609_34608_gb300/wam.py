@@ -130,6 +130,7 @@ def lib() -> ctypes.CDLL:
                                                  _i32, _i32, _vp, ctypes.c_size_t, _vp]),
         "wam_op_gemm_workspace_bytes": (ctypes.c_size_t, []),
         "wam_gemm_tile_width": (ctypes.c_int, [_vp, _i32, _i32, _i32, _i32]),
+        "wam_set_graph_replay": (ctypes.c_int, [_vp, _i32]),
         "wam_op_attention": (ctypes.c_int, [_vp, _vp, _i32, _i32, _i32, _i32, _i32, _vp]),
         "wam_op_ln_modulate": (ctypes.c_int, [_vp, _vp, _vp, ctypes.c_int64, _vp, _i32, _i32, _i32, _i32, _vp]),
         "wam_op_last_error": (ctypes.c_char_p, []),
@@ -274,6 +275,10 @@ class Context:
 
     def sync(self):
         self._check(lib().wam_sync(self.handle))
+
+    def set_graph_replay(self, enable: bool):
+        """CUDA-graph replay of the layer stack (default on); off launches every kernel."""
+        self._check(lib().wam_set_graph_replay(self.handle, 1 if enable else 0))
 
     def gemm_tile_width(self, M: int, N: int, K: int, epilogue: int) -> int:
         """Output tile width the context uses for this GEMM shape (chosen from the shape alone)."""
