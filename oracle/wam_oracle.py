@@ -17,7 +17,9 @@ States", arXiv 2609.34608):
   normaliser),
 * Observation Rebinding (§3.2, Eq. 4 consistency score and the kappa rule),
 * Residual Rescaling (§3.3, Eqs. 5-9),
-* the coordinating state machine (§3.4) and the reuse statistics (App. D.2, Eqs. 14-15).
+* the coordinating state machine (§3.4) and the reuse statistics (App. D.2, Eqs. 14-15),
+* the state-continuity diagnostics (App. E): latent similarity across replans, action RMSE and
+  the per-layer hidden-state change.
 
 Precision: every array is promoted to float64 and every reduction is a float64 numpy reduction.
 
@@ -604,6 +606,32 @@ class OracleEpisode:
     def actions(self):
         cfg = self.cfg
         return self.hist[cfg.n_steps][cfg.video_len:].reshape(cfg.n_action, cfg.action_dim)
+
+
+def latent_similarity(x_t, x_prev):
+    """App. E trajectory diagnostic: cosine similarity and relative L2 distance between the latent
+    of the current replan x_t^r and the preceding replan's x_{t-1}^r at the same stage; the
+    preceding latent is the reference of the relative distance."""
+    a = np.asarray(x_t, dtype=F64).ravel()
+    b = np.asarray(x_prev, dtype=F64).ravel()
+    na, nb = float(np.linalg.norm(a)), float(np.linalg.norm(b))
+    cos = float(a @ b) / (na * nb) if na > 0.0 and nb > 0.0 else 0.0
+    dist = float(np.linalg.norm(a - b))
+    rel = dist / nb if nb > 0.0 else (0.0 if dist == 0.0 else math.inf)
+    return cos, rel
+
+
+def layer_deltas(W, cfg: OracleConfig, x_traj, obs, sigma: float):
+    """App. E layer diagnostic: relative L2 change of the hidden state across each layer of the
+    full forward at sigma, Delta_l = ||h_{l+1} - h_l|| / ||h_l|| with h_0 the token embedding."""
+    mods, _ = conditioning(W, cfg, sigma)
+    h = embed(W, cfg, x_traj, obs)
+    out = []
+    for l in range(cfg.n_layers):
+        h1 = dit_layer(W, cfg, h, l, mods[l])
+        out.append(float(np.linalg.norm(h1 - h) / np.linalg.norm(h)))
+        h = h1
+    return out
 
 
 def action_rmse(a, b, dims=None):

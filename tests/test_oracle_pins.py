@@ -456,3 +456,60 @@ def test_reuse_rates_definitions():
     s = O.Stats(n_attempt=8, n_reuse=6, b_skip=24, b_dense=96, n_start=5, n_bind=4, n_noninitial=9)
     r = s.rates()
     assert r == dict(r_rr=0.75, f_skip=0.25, r_or=0.8, coverage=4 / 9)
+
+
+# ----------------------------------------------------------------------------- diagnostics (App. E)
+def test_latent_similarity_closed_forms_and_bruteforce():
+    rng = np.random.default_rng(11)
+    a = rng.standard_normal(37)
+    assert O.latent_similarity(a, a) == pytest.approx((1.0, 0.0), abs=1e-15)
+    assert O.latent_similarity(2.0 * a, a) == pytest.approx((1.0, 1.0), abs=1e-15)
+    assert O.latent_similarity(-a, a) == pytest.approx((-1.0, 2.0), abs=1e-15)
+    e1, e2 = np.eye(4)[0] * 3.0, np.eye(4)[1] * 4.0
+    assert O.latent_similarity(e1, e2) == pytest.approx((0.0, 5.0 / 4.0), abs=1e-15)   # 3-4-5 triangle
+    b = rng.standard_normal(37)
+    dot = sum(float(x) * float(y) for x, y in zip(a, b))
+    na = math.sqrt(sum(float(x) ** 2 for x in a))
+    nb = math.sqrt(sum(float(y) ** 2 for y in b))
+    dd = math.sqrt(sum((float(x) - float(y)) ** 2 for x, y in zip(a, b)))
+    cos, rel = O.latent_similarity(a, b)
+    assert cos == pytest.approx(dot / (na * nb), rel=1e-13) and rel == pytest.approx(dd / nb, rel=1e-13)
+
+
+def test_action_rmse_constant_offset_and_ignored_dims():
+    rng = np.random.default_rng(12)
+    b = rng.standard_normal((16, 7))
+    assert O.action_rmse(b + 0.25, b, dims=6) == pytest.approx(0.25, abs=1e-15)
+    a = b.copy()
+    a[:, 6] += 9.0                     # only the dimension outside the first six differs
+    assert O.action_rmse(a, b, dims=6) == 0.0
+    assert O.action_rmse(a, b) == pytest.approx(9.0 / math.sqrt(7.0), abs=1e-12)
+
+
+def _zero_gate_weights(W, cfg, which):
+    d = cfg.d_model
+    for l in range(cfg.n_layers):
+        for g in which:   # modulation rows 2 (attention gate) and 5 (MLP gate)
+            W[f"layers.{l}.ada_w"][:, g * d:(g + 1) * d] = 0.0
+            W[f"layers.{l}.ada_b"][g * d:(g + 1) * d] = 0.0
+    return W
+
+
+def test_layer_deltas_zero_gates_and_gate_scaling():
+    cfgd = micro_config()
+    W, cfg = _setup(cfgd, std=0.2)
+    rng = np.random.default_rng(13)
+    x = rng.standard_normal(cfg.traj_len)
+    obs = rng.standard_normal((cfg.n_obs, cfg.d_model))
+    Wz = _zero_gate_weights({k: v.copy() for k, v in W.items()}, cfg, (2, 5))
+    assert O.layer_deltas(Wz, cfg, x, obs, 0.6) == [0.0] * cfg.n_layers
+    # with the MLP gate zero a layer adds g1 * Attn(...): scaling the attention-gate weights by c
+    # scales the first layer's change by |c|
+    W1 = _zero_gate_weights({k: v.astype(np.float64) for k, v in W.items()}, cfg, (5,))   # exact scaling
+    W2 = {k: v.copy() for k, v in W1.items()}
+    d = cfg.d_model
+    W2["layers.0.ada_w"][:, 2 * d:3 * d] *= -3.0
+    W2["layers.0.ada_b"][2 * d:3 * d] *= -3.0
+    d1 = O.layer_deltas(W1, cfg, x, obs, 0.6)[0]
+    d2 = O.layer_deltas(W2, cfg, x, obs, 0.6)[0]
+    assert d1 > 0.0 and d2 == pytest.approx(3.0 * d1, rel=1e-12)
