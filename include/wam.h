@@ -258,6 +258,30 @@ int wam_profile_enable(wam_ctx* ctx, int32_t enable);
 int wam_profile_read(wam_ctx* ctx, wam_kclass_timing* out /* [WAM_KCLASS_COUNT] */);
 
 /*
+ * State-continuity diagnostics (paper App. E), computed on the device in float64.  Inputs may be
+ * host or device pointers; the calls synchronise the context's stream and return the values.
+ *
+ * wam_diag_similarity: cosine similarity <a,b>/(|a||b|) and relative L2 distance |a-b|/|b| of
+ *   two vectors of n floats (App. E: the latent x_t^r of the current replan against the
+ *   preceding replan's x_{t-1}^r at the same stage r, the preceding one being b).  A zero-norm
+ *   input gives cos 0; |b| = 0 gives rel_l2 0 if a == b, else HUGE_VAL.
+ * wam_diag_action_rmse: sqrt(mean over rows j and the first `dims` of each row's `row_len`
+ *   values of (a - b)^2) (App. E Eq. 17 with dims = 6; actions [n_rows, row_len]).
+ * wam_diag_layer_deltas: for one episode of a state at its pending stage k (0 <= k < K), runs
+ *   the full forward at sigma_k on its current latent and bound observation and writes
+ *   out[l] = |h_{l+1} - h_l| / |h_l| for every layer l (h_0 = the token embedding), the hidden
+ *   state change of App. E.  The state is not modified (context scratch only).
+ * n (resp. n_rows * row_len) is at most batch_max * tokens * d_model.  Errors:
+ * WAM_ERR_INVALID_ARG (null, sizes), WAM_ERR_BAD_STATE (episode finished or not started).
+ */
+int wam_diag_similarity(wam_ctx* ctx, const float* a, const float* b, int64_t n, double* cos_out,
+                        double* rel_l2_out);
+int wam_diag_action_rmse(wam_ctx* ctx, const float* a, const float* b, int32_t n_rows,
+                         int32_t row_len, int32_t dims, double* out);
+int wam_diag_layer_deltas(wam_ctx* ctx, wam_state* state, int32_t episode,
+                          double* out /* [n_layers] */);
+
+/*
  * CUDA-graph replay of the layer stack (default on).  Each contiguous range of DiT layers a step
  * runs (all layers; or the head, the gathered middle and the tail around Residual Rescaling) is
  * captured into a CUDA graph the second time the same range, batch width and buffers occur, and

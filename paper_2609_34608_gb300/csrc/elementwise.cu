@@ -627,6 +627,38 @@ __global__ void __launch_bounds__(256) rr_gather_kernel(float* __restrict__ hm, 
     dst[i] = src[i];
 }
 
+// ---------------------------------------------------------------- diagnostics (App. E)
+// Per-block float64 partial sums of a.b, a.a, b.b and (a-b).(a-b) over the elements i < n whose
+// column i mod row_len is below cols (row_len = cols = n for a whole vector).
+__global__ void __launch_bounds__(256) diag_partial_kernel(const float* __restrict__ a, const float* __restrict__ b,
+                                                           int64_t n, int64_t row_len, int64_t cols,
+                                                           double* __restrict__ partial) {
+  pdl_wait();
+  pdl_launch_dependents();
+  __shared__ double red[8];
+  double s0 = 0.0, s1 = 0.0, s2 = 0.0, s3 = 0.0;
+  for (int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; i < n;
+       i += static_cast<int64_t>(gridDim.x) * blockDim.x) {
+    if (i % row_len >= cols) continue;
+    const double x = a[i], y = b[i], e = x - y;
+    s0 += x * y;
+    s1 += x * x;
+    s2 += y * y;
+    s3 += e * e;
+  }
+  s0 = block_sum_d(s0, red);
+  s1 = block_sum_d(s1, red);
+  s2 = block_sum_d(s2, red);
+  s3 = block_sum_d(s3, red);
+  if (threadIdx.x == 0) {
+    double* p = partial + static_cast<int64_t>(blockIdx.x) * 4;
+    p[0] = s0;
+    p[1] = s1;
+    p[2] = s2;
+    p[3] = s3;
+  }
+}
+
 // ---------------------------------------------------------------- preparation
 __global__ void cast_kernel(const float* __restrict__ in, bf16* __restrict__ out, int64_t n) {
   pdl_wait();
@@ -866,6 +898,13 @@ cudaError_t rr_gather(float* hm, const float* h, const int* map, int nmid, int64
   const int64_t item4 = item_elems / 4;
   const int bx = static_cast<int>((item4 + 255) / 256 < 512 ? (item4 + 255) / 256 : 512);
   launch_pdl(rr_gather_kernel, dim3(bx, nmid), dim3(256), 0, s, hm, h, map, item4);
+  return cudaGetLastError();
+}
+
+cudaError_t diag_partial(const float* a, const float* b, int64_t n, int64_t row_len, int64_t cols, int nblocks,
+                         double* partial, cudaStream_t s) {
+  if (n <= 0 || nblocks <= 0 || row_len <= 0) return cudaErrorInvalidValue;
+  launch_pdl(diag_partial_kernel, dim3(nblocks), dim3(256), 0, s, a, b, n, row_len, cols, partial);
   return cudaGetLastError();
 }
 

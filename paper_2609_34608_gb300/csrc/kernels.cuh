@@ -100,6 +100,10 @@ cudaError_t rr_gate(const double* partial, int Bw, int nch, int64_t n0, int64_t 
                     cudaStream_t s);
 // hm[c] = h[map[c]] for the nmid items that run the middle layers (rows of N*d floats)
 cudaError_t rr_gather(float* hm, const float* h, const int* map, int nmid, int64_t item_elems, cudaStream_t s);
+// App. E diagnostics: nblocks x {a.b, a.a, b.b, (a-b).(a-b)} float64 partials over the elements
+// whose column (index mod row_len) is below cols.
+cudaError_t diag_partial(const float* a, const float* b, int64_t n, int64_t row_len, int64_t cols, int nblocks,
+                         double* partial, cudaStream_t s);
 cudaError_t rr_apply(float* h, const float* hm, const float* hq, float* pa, float* ra,
                      const StepItem* items, const RRApply* ap, int Bw, int N, int d,
                      int split_row, cudaStream_t s);

@@ -1217,6 +1217,97 @@ int wam_sync(wam_ctx* c) {
   return sync_check(c);
 }
 
+// ------------------------------------------------------------------- diagnostics (App. E)
+namespace {
+
+// {a.b, a.a, b.b, (a-b).(a-b)} in float64 over the elements whose column (index mod row_len) is
+// below cols; host inputs are staged into the context's scratch first.  Blocks' partials are
+// summed on the host in block order.
+int diag_sums(wam_ctx* c, const float* a, const float* b, int64_t n, int64_t row_len, int64_t cols, double out[4]) {
+  const size_t cap = size_t(c->Bmax) * c->N * c->d;
+  if (n <= 0 || size_t(n) > cap) return fail(c, WAM_ERR_INVALID_ARG, "diagnostic length outside [1, batch_max*tokens*d_model]");
+  const float* da = a;
+  const float* db = b;
+  if (!is_device_ptr(a)) {
+    CK(cudaMemcpyAsync(c->hq, a, size_t(n) * sizeof(float), cudaMemcpyHostToDevice, c->stream));
+    da = c->hq;
+  }
+  if (!is_device_ptr(b)) {
+    CK(cudaMemcpyAsync(c->hm, b, size_t(n) * sizeof(float), cudaMemcpyHostToDevice, c->stream));
+    db = c->hm;
+  }
+  int nb = static_cast<int>(std::min<int64_t>(256, (n + 1023) / 1024));
+  nb = std::max(1, std::min<int>(nb, static_cast<int>(c->part_doubles / 4)));
+  CK(diag_partial(da, db, n, row_len, cols, nb, c->d_part, c->stream));
+  std::vector<double> p(size_t(nb) * 4);
+  TRY(readback(c, p.data(), c->d_part, sizeof(double) * p.size()));
+  for (int q = 0; q < 4; ++q) out[q] = 0.0;
+  for (int i = 0; i < nb; ++i)
+    for (int q = 0; q < 4; ++q) out[q] += p[size_t(i) * 4 + q];
+  return WAM_OK;
+}
+
+}  // namespace
+
+int wam_diag_similarity(wam_ctx* c, const float* a, const float* b, int64_t n, double* cos_out, double* rel_l2_out) {
+  if (c == nullptr || a == nullptr || b == nullptr || cos_out == nullptr || rel_l2_out == nullptr) return WAM_ERR_INVALID_ARG;
+  double v[4];
+  TRY(diag_sums(c, a, b, n, n, n, v));
+  const double na = std::sqrt(v[1]), nb = std::sqrt(v[2]), dist = std::sqrt(v[3]);
+  *cos_out = (na > 0.0 && nb > 0.0) ? v[0] / (na * nb) : 0.0;
+  *rel_l2_out = nb > 0.0 ? dist / nb : (dist == 0.0 ? 0.0 : HUGE_VAL);
+  return WAM_OK;
+}
+
+int wam_diag_action_rmse(wam_ctx* c, const float* a, const float* b, int32_t n_rows, int32_t row_len, int32_t dims,
+                         double* out) {
+  if (c == nullptr || a == nullptr || b == nullptr || out == nullptr || n_rows <= 0 || row_len <= 0 || dims <= 0 ||
+      dims > row_len)
+    return WAM_ERR_INVALID_ARG;
+  double v[4];
+  TRY(diag_sums(c, a, b, int64_t(n_rows) * row_len, row_len, dims, v));
+  *out = std::sqrt(v[3] / (double(n_rows) * dims));
+  return WAM_OK;
+}
+
+int wam_diag_layer_deltas(wam_ctx* c, wam_state* st, int32_t episode, double* out) {
+  if (c == nullptr || st == nullptr || st->ctx != c || out == nullptr || episode < 0 || episode >= st->B)
+    return WAM_ERR_INVALID_ARG;
+  const int k = st->meta[episode].stage;
+  if (k < 0 || k >= c->K) return fail(c, WAM_ERR_BAD_STATE, "the episode has no pending denoising stage");
+  const int d = c->d, N = c->N;
+  StepItem it;
+  it.ep = episode;
+  it.stage = k;
+  it.sigma = c->sigma[k];
+  it.dsigma = c->sigma[k + 1] - c->sigma[k];
+  TRY(upload(c, c->d_items, &it, sizeof(StepItem)));
+  {
+    const CondGemv g{nullptr, 0, nullptr, 0, 1, c->d_items, c->t_w1, false, 256, d, 1, kT1Splits, c->t1, nullptr};
+    CK(cond_gemv(g, c->stream));
+  }
+  {
+    const CondGemv g{c->t1, kT1Splits, c->t_b1, 1, 0, c->d_items, c->t_w2, false, d, d, 1, kT2Splits, c->cvec, nullptr};
+    CK(cond_gemv(g, c->stream));
+  }
+  {
+    const CondGemv g{c->cvec, kT2Splits, c->t_b2, 1, 0, c->d_items, c->mod_w, c->bf16, d, static_cast<int>(c->mod_n),
+                     1, 1, c->mods, c->mod_b};
+    CK(cond_gemv(g, c->stream));
+  }
+  // the embedding records the latent it reads: point that record at scratch (stage stride 0)
+  CK(embed_tokens(c->h, c->hq, 0, c->d_items, st->x, c->T, st->obs_emb, c->vid_w, c->vid_b, c->act_w, c->act_b,
+                  c->pos, 1, c->No, c->Nv, c->vd, c->Na, c->ad, d, c->stream));
+  for (int l = 0; l < c->L; ++l) {
+    CK(cudaMemcpyAsync(c->hm, c->h, size_t(N) * d * sizeof(float), cudaMemcpyDeviceToDevice, c->stream));
+    TRY(run_layer(c, l, c->h, 1, nullptr, nullptr));
+    double v[4];
+    TRY(diag_sums(c, c->h, c->hm, int64_t(N) * d, int64_t(N) * d, int64_t(N) * d, v));
+    out[l] = std::sqrt(v[3]) / std::sqrt(v[2]);
+  }
+  return WAM_OK;
+}
+
 int wam_set_graph_replay(wam_ctx* c, int32_t enable) {
   if (c == nullptr) return WAM_ERR_INVALID_ARG;
   c->graph_replay = enable != 0;

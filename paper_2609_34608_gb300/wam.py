@@ -131,6 +131,9 @@ def lib() -> ctypes.CDLL:
         "wam_op_gemm_workspace_bytes": (ctypes.c_size_t, []),
         "wam_gemm_tile_width": (ctypes.c_int, [_vp, _i32, _i32, _i32, _i32]),
         "wam_set_graph_replay": (ctypes.c_int, [_vp, _i32]),
+        "wam_diag_similarity": (ctypes.c_int, [_vp, _vp, _vp, ctypes.c_int64, _vp, _vp]),
+        "wam_diag_action_rmse": (ctypes.c_int, [_vp, _vp, _vp, _i32, _i32, _i32, _vp]),
+        "wam_diag_layer_deltas": (ctypes.c_int, [_vp, _vp, _i32, _vp]),
         "wam_op_attention": (ctypes.c_int, [_vp, _vp, _i32, _i32, _i32, _i32, _i32, _vp]),
         "wam_op_ln_modulate": (ctypes.c_int, [_vp, _vp, _vp, ctypes.c_int64, _vp, _i32, _i32, _i32, _i32, _vp]),
         "wam_op_last_error": (ctypes.c_char_p, []),
@@ -275,6 +278,27 @@ class Context:
 
     def sync(self):
         self._check(lib().wam_sync(self.handle))
+
+    def diag_similarity(self, a, b) -> tuple[float, float]:
+        """App. E: (cosine, relative L2 against b) of two float32 vectors (host or device)."""
+        c, r = ctypes.c_double(), ctypes.c_double()
+        n = a.numel() if hasattr(a, "numel") else int(np.asarray(a).size)
+        self._check(lib().wam_diag_similarity(self.handle, ptr(a), ptr(b), n, ctypes.byref(c), ctypes.byref(r)))
+        return c.value, r.value
+
+    def diag_action_rmse(self, a, b, dims: int = 6) -> float:
+        """App. E Eq. 17: RMSE over the first `dims` values of each action row."""
+        shape = tuple(a.shape)
+        out = ctypes.c_double()
+        self._check(lib().wam_diag_action_rmse(self.handle, ptr(a), ptr(b), int(np.prod(shape[:-1])), int(shape[-1]),
+                                               int(dims), ctypes.byref(out)))
+        return out.value
+
+    def diag_layer_deltas(self, st: "State", episode: int) -> np.ndarray:
+        """App. E: relative hidden-state change across each layer at the episode's pending stage."""
+        out = np.zeros(int(self.cfg["n_layers"]), dtype=np.float64)
+        self._check(lib().wam_diag_layer_deltas(self.handle, st.handle, int(episode), out.ctypes.data))
+        return out
 
     def set_graph_replay(self, enable: bool):
         """CUDA-graph replay of the layer stack (default on); off launches every kernel."""
