@@ -14,7 +14,8 @@ steps after it); `cold` = a native cold 10-step sample; `e2e` = the same control
 the C ABI with pinned host buffers (host<->device copies inside the timed region);
 `roofline` = the dominant kernel class (tcgen05 GEMM) against the measured bf16 peak;
 `ablation` = the same control steps with the layer stack launched kernel by kernel instead of
-replayed from CUDA graphs; `cpu_baseline` = the float64 CPU oracle on the host cores for one
+replayed from CUDA graphs; `independent` = the separate video / action models of independent
+execution, their continuations overlapped on two streams and in sequence; `cpu_baseline` = the float64 CPU oracle on the host cores for one
 control step.
 
 Usage: python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
@@ -369,11 +370,13 @@ def main_ours(args):
     prof = ctx.profile_read()
     ctx.profile_enable(False)
 
-    serving = serving_rr = None
+    serving = serving_rr = independent = None
     if not args.no_serving:
         ctx.close()
         serving = run_serving(dev, stream, _peaks())
         serving_rr = run_serving(dev, stream, _peaks(), relax_gate=True)
+    if not args.no_independent:
+        independent = run_independent(dev)
 
     if rank != 0:
         return 0
@@ -408,6 +411,8 @@ def main_ours(args):
     if serving is not None:
         line["serving"] = serving
         line["serving_rr_accept"] = serving_rr
+    if independent is not None:
+        line["independent"] = independent
     if cpu_times:
         ct = cpu_times[-1]
         line["cpu_baseline"] = {"value": 1.0 / ct, "unit": "chunks/s", "cores": cpu_cores, "kind": "oracle",
@@ -484,6 +489,112 @@ def run_serving(dev, stream, peaks, warm_batches=2, batches=3, relax_gate=False)
     return res
 
 
+def run_independent(dev, n_steps=50, warmup=5):
+    """Independent execution (§3.3; the Fast-WAM-IDM profile of App. B.1): a video-only and an
+    action-only 12-block d768 model, each with its own replan state, on its own stream.  One
+    control step: the video branch remaps stage 5 to entry 4 (shifted schedule) and runs its
+    2-step anticipatory prefix under the predicted observation; when the real observation
+    arrives the video branch rebinds and finishes its 4 steps while the action branch remaps
+    with the executed shift 8, enters stage 5 and runs 5 steps.  Timed twice: the two
+    continuations through wam_continue_many (one host thread per context, overlapping on the
+    GPU) and as two wam_continue calls in sequence.  O2A = real observation to action chunk."""
+    import torch
+
+    from paper_2609_34608_gb300 import inputs as I
+    from paper_2609_34608_gb300 import wam as W
+
+    cv, ca = I.get_config("idm_video"), I.get_config("idm_action")
+    K = cv["n_steps"]
+    sv, sa = torch.cuda.Stream(dev), torch.cuda.Stream(dev)
+    ctxs = []
+    for cfg, s in ((cv, sv), (ca, sa)):
+        flat = torch.from_numpy(I.flatten_weights(I.make_weights(cfg))).to(dev)
+        ctxs.append(W.Context(cfg, flat, stream=s.cuda_stream))
+        del flat
+    vctx, actx = ctxs
+    total = 2 * (warmup + n_steps) + 1
+    proc = I.ObsProcess(cv, 1, seed=5)
+    with torch.cuda.stream(sv):
+        obs0 = torch.from_numpy(proc.obs.copy()).to(dev)
+        inputs = []
+        for t in range(total):
+            pred, real = proc.predicted(), proc.step()
+            inputs.append((torch.from_numpy(pred).to(dev), torch.from_numpy(real).to(dev),
+                           torch.from_numpy(I.make_fresh_eps(cv, 1, t)).to(dev),
+                           torch.from_numpy(I.make_fresh_eps(ca, 1, 500 + t)).to(dev)))
+        vout = torch.zeros((1, cv["n_video"], cv["video_dim"]), device=dev)
+        aout = torch.zeros((1, ca["n_action"], ca["action_dim"]), device=dev)
+        vst, ast = vctx.state(1), actx.state(1)
+        vctx.sample_cold(vst, obs0, torch.from_numpy(I.make_noise(cv, 1)).to(dev), K)
+    with torch.cuda.stream(sa):
+        actx.sample_cold(ast, obs0, torch.from_numpy(I.make_noise(ca, 1, seed=2)).to(dev), K)
+    torch.cuda.synchronize(dev)
+    b0v, pv = cv["tr_entry_stage"], cv["prefix_steps"]
+    ev = lambda: torch.cuda.Event(enable_timing=True)
+
+    def control_step(inp, concurrent, marks=None):
+        pred, real, eps_v, eps_a = inp
+        if marks is not None:
+            marks[0].record(sv)
+            sa.wait_event(marks[0])
+        s1 = vctx.adapt(vst, pred, shift=0, fresh_noise=eps_v)[0]
+        if s1 == W.ADAPT_TR_INIT:
+            vctx.continue_(vst, pv)
+        if marks is not None:
+            marks[1].record(sv)          # the real observation arrives
+            sa.wait_event(marks[1])
+        s2 = vctx.adapt(vst, real)[0]
+        actx.adapt(ast, real, shift=ca["shift"], fresh_noise=eps_a)
+        kv = b0v + pv if s2 == W.ADAPT_REBIND_ACCEPT else b0v
+        calls = [(vctx, vst, K - kv, None, vout), (actx, ast, K - ca["tr_entry_stage"], aout, None)]
+        if concurrent:
+            W.Context.continue_many(calls)
+        else:
+            for c in calls:
+                c[0].continue_(c[1], c[2], c[3], c[4])
+        if marks is not None:
+            marks[2].record(sa)          # action chunk ready
+            sv.wait_event(marks[2])
+            marks[3].record(sv)          # both branches done
+
+    res = {}
+    t = 0
+    for concurrent in (True, False):
+        for _ in range(warmup):
+            control_step(inputs[t], concurrent)
+            t += 1
+        vctx.reset_stats()
+        actx.reset_stats()
+        torch.cuda.synchronize(dev)
+        marks = [[ev() for _ in range(4)] for _ in range(n_steps)]
+        for i in range(n_steps):
+            control_step(inputs[t], concurrent, marks[i])
+            t += 1
+        torch.cuda.synchronize(dev)
+        total_ms = marks[0][0].elapsed_time(marks[-1][3])
+        step_ms = [m[0].elapsed_time(m[3]) for m in marks]
+        o2a_ms = [m[1].elapsed_time(m[2]) for m in marks]
+        key = "concurrent" if concurrent else "sequential"
+        res[key] = {"chunks_per_s": n_steps / (total_ms * 1e-3), "ms_per_step": total_ms / n_steps,
+                    "step_ms_p50": float(np.percentile(step_ms, 50)),
+                    "o2a_ms_p50": float(np.percentile(o2a_ms, 50)),
+                    "o2a_ms_p99": float(np.percentile(o2a_ms, 99))}
+        if concurrent:
+            for name, c in (("video", vctx), ("action", actx)):
+                st = c.stats()
+                res.setdefault("reuse", {})[name] = {
+                    "r_rr": st["n_reuse"] / max(1, st["n_attempt"]), "f_skip": st["b_skip"] / max(1, st["b_dense"]),
+                    "r_or": st["n_bind"] / max(1, st["n_start"])}
+    vctx.close()
+    actx.close()
+    res["workload"] = ("independent execution (Fast-WAM-IDM profile): video-only 12-block d768 model "
+                       "(256 obs + 1024 video tokens, shifted schedule s=5, stage 5 -> entry 4, 2+4 steps) and "
+                       "action-only 12-block d768 model (256 obs + 16x7 action tokens, shift 8, entry 5, 5 steps), "
+                       "batch 1, RR gates cos >= 0.80, fit <= 0.60; each on its own stream")
+    res["steps"] = n_steps
+    return res
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -492,6 +603,7 @@ def main():
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-serving", action="store_true", help="skip the batched serving section")
+    ap.add_argument("--no-independent", action="store_true", help="skip the independent-execution section")
     args = ap.parse_args()
     if args.warmup < 3:
         raise SystemExit("--warmup must be >= 3")

@@ -21,7 +21,8 @@
  *     only after the output has been written.  With device buffers only, a call returns
  *     once its work is enqueued on the context's stream.
  *   - Contexts and states own their device memory.  A context is used from one host thread
- *     at a time; it is not thread-safe.
+ *     at a time; it is not thread-safe.  Different contexts may be driven from different host
+ *     threads at the same time (they share no mutable state).
  *   - All float buffers are IEEE float32, row-major, contiguous.
  *
  * Layouts (B = episodes in a state, No/Nv/Na = observation/video/action tokens,
@@ -87,6 +88,14 @@ extern "C" {
  * and epsilon of Eq. 7; gate thresholds of Eq. 8.  Branches (joint execution): observation and
  * video rows form one branch, action rows the other; each gets its own alpha and the middle
  * layers are skipped only if both pass.
+ *
+ * Independent execution (§3.3, App. B.1 Fast-WAM-IDM profile): n_video = 0 makes an
+ * action-only model and n_action = 0 a video-only one (not both).  Such a model is one branch:
+ * all of its rows share one alpha and one gate decision, its TR direction is normalised over
+ * its own trajectory, and its context keeps its own replan state, schedule (sched_shift) and
+ * retained / entry stages.  Two contexts then form the video and action branches; video_dim and
+ * action_dim stay >= 1 and the unused branch's embedding / output weights stay in the weight
+ * layout (ignored).  wam_continue_many advances both concurrently.
  *
  * OR (§3.2): Eq. 4 over or_n_components (1..4) equal contiguous blocks of observation tokens
  * with per-component scale or_deltas[m] and weight or_weights[m]; accept iff S < or_tau and
@@ -209,6 +218,20 @@ int wam_adapt_state(wam_ctx* ctx, wam_state* st, const float* new_obs,
  */
 int wam_continue(wam_ctx* ctx, wam_state* st, const int32_t* n_steps, float* actions_out,
                  float* video_out);
+
+/*
+ * wam_continue on n (>= 1) distinct contexts at once, each from its own host thread (the
+ * calling thread runs the first), so the branches of independent execution overlap on the GPU
+ * when their contexts use different streams.  Element i of every array belongs to context i:
+ * states[i] belongs to ctxs[i]; n_steps[i] has states[i]'s batch entries; actions_out and
+ * video_out (each nullable, as are their elements) as in wam_continue.  Results are those of
+ * n separate wam_continue calls.  status_out [n] (nullable) receives each call's status; the
+ * return value is the first non-zero of them, or WAM_OK.  Each context's last error names its
+ * own failure.  Errors: INVALID_ARG (null arrays, a state of another context, a context twice).
+ */
+int wam_continue_many(int32_t n, wam_ctx* const* ctxs, wam_state* const* states,
+                      const int32_t* const* n_steps, float* const* actions_out,
+                      float* const* video_out, int32_t* status_out);
 
 /* Reuse statistics accumulated on the context since creation / the last reset. */
 int wam_get_stats(wam_ctx* ctx, wam_stats* out);

@@ -262,8 +262,15 @@ class RRCheck:
 
 
 def rr_branch_rows(cfg: OracleConfig):
-    """Token-row ranges of the two jointly executed branches: observation + video rows form
-    the video branch, action rows the action branch (joint execution, §3.3)."""
+    """Token-row ranges of the branches whose rescaling factors and checks are separate.
+
+    Joint execution (§3.3): observation + video rows form the video branch, action rows the
+    action branch.  Independent execution (§3.3, the Fast-WAM-IDM profile of App. B.1) runs
+    each branch as its own model (no action tokens, or no video tokens): that model is one
+    branch, all of its rows.
+    """
+    if cfg.n_video == 0 or cfg.n_action == 0:
+        return [(0, cfg.n_tokens)]
     a1 = cfg.n_obs + cfg.n_video
     return [(0, a1), (a1, cfg.n_tokens)]
 
@@ -374,7 +381,9 @@ def tr_remap(cfg: OracleConfig, x_bar, x_r, sigma_r: float, sigma_b0: float, shi
     Video: no temporal shift (every slot receives state), or fresh noise when
     ``tr_video_mode == 1`` (Motus profile, App. B.1).  Action: slot j receives the retained
     slot j + shift while that stays inside the horizon; the uncovered tail gets fresh noise.
-    Fresh noise at level sigma_b0 is sigma_b0 * eps.
+    Fresh noise at level sigma_b0 is sigma_b0 * eps.  Each branch's direction is normalised over
+    that branch alone, so a single-branch model of independent execution (App. B.1: video and
+    action keep separate replan states) remaps exactly its part of the joint trajectory.
     """
     x_bar = np.asarray(x_bar, dtype=F64)
     x_r = np.asarray(x_r, dtype=F64)
@@ -382,11 +391,15 @@ def tr_remap(cfg: OracleConfig, x_bar, x_r, sigma_r: float, sigma_b0: float, shi
     V, Na, ad = cfg.video_len, cfg.n_action, cfg.action_dim
     norm = bool(cfg.tr_normalize)
     out = np.empty(cfg.traj_len, dtype=F64)
-    if cfg.tr_video_mode == 1:
+    if V == 0:
+        pass  # action-only model (independent execution): no video branch
+    elif cfg.tr_video_mode == 1:
         out[:V] = sigma_b0 * eps[:V]
     else:
         d_v = tr_direction(x_r[:V], x_bar[:V], sigma_r, norm)
         out[:V] = x_bar[:V] + sigma_b0 * d_v
+    if Na == 0:
+        return out  # video-only model (independent execution): no action branch
     d_a = tr_direction(x_r[V:], x_bar[V:], sigma_r, norm).reshape(Na, ad)
     xb_a = x_bar[V:].reshape(Na, ad)
     ea = eps[V:].reshape(Na, ad)

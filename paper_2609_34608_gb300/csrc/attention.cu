@@ -305,12 +305,12 @@ __global__ void __launch_bounds__(256) attn_f32_kernel(const float* __restrict__
 template <int DH>
 cudaError_t launch_bf16(const bf16* qkv, bf16* out, int B, int N, int d, int H, cudaStream_t s) {
   using C = AttnCfg<DH>;
-  static bool attr_set = false;
-  if (!attr_set) {
+  static std::atomic<bool> attr_set{false};  // contexts may run on several host threads
+  if (!attr_set.load(std::memory_order_acquire)) {
     cudaError_t e = cudaFuncSetAttribute(attn_bf16_kernel<DH>,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize, C::kSmem);
     if (e != cudaSuccess) return e;
-    attr_set = true;
+    attr_set.store(true, std::memory_order_release);
   }
   dim3 grid((N + C::kBQ - 1) / C::kBQ, H, B);
   const float scale_log2 = 1.4426950408889634f / sqrtf(static_cast<float>(DH));

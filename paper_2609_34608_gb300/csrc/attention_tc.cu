@@ -323,11 +323,11 @@ cudaError_t attention_tc(const CUtensorMap& tm_qk, const CUtensorMap& tm_vt, bf1
                          int H, int* dev_err, cudaStream_t s) {
   if (B <= 0 || N <= 0) return cudaSuccess;
   if (d / H != kDH) return cudaErrorInvalidValue;
-  static bool attr_set = false;
-  if (!attr_set) {
+  static std::atomic<bool> attr_set{false};  // contexts may run on several host threads
+  if (!attr_set.load(std::memory_order_acquire)) {
     cudaError_t e = cudaFuncSetAttribute(attn_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemAttn);
     if (e != cudaSuccess) return e;
-    attr_set = true;
+    attr_set.store(true, std::memory_order_release);
   }
   const float scale_log2 = 1.4426950408889634f / 8.0f;  // log2(e) / sqrt(64)
   dim3 grid((N + kQ - 1) / kQ, H, B);

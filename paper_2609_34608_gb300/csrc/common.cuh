@@ -7,6 +7,8 @@
 #include <cuda_runtime.h>
 #include <stdint.h>
 
+#include <atomic>
+
 #define WAM_DEV __device__ __forceinline__
 
 namespace wam {

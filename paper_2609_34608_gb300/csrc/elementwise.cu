@@ -787,11 +787,14 @@ cudaError_t final_euler(const float* h, const StepItem* items, const float* mods
   if (d % 128 != 0 || vd > 16 || ad > 16) return cudaErrorInvalidValue;  // heads padded to 16
   // One block per SM (or fewer), each staging both output heads once; warps stride over the
   // row pairs.
-  static int num_sms = 0;
+  static std::atomic<int> sms_cached{0};  // contexts may run on several host threads
+  int num_sms = sms_cached.load(std::memory_order_relaxed);
   if (num_sms == 0) {
     int dev = 0;
     cudaGetDevice(&dev);
     cudaDeviceGetAttribute(&num_sms, cudaDevAttrMultiProcessorCount, dev);
+    if (num_sms < 1) num_sms = 1;
+    sms_cached.store(num_sms, std::memory_order_relaxed);
   }
   const int64_t units = static_cast<int64_t>(Bw) * ((Nv + 1) / 2 + (Na + 1) / 2);
   const int64_t want = (units + kRowWarps - 1) / kRowWarps;
@@ -799,13 +802,16 @@ cudaError_t final_euler(const float* h, const StepItem* items, const float* mods
   const size_t smem = static_cast<size_t>(2) * d * 16 * sizeof(float);
 #define WAM_FE_CASE(NV)                                                                       \
   case NV: {                                                                                  \
-    static int smem_set = 0;                                                                  \
-    if (smem_set < static_cast<int>(smem)) {                                                  \
+    static std::atomic<int> smem_set{0};                                                      \
+    if (smem_set.load(std::memory_order_acquire) < static_cast<int>(smem)) {                  \
       cudaError_t e = cudaFuncSetAttribute(final_euler_kernel<NV>,                           \
                                            cudaFuncAttributeMaxDynamicSharedMemorySize,       \
                                            static_cast<int>(smem));                           \
       if (e != cudaSuccess) return e;                                                         \
-      smem_set = static_cast<int>(smem);                                                      \
+      int prev = smem_set.load(std::memory_order_relaxed);                                    \
+      while (prev < static_cast<int>(smem) &&                                                 \
+             !smem_set.compare_exchange_weak(prev, static_cast<int>(smem)))                   \
+        ;                                                                                     \
     }                                                                                         \
     launch_pdl(final_euler_kernel<NV>, dim3(grid), dim3(256), smem, s, h, items, mods, mod_stride, fin_off, vout_w,  \
                                                 vout_b, aout_w, aout_b, x, xhist, vhist,      \

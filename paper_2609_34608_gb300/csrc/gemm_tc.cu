@@ -472,12 +472,12 @@ template <int BN, int EPI, int KA>
 cudaError_t launch(const CUtensorMap& ta, const CUtensorMap& tb, int M, int N, int K,
                    const EpiArgs& e, const SplitArgs& sp, int num_sms, int* dev_err, cudaStream_t s) {
   using C = TileCfg<BN, KA>;
-  static bool attr_set = false;
-  if (!attr_set) {
+  static std::atomic<bool> attr_set{false};  // contexts may run on several host threads
+  if (!attr_set.load(std::memory_order_acquire)) {
     cudaError_t err = cudaFuncSetAttribute(gemm_tc_kernel<BN, EPI, KA>,
                                            cudaFuncAttributeMaxDynamicSharedMemorySize, C::kSmemBytes);
     if (err != cudaSuccess) return err;
-    attr_set = true;
+    attr_set.store(true, std::memory_order_release);
   }
   const int units = ((M + kBM - 1) / kBM) * (N / BN) * sp.splits;
   const int grid = units < num_sms ? units : num_sms;

@@ -11,6 +11,7 @@
 #include <map>
 #include <new>
 #include <string>
+#include <thread>
 #include <tuple>
 #include <vector>
 
@@ -65,6 +66,9 @@ struct EpisodeMeta {
 struct wam_ctx {
   wam_config cfg;
   int L, d, H, R, No, Nv, vd, Na, ad, N, T, V, K, dff, Bmax;
+  // first row of the RR action branch: No + Nv for a joint model; N for a video-only model
+  // (one branch, all rows) and 0 for an action-only model (one branch, all rows)
+  int split;
   int64_t mod_n;
   bool bf16;
   cudaStream_t stream = nullptr;
@@ -397,7 +401,7 @@ int run_steps(wam_ctx* c, wam_state* st, const std::vector<int>& n) {
   const int64_t stage_stride = int64_t(B) * c->T;
   const bool rr_on = rr_enabled(c);
   const int q = c->cfg.rr_q, s = c->cfg.rr_s, e = c->cfg.rr_e;
-  const int split_row = c->No + c->Nv;
+  const int split_row = c->split;
   TRY(obs_embed(c, st));
   int max_n = 0;
   for (int b = 0; b < B; ++b) max_n = std::max(max_n, n[b]);
@@ -501,8 +505,10 @@ int run_steps(wam_ctx* c, wam_state* st, const std::vector<int>& n) {
                      c->cfg.rr_alpha_max, c->cfg.rr_eps, c->cfg.rr_gamma_cos, c->cfg.rr_gamma_fit, c->d_gate, c->stream));
         }
         TRY(readback(c, gates.data(), c->d_gate, sizeof(RRGate) * 2 * Bw));
+        // every non-empty branch must pass (§3.3); a single-branch model has one
         for (int w = 0; w < Bw; ++w)
-          if (gate_ok[w] && gates[2 * w].pass && gates[2 * w + 1].pass) accepted[w] = 1;
+          if (gate_ok[w] && (split_row == 0 || gates[2 * w].pass) && (split_row == N || gates[2 * w + 1].pass))
+            accepted[w] = 1;
       }
       midmap.clear();
       for (int w = 0; w < Bw; ++w) {
@@ -557,6 +563,7 @@ int run_steps(wam_ctx* c, wam_state* st, const std::vector<int>& n) {
       rec.rr_accept = accepted[w];
       if (gate_ok[w]) {
         for (int br = 0; br < 2; ++br) {
+          if (br == 0 ? split_row == 0 : split_row == N) continue;  // empty branch
           rec.alpha[br] = static_cast<float>(gates[2 * w + br].alpha);
           rec.cos[br] = static_cast<float>(gates[2 * w + br].cos);
           rec.fit[br] = static_cast<float>(gates[2 * w + br].fit);
@@ -584,12 +591,12 @@ int run_steps(wam_ctx* c, wam_state* st, const std::vector<int>& n) {
 }
 
 int copy_out(wam_ctx* c, wam_state* st, float* actions_out, float* video_out, bool& host_out) {
-  if (actions_out != nullptr) {
+  if (actions_out != nullptr && c->Na > 0) {
     const size_t w = sizeof(float) * c->Na * c->ad;
     CK(cudaMemcpy2DAsync(actions_out, w, st->x + c->V, sizeof(float) * c->T, w, st->B, cudaMemcpyDefault, c->stream));
     host_out = host_out || !is_device_ptr(actions_out);
   }
-  if (video_out != nullptr) {
+  if (video_out != nullptr && c->V > 0) {
     const size_t w = sizeof(float) * c->V;
     CK(cudaMemcpy2DAsync(video_out, w, st->x, sizeof(float) * c->T, w, st->B, cudaMemcpyDefault, c->stream));
     host_out = host_out || !is_device_ptr(video_out);
@@ -600,9 +607,10 @@ int copy_out(wam_ctx* c, wam_state* st, float* actions_out, float* video_out, bo
 int validate_cfg(const wam_config* g, std::string& why) {
   if (g == nullptr) return why = "null config", WAM_ERR_INVALID_ARG;
   if (g->n_layers < 1 || g->d_model < 1 || g->n_heads < 1 || g->mlp_ratio < 1 || g->n_obs < 1 ||
-      g->n_video < 1 || g->video_dim < 1 || g->n_action < 1 || g->action_dim < 1 || g->n_steps < 1 ||
-      g->batch_max < 1)
+      g->video_dim < 1 || g->action_dim < 1 || g->n_steps < 1 || g->batch_max < 1)
     return why = "every size must be >= 1", WAM_ERR_INVALID_ARG;
+  if (g->n_video < 0 || g->n_action < 0 || g->n_video + g->n_action < 1)
+    return why = "n_video and n_action must be >= 0, not both 0", WAM_ERR_INVALID_ARG;
   if (g->d_model % g->n_heads != 0) return why = "d_model must be a multiple of n_heads", WAM_ERR_INVALID_ARG;
   if (g->precision != WAM_PREC_FP32 && g->precision != WAM_PREC_BF16) return why = "unknown precision", WAM_ERR_INVALID_ARG;
   if (g->batch_max > kMaxBatch) return why = "batch_max above 256", WAM_ERR_UNSUPPORTED;
@@ -735,6 +743,7 @@ int create_impl(wam_ctx* c, const wam_config* cfg, const float* weights, size_t 
   c->Na = cfg->n_action;
   c->ad = cfg->action_dim;
   c->N = c->No + c->Nv + c->Na;
+  c->split = c->Na == 0 ? c->N : (c->Nv == 0 ? 0 : c->No + c->Nv);
   c->V = c->Nv * c->vd;
   c->T = c->V + c->Na * c->ad;
   c->K = cfg->n_steps;
@@ -812,7 +821,7 @@ int create_impl(wam_ctx* c, const wam_config* cfg, const float* weights, size_t 
   TRY(dalloc(c, c->allocs, &c->d_err, 1));
   CK(cudaMemset(c->d_err, 0, sizeof(int)));
   // scratch for the float64 partial sums of TR / OR / RR reductions
-  const int split = c->No + c->Nv;
+  const int split = c->split;
   const size_t p_tr = size_t(c->Bmax) * 2 * tr_num_chunks(c->T, c->V);
   const size_t p_or = size_t(c->Bmax) * cfg->or_n_components * or_num_chunks(int64_t(c->No / cfg->or_n_components) * c->d);
   const size_t p_rr = size_t(c->Bmax) * 2 * 3 * rr_num_chunks(int64_t(std::max(split, c->N - split)) * c->d);
@@ -1124,6 +1133,47 @@ int wam_continue(wam_ctx* c, wam_state* st, const int32_t* n_steps, float* actio
   TRY(copy_out(c, st, actions_out, video_out, host_out));
   if (host_out) TRY(sync_check(c));
   return WAM_OK;
+}
+
+int wam_continue_many(int32_t n, wam_ctx* const* ctxs, wam_state* const* states, const int32_t* const* n_steps,
+                      float* const* actions_out, float* const* video_out, int32_t* status_out) {
+  if (n < 1 || ctxs == nullptr || states == nullptr || n_steps == nullptr) return WAM_ERR_INVALID_ARG;
+  for (int i = 0; i < n; ++i) {
+    if (ctxs[i] == nullptr || states[i] == nullptr || states[i]->ctx != ctxs[i] || n_steps[i] == nullptr)
+      return WAM_ERR_INVALID_ARG;
+    for (int j = 0; j < i; ++j)
+      if (ctxs[j] == ctxs[i]) return fail(ctxs[i], WAM_ERR_INVALID_ARG, "a context appears twice");
+  }
+  std::vector<int> rc(n, WAM_OK);
+  auto run = [&](int i) {
+    wam_ctx* c = ctxs[i];
+    if (cudaSetDevice(c->device) != cudaSuccess) {
+      cudaGetLastError();
+      rc[i] = fail(c, WAM_ERR_CUDA, "cudaSetDevice failed on a worker thread");
+      return;
+    }
+    rc[i] = wam_continue(c, states[i], n_steps[i], actions_out ? actions_out[i] : nullptr,
+                         video_out ? video_out[i] : nullptr);
+  };
+  // One host thread per context, so the host-side gate decisions of one branch never hold back
+  // the launches of another; the GPU overlaps the contexts' streams.
+  std::vector<std::thread> workers;
+  int spawned = 1;
+  try {
+    workers.reserve(n - 1);
+    for (; spawned < n; ++spawned) workers.emplace_back(run, spawned);
+  } catch (...) {
+    // no thread available: the rest run on this thread after the spawned ones
+  }
+  run(0);
+  for (auto& t : workers) t.join();
+  for (int i = spawned; i < n; ++i) run(i);
+  int first = WAM_OK;
+  for (int i = 0; i < n; ++i) {
+    if (status_out) status_out[i] = rc[i];
+    if (first == WAM_OK) first = rc[i];
+  }
+  return first;
 }
 
 int wam_sample_cold(wam_ctx* c, wam_state* st, const float* obs, const float* noise, int32_t n_steps, float* actions_out) {

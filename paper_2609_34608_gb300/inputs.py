@@ -19,6 +19,9 @@ none of which exists here; these synthetic shapes stand in for them):
                   (7-DoF); 16 cold (10 steps) + 16 warm (2 of 10 steps).
 * ``bimanual``    28 blocks, d=1152, 16 heads (head dim 72); B=8; 768 obs + 4096 video +
                   50 action (14-DoF); cold 10 + warm sweep over 1..9 retained steps, shift 25.
+* ``tiny_video`` / ``tiny_action``, ``idm_video`` / ``idm_action``: independent execution, a
+                  video-only and an action-only model with separate replan states (the
+                  Fast-WAM-IDM profile), at the ``tiny_rr`` and ``latency`` sizes.
 
 Weight tensors are N(0, 0.02) from seed 0 in the fixed order of ``weight_spec`` (the same
 order the C header ``include/wam.h`` documents for the flat weight buffer).
@@ -82,6 +85,42 @@ NAMED_CONFIGS: dict[str, dict] = {
         n_steps=10, precision="bf16", batch=8,
         tr_entry_stage=5, tr_retain_stage=5, shift=25,
         rr_policy=1, rr_q=2, rr_s=4, rr_e=24,
+    ),
+    # Independent execution (§3.3; App. B.1 Fast-WAM-IDM profile): the video branch and the
+    # action branch are separate models, each with its own replan state and RR decisions.
+    # Video: shifted schedule s = 5, retained stage 5 remapped to entry stage 4 without a
+    # temporal shift, 2 anticipatory + 4 real steps.  Action: linear schedule, enters stage 5
+    # with the horizon shifted by the executed count, 5 steps under the real observation.  RR
+    # thresholds of the Fast-WAM-IDM column of Table 7 (cos >= 0.80, fit <= 0.60).
+    "tiny_video": dict(
+        n_layers=6, d_model=128, n_heads=4, mlp_ratio=4,
+        n_obs=16, n_video=32, video_dim=16, n_action=0, action_dim=7,
+        n_steps=10, precision="fp32", batch=1, sched_shift=5.0,
+        tr_entry_stage=4, tr_retain_stage=5, shift=0, prefix_steps=2,
+        rr_policy=1, rr_q=1, rr_s=2, rr_e=5, rr_gamma_cos=0.80, rr_gamma_fit=0.60,
+    ),
+    "tiny_action": dict(
+        n_layers=6, d_model=128, n_heads=4, mlp_ratio=4,
+        n_obs=16, n_video=0, video_dim=16, n_action=8, action_dim=7,
+        n_steps=10, precision="fp32", batch=1, sched_shift=1.0,
+        tr_entry_stage=5, tr_retain_stage=5, shift=4, prefix_steps=0,
+        rr_policy=1, rr_q=1, rr_s=2, rr_e=5, rr_gamma_cos=0.80, rr_gamma_fit=0.60,
+    ),
+    # The same pair at the size of the ``latency`` model: 12 blocks, d=768, 12 heads each;
+    # video 256 obs + 1024 video tokens, action 256 obs + 16 action tokens (7-DoF).
+    "idm_video": dict(
+        n_layers=12, d_model=768, n_heads=12, mlp_ratio=4,
+        n_obs=256, n_video=1024, video_dim=16, n_action=0, action_dim=7,
+        n_steps=10, precision="bf16", batch=1, sched_shift=5.0,
+        tr_entry_stage=4, tr_retain_stage=5, shift=0, prefix_steps=2,
+        rr_policy=1, rr_q=2, rr_s=4, rr_e=8, rr_gamma_cos=0.80, rr_gamma_fit=0.60,
+    ),
+    "idm_action": dict(
+        n_layers=12, d_model=768, n_heads=12, mlp_ratio=4,
+        n_obs=256, n_video=0, video_dim=16, n_action=16, action_dim=7,
+        n_steps=10, precision="bf16", batch=1, sched_shift=1.0,
+        tr_entry_stage=5, tr_retain_stage=5, shift=8, prefix_steps=0,
+        rr_policy=1, rr_q=2, rr_s=4, rr_e=8, rr_gamma_cos=0.80, rr_gamma_fit=0.60,
     ),
 }
 

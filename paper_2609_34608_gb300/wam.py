@@ -116,6 +116,7 @@ def lib() -> ctypes.CDLL:
         "wam_sample_cold": (ctypes.c_int, [_vp, _vp, _vp, _vp, _i32, _vp]),
         "wam_adapt_state": (ctypes.c_int, [_vp, _vp, _vp, _vp, _vp, _vp, _vp]),
         "wam_continue": (ctypes.c_int, [_vp, _vp, _vp, _vp, _vp]),
+        "wam_continue_many": (ctypes.c_int, [_i32, _vp, _vp, _vp, _vp, _vp, _vp]),
         "wam_get_stats": (ctypes.c_int, [_vp, ctypes.POINTER(Stats)]),
         "wam_reset_stats": (ctypes.c_int, [_vp]),
         "wam_state_log": (ctypes.c_int, [_vp, _vp, _i32, ctypes.POINTER(_i32)]),
@@ -267,6 +268,24 @@ class Context:
     def continue_(self, st: State, n_steps, actions_out=None, video_out=None):
         n = _i32_array(n_steps, st.batch)
         self._check(lib().wam_continue(self.handle, st.handle, ptr(n), ptr(actions_out), ptr(video_out)))
+
+    @staticmethod
+    def continue_many(calls):
+        """wam_continue_many: `calls` is a list of (context, state, n_steps, actions_out, video_out)
+        on distinct contexts, advanced concurrently (one host thread each)."""
+        n = len(calls)
+        ctxs = (_vp * n)(*[c[0].handle.value for c in calls])
+        states = (_vp * n)(*[c[1].handle.value for c in calls])
+        steps = [_i32_array(c[2], c[1].batch) for c in calls]
+        step_ptrs = (_vp * n)(*[s.ctypes.data for s in steps])
+        outs_a = (_vp * n)(*[ptr(c[3]) if len(c) > 3 else None for c in calls])
+        outs_v = (_vp * n)(*[ptr(c[4]) if len(c) > 4 else None for c in calls])
+        status = np.zeros(n, dtype=np.int32)
+        code = lib().wam_continue_many(n, ctxs, states, step_ptrs, outs_a, outs_v, status.ctypes.data)
+        if code != WAM_OK:
+            i = int(np.flatnonzero(status)[0]) if status.any() else 0
+            calls[i][0]._check(code)
+        return status
 
     def stats(self) -> dict:
         s = Stats()

@@ -46,6 +46,8 @@ def _create(cfg):
     (dict(batch=0), 1),                              # batch_max below 1
     (dict(d_model=96, n_heads=3), 6),                # width not a multiple of 128
     (dict(video_dim=32), 6),                         # output head wider than 16
+    (dict(n_video=0, n_action=0), 1),                # a model needs video or action tokens
+    (dict(n_action=-1), 1),                          # negative token count
 ])
 def test_invalid_configs_are_rejected_before_device_work(lib, bad, code):
     cfg = inputs.get_config("tiny", **bad)

@@ -513,3 +513,96 @@ def test_layer_deltas_zero_gates_and_gate_scaling():
     d1 = O.layer_deltas(W1, cfg, x, obs, 0.6)[0]
     d2 = O.layer_deltas(W2, cfg, x, obs, 0.6)[0]
     assert d1 > 0.0 and d2 == pytest.approx(3.0 * d1, rel=1e-12)
+
+
+# ----------------------------------------------------------------------------- independent execution
+def test_independent_profiles_match_appendix_b():
+    """The video / action pair follows the Fast-WAM-IDM profile of App. B.1-B.2: K = 10, the
+    video branch remaps stage 5 (sigma 0.83333) to stage 4 (0.88235) on the shifted schedule and
+    runs 2 + 4 steps, the action branch enters stage 5 for 5 steps, gates of Table 7."""
+    rows = _golden("profiles.txt")
+    gate = [r for r in rows if r[0] == "gate" and r[1] == "fastwam"][0]
+    sched = {(int(r[2])): float(r[3]) for r in _golden("fastwam_schedule.txt")}
+    for size in ("tiny", "idm"):
+        v = I.get_config(f"{size}_video" if size == "idm" else "tiny_video")
+        a = I.get_config(f"{size}_action" if size == "idm" else "tiny_action")
+        steps_v = [r for r in rows if r[0] == "steps" and r[1] == "fastwam_video"][0]
+        steps_a = [r for r in rows if r[0] == "steps" and r[1] == "fastwam_action"][0]
+        assert v["n_action"] == 0 and a["n_video"] == 0
+        assert v["n_steps"] == a["n_steps"] == int(steps_v[2]) == int(steps_a[2])
+        sig = O.schedule(v["n_steps"], v["sched_shift"])
+        assert round(sig[v["tr_retain_stage"]], 5) == sched[v["tr_retain_stage"]]
+        assert round(sig[v["tr_entry_stage"]], 5) == sched[v["tr_entry_stage"]]
+        assert (v["prefix_steps"], v["n_steps"] - v["tr_entry_stage"] - v["prefix_steps"]) == \
+            (int(steps_v[3]), int(steps_v[4]))
+        assert (a["prefix_steps"], a["n_steps"] - a["tr_entry_stage"]) == (int(steps_a[3]), int(steps_a[4]))
+        for c in (v, a):
+            assert (c["rr_gamma_cos"], c["rr_gamma_fit"]) == (float(gate[2]), float(gate[3]))
+
+
+def test_single_branch_remap_is_the_joint_remap_of_its_branch():
+    """App. B.1: video and action keep separate replan states, each normalised over its own
+    trajectory; since Eq. 12 normalises per branch, a one-branch model remaps exactly the slice
+    a joint model gives its branch."""
+    joint = O.OracleConfig.from_dict(micro_config())
+    vid = O.OracleConfig.from_dict(micro_config(n_action=0))
+    act = O.OracleConfig.from_dict(micro_config(n_video=0))
+    V = joint.video_len
+    assert vid.traj_len == V and act.traj_len == joint.traj_len - V
+    rng = np.random.default_rng(30)
+    x_bar, x_r, eps = (rng.standard_normal(joint.traj_len) for _ in range(3))
+    for shift in (0, 2, 7):
+        out = O.tr_remap(joint, x_bar, x_r, 0.6, 0.8, shift, eps)
+        assert np.array_equal(O.tr_remap(vid, x_bar[:V], x_r[:V], 0.6, 0.8, shift, eps[:V]), out[:V])
+        assert np.array_equal(O.tr_remap(act, x_bar[V:], x_r[V:], 0.6, 0.8, shift, eps[V:]), out[V:])
+
+
+def test_single_branch_rr_uses_one_factor_over_all_rows():
+    """§3.3: a branch executed on its own decides reuse by itself, over all of its rows (one
+    alpha, one check); a joint model checks observation + video and action rows separately.
+    The probe residual is scaled by 1.1 on the first rows and 1.2 on the rest against the
+    retained one, and alpha is checked against the least-squares ratio written out by loops."""
+    for over, n_checks in ((dict(n_action=0), 1), (dict(n_video=0), 1), (dict(), 2)):
+        cfgd = micro_config(n_layers=6, rr_policy=1, rr_q=1, rr_s=2, rr_e=5, rr_alpha_max=2.0, **over)
+        W, cfg = _setup(cfgd, std=0.3)
+        rng = np.random.default_rng(31)
+        x = rng.standard_normal(cfg.traj_len)
+        obs = rng.standard_normal((cfg.n_obs, cfg.d_model))
+        _, st, _ = O.velocity_rr(W, cfg, x, obs, 0.5, None, True)
+        p_i = st.p_a
+        half = cfg.n_tokens // 2
+        scale = np.where(np.arange(cfg.n_tokens)[:, None] < half, 1.1, 1.2)
+        crafted = O.LayerState(p_a=p_i / scale, R_a=st.R_a)
+        _, _, rec = O.velocity_rr(W, cfg, x, obs, 0.5, crafted, True)
+        assert rec.rr_attempt and len(rec.checks) == n_checks
+        for (a, b), chk in zip(O.rr_branch_rows(cfg), rec.checks):
+            pi = p_i[a:b].ravel().tolist()
+            pa = crafted.p_a[a:b].ravel().tolist()
+            num = sum(u * w for u, w in zip(pi, pa))
+            den = sum(w * w for w in pa)
+            assert chk.alpha == pytest.approx(min(max(num / den, 1.0), 2.0), rel=1e-12)
+        if n_checks == 1:
+            assert O.rr_branch_rows(cfg) == [(0, cfg.n_tokens)]
+            assert 1.1 < rec.checks[0].alpha < 1.2
+
+
+def test_single_branch_models_denoise_their_own_trajectory():
+    """A video-only model outputs only video velocities and an action-only one only action
+    velocities; with zero gates every layer is the identity, so each equals the output head
+    applied to its own embedded tokens (the branches do not see each other)."""
+    for over in (dict(n_action=0), dict(n_video=0)):
+        cfgd = micro_config(**over)
+        W, cfg = _setup(cfgd, std=0.3)
+        W = _zero_gate_weights(W, cfg, (2, 5))
+        rng = np.random.default_rng(32)
+        x = rng.standard_normal(cfg.traj_len)
+        obs = rng.standard_normal((cfg.n_obs, cfg.d_model))
+        v = O.velocity(W, cfg, x, obs, 0.3)
+        assert v.shape == (cfg.traj_len,)
+        _, fin = O.conditioning(W, cfg, 0.3)
+        h = O.embed(W, cfg, x, obs)
+        y = O.layer_norm(h) * (1.0 + fin[1]) + fin[0]
+        a0, a1 = cfg.n_obs, cfg.n_obs + cfg.n_video
+        want = np.concatenate([(y[a0:a1] @ W["vout_w"].astype(np.float64) + W["vout_b"]).ravel(),
+                               (y[a1:] @ W["aout_w"].astype(np.float64) + W["aout_b"]).ravel()])
+        assert np.allclose(v, want, atol=1e-12)
