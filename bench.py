@@ -497,7 +497,8 @@ def run_independent(dev, n_steps=50, warmup=5):
     arrives the video branch rebinds and finishes its 4 steps while the action branch remaps
     with the executed shift 8, enters stage 5 and runs 5 steps.  Timed twice: the two
     continuations through wam_continue_many (one host thread per context, overlapping on the
-    GPU) and as two wam_continue calls in sequence.  O2A = real observation to action chunk."""
+    GPU; the action stream has the higher priority) and as two wam_continue calls in sequence.
+    O2A = real observation to action chunk."""
     import torch
 
     from paper_2609_34608_gb300 import inputs as I
@@ -505,7 +506,9 @@ def run_independent(dev, n_steps=50, warmup=5):
 
     cv, ca = I.get_config("idm_video"), I.get_config("idm_action")
     K = cv["n_steps"]
-    sv, sa = torch.cuda.Stream(dev), torch.cuda.Stream(dev)
+    # the action branch produces the chunk the robot waits for: its stream gets the higher
+    # priority, so its blocks are scheduled first whenever both branches have work queued
+    sv, sa = torch.cuda.Stream(dev), torch.cuda.Stream(dev, priority=-1)
     ctxs = []
     for cfg, s in ((cv, sv), (ca, sa)):
         flat = torch.from_numpy(I.flatten_weights(I.make_weights(cfg))).to(dev)
@@ -543,8 +546,8 @@ def run_independent(dev, n_steps=50, warmup=5):
         if marks is not None:
             marks[1].record(sv)          # the real observation arrives
             sa.wait_event(marks[1])
-        s2 = vctx.adapt(vst, real)[0]
         actx.adapt(ast, real, shift=ca["shift"], fresh_noise=eps_a)
+        s2 = vctx.adapt(vst, real)[0]
         kv = b0v + pv if s2 == W.ADAPT_REBIND_ACCEPT else b0v
         calls = [(vctx, vst, K - kv, None, vout), (actx, ast, K - ca["tr_entry_stage"], aout, None)]
         if concurrent:

@@ -257,28 +257,18 @@ __global__ void __launch_bounds__(256) ln_mod_kernel(const float* __restrict__ h
 }
 
 // ---------------------------------------------------------------- final layer + Euler
-// Modulated LN of a token row, the output head (16 columns; the zero-padded [d, 16] video and
-// action heads are staged once per block in shared memory, transposed to [16, d] so a lane's
-// float4 reads are consecutive across the warp), the Euler update of that token's trajectory
-// values and their retention.  Work unit: up to two consecutive token rows of the same head of
-// one item, processed by one warp so each weight element read from shared memory serves both.
-template <int NV4>
-WAM_DEV void ln_mod_row(const float* __restrict__ hrow, const float* shift, const float* scale, int d,
-                        int lane, float4 (&y)[NV4]) {
-  const float4* hr = reinterpret_cast<const float4*>(hrow);
-#pragma unroll
-  for (int i = 0; i < NV4; ++i) y[i] = hr[lane + 32 * i];
-  float mean, rstd;
-  row_stats<NV4>(y, d, mean, rstd);
-#pragma unroll
-  for (int i = 0; i < NV4; ++i) {
-    const int c = (lane + 32 * i) * 4;
-    const float4 sh = *reinterpret_cast<const float4*>(shift + c);
-    const float4 sc = *reinterpret_cast<const float4*>(scale + c);
-    y[i] = make_float4(fmaf((y[i].x - mean) * rstd, 1.0f + sc.x, sh.x), fmaf((y[i].y - mean) * rstd, 1.0f + sc.y, sh.y),
-                       fmaf((y[i].z - mean) * rstd, 1.0f + sc.z, sh.z), fmaf((y[i].w - mean) * rstd, 1.0f + sc.w, sh.w));
-  }
-}
+// Modulated LN of a token row, the output head (16 columns; the [d, 16] heads are zero-padded),
+// the Euler update of that token's trajectory values and their retention.  The modulation is
+// folded into the head once per block: LN(h)(1+scale)+shift times W equals
+// xhat . W' + c with W'[k][j] = (1+scale[k]) W[k][j] and c[j] = b[j] + sum_k shift[k] W[k][j],
+// where xhat = (h - mean) rstd.  A block serves a contiguous range of one item's video (or
+// action) rows and stages only that head's W'.
+//
+// Float32 precision mode: SIMT dot products, a warp per row pair (each weight read from shared
+// memory serves both rows).  Bf16 precision mode: the head is a [rows, d] x [d, 16] product on
+// the tensor cores (mma.sync m16n8k16, bf16 operands, float32 accumulation), a warp per 16-row
+// tile, with the row statistics gathered from the same loads; 16 products per loaded element
+// would otherwise bound the kernel on the FMA pipe instead of HBM.
 
 // Reduce-scatter 16 partial outputs over the warp: lane l ends with output (l & 15).
 WAM_DEV float reduce_scatter16(float (&acc)[16], int lane) {
@@ -295,45 +285,97 @@ WAM_DEV float reduce_scatter16(float (&acc)[16], int lane) {
   return acc[0] + __shfl_xor_sync(0xffffffffu, acc[0], 16);
 }
 
+// Normalised row: xhat = (h - mean) rstd, lane-strided float4s (element c = 4 (lane + 32 i)).
 template <int NV4>
-__global__ void __launch_bounds__(256) final_euler_kernel(
+WAM_DEV void ln_row(const float* __restrict__ hrow, int d, int lane, float4 (&y)[NV4]) {
+  const float4* hr = reinterpret_cast<const float4*>(hrow);
+#pragma unroll
+  for (int i = 0; i < NV4; ++i) y[i] = hr[lane + 32 * i];
+  float mean, rstd;
+  row_stats<NV4>(y, d, mean, rstd);
+#pragma unroll
+  for (int i = 0; i < NV4; ++i)
+    y[i] = make_float4((y[i].x - mean) * rstd, (y[i].y - mean) * rstd, (y[i].z - mean) * rstd, (y[i].w - mean) * rstd);
+}
+
+// Which rows a block of the final kernel serves: blocks [0, vblocks) split an item's video rows,
+// the rest its action rows, in contiguous ranges of `gran`-row units.
+struct HeadRange {
+  bool video;
+  int beg, end;  // token rows within the head
+};
+WAM_DEV HeadRange head_range(int bx, int vblocks, int ablocks, int Nv, int Na, int gran) {
+  HeadRange r;
+  r.video = bx < vblocks;
+  const int part = r.video ? bx : bx - vblocks;
+  const int nparts = r.video ? vblocks : ablocks;
+  const int nrows = r.video ? Nv : Na;
+  const int units = (nrows + gran - 1) / gran;
+  const int per = (units + nparts - 1) / nparts;
+  r.beg = min(nrows, part * per * gran);
+  r.end = min(nrows, (part + 1) * per * gran);
+  return r;
+}
+
+// Euler update x <- x + dsigma v of one trajectory value, retained as x^{k+1} and v^k.
+WAM_DEV void euler_store(const StepItem& it, int64_t idx, float vel, float* __restrict__ x,
+                         float* __restrict__ xhist, float* __restrict__ vhist, int64_t stage_stride) {
+  const float xn = static_cast<float>(static_cast<double>(x[idx]) + it.dsigma * static_cast<double>(vel));
+  x[idx] = xn;
+  xhist[static_cast<int64_t>(it.stage + 1) * stage_stride + idx] = xn;
+  vhist[static_cast<int64_t>(it.stage) * stage_stride + idx] = vel;
+}
+
+// grid (video blocks + action blocks per item, items); block = 8 warps.
+template <int NV4>
+__global__ void __launch_bounds__(256, NV4 <= 8 ? 2 : 1) final_euler_kernel(
     const float* __restrict__ h, const StepItem* __restrict__ items,
     const float* __restrict__ mods, int64_t mod_stride, int fin_off,
     const float* __restrict__ vout_w, const float* __restrict__ vout_b,
     const float* __restrict__ aout_w, const float* __restrict__ aout_b, float* __restrict__ x,
-    float* __restrict__ xhist, float* __restrict__ vhist, int64_t stage_stride, int T, int Bw,
-    int No, int Nv, int vd, int Na, int ad, int d) {
-  extern __shared__ float swt[];  // [2 heads][16 outputs][d]
+    float* __restrict__ xhist, float* __restrict__ vhist, int64_t stage_stride, int T, int No,
+    int Nv, int vd, int Na, int ad, int d, int vblocks, int ablocks) {
+  extern __shared__ __align__(16) uint8_t fe_smem[];
+  __shared__ float cvec[16];
   pdl_wait();
   pdl_launch_dependents();
-  const int lane = threadIdx.x & 31;
-  // Coalesced float4 reads of the [d, 16] heads, transposed into shared memory.
-  for (int i = threadIdx.x; i < 2 * 4 * d; i += blockDim.x) {
-    const int head = i / (4 * d), k = i - head * 4 * d, c = k >> 2, q = k & 3;
-    const float4 w = reinterpret_cast<const float4*>(head == 0 ? vout_w : aout_w)[k];
-    float* dst = swt + head * 16 * d + (4 * q) * d + c;
-    dst[0] = w.x;
-    dst[d] = w.y;
-    dst[2 * d] = w.z;
-    dst[3 * d] = w.w;
+  const int w = blockIdx.y;
+  const HeadRange hr = head_range(blockIdx.x, vblocks, ablocks, Nv, Na, 2);
+  if (hr.beg >= hr.end) return;  // whole block: no barrier below is skipped by only some threads
+  const bool video = hr.video;
+  const float* Wg = video ? vout_w : aout_w;
+  const float* shift = mods + w * mod_stride + fin_off;
+  const float* scale = shift + d;
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  float* Ws = reinterpret_cast<float*>(fe_smem);  // [16][d]
+  // Stage W' = (1 + scale) W from the [d, 16] head: 4 consecutive outputs of one k per thread.
+  for (int t = threadIdx.x; t < 4 * d; t += blockDim.x) {
+    const int k = t >> 2, q = t & 3;
+    const float4 wv = reinterpret_cast<const float4*>(Wg)[t];  // W[k][4q .. 4q+3]
+    const float sc = 1.0f + scale[k];
+    Ws[(4 * q) * d + k] = wv.x * sc;
+    Ws[(4 * q + 1) * d + k] = wv.y * sc;
+    Ws[(4 * q + 2) * d + k] = wv.z * sc;
+    Ws[(4 * q + 3) * d + k] = wv.w * sc;
+  }
+  // c[j] = b[j] + sum_k shift[k] W[k][j]: warp w sums outputs w and w + 8.
+  const int od = video ? vd : ad;
+  for (int j = warp; j < 16; j += kRowWarps) {
+    float sacc = 0.0f;
+    for (int k = lane; k < d; k += 32) sacc = fmaf(shift[k], Wg[k * 16 + j], sacc);
+    sacc = warp_sum(sacc);
+    if (lane == 0) cvec[j] = sacc + (j < od ? (video ? vout_b : aout_b)[j] : 0.0f);
   }
   __syncthreads();
+  const StepItem it = items[w];
   const int N = No + Nv + Na;
-  const int gv = (Nv + 1) / 2, ga = (Na + 1) / 2, groups = gv + ga;
-  const int64_t total = static_cast<int64_t>(Bw) * groups;
-  for (int64_t g = static_cast<int64_t>(blockIdx.x) * kRowWarps + (threadIdx.x >> 5); g < total;
-       g += static_cast<int64_t>(gridDim.x) * kRowWarps) {
-    const int w = static_cast<int>(g / groups), gi = static_cast<int>(g % groups);
-    const bool video = gi < gv;
-    const int r0 = video ? 2 * gi : Nv + 2 * (gi - gv);  // row among the item's video + action rows
-    const int nrows = video ? min(2, Nv - 2 * gi) : min(2, Na - 2 * (gi - gv));
-    const StepItem it = items[w];
-    const float* shift = mods + w * mod_stride + fin_off;
-    const float* scale = shift + d;
+  const int row0 = No + (video ? 0 : Nv);  // first token row of this head
+  const int64_t tbase = static_cast<int64_t>(it.ep) * T + (video ? 0 : static_cast<int64_t>(Nv) * vd);
+  for (int r = hr.beg + 2 * warp; r < hr.end; r += 2 * kRowWarps) {
+    const bool two = r + 1 < hr.end;
     float4 y0[NV4], y1[NV4];
-    ln_mod_row<NV4>(h + (static_cast<int64_t>(w) * N + No + r0) * d, shift, scale, d, lane, y0);
-    if (nrows == 2) ln_mod_row<NV4>(h + (static_cast<int64_t>(w) * N + No + r0 + 1) * d, shift, scale, d, lane, y1);
-    const float* Wt = swt + (video ? 0 : 16 * d);
+    ln_row<NV4>(h + (static_cast<int64_t>(w) * N + row0 + r) * d, d, lane, y0);
+    if (two) ln_row<NV4>(h + (static_cast<int64_t>(w) * N + row0 + r + 1) * d, d, lane, y1);
     float acc0[16], acc1[16];
 #pragma unroll
     for (int j = 0; j < 16; ++j) acc0[j] = acc1[j] = 0.0f;
@@ -342,28 +384,163 @@ __global__ void __launch_bounds__(256) final_euler_kernel(
       const int c = (lane + 32 * i) * 4;
 #pragma unroll
       for (int j = 0; j < 16; ++j) {
-        const float4 wv = *reinterpret_cast<const float4*>(Wt + j * d + c);
+        const float4 wv = *reinterpret_cast<const float4*>(Ws + j * d + c);
         acc0[j] = fmaf(y0[i].x, wv.x, fmaf(y0[i].y, wv.y, fmaf(y0[i].z, wv.z, fmaf(y0[i].w, wv.w, acc0[j]))));
-        if (nrows == 2)
+        if (two)
           acc1[j] = fmaf(y1[i].x, wv.x, fmaf(y1[i].y, wv.y, fmaf(y1[i].z, wv.z, fmaf(y1[i].w, wv.w, acc1[j]))));
       }
     }
     const float out0 = reduce_scatter16(acc0, lane);
     const float out1 = reduce_scatter16(acc1, lane);
-    const int od = video ? vd : ad;
-    const float bias = lane < od ? (video ? vout_b : aout_b)[lane] : 0.0f;
-    for (int rr = 0; rr < nrows; ++rr) {
-      if (lane < od) {
-        const int r = r0 + rr;
-        const float vel = (rr == 0 ? out0 : out1) + bias;
-        const int64_t idx = static_cast<int64_t>(it.ep) * T +
-                            (video ? static_cast<int64_t>(r) * vd
-                                   : static_cast<int64_t>(Nv) * vd + static_cast<int64_t>(r - Nv) * ad) +
-                            lane;
-        const float xn = static_cast<float>(static_cast<double>(x[idx]) + it.dsigma * static_cast<double>(vel));
-        x[idx] = xn;
-        xhist[static_cast<int64_t>(it.stage + 1) * stage_stride + idx] = xn;
-        vhist[static_cast<int64_t>(it.stage) * stage_stride + idx] = vel;
+    if (lane < od) {
+      const float cj = cvec[lane];
+      euler_store(it, tbase + static_cast<int64_t>(r) * od + lane, out0 + cj, x, xhist, vhist, stage_stride);
+      if (two) euler_store(it, tbase + static_cast<int64_t>(r + 1) * od + lane, out1 + cj, x, xhist, vhist, stage_stride);
+    }
+  }
+}
+
+WAM_DEV uint32_t bf16x2_bits(float lo, float hi) {
+  __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
+  return *reinterpret_cast<uint32_t*>(&v);
+}
+
+WAM_DEV void mma_bf16_16816(float (&c)[4], uint32_t a0, uint32_t a1, uint32_t a2, uint32_t a3, uint32_t b0,
+                            uint32_t b1) {
+  asm volatile(
+      "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, "
+      "{%0,%1,%2,%3};"
+      : "+f"(c[0]), "+f"(c[1]), "+f"(c[2]), "+f"(c[3])
+      : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
+}
+
+constexpr int kFtWarps = 4;   // warps per block of the tensor-core final kernel
+constexpr int kFtUnroll = 4;  // k-steps of 16 whose loads are issued together
+
+// Bf16 precision mode.  A warp owns 16 rows: lane (g = lane / 4, c = lane % 4) loads rows g and
+// g + 8 at columns k0 + 4c .. k0 + 4c + 3 of every 16-column step.  The fragment's logical k
+// order {2c, 2c+1, 2c+8, 2c+9} is mapped to these physical columns for both operands (a sum over
+// k does not depend on the order), so each row slice is one 16-byte load.  Row statistics are
+// accumulated from the same values around a per-row reference K (the row's first element), and
+// the tensor cores see bf16(h - K):  sum_k (h_k - mean) W'_kj = acc_j - (mean - K) colsum_j.
+// W' is staged as bf16 [16][d + 8] (the pad makes the 8-byte reads of a warp conflict-free).
+__global__ void __launch_bounds__(32 * kFtWarps) final_euler_tc_kernel(
+    const float* __restrict__ h, const StepItem* __restrict__ items,
+    const float* __restrict__ mods, int64_t mod_stride, int fin_off,
+    const float* __restrict__ vout_w, const float* __restrict__ vout_b,
+    const float* __restrict__ aout_w, const float* __restrict__ aout_b, float* __restrict__ x,
+    float* __restrict__ xhist, float* __restrict__ vhist, int64_t stage_stride, int T, int No,
+    int Nv, int vd, int Na, int ad, int d, int vblocks, int ablocks) {
+  extern __shared__ __align__(16) uint8_t fe_smem[];
+  __shared__ float cvec[16], colsum[16];
+  pdl_wait();
+  pdl_launch_dependents();
+  const int w = blockIdx.y;
+  const HeadRange hr = head_range(blockIdx.x, vblocks, ablocks, Nv, Na, 16);
+  if (hr.beg >= hr.end) return;  // whole block: no barrier below is skipped by only some threads
+  const bool video = hr.video;
+  const float* Wg = video ? vout_w : aout_w;
+  const float* shift = mods + w * mod_stride + fin_off;
+  const float* scale = shift + d;
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int ld = d + 8;
+  bf16* Ws = reinterpret_cast<bf16*>(fe_smem);  // [16][d + 8]
+#pragma unroll 4
+  for (int t = threadIdx.x; t < 4 * d; t += blockDim.x) {
+    const int k = t >> 2, q = t & 3;
+    const float4 wv = reinterpret_cast<const float4*>(Wg)[t];  // W[k][4q .. 4q+3]
+    const float sc = 1.0f + scale[k];
+    Ws[(4 * q) * ld + k] = __float2bfloat16(wv.x * sc);
+    Ws[(4 * q + 1) * ld + k] = __float2bfloat16(wv.y * sc);
+    Ws[(4 * q + 2) * ld + k] = __float2bfloat16(wv.z * sc);
+    Ws[(4 * q + 3) * ld + k] = __float2bfloat16(wv.w * sc);
+  }
+  __syncthreads();
+  // c[j] = b[j] + sum_k shift[k] W[k][j] and colsum[j] = sum_k W'_bf16[k][j]: warp w sums
+  // outputs w, w + 4, w + 8, w + 12.
+  const int od = video ? vd : ad;
+  for (int j = warp; j < 16; j += kFtWarps) {
+    float sc_acc = 0.0f, cs_acc = 0.0f;
+    for (int k = lane; k < d; k += 32) {
+      sc_acc = fmaf(shift[k], Wg[k * 16 + j], sc_acc);
+      cs_acc += __bfloat162float(Ws[j * ld + k]);
+    }
+    sc_acc = warp_sum(sc_acc);
+    cs_acc = warp_sum(cs_acc);
+    if (lane == 0) {
+      cvec[j] = sc_acc + (j < od ? (video ? vout_b : aout_b)[j] : 0.0f);
+      colsum[j] = cs_acc;
+    }
+  }
+  __syncthreads();
+  const StepItem it = items[w];
+  const int N = No + Nv + Na;
+  const int row0 = No + (video ? 0 : Nv);
+  const int64_t tbase = static_cast<int64_t>(it.ep) * T + (video ? 0 : static_cast<int64_t>(Nv) * vd);
+  const int g = lane >> 2, c = lane & 3;
+  const uint32_t wsa = static_cast<uint32_t>(__cvta_generic_to_shared(Ws));
+  for (int r0 = hr.beg + 16 * warp; r0 < hr.end; r0 += 16 * kFtWarps) {
+    const int ra = r0 + g, rb = r0 + g + 8;
+    const bool va = ra < hr.end, vb = rb < hr.end;
+    const float* pa = h + (static_cast<int64_t>(w) * N + row0 + (va ? ra : r0)) * d + 4 * c;
+    const float* pb = h + (static_cast<int64_t>(w) * N + row0 + (vb ? rb : r0)) * d + 4 * c;
+    const float Ka = va ? pa[-4 * c] : 0.0f, Kb = vb ? pb[-4 * c] : 0.0f;
+    float acc0[4] = {0.f, 0.f, 0.f, 0.f}, acc1[4] = {0.f, 0.f, 0.f, 0.f};
+    float s1a = 0.f, s2a = 0.f, s1b = 0.f, s2b = 0.f;
+    for (int k0 = 0; k0 < d; k0 += 16 * kFtUnroll) {
+      float4 xa[kFtUnroll], xb[kFtUnroll];
+#pragma unroll
+      for (int u = 0; u < kFtUnroll; ++u) {
+        const bool in = k0 + 16 * u < d;
+        xa[u] = (va && in) ? *reinterpret_cast<const float4*>(pa + k0 + 16 * u) : make_float4(Ka, Ka, Ka, Ka);
+        xb[u] = (vb && in) ? *reinterpret_cast<const float4*>(pb + k0 + 16 * u) : make_float4(Kb, Kb, Kb, Kb);
+      }
+#pragma unroll
+      for (int u = 0; u < kFtUnroll; ++u) {
+        const int kk = k0 + 16 * u;
+        if (kk >= d) break;
+        const float a0 = xa[u].x - Ka, a1 = xa[u].y - Ka, a2 = xa[u].z - Ka, a3 = xa[u].w - Ka;
+        const float b0 = xb[u].x - Kb, b1 = xb[u].y - Kb, b2 = xb[u].z - Kb, b3 = xb[u].w - Kb;
+        s1a += (a0 + a1) + (a2 + a3);
+        s2a = fmaf(a0, a0, fmaf(a1, a1, fmaf(a2, a2, fmaf(a3, a3, s2a))));
+        s1b += (b0 + b1) + (b2 + b3);
+        s2b = fmaf(b0, b0, fmaf(b1, b1, fmaf(b2, b2, fmaf(b3, b3, s2b))));
+        const uint32_t A0 = bf16x2_bits(a0, a1), A2 = bf16x2_bits(a2, a3);
+        const uint32_t A1 = bf16x2_bits(b0, b1), A3 = bf16x2_bits(b2, b3);
+        uint32_t B0, B1, C0, C1;  // outputs g (n-tile 0) and g + 8 (n-tile 1), columns kk + 4c ..
+        asm volatile("ld.shared.v2.b32 {%0, %1}, [%2];"
+                     : "=r"(B0), "=r"(B1)
+                     : "r"(wsa + static_cast<uint32_t>((g * ld + kk + 4 * c) * 2)));
+        asm volatile("ld.shared.v2.b32 {%0, %1}, [%2];"
+                     : "=r"(C0), "=r"(C1)
+                     : "r"(wsa + static_cast<uint32_t>(((g + 8) * ld + kk + 4 * c) * 2)));
+        mma_bf16_16816(acc0, A0, A1, A2, A3, B0, B1);
+        mma_bf16_16816(acc1, A0, A1, A2, A3, C0, C1);
+      }
+    }
+    // row statistics over the 4 lanes that share rows g and g + 8
+#pragma unroll
+    for (int m = 1; m <= 2; m <<= 1) {
+      s1a += __shfl_xor_sync(0xffffffffu, s1a, m);
+      s2a += __shfl_xor_sync(0xffffffffu, s2a, m);
+      s1b += __shfl_xor_sync(0xffffffffu, s1b, m);
+      s2b += __shfl_xor_sync(0xffffffffu, s2b, m);
+    }
+    const float inv_d = 1.0f / static_cast<float>(d);
+    const float ma = s1a * inv_d, mb = s1b * inv_d;  // mean - K
+    const float ra_std = rsqrtf(fmaxf(s2a * inv_d - ma * ma, 0.0f) + 1e-6f);
+    const float rb_std = rsqrtf(fmaxf(s2b * inv_d - mb * mb, 0.0f) + 1e-6f);
+    // accumulator layout: acc[0..1] row g, acc[2..3] row g + 8; columns 2c, 2c + 1 of the n-tile
+#pragma unroll
+    for (int nt = 0; nt < 2; ++nt) {
+      const float* acc = nt == 0 ? acc0 : acc1;
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        const int j = 8 * nt + 2 * c + (e & 1);
+        const bool top = e < 2;
+        if (j >= od || !(top ? va : vb)) continue;
+        const float vel = (top ? ra_std : rb_std) * (acc[e] - (top ? ma : mb) * colsum[j]) + cvec[j];
+        euler_store(it, tbase + static_cast<int64_t>(top ? ra : rb) * od + j, vel, x, xhist, vhist, stage_stride);
       }
     }
   }
@@ -387,10 +564,24 @@ __global__ void __launch_bounds__(256) tr_rms_partial_kernel(const AdaptItem* __
     const float* xr = xhist + it.r * stage_stride + static_cast<int64_t>(b) * T + beg;
     const float* xb = xhist + K * stage_stride + static_cast<int64_t>(b) * T + beg;
     const int end = min(len, (ch + 1) * kTrChunk);
-    for (int i = ch * kTrChunk + threadIdx.x; i < end; i += blockDim.x) {
-      const double u = (static_cast<double>(xr[i]) - static_cast<double>(xb[i])) / it.sigma_r;
-      s += u * u;
+    // every load of the chunk issued before the first use (the chunk is 8 rows of the block)
+    constexpr int kPer = kTrChunk / 256;
+    static_assert(kTrChunk % 256 == 0, "TR chunk is whole rows of the block");
+    float a[kPer], c[kPer];
+#pragma unroll
+    for (int u = 0; u < kPer; ++u) {
+      const int i = ch * kTrChunk + u * 256 + threadIdx.x;
+      a[u] = i < end ? xr[i] : 0.0f;
+      c[u] = i < end ? xb[i] : 0.0f;
     }
+    // sum of (x^r - x_bar)^2, scaled by 1 / sigma_r^2 once (no float64 division per element:
+    // float64 runs at a small fraction of the float32 rate on this part)
+#pragma unroll
+    for (int u = 0; u < kPer; ++u) {
+      const double v = static_cast<double>(a[u]) - static_cast<double>(c[u]);
+      s = fma(v, v, s);
+    }
+    s *= 1.0 / (it.sigma_r * it.sigma_r);
   }
   s = block_sum_d(s, red);
   if (threadIdx.x == 0) partial[(static_cast<int64_t>(b) * 2 + br) * nch + ch] = s;
@@ -407,17 +598,27 @@ __global__ void __launch_bounds__(256) adapt_apply_kernel(
     int64_t obs_elems, int normalize, int video_mode, int traj_blocks) {
   pdl_wait();
   pdl_launch_dependents();
-  __shared__ double rms[2];
+  __shared__ double rms[2], gain[2];
   __shared__ int zero[2];
   const int b = blockIdx.y;
   const AdaptItem it = items[b];
   if (it.op == kAdaptNone && !it.bind_obs) return;
   if (static_cast<int>(blockIdx.x) >= traj_blocks) {
     if (!it.bind_obs) return;
-    const int64_t base = static_cast<int64_t>(b) * obs_elems;
-    const int64_t start = static_cast<int64_t>(blockIdx.x - traj_blocks) * blockDim.x + threadIdx.x;
+    // obs_elems = No * d with d a multiple of 128: whole float4s, four in flight per thread
+    const int64_t n4 = obs_elems / 4;
+    const float4* src = reinterpret_cast<const float4*>(obs_new + static_cast<int64_t>(b) * obs_elems);
+    float4* dst = reinterpret_cast<float4*>(obs + static_cast<int64_t>(b) * obs_elems);
     const int64_t stride = static_cast<int64_t>(gridDim.x - traj_blocks) * blockDim.x;
-    for (int64_t i = start; i < obs_elems; i += stride) obs[base + i] = obs_new[base + i];
+    int64_t i = static_cast<int64_t>(blockIdx.x - traj_blocks) * blockDim.x + threadIdx.x;
+    for (; i + 3 * stride < n4; i += 4 * stride) {
+      const float4 v0 = src[i], v1 = src[i + stride], v2 = src[i + 2 * stride], v3 = src[i + 3 * stride];
+      dst[i] = v0;
+      dst[i + stride] = v1;
+      dst[i + 2 * stride] = v2;
+      dst[i + 3 * stride] = v3;
+    }
+    for (; i < n4; i += stride) dst[i] = src[i];
     return;
   }
   if (it.op == kAdaptNone) return;
@@ -430,39 +631,54 @@ __global__ void __launch_bounds__(256) adapt_apply_kernel(
     }
     rms[threadIdx.x] = normalize ? sqrt(ms) : 1.0;
     zero[threadIdx.x] = normalize && !(ms > 0.0);
+    // direction scale of Eq. 2 for this branch: sigma_b0 / (sigma_r rms); one float64 division
+    // here instead of two per element
+    gain[threadIdx.x] = zero[threadIdx.x] ? 0.0 : it.sigma_b0 / (it.sigma_r * rms[threadIdx.x]);
   }
   __syncthreads();
   const int64_t bo = static_cast<int64_t>(b) * T;
   const float* xr = xhist + it.r * stage_stride + bo;
   const float* xb = xhist + K * stage_stride + bo;
-  for (int j = blockIdx.x * blockDim.x + threadIdx.x; j < T; j += traj_blocks * blockDim.x) {
-    float val;
-    if (it.op == kAdaptCold) {
-      val = eps[bo + j];
-    } else if (it.op == kAdaptRestart) {
-      val = xb0[bo + j];
-    } else {
-      int src = -1;
-      int br = 0;
-      if (j < V) {
-        if (video_mode == 0) src = j;
+  const int stride = traj_blocks * blockDim.x;
+  // Four elements per thread and pass, every load issued before the first store.
+  for (int j0 = blockIdx.x * blockDim.x + threadIdx.x; j0 < T; j0 += 4 * stride) {
+    float val[4];
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      const int j = j0 + u * stride;
+      val[u] = 0.0f;
+      if (j >= T) continue;
+      if (it.op == kAdaptCold) {
+        val[u] = eps[bo + j];
+      } else if (it.op == kAdaptRestart) {
+        val[u] = xb0[bo + j];
       } else {
-        br = 1;
-        const int ja = j - V;
-        const int row = ja / ad, col = ja - row * ad;
-        const int srow = row + it.shift;
-        if (srow < Na) src = V + srow * ad + col;
-      }
-      if (src >= 0) {
-        const double u = (static_cast<double>(xr[src]) - static_cast<double>(xb[src])) / it.sigma_r;
-        const double dir = zero[br] ? 0.0 : u / rms[br];
-        val = static_cast<float>(static_cast<double>(xb[src]) + it.sigma_b0 * dir);
-      } else {
-        val = static_cast<float>(it.sigma_b0 * static_cast<double>(eps[bo + j]));
+        int src = -1;
+        int br = 0;
+        if (j < V) {
+          if (video_mode == 0) src = j;
+        } else {
+          br = 1;
+          const int ja = j - V;
+          const int row = ja / ad, col = ja - row * ad;
+          const int srow = row + it.shift;
+          if (srow < Na) src = V + srow * ad + col;
+        }
+        if (src >= 0) {
+          const double xbs = static_cast<double>(xb[src]);
+          val[u] = static_cast<float>(fma(gain[br], static_cast<double>(xr[src]) - xbs, xbs));
+        } else {
+          val[u] = static_cast<float>(it.sigma_b0 * static_cast<double>(eps[bo + j]));
+        }
       }
     }
-    x[bo + j] = val;
-    if (it.op != kAdaptRestart) xb0[bo + j] = val;
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      const int j = j0 + u * stride;
+      if (j >= T) continue;
+      x[bo + j] = val[u];
+      if (it.op != kAdaptRestart) xb0[bo + j] = val[u];
+    }
   }
 }
 
@@ -499,7 +715,7 @@ __global__ void __launch_bounds__(256) rr_probe_kernel(const float* __restrict__
                                                        double* __restrict__ partial) {
   pdl_wait();
   pdl_launch_dependents();
-  __shared__ double red[8];
+  __shared__ double red3[8][3];
   const int w = blockIdx.z, br = blockIdx.y, ch = blockIdx.x;
   const int ep = items[w].ep;
   const int64_t row0 = br == 0 ? 0 : split_row;
@@ -512,17 +728,41 @@ __global__ void __launch_bounds__(256) rr_probe_kernel(const float* __restrict__
   const int64_t beg4 = static_cast<int64_t>(ch) * (kProbeChunk / 4);
   const int64_t end4 = min(n_el / 4, beg4 + kProbeChunk / 4);
   float sia = 0.0f, saa = 0.0f, sii = 0.0f;
-  for (int64_t i = beg4 + threadIdx.x; i < end4; i += blockDim.x) {
-    const float4 hv = h4[i], qv = q4[i], av = a4[i];
-    const float p0 = hv.x - qv.x, p1 = hv.y - qv.y, p2 = hv.z - qv.z, p3 = hv.w - qv.w;
-    sia += (p0 * av.x + p1 * av.y) + (p2 * av.z + p3 * av.w);
-    saa += (av.x * av.x + av.y * av.y) + (av.z * av.z + av.w * av.w);
-    sii += (p0 * p0 + p1 * p1) + (p2 * p2 + p3 * p3);
+  // the chunk is 8 float4 rows of the block: two batches of four rows, loads issued first
+  for (int64_t i0 = beg4 + threadIdx.x; i0 < end4; i0 += 4 * blockDim.x) {
+    float4 hv[4], qv[4], av[4];
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      const int64_t i = i0 + u * blockDim.x;
+      const bool in = i < end4;
+      hv[u] = in ? h4[i] : make_float4(0.f, 0.f, 0.f, 0.f);
+      qv[u] = in ? q4[i] : make_float4(0.f, 0.f, 0.f, 0.f);
+      av[u] = in ? a4[i] : make_float4(0.f, 0.f, 0.f, 0.f);
+    }
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      const float p0 = hv[u].x - qv[u].x, p1 = hv[u].y - qv[u].y, p2 = hv[u].z - qv[u].z, p3 = hv[u].w - qv[u].w;
+      sia += (p0 * av[u].x + p1 * av[u].y) + (p2 * av[u].z + p3 * av[u].w);
+      saa += (av[u].x * av[u].x + av[u].y * av[u].y) + (av[u].z * av[u].z + av[u].w * av[u].w);
+      sii += (p0 * p0 + p1 * p1) + (p2 * p2 + p3 * p3);
+    }
   }
-  const double t0 = block_sum_d(sia, red);
-  const double t1 = block_sum_d(saa, red);
-  const double t2 = block_sum_d(sii, red);
+  // the three block sums share one barrier: warp sums, then thread 0 adds the warps in order
+  const double w0 = warp_sum_d(sia), w1 = warp_sum_d(saa), w2 = warp_sum_d(sii);
+  const int wi = threadIdx.x >> 5;
+  if ((threadIdx.x & 31) == 0) {
+    red3[wi][0] = w0;
+    red3[wi][1] = w1;
+    red3[wi][2] = w2;
+  }
+  __syncthreads();
   if (threadIdx.x == 0) {
+    double t0 = 0.0, t1 = 0.0, t2 = 0.0;
+    for (int v = 0; v < (blockDim.x >> 5); ++v) {
+      t0 += red3[v][0];
+      t1 += red3[v][1];
+      t2 += red3[v][2];
+    }
     double* out = partial + ((static_cast<int64_t>(w) * 2 + br) * nch + ch) * 3;
     out[0] = t0;
     out[1] = t1;
@@ -782,11 +1022,9 @@ cudaError_t final_euler(const float* h, const StepItem* items, const float* mods
                         int64_t mod_stride, int fin_off, const float* vout_w,
                         const float* vout_b, const float* aout_w, const float* aout_b, float* x,
                         float* xhist, float* vhist, int64_t stage_stride, int T, int Bw, int No,
-                        int Nv, int vd, int Na, int ad, int d, cudaStream_t s) {
+                        int Nv, int vd, int Na, int ad, int d, bool head_bf16, cudaStream_t s) {
   if (Bw <= 0) return cudaSuccess;
   if (d % 128 != 0 || vd > 16 || ad > 16) return cudaErrorInvalidValue;  // heads padded to 16
-  // One block per SM (or fewer), each staging both output heads once; warps stride over the
-  // row pairs.
   static std::atomic<int> sms_cached{0};  // contexts may run on several host threads
   int num_sms = sms_cached.load(std::memory_order_relaxed);
   if (num_sms == 0) {
@@ -796,33 +1034,49 @@ cudaError_t final_euler(const float* h, const StepItem* items, const float* mods
     if (num_sms < 1) num_sms = 1;
     sms_cached.store(num_sms, std::memory_order_relaxed);
   }
-  const int64_t units = static_cast<int64_t>(Bw) * ((Nv + 1) / 2 + (Na + 1) / 2);
-  const int64_t want = (units + kRowWarps - 1) / kRowWarps;
-  const unsigned grid = static_cast<unsigned>(want < 2 * num_sms ? want : 2 * num_sms);
-  const size_t smem = static_cast<size_t>(2) * d * 16 * sizeof(float);
-#define WAM_FE_CASE(NV)                                                                       \
-  case NV: {                                                                                  \
-    static std::atomic<int> smem_set{0};                                                      \
-    if (smem_set.load(std::memory_order_acquire) < static_cast<int>(smem)) {                  \
-      cudaError_t e = cudaFuncSetAttribute(final_euler_kernel<NV>,                           \
-                                           cudaFuncAttributeMaxDynamicSharedMemorySize,       \
-                                           static_cast<int>(smem));                           \
-      if (e != cudaSuccess) return e;                                                         \
-      int prev = smem_set.load(std::memory_order_relaxed);                                    \
-      while (prev < static_cast<int>(smem) &&                                                 \
-             !smem_set.compare_exchange_weak(prev, static_cast<int>(smem)))                   \
-        ;                                                                                     \
-    }                                                                                         \
-    launch_pdl(final_euler_kernel<NV>, dim3(grid), dim3(256), smem, s, h, items, mods, mod_stride, fin_off, vout_w,  \
-                                                vout_b, aout_w, aout_b, x, xhist, vhist,      \
-                                                stage_stride, T, Bw, No, Nv, vd, Na, ad, d); \
-    break;                                                                                    \
+  // An item's video rows are split over blocks (about four blocks per SM in all; at least a
+  // row pair per warp of the SIMT kernel, a 16-row tile per warp of the tensor-core kernel);
+  // its action rows take one block.
+  const int rows_per_block = head_bf16 ? 16 * kFtWarps : 2 * kRowWarps;
+  const int want = (4 * num_sms + Bw - 1) / Bw;
+  const int vmax = (Nv + rows_per_block - 1) / rows_per_block;
+  const int vblocks = Nv == 0 ? 0 : (want < vmax ? (want > 1 ? want : 1) : vmax);
+  const int ablocks = Na == 0 ? 0 : 1;
+  const size_t smem = head_bf16 ? static_cast<size_t>(16) * (d + 8) * sizeof(bf16) : static_cast<size_t>(16) * d * 4;
+  dim3 grid(vblocks + ablocks, Bw);
+#define WAM_SET_SMEM(KERNEL)                                                                       \
+  {                                                                                                \
+    static std::atomic<int> smem_set{0};                                                           \
+    if (smem_set.load(std::memory_order_acquire) < static_cast<int>(smem)) {                       \
+      cudaError_t e = cudaFuncSetAttribute(KERNEL, cudaFuncAttributeMaxDynamicSharedMemorySize,    \
+                                           static_cast<int>(smem));                                \
+      if (e != cudaSuccess) return e;                                                              \
+      int prev = smem_set.load(std::memory_order_relaxed);                                         \
+      while (prev < static_cast<int>(smem) &&                                                      \
+             !smem_set.compare_exchange_weak(prev, static_cast<int>(smem)))                        \
+        ;                                                                                          \
+    }                                                                                              \
   }
+  if (head_bf16) {
+    WAM_SET_SMEM(final_euler_tc_kernel)
+    launch_pdl(final_euler_tc_kernel, grid, dim3(32 * kFtWarps), smem, s, h, items, mods, mod_stride, fin_off,
+               vout_w, vout_b, aout_w, aout_b, x, xhist, vhist, stage_stride, T, No, Nv, vd, Na, ad, d, vblocks,
+               ablocks);
+    return cudaGetLastError();
+  }
+#define WAM_FE_CASE(NV)                                                                             \
+  case NV:                                                                                          \
+    WAM_SET_SMEM(final_euler_kernel<NV>)                                                            \
+    launch_pdl(final_euler_kernel<NV>, grid, dim3(256), smem, s, h, items, mods, mod_stride, fin_off, \
+               vout_w, vout_b, aout_w, aout_b, x, xhist, vhist, stage_stride, T, No, Nv, vd, Na, ad, d, \
+               vblocks, ablocks);                                                                   \
+    break;
   switch (d / 128) {
     WAM_NV4_CASES(WAM_FE_CASE)
     default: return cudaErrorInvalidValue;
   }
 #undef WAM_FE_CASE
+#undef WAM_SET_SMEM
   return cudaGetLastError();
 }
 
@@ -844,7 +1098,7 @@ cudaError_t adapt_apply(const AdaptItem* items, const double* partial, int nch, 
                         const float* eps, const float* obs_new, float* obs, int B, int T, int V,
                         int Na, int ad, int64_t obs_elems, int normalize, int video_mode,
                         cudaStream_t s) {
-  const int traj_blocks = (T + 255) / 256 < 64 ? (T + 255) / 256 : 64;
+  const int traj_blocks = (T + 1023) / 1024 < 64 ? (T + 1023) / 1024 : 64;  // ~4 elements per thread
   const int obs_blocks = static_cast<int>((obs_elems + 255) / 256 < 64 ? (obs_elems + 255) / 256 : 64);
   dim3 grid(traj_blocks + obs_blocks, B);
   launch_pdl(adapt_apply_kernel, dim3(grid), dim3(256), 0, s, items, partial, nch, x, xb0, xhist, stage_stride, K,

@@ -75,7 +75,7 @@ cudaError_t final_euler(const float* h, const StepItem* items, const float* mods
                         int64_t mod_stride, int fin_off, const float* vout_w,
                         const float* vout_b, const float* aout_w, const float* aout_b, float* x,
                         float* xhist, float* vhist, int64_t stage_stride, int T, int Bw, int No,
-                        int Nv, int vd, int Na, int ad, int d, cudaStream_t s);
+                        int Nv, int vd, int Na, int ad, int d, bool head_bf16, cudaStream_t s);
 
 int tr_num_chunks(int T, int V);
 cudaError_t tr_rms_partial(const AdaptItem* items, const float* xhist, int64_t stage_stride,

@@ -549,7 +549,7 @@ int run_steps(wam_ctx* c, wam_state* st, const std::vector<int>& n) {
               4.0 * Bw * double(c->Nv + c->Na) * d + 16.0 * Bw * c->T);
       CK(final_euler(c->h, c->d_items, c->mods, c->mod_n, 6 * L * d, c->vout_w, c->vout_b, c->aout_w, c->aout_b,
                      st->x, st->xhist, st->vhist, stage_stride, c->T, Bw, c->No, c->Nv, c->vd, c->Na, c->ad, d,
-                     c->stream));
+                     c->bf16, c->stream));
     }
     // bookkeeping (§3.4) and reuse statistics (App. D.2)
     for (int w = 0; w < Bw; ++w) {
