@@ -259,10 +259,10 @@ __global__ void __launch_bounds__(256) ln_mod_kernel(const float* __restrict__ h
 // ---------------------------------------------------------------- final layer + Euler
 // Modulated LN of a token row, the output head (16 columns; the [d, 16] heads are zero-padded),
 // the Euler update of that token's trajectory values and their retention.  The modulation is
-// folded into the head once per block: LN(h)(1+scale)+shift times W equals
-// xhat . W' + c with W'[k][j] = (1+scale[k]) W[k][j] and c[j] = b[j] + sum_k shift[k] W[k][j],
-// where xhat = (h - mean) rstd.  A block serves a contiguous range of one item's video (or
-// action) rows and stages only that head's W'.
+// folded into the head once per work item (final_head_prep_kernel): LN(h)(1+scale)+shift
+// times W equals xhat . W' + c with W'[k][j] = (1+scale[k]) W[k][j] and
+// c[j] = b[j] + sum_k shift[k] W[k][j], where xhat = (h - mean) rstd.  A block serves a
+// contiguous range of one item's video (or action) rows and copies only that head's W'.
 //
 // Float32 precision mode: SIMT dot products, a warp per row pair (each weight read from shared
 // memory serves both rows).  Bf16 precision mode: the head is a [rows, d] x [d, 16] product on
@@ -317,24 +317,108 @@ WAM_DEV HeadRange head_range(int bx, int vblocks, int ablocks, int Nv, int Na, i
   return r;
 }
 
-// Euler update x <- x + dsigma v of one trajectory value, retained as x^{k+1} and v^k.
-WAM_DEV void euler_store(const StepItem& it, int64_t idx, float vel, float* __restrict__ x,
+// Euler update x <- x + dsigma v of one trajectory value (its current value xv read earlier, so
+// that callers can issue those loads before any store), retained as x^{k+1} and v^k.
+WAM_DEV void euler_store(const StepItem& it, int64_t idx, float xv, float vel, float* __restrict__ x,
                          float* __restrict__ xhist, float* __restrict__ vhist, int64_t stage_stride) {
-  const float xn = static_cast<float>(static_cast<double>(x[idx]) + it.dsigma * static_cast<double>(vel));
+  const float xn = static_cast<float>(static_cast<double>(xv) + it.dsigma * static_cast<double>(vel));
   x[idx] = xn;
   xhist[static_cast<int64_t>(it.stage + 1) * stage_stride + idx] = xn;
   vhist[static_cast<int64_t>(it.stage) * stage_stride + idx] = vel;
 }
 
+// Head preparation, one block per (head, work item): W' = (1 + scale) W in the layout its
+// final kernel reads (float32 [16][d], or bf16 [16][d + 8]), c[j] = b[j] + sum_k shift[k] W[k][j]
+// and, for the bf16 layout, colsum[j] = sum_k W'_bf16[k][j].  Thread t covers k = t, t + 256, ..:
+// one pass over the [d, 16] head with every load of the pass issued together, then a block
+// reduction of the 32 sums.  Writes hw + (item * 2 + head) * head_stride bytes and
+// hc[(item * 2 + head) * 32 + (0..15: c, 16..31: colsum)].
+template <bool HB>
+__global__ void __launch_bounds__(256) final_head_prep_kernel(
+    const float* __restrict__ mods, int64_t mod_stride, int fin_off, const float* __restrict__ vout_w,
+    const float* __restrict__ vout_b, const float* __restrict__ aout_w, const float* __restrict__ aout_b,
+    int d, int vd, int ad, int Nv, int Na, uint8_t* __restrict__ hw, int64_t head_stride, float* __restrict__ hc) {
+  __shared__ float red[8][32];
+  pdl_wait();
+  pdl_launch_dependents();
+  const int head = blockIdx.x, w = blockIdx.y;
+  if ((head == 0 ? Nv : Na) == 0) return;
+  const float* Wg = head == 0 ? vout_w : aout_w;
+  const float* shift = mods + w * mod_stride + fin_off;
+  const float* scale = shift + d;
+  uint8_t* dst = hw + (static_cast<int64_t>(w) * 2 + head) * head_stride;
+  const int ld = d + 8;
+  float cacc[16], sacc[16];
+#pragma unroll
+  for (int j = 0; j < 16; ++j) cacc[j] = sacc[j] = 0.0f;
+  for (int k = threadIdx.x; k < d; k += blockDim.x) {
+    const float4* wr = reinterpret_cast<const float4*>(Wg + static_cast<int64_t>(k) * 16);
+    const float4 q0 = wr[0], q1 = wr[1], q2 = wr[2], q3 = wr[3];
+    const float wv[16] = {q0.x, q0.y, q0.z, q0.w, q1.x, q1.y, q1.z, q1.w,
+                          q2.x, q2.y, q2.z, q2.w, q3.x, q3.y, q3.z, q3.w};
+    const float sc = 1.0f + scale[k], sh = shift[k];
+#pragma unroll
+    for (int j = 0; j < 16; ++j) {
+      const float wp = wv[j] * sc;
+      cacc[j] = fmaf(sh, wv[j], cacc[j]);
+      if constexpr (HB) {
+        const bf16 b = __float2bfloat16(wp);
+        reinterpret_cast<bf16*>(dst)[j * ld + k] = b;
+        sacc[j] += __bfloat162float(b);
+      } else {
+        reinterpret_cast<float*>(dst)[j * d + k] = wp;
+      }
+    }
+  }
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+#pragma unroll
+  for (int j = 0; j < 16; ++j) {
+    const float a = warp_sum(cacc[j]);
+    const float b = warp_sum(sacc[j]);
+    if (lane == 0) {
+      red[warp][j] = a;
+      red[warp][16 + j] = b;
+    }
+  }
+  __syncthreads();
+  if (threadIdx.x < 32) {
+    float v = 0.0f;
+    for (int q = 0; q < static_cast<int>(blockDim.x >> 5); ++q) v += red[q][threadIdx.x];
+    const int j = threadIdx.x & 15;
+    const int od = head == 0 ? vd : ad;
+    if (threadIdx.x < 16) v += j < od ? (head == 0 ? vout_b : aout_b)[j] : 0.0f;
+    hc[(static_cast<int64_t>(w) * 2 + head) * 32 + threadIdx.x] = v;
+  }
+}
+
+// Copy `bytes` (a multiple of 16) from global to shared memory, eight 16-byte loads in flight
+// per thread.
+WAM_DEV void copy_to_smem(void* sdst, const void* gsrc, int bytes) {
+  const uint4* src = static_cast<const uint4*>(gsrc);
+  uint4* dst = static_cast<uint4*>(sdst);
+  const int n = bytes / 16;
+  for (int i0 = threadIdx.x; i0 < n; i0 += 8 * blockDim.x) {
+    uint4 v[8];
+#pragma unroll
+    for (int u = 0; u < 8; ++u) {
+      const int i = i0 + u * blockDim.x;
+      if (i < n) v[u] = src[i];
+    }
+#pragma unroll
+    for (int u = 0; u < 8; ++u) {
+      const int i = i0 + u * blockDim.x;
+      if (i < n) dst[i] = v[u];
+    }
+  }
+}
+
 // grid (video blocks + action blocks per item, items); block = 8 warps.
 template <int NV4>
 __global__ void __launch_bounds__(256, NV4 <= 8 ? 2 : 1) final_euler_kernel(
-    const float* __restrict__ h, const StepItem* __restrict__ items,
-    const float* __restrict__ mods, int64_t mod_stride, int fin_off,
-    const float* __restrict__ vout_w, const float* __restrict__ vout_b,
-    const float* __restrict__ aout_w, const float* __restrict__ aout_b, float* __restrict__ x,
+    const float* __restrict__ h, const StepItem* __restrict__ items, float* __restrict__ x,
     float* __restrict__ xhist, float* __restrict__ vhist, int64_t stage_stride, int T, int No,
-    int Nv, int vd, int Na, int ad, int d, int vblocks, int ablocks) {
+    int Nv, int vd, int Na, int ad, int d, int vblocks, int ablocks, const uint8_t* __restrict__ hw,
+    int64_t head_stride, const float* __restrict__ hc) {
   extern __shared__ __align__(16) uint8_t fe_smem[];
   __shared__ float cvec[16];
   pdl_wait();
@@ -343,29 +427,12 @@ __global__ void __launch_bounds__(256, NV4 <= 8 ? 2 : 1) final_euler_kernel(
   const HeadRange hr = head_range(blockIdx.x, vblocks, ablocks, Nv, Na, 2);
   if (hr.beg >= hr.end) return;  // whole block: no barrier below is skipped by only some threads
   const bool video = hr.video;
-  const float* Wg = video ? vout_w : aout_w;
-  const float* shift = mods + w * mod_stride + fin_off;
-  const float* scale = shift + d;
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  float* Ws = reinterpret_cast<float*>(fe_smem);  // [16][d]
-  // Stage W' = (1 + scale) W from the [d, 16] head: 4 consecutive outputs of one k per thread.
-  for (int t = threadIdx.x; t < 4 * d; t += blockDim.x) {
-    const int k = t >> 2, q = t & 3;
-    const float4 wv = reinterpret_cast<const float4*>(Wg)[t];  // W[k][4q .. 4q+3]
-    const float sc = 1.0f + scale[k];
-    Ws[(4 * q) * d + k] = wv.x * sc;
-    Ws[(4 * q + 1) * d + k] = wv.y * sc;
-    Ws[(4 * q + 2) * d + k] = wv.z * sc;
-    Ws[(4 * q + 3) * d + k] = wv.w * sc;
-  }
-  // c[j] = b[j] + sum_k shift[k] W[k][j]: warp w sums outputs w and w + 8.
+  const int hidx = w * 2 + (video ? 0 : 1);
+  float* Ws = reinterpret_cast<float*>(fe_smem);  // [16][d], prepared by final_head_prep_kernel
+  copy_to_smem(Ws, hw + hidx * head_stride, 16 * d * 4);
+  if (threadIdx.x < 16) cvec[threadIdx.x] = hc[hidx * 32 + threadIdx.x];
   const int od = video ? vd : ad;
-  for (int j = warp; j < 16; j += kRowWarps) {
-    float sacc = 0.0f;
-    for (int k = lane; k < d; k += 32) sacc = fmaf(shift[k], Wg[k * 16 + j], sacc);
-    sacc = warp_sum(sacc);
-    if (lane == 0) cvec[j] = sacc + (j < od ? (video ? vout_b : aout_b)[j] : 0.0f);
-  }
   __syncthreads();
   const StepItem it = items[w];
   const int N = No + Nv + Na;
@@ -373,6 +440,9 @@ __global__ void __launch_bounds__(256, NV4 <= 8 ? 2 : 1) final_euler_kernel(
   const int64_t tbase = static_cast<int64_t>(it.ep) * T + (video ? 0 : static_cast<int64_t>(Nv) * vd);
   for (int r = hr.beg + 2 * warp; r < hr.end; r += 2 * kRowWarps) {
     const bool two = r + 1 < hr.end;
+    const int64_t i0 = tbase + static_cast<int64_t>(r) * od + lane, i1 = i0 + od;
+    const float x0 = lane < od ? x[i0] : 0.0f;
+    const float x1 = (lane < od && two) ? x[i1] : 0.0f;
     float4 y0[NV4], y1[NV4];
     ln_row<NV4>(h + (static_cast<int64_t>(w) * N + row0 + r) * d, d, lane, y0);
     if (two) ln_row<NV4>(h + (static_cast<int64_t>(w) * N + row0 + r + 1) * d, d, lane, y1);
@@ -394,8 +464,8 @@ __global__ void __launch_bounds__(256, NV4 <= 8 ? 2 : 1) final_euler_kernel(
     const float out1 = reduce_scatter16(acc1, lane);
     if (lane < od) {
       const float cj = cvec[lane];
-      euler_store(it, tbase + static_cast<int64_t>(r) * od + lane, out0 + cj, x, xhist, vhist, stage_stride);
-      if (two) euler_store(it, tbase + static_cast<int64_t>(r + 1) * od + lane, out1 + cj, x, xhist, vhist, stage_stride);
+      euler_store(it, i0, x0, out0 + cj, x, xhist, vhist, stage_stride);
+      if (two) euler_store(it, i1, x1, out1 + cj, x, xhist, vhist, stage_stride);
     }
   }
 }
@@ -414,91 +484,80 @@ WAM_DEV void mma_bf16_16816(float (&c)[4], uint32_t a0, uint32_t a1, uint32_t a2
       : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
 }
 
-constexpr int kFtWarps = 4;   // warps per block of the tensor-core final kernel
-constexpr int kFtUnroll = 4;  // k-steps of 16 whose loads are issued together
+constexpr int kFtWarps = 4;   // warps per block of the tensor-core final kernel (one K quarter each)
+constexpr int kFtUnroll = 8;  // k-steps of 16 whose loads are issued together
 
-// Bf16 precision mode.  A warp owns 16 rows: lane (g = lane / 4, c = lane % 4) loads rows g and
-// g + 8 at columns k0 + 4c .. k0 + 4c + 3 of every 16-column step.  The fragment's logical k
-// order {2c, 2c+1, 2c+8, 2c+9} is mapped to these physical columns for both operands (a sum over
-// k does not depend on the order), so each row slice is one 16-byte load.  Row statistics are
-// accumulated from the same values around a per-row reference K (the row's first element), and
+// Bf16 precision mode.  A block takes 16-row tiles one at a time; warp q covers the K quarter
+// [q d / 4, (q + 1) d / 4) of the tile, so a row tile costs few dependent load batches even at
+// one episode.  Lane (g = lane / 4, c = lane % 4) loads rows g and g + 8 at columns
+// k0 + 4c .. k0 + 4c + 3 of every 16-column step; the fragment's logical k order
+// {2c, 2c+1, 2c+8, 2c+9} is mapped to these physical columns for both operands (a sum over k
+// does not depend on the order), so each row slice is one 16-byte load.  Row statistics are
+// accumulated from the same values around a per-row reference K (the row's first element) and
 // the tensor cores see bf16(h - K):  sum_k (h_k - mean) W'_kj = acc_j - (mean - K) colsum_j.
-// W' is staged as bf16 [16][d + 8] (the pad makes the 8-byte reads of a warp conflict-free).
+// The four quarters' partial accumulators and sums meet in shared memory and are added in
+// warp order by warp 0, which applies the Euler update.  W' is the prepared bf16 [16][d + 8]
+// copy (the pad makes the 8-byte reads of a warp conflict-free).
 __global__ void __launch_bounds__(32 * kFtWarps) final_euler_tc_kernel(
-    const float* __restrict__ h, const StepItem* __restrict__ items,
-    const float* __restrict__ mods, int64_t mod_stride, int fin_off,
-    const float* __restrict__ vout_w, const float* __restrict__ vout_b,
-    const float* __restrict__ aout_w, const float* __restrict__ aout_b, float* __restrict__ x,
+    const float* __restrict__ h, const StepItem* __restrict__ items, float* __restrict__ x,
     float* __restrict__ xhist, float* __restrict__ vhist, int64_t stage_stride, int T, int No,
-    int Nv, int vd, int Na, int ad, int d, int vblocks, int ablocks) {
+    int Nv, int vd, int Na, int ad, int d, int vblocks, int ablocks, const uint8_t* __restrict__ hw,
+    int64_t head_stride, const float* __restrict__ hc) {
   extern __shared__ __align__(16) uint8_t fe_smem[];
   __shared__ float cvec[16], colsum[16];
+  __shared__ float part[kFtWarps][12][32];  // per quarter: 8 accumulators + 4 row sums, per lane
   pdl_wait();
   pdl_launch_dependents();
   const int w = blockIdx.y;
   const HeadRange hr = head_range(blockIdx.x, vblocks, ablocks, Nv, Na, 16);
   if (hr.beg >= hr.end) return;  // whole block: no barrier below is skipped by only some threads
   const bool video = hr.video;
-  const float* Wg = video ? vout_w : aout_w;
-  const float* shift = mods + w * mod_stride + fin_off;
-  const float* scale = shift + d;
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const int ld = d + 8;
-  bf16* Ws = reinterpret_cast<bf16*>(fe_smem);  // [16][d + 8]
-#pragma unroll 4
-  for (int t = threadIdx.x; t < 4 * d; t += blockDim.x) {
-    const int k = t >> 2, q = t & 3;
-    const float4 wv = reinterpret_cast<const float4*>(Wg)[t];  // W[k][4q .. 4q+3]
-    const float sc = 1.0f + scale[k];
-    Ws[(4 * q) * ld + k] = __float2bfloat16(wv.x * sc);
-    Ws[(4 * q + 1) * ld + k] = __float2bfloat16(wv.y * sc);
-    Ws[(4 * q + 2) * ld + k] = __float2bfloat16(wv.z * sc);
-    Ws[(4 * q + 3) * ld + k] = __float2bfloat16(wv.w * sc);
-  }
-  __syncthreads();
-  // c[j] = b[j] + sum_k shift[k] W[k][j] and colsum[j] = sum_k W'_bf16[k][j]: warp w sums
-  // outputs w, w + 4, w + 8, w + 12.
+  const int hidx = w * 2 + (video ? 0 : 1);
+  bf16* Ws = reinterpret_cast<bf16*>(fe_smem);  // [16][d + 8], prepared by final_head_prep_kernel
+  copy_to_smem(Ws, hw + hidx * head_stride, 16 * ld * 2);
+  if (threadIdx.x < 32) (threadIdx.x < 16 ? cvec : colsum)[threadIdx.x & 15] = hc[hidx * 32 + threadIdx.x];
   const int od = video ? vd : ad;
-  for (int j = warp; j < 16; j += kFtWarps) {
-    float sc_acc = 0.0f, cs_acc = 0.0f;
-    for (int k = lane; k < d; k += 32) {
-      sc_acc = fmaf(shift[k], Wg[k * 16 + j], sc_acc);
-      cs_acc += __bfloat162float(Ws[j * ld + k]);
-    }
-    sc_acc = warp_sum(sc_acc);
-    cs_acc = warp_sum(cs_acc);
-    if (lane == 0) {
-      cvec[j] = sc_acc + (j < od ? (video ? vout_b : aout_b)[j] : 0.0f);
-      colsum[j] = cs_acc;
-    }
-  }
   __syncthreads();
   const StepItem it = items[w];
   const int N = No + Nv + Na;
   const int row0 = No + (video ? 0 : Nv);
   const int64_t tbase = static_cast<int64_t>(it.ep) * T + (video ? 0 : static_cast<int64_t>(Nv) * vd);
   const int g = lane >> 2, c = lane & 3;
-  const uint32_t wsa = static_cast<uint32_t>(__cvta_generic_to_shared(Ws));
-  for (int r0 = hr.beg + 16 * warp; r0 < hr.end; r0 += 16 * kFtWarps) {
+  const int ks = d / kFtWarps;  // K quarter (a multiple of 32: d is a multiple of 128)
+  const uint32_t wsa = static_cast<uint32_t>(__cvta_generic_to_shared(Ws)) + static_cast<uint32_t>(warp * ks * 2);
+  for (int r0 = hr.beg; r0 < hr.end; r0 += 16) {
     const int ra = r0 + g, rb = r0 + g + 8;
     const bool va = ra < hr.end, vb = rb < hr.end;
-    const float* pa = h + (static_cast<int64_t>(w) * N + row0 + (va ? ra : r0)) * d + 4 * c;
-    const float* pb = h + (static_cast<int64_t>(w) * N + row0 + (vb ? rb : r0)) * d + 4 * c;
-    const float Ka = va ? pa[-4 * c] : 0.0f, Kb = vb ? pb[-4 * c] : 0.0f;
+    const float* rowa = h + (static_cast<int64_t>(w) * N + row0 + (va ? ra : r0)) * d;
+    const float* rowb = h + (static_cast<int64_t>(w) * N + row0 + (vb ? rb : r0)) * d;
+    const float Ka = va ? rowa[0] : 0.0f, Kb = vb ? rowb[0] : 0.0f;
+    const float* pa = rowa + warp * ks + 4 * c;
+    const float* pb = rowb + warp * ks + 4 * c;
+    // This warp finishes accumulator entries 2 warp and 2 warp + 1 (n-tile warp / 2; row g for
+    // even warps, g + 8 for odd; columns 2c, 2c + 1): their trajectory values are read now.
+    const bool top = (warp & 1) == 0;
+    const int jbase = 8 * (warp >> 1) + 2 * c;
+    const bool vrow = top ? va : vb;
+    const int64_t ibase = tbase + static_cast<int64_t>(top ? ra : rb) * od;
+    float xv[2];
+#pragma unroll
+    for (int e = 0; e < 2; ++e) xv[e] = (vrow && jbase + e < od) ? x[ibase + jbase + e] : 0.0f;
     float acc0[4] = {0.f, 0.f, 0.f, 0.f}, acc1[4] = {0.f, 0.f, 0.f, 0.f};
     float s1a = 0.f, s2a = 0.f, s1b = 0.f, s2b = 0.f;
-    for (int k0 = 0; k0 < d; k0 += 16 * kFtUnroll) {
+    for (int k0 = 0; k0 < ks; k0 += 16 * kFtUnroll) {
       float4 xa[kFtUnroll], xb[kFtUnroll];
 #pragma unroll
       for (int u = 0; u < kFtUnroll; ++u) {
-        const bool in = k0 + 16 * u < d;
+        const bool in = k0 + 16 * u < ks;
         xa[u] = (va && in) ? *reinterpret_cast<const float4*>(pa + k0 + 16 * u) : make_float4(Ka, Ka, Ka, Ka);
         xb[u] = (vb && in) ? *reinterpret_cast<const float4*>(pb + k0 + 16 * u) : make_float4(Kb, Kb, Kb, Kb);
       }
 #pragma unroll
       for (int u = 0; u < kFtUnroll; ++u) {
         const int kk = k0 + 16 * u;
-        if (kk >= d) break;
+        if (kk >= ks) break;
         const float a0 = xa[u].x - Ka, a1 = xa[u].y - Ka, a2 = xa[u].z - Ka, a3 = xa[u].w - Ka;
         const float b0 = xb[u].x - Kb, b1 = xb[u].y - Kb, b2 = xb[u].z - Kb, b3 = xb[u].w - Kb;
         s1a += (a0 + a1) + (a2 + a3);
@@ -518,31 +577,47 @@ __global__ void __launch_bounds__(32 * kFtWarps) final_euler_tc_kernel(
         mma_bf16_16816(acc1, A0, A1, A2, A3, C0, C1);
       }
     }
-    // row statistics over the 4 lanes that share rows g and g + 8
 #pragma unroll
-    for (int m = 1; m <= 2; m <<= 1) {
-      s1a += __shfl_xor_sync(0xffffffffu, s1a, m);
-      s2a += __shfl_xor_sync(0xffffffffu, s2a, m);
-      s1b += __shfl_xor_sync(0xffffffffu, s1b, m);
-      s2b += __shfl_xor_sync(0xffffffffu, s2b, m);
+    for (int e = 0; e < 4; ++e) {
+      part[warp][e][lane] = acc0[e];
+      part[warp][4 + e][lane] = acc1[e];
     }
-    const float inv_d = 1.0f / static_cast<float>(d);
-    const float ma = s1a * inv_d, mb = s1b * inv_d;  // mean - K
-    const float ra_std = rsqrtf(fmaxf(s2a * inv_d - ma * ma, 0.0f) + 1e-6f);
-    const float rb_std = rsqrtf(fmaxf(s2b * inv_d - mb * mb, 0.0f) + 1e-6f);
-    // accumulator layout: acc[0..1] row g, acc[2..3] row g + 8; columns 2c, 2c + 1 of the n-tile
+    part[warp][8][lane] = s1a;
+    part[warp][9][lane] = s2a;
+    part[warp][10][lane] = s1b;
+    part[warp][11][lane] = s2b;
+    __syncthreads();
+    {
+      // the row's sums (entries 8, 9 for row g; 10, 11 for row g + 8), added over the quarters in
+      // warp order, then over the 4 lanes that share the row
+      const int se = top ? 8 : 10;
+      float s1 = part[0][se][lane], s2 = part[0][se + 1][lane];
 #pragma unroll
-    for (int nt = 0; nt < 2; ++nt) {
-      const float* acc = nt == 0 ? acc0 : acc1;
+      for (int q = 1; q < kFtWarps; ++q) {
+        s1 += part[q][se][lane];
+        s2 += part[q][se + 1][lane];
+      }
+      s1 += __shfl_xor_sync(0xffffffffu, s1, 1);
+      s1 += __shfl_xor_sync(0xffffffffu, s1, 2);
+      s2 += __shfl_xor_sync(0xffffffffu, s2, 1);
+      s2 += __shfl_xor_sync(0xffffffffu, s2, 2);
+      const float inv_d = 1.0f / static_cast<float>(d);
+      const float m = s1 * inv_d;  // mean - K
+      const float rs = rsqrtf(fmaxf(s2 * inv_d - m * m, 0.0f) + 1e-6f);
+      // accumulator layout: entries 4 n + {0, 1} row g, 4 n + {2, 3} row g + 8 of n-tile n
 #pragma unroll
-      for (int e = 0; e < 4; ++e) {
-        const int j = 8 * nt + 2 * c + (e & 1);
-        const bool top = e < 2;
-        if (j >= od || !(top ? va : vb)) continue;
-        const float vel = (top ? ra_std : rb_std) * (acc[e] - (top ? ma : mb) * colsum[j]) + cvec[j];
-        euler_store(it, tbase + static_cast<int64_t>(top ? ra : rb) * od + j, vel, x, xhist, vhist, stage_stride);
+      for (int e = 0; e < 2; ++e) {
+        const int pe = 2 * warp + e;
+        const int j = jbase + e;
+        if (!vrow || j >= od) continue;
+        float tot = part[0][pe][lane];
+#pragma unroll
+        for (int q = 1; q < kFtWarps; ++q) tot += part[q][pe][lane];
+        const float vel = rs * (tot - m * colsum[j]) + cvec[j];
+        euler_store(it, ibase + j, xv[e], vel, x, xhist, vhist, stage_stride);
       }
     }
+    __syncthreads();
   }
 }
 
@@ -715,7 +790,7 @@ __global__ void __launch_bounds__(256) rr_probe_kernel(const float* __restrict__
                                                        double* __restrict__ partial) {
   pdl_wait();
   pdl_launch_dependents();
-  __shared__ double red3[8][3];
+  __shared__ float red3[8][3];
   const int w = blockIdx.z, br = blockIdx.y, ch = blockIdx.x;
   const int ep = items[w].ep;
   const int64_t row0 = br == 0 ? 0 : split_row;
@@ -747,8 +822,10 @@ __global__ void __launch_bounds__(256) rr_probe_kernel(const float* __restrict__
       sii += (p0 * p0 + p1 * p1) + (p2 * p2 + p3 * p3);
     }
   }
-  // the three block sums share one barrier: warp sums, then thread 0 adds the warps in order
-  const double w0 = warp_sum_d(sia), w1 = warp_sum_d(saa), w2 = warp_sum_d(sii);
+  // The three block sums share one barrier: float32 warp trees, then thread 0 adds the warps in
+  // order; the chunk partials are combined in float64 by the gate.  (Float64 arithmetic runs at
+  // a small fraction of the float32 rate here: a float64 tree per chunk bounded this kernel.)
+  const float w0 = warp_sum(sia), w1 = warp_sum(saa), w2 = warp_sum(sii);
   const int wi = threadIdx.x >> 5;
   if ((threadIdx.x & 31) == 0) {
     red3[wi][0] = w0;
@@ -757,7 +834,7 @@ __global__ void __launch_bounds__(256) rr_probe_kernel(const float* __restrict__
   }
   __syncthreads();
   if (threadIdx.x == 0) {
-    double t0 = 0.0, t1 = 0.0, t2 = 0.0;
+    float t0 = 0.0f, t1 = 0.0f, t2 = 0.0f;
     for (int v = 0; v < (blockDim.x >> 5); ++v) {
       t0 += red3[v][0];
       t1 += red3[v][1];
@@ -1018,11 +1095,18 @@ cudaError_t ln_modulate(const float* h, float* hcopy, const float* mods, int64_t
   return cudaGetLastError();
 }
 
+int64_t final_head_bytes(int d) {
+  const int64_t a = static_cast<int64_t>(16) * (d + 8) * 2, b = static_cast<int64_t>(16) * d * 4;
+  const int64_t m = a > b ? a : b;
+  return (m + 15) / 16 * 16;
+}
+
 cudaError_t final_euler(const float* h, const StepItem* items, const float* mods,
                         int64_t mod_stride, int fin_off, const float* vout_w,
                         const float* vout_b, const float* aout_w, const float* aout_b, float* x,
                         float* xhist, float* vhist, int64_t stage_stride, int T, int Bw, int No,
-                        int Nv, int vd, int Na, int ad, int d, bool head_bf16, cudaStream_t s) {
+                        int Nv, int vd, int Na, int ad, int d, bool head_bf16, uint8_t* head_ws,
+                        float* head_const, cudaStream_t s) {
   if (Bw <= 0) return cudaSuccess;
   if (d % 128 != 0 || vd > 16 || ad > 16) return cudaErrorInvalidValue;  // heads padded to 16
   static std::atomic<int> sms_cached{0};  // contexts may run on several host threads
@@ -1034,14 +1118,22 @@ cudaError_t final_euler(const float* h, const StepItem* items, const float* mods
     if (num_sms < 1) num_sms = 1;
     sms_cached.store(num_sms, std::memory_order_relaxed);
   }
-  // An item's video rows are split over blocks (about four blocks per SM in all; at least a
-  // row pair per warp of the SIMT kernel, a 16-row tile per warp of the tensor-core kernel);
-  // its action rows take one block.
-  const int rows_per_block = head_bf16 ? 16 * kFtWarps : 2 * kRowWarps;
-  const int want = (4 * num_sms + Bw - 1) / Bw;
+  const int64_t hstride = final_head_bytes(d);
+  if (head_bf16)
+    launch_pdl(final_head_prep_kernel<true>, dim3(2, Bw), dim3(256), 0, s, mods, mod_stride, fin_off, vout_w, vout_b,
+               aout_w, aout_b, d, vd, ad, Nv, Na, head_ws, hstride, head_const);
+  else
+    launch_pdl(final_head_prep_kernel<false>, dim3(2, Bw), dim3(256), 0, s, mods, mod_stride, fin_off, vout_w, vout_b,
+               aout_w, aout_b, d, vd, ad, Nv, Na, head_ws, hstride, head_const);
+  // An item's video rows are split over blocks so that all blocks are resident at once (the
+  // register limit: four 4-warp blocks of the tensor-core kernel or two 8-warp blocks of the SIMT
+  // kernel per SM), with at least a 16-row tile per tensor-core block or a row pair per SIMT
+  // warp; its action rows take one block (one per 16-row tile).
+  const int rows_per_block = head_bf16 ? 16 : 2 * kRowWarps;
+  const int want = ((head_bf16 ? 4 : 2) * num_sms + Bw - 1) / Bw;
   const int vmax = (Nv + rows_per_block - 1) / rows_per_block;
   const int vblocks = Nv == 0 ? 0 : (want < vmax ? (want > 1 ? want : 1) : vmax);
-  const int ablocks = Na == 0 ? 0 : 1;
+  const int ablocks = Na == 0 ? 0 : (head_bf16 ? (Na + 15) / 16 : 1);
   const size_t smem = head_bf16 ? static_cast<size_t>(16) * (d + 8) * sizeof(bf16) : static_cast<size_t>(16) * d * 4;
   dim3 grid(vblocks + ablocks, Bw);
 #define WAM_SET_SMEM(KERNEL)                                                                       \
@@ -1059,17 +1151,17 @@ cudaError_t final_euler(const float* h, const StepItem* items, const float* mods
   }
   if (head_bf16) {
     WAM_SET_SMEM(final_euler_tc_kernel)
-    launch_pdl(final_euler_tc_kernel, grid, dim3(32 * kFtWarps), smem, s, h, items, mods, mod_stride, fin_off,
-               vout_w, vout_b, aout_w, aout_b, x, xhist, vhist, stage_stride, T, No, Nv, vd, Na, ad, d, vblocks,
-               ablocks);
+    launch_pdl(final_euler_tc_kernel, grid, dim3(32 * kFtWarps), smem, s, h, items, x, xhist, vhist, stage_stride, T,
+               No, Nv, vd, Na, ad, d, vblocks, ablocks, static_cast<const uint8_t*>(head_ws), hstride,
+               static_cast<const float*>(head_const));
     return cudaGetLastError();
   }
 #define WAM_FE_CASE(NV)                                                                             \
   case NV:                                                                                          \
     WAM_SET_SMEM(final_euler_kernel<NV>)                                                            \
-    launch_pdl(final_euler_kernel<NV>, grid, dim3(256), smem, s, h, items, mods, mod_stride, fin_off, \
-               vout_w, vout_b, aout_w, aout_b, x, xhist, vhist, stage_stride, T, No, Nv, vd, Na, ad, d, \
-               vblocks, ablocks);                                                                   \
+    launch_pdl(final_euler_kernel<NV>, grid, dim3(256), smem, s, h, items, x, xhist, vhist, stage_stride, T, No, \
+               Nv, vd, Na, ad, d, vblocks, ablocks, static_cast<const uint8_t*>(head_ws), hstride,  \
+               static_cast<const float*>(head_const));                                              \
     break;
   switch (d / 128) {
     WAM_NV4_CASES(WAM_FE_CASE)

@@ -75,7 +75,11 @@ cudaError_t final_euler(const float* h, const StepItem* items, const float* mods
                         int64_t mod_stride, int fin_off, const float* vout_w,
                         const float* vout_b, const float* aout_w, const float* aout_b, float* x,
                         float* xhist, float* vhist, int64_t stage_stride, int T, int Bw, int No,
-                        int Nv, int vd, int Na, int ad, int d, bool head_bf16, cudaStream_t s);
+                        int Nv, int vd, int Na, int ad, int d, bool head_bf16, uint8_t* head_ws,
+                        float* head_const, cudaStream_t s);
+// Bytes per (work item, head) of the prepared-head scratch of final_euler (head_ws holds
+// 2 * items of them; head_const 64 floats per item).
+int64_t final_head_bytes(int d);
 
 int tr_num_chunks(int T, int V);
 cudaError_t tr_rms_partial(const AdaptItem* items, const float* xhist, int64_t stage_stride,

@@ -116,6 +116,9 @@ struct wam_ctx {
   size_t part_doubles = 0;
   float* d_eps = nullptr;
   float* d_obs_new = nullptr;
+  // final layer: each work item's modulated output heads, prepared once per step
+  uint8_t* d_fhead = nullptr;
+  float* d_fconst = nullptr;
   int* d_err = nullptr;
   // pinned host staging
   uint8_t* ring = nullptr;
@@ -549,7 +552,7 @@ int run_steps(wam_ctx* c, wam_state* st, const std::vector<int>& n) {
               4.0 * Bw * double(c->Nv + c->Na) * d + 16.0 * Bw * c->T);
       CK(final_euler(c->h, c->d_items, c->mods, c->mod_n, 6 * L * d, c->vout_w, c->vout_b, c->aout_w, c->aout_b,
                      st->x, st->xhist, st->vhist, stage_stride, c->T, Bw, c->No, c->Nv, c->vd, c->Na, c->ad, d,
-                     c->bf16, c->stream));
+                     c->bf16, c->d_fhead, c->d_fconst, c->stream));
     }
     // bookkeeping (§3.4) and reuse statistics (App. D.2)
     for (int w = 0; w < Bw; ++w) {
@@ -818,6 +821,8 @@ int create_impl(wam_ctx* c, const wam_config* cfg, const float* weights, size_t 
   TRY(dalloc(c, c->allocs, &c->d_adapt, c->Bmax));
   TRY(dalloc(c, c->allocs, &c->d_eps, size_t(c->Bmax) * c->T));
   TRY(dalloc(c, c->allocs, &c->d_obs_new, size_t(c->Bmax) * c->No * c->d));
+  TRY(dalloc(c, c->allocs, &c->d_fhead, size_t(c->Bmax) * 2 * size_t(final_head_bytes(c->d))));
+  TRY(dalloc(c, c->allocs, &c->d_fconst, size_t(c->Bmax) * 64));
   TRY(dalloc(c, c->allocs, &c->d_err, 1));
   CK(cudaMemset(c->d_err, 0, sizeof(int)));
   // scratch for the float64 partial sums of TR / OR / RR reductions
