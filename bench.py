@@ -497,7 +497,8 @@ def run_independent(dev, n_steps=50, warmup=5):
     arrives the video branch rebinds and finishes its 4 steps while the action branch remaps
     with the executed shift 8, enters stage 5 and runs 5 steps.  Timed twice: the two
     continuations through wam_continue_many (one host thread per context, overlapping on the
-    GPU; the action stream has the higher priority) and as two wam_continue calls in sequence.
+    GPU; the action stream has the higher priority), as two wam_continue calls in sequence, and
+    in sequence with the action branch first (the shortest observation-to-action time).
     O2A = real observation to action chunk."""
     import torch
 
@@ -515,7 +516,7 @@ def run_independent(dev, n_steps=50, warmup=5):
         ctxs.append(W.Context(cfg, flat, stream=s.cuda_stream))
         del flat
     vctx, actx = ctxs
-    total = 2 * (warmup + n_steps) + 1
+    total = 3 * (warmup + n_steps) + 1
     proc = I.ObsProcess(cv, 1, seed=5)
     with torch.cuda.stream(sv):
         obs0 = torch.from_numpy(proc.obs.copy()).to(dev)
@@ -535,7 +536,7 @@ def run_independent(dev, n_steps=50, warmup=5):
     b0v, pv = cv["tr_entry_stage"], cv["prefix_steps"]
     ev = lambda: torch.cuda.Event(enable_timing=True)
 
-    def control_step(inp, concurrent, marks=None):
+    def control_step(inp, mode, marks=None):
         pred, real, eps_v, eps_a = inp
         if marks is not None:
             marks[0].record(sv)
@@ -550,10 +551,10 @@ def run_independent(dev, n_steps=50, warmup=5):
         s2 = vctx.adapt(vst, real)[0]
         kv = b0v + pv if s2 == W.ADAPT_REBIND_ACCEPT else b0v
         calls = [(vctx, vst, K - kv, None, vout), (actx, ast, K - ca["tr_entry_stage"], aout, None)]
-        if concurrent:
+        if mode == "concurrent":
             W.Context.continue_many(calls)
         else:
-            for c in calls:
+            for c in (calls if mode == "sequential" else calls[::-1]):
                 c[0].continue_(c[1], c[2], c[3], c[4])
         if marks is not None:
             marks[2].record(sa)          # action chunk ready
@@ -562,27 +563,26 @@ def run_independent(dev, n_steps=50, warmup=5):
 
     res = {}
     t = 0
-    for concurrent in (True, False):
+    for mode in ("concurrent", "sequential", "action_first"):
         for _ in range(warmup):
-            control_step(inputs[t], concurrent)
+            control_step(inputs[t], mode)
             t += 1
         vctx.reset_stats()
         actx.reset_stats()
         torch.cuda.synchronize(dev)
         marks = [[ev() for _ in range(4)] for _ in range(n_steps)]
         for i in range(n_steps):
-            control_step(inputs[t], concurrent, marks[i])
+            control_step(inputs[t], mode, marks[i])
             t += 1
         torch.cuda.synchronize(dev)
         total_ms = marks[0][0].elapsed_time(marks[-1][3])
         step_ms = [m[0].elapsed_time(m[3]) for m in marks]
         o2a_ms = [m[1].elapsed_time(m[2]) for m in marks]
-        key = "concurrent" if concurrent else "sequential"
-        res[key] = {"chunks_per_s": n_steps / (total_ms * 1e-3), "ms_per_step": total_ms / n_steps,
+        res[mode] = {"chunks_per_s": n_steps / (total_ms * 1e-3), "ms_per_step": total_ms / n_steps,
                     "step_ms_p50": float(np.percentile(step_ms, 50)),
                     "o2a_ms_p50": float(np.percentile(o2a_ms, 50)),
                     "o2a_ms_p99": float(np.percentile(o2a_ms, 99))}
-        if concurrent:
+        if mode == "concurrent":
             for name, c in (("video", vctx), ("action", actx)):
                 st = c.stats()
                 res.setdefault("reuse", {})[name] = {
