@@ -3,10 +3,17 @@
     python -m paper_2609_34608_gb300.kernel_bench gemm M N K [--iters I]
     python -m paper_2609_34608_gb300.kernel_bench attn B N H [--iters I] [--impl tc|mma]
     python -m paper_2609_34608_gb300.kernel_bench step CONFIG [--batch B] [--rounds R] [--relax-gate]
+    python -m paper_2609_34608_gb300.kernel_bench sweep CONFIG B1 B2 ... [--relax-gate]
 
 Each invocation builds the library if needed, warms up, captures `iters` back-to-back launches in
 a CUDA graph, times a replay with CUDA events and prints one JSON line (microseconds per launch
 and algorithmic TFLOP/s: 2MNK for the GEMM, 4 B N^2 d for attention).
+
+`sweep` runs one warm round (the profile's Trajectory Remapping, then its remaining steps) at
+each batch size with the library's kernel-class timing on
+(CUDA events on its stream) and prints, per size, the achieved algorithmic bandwidth of the
+residual-stream and adaptation kernel classes (final layer + Euler, TR / OR adaptation, RR probe,
+RR apply, LN) as fractions of the measured copy bandwidth.
 
 `step` drives a named model configuration (inputs.NAMED_CONFIGS) through the library's public
 calls with seeded synthetic inputs: a cold sample of all episodes, then R warm rounds, each a
@@ -109,9 +116,56 @@ def bench_step(name: str, batch: int, rounds: int, relax_gate: bool) -> dict:
     return out
 
 
+def bench_sweep(name: str, batches: list, relax_gate: bool) -> list:
+    import json as _json
+    import os
+
+    import numpy as np
+
+    from . import inputs as I
+    root = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+    peaks_path = os.path.join(root, "MEASURED_PEAKS.json")
+    hbm = _json.load(open(peaks_path))["hbm_gbs"] if os.path.exists(peaks_path) else 6800.0
+    dev = torch.device("cuda")
+    over = dict(rr_gamma_cos=-1.0, rr_gamma_fit=1e30) if relax_gate else {}
+    out = []
+    bmax = max(batches)
+    cfg = I.get_config(name, batch=bmax, **over)
+    K = cfg["n_steps"]
+    stream = torch.cuda.Stream()
+    ctx = W.Context(cfg, I.flatten_weights(I.make_weights(cfg)), stream=stream.cuda_stream, batch_max=bmax)
+    for batch in batches:
+        st = ctx.state(batch)
+        shift = np.full(batch, int(cfg["shift"]), np.int32)
+        b0 = int(cfg["tr_entry_stage"])  # the profile's entry stage (its retained stage is valid)
+        with torch.cuda.stream(stream):
+            obs = [torch.from_numpy(I.make_obs(cfg, batch, seed=100 + i)).to(dev) for i in range(3)]
+            eps = [torch.from_numpy(I.make_fresh_eps(cfg, batch, i)).to(dev) for i in range(3)]
+            noise = torch.from_numpy(I.make_noise(cfg, batch)).to(dev)
+            ctx.sample_cold(st, obs[0], noise, K)
+            ctx.adapt(st, obs[1], shift=shift, fresh_noise=eps[1])
+            ctx.continue_(st, np.full(batch, K - b0, np.int32))
+            ctx.profile_enable(True)
+            ctx.adapt(st, obs[2], shift=shift, fresh_noise=eps[2])
+            ctx.continue_(st, np.full(batch, K - b0, np.int32))
+            prof = ctx.profile_read()
+            ctx.profile_enable(False)
+        row = {"config": name, "batch": batch}
+        for k in ("final", "adapt", "rr_probe", "rr_apply", "norm"):
+            v = prof[k]
+            if v["ms"] > 0:
+                gbs = v["bytes"] / (v["ms"] * 1e-3) / 1e9
+                row[k] = {"launches": v["launches"], "us_per_launch": 1e3 * v["ms"] / max(1, v["launches"]),
+                          "gbs": gbs, "frac": gbs / hbm}
+        out.append(row)
+        st.close()
+    ctx.close()
+    return out
+
+
 def main() -> None:
     ap = argparse.ArgumentParser()
-    ap.add_argument("kind", choices=["gemm", "attn", "step"])
+    ap.add_argument("kind", choices=["gemm", "attn", "step", "sweep"])
     ap.add_argument("dims", nargs="+")
     ap.add_argument("--iters", type=int, default=20)
     ap.add_argument("--impl", choices=["tc", "mma"], default="tc")
@@ -124,6 +178,9 @@ def main() -> None:
         print(json.dumps(bench_gemm(*map(int, a.dims), a.iters)))
     elif a.kind == "attn":
         print(json.dumps(bench_attn(*map(int, a.dims), a.iters, a.impl)))
+    elif a.kind == "sweep":
+        for row in bench_sweep(a.dims[0], [int(b) for b in a.dims[1:]], a.relax_gate):
+            print(json.dumps(row))
     else:
         print(json.dumps(bench_step(a.dims[0], a.batch, a.rounds, a.relax_gate)))
 
