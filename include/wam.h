@@ -294,6 +294,14 @@ int wam_profile_read(wam_ctx* ctx, wam_kclass_timing* out /* [WAM_KCLASS_COUNT] 
  *   the full forward at sigma_k on its current latent and bound observation and writes
  *   out[l] = |h_{l+1} - h_l| / |h_l| for every layer l (h_0 = the token embedding), the hidden
  *   state change of App. E.  The state is not modified (context scratch only).
+ * wam_diag_reuse_error: for one episode at its pending stage k with a retained RR layer state,
+ *   the residual-reuse output error of App. E, E_out = |y_reuse - y_full| / |y_full| on identical
+ *   inputs: y_full the full forward at sigma_k, y_reuse the forward whose middle layers [s, e) are
+ *   replaced by h_s + alpha R_a (Eq. 9) with alpha per branch from Eq. 7 against the retained
+ *   layer state, whatever the Eq. 8 checks say.  alpha_out [2] (nullable) receives the factors
+ *   (0 for a branch the model does not have).  The state is not modified.  Errors:
+ *   WAM_ERR_INVALID_ARG also when the profile has no RR boundaries; WAM_ERR_BAD_STATE also when
+ *   the episode has no retained layer state yet.
  * n (resp. n_rows * row_len) is at most batch_max * tokens * d_model.  Errors:
  * WAM_ERR_INVALID_ARG (null, sizes), WAM_ERR_BAD_STATE (episode finished or not started).
  */
@@ -301,6 +309,8 @@ int wam_diag_similarity(wam_ctx* ctx, const float* a, const float* b, int64_t n,
                         double* rel_l2_out);
 int wam_diag_action_rmse(wam_ctx* ctx, const float* a, const float* b, int32_t n_rows,
                          int32_t row_len, int32_t dims, double* out);
+int wam_diag_reuse_error(wam_ctx* ctx, wam_state* state, int32_t episode, double* e_out,
+                         double* alpha_out);
 int wam_diag_layer_deltas(wam_ctx* ctx, wam_state* state, int32_t episode,
                           double* out /* [n_layers] */);
 

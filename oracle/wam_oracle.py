@@ -18,8 +18,8 @@ States", arXiv 2609.34608):
 * Observation Rebinding (§3.2, Eq. 4 consistency score and the kappa rule),
 * Residual Rescaling (§3.3, Eqs. 5-9),
 * the coordinating state machine (§3.4) and the reuse statistics (App. D.2, Eqs. 14-15),
-* the state-continuity diagnostics (App. E): latent similarity across replans, action RMSE and
-  the per-layer hidden-state change.
+* the state-continuity diagnostics (App. E): latent similarity across replans, action RMSE, the
+  per-layer hidden-state change and the residual-reuse output error.
 
 Precision: every array is promoted to float64 and every reduction is a float64 numpy reduction.
 
@@ -645,6 +645,18 @@ def layer_deltas(W, cfg: OracleConfig, x_traj, obs, sigma: float):
         out.append(float(np.linalg.norm(h1 - h) / np.linalg.norm(h)))
         h = h1
     return out
+
+
+def reuse_output_error(W, cfg: OracleConfig, x_traj, obs, sigma: float, layer: LayerState):
+    """App. E residual-reuse diagnostic at one step: E_out = |y_reuse - y_full| / |y_full| on
+    identical inputs, y_full the full forward and y_reuse the forward whose middle layers are
+    replaced by h_s + alpha R_a (Eq. 9), alpha per branch from Eq. 7 against the retained layer
+    state whatever the Eq. 8 checks say.  Returns (E_out, [alpha per branch])."""
+    y_full = velocity(W, cfg, x_traj, obs, sigma)
+    y_reuse, _, rec = velocity_rr(W, cfg, x_traj, obs, sigma, layer, True, forced_accept=True,
+                                  margin_tol=math.inf)
+    err = float(np.linalg.norm(y_reuse - y_full) / np.linalg.norm(y_full))
+    return err, [c.alpha for c in rec.checks]
 
 
 def action_rmse(a, b, dims=None):

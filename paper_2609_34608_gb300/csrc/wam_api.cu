@@ -1325,18 +1325,23 @@ int wam_diag_action_rmse(wam_ctx* c, const float* a, const float* b, int32_t n_r
   return WAM_OK;
 }
 
-int wam_diag_layer_deltas(wam_ctx* c, wam_state* st, int32_t episode, double* out) {
-  if (c == nullptr || st == nullptr || st->ctx != c || out == nullptr || episode < 0 || episode >= st->B)
-    return WAM_ERR_INVALID_ARG;
+}  // extern "C"
+
+namespace {
+
+// Conditioning and token embedding of one episode at its pending stage k into context scratch
+// (work item 0: modulations row 0, residual stream c->h); the state itself is not modified (the
+// observation embedding is recomputed from the bound observation, which it derives from).
+int diag_embed_item(wam_ctx* c, wam_state* st, int episode) {
   const int k = st->meta[episode].stage;
-  if (k < 0 || k >= c->K) return fail(c, WAM_ERR_BAD_STATE, "the episode has no pending denoising stage");
-  const int d = c->d, N = c->N;
+  const int d = c->d;
   StepItem it;
   it.ep = episode;
   it.stage = k;
   it.sigma = c->sigma[k];
   it.dsigma = c->sigma[k + 1] - c->sigma[k];
   TRY(upload(c, c->d_items, &it, sizeof(StepItem)));
+  TRY(obs_embed(c, st));
   {
     const CondGemv g{nullptr, 0, nullptr, 0, 1, c->d_items, c->t_w1, false, 256, d, 1, kT1Splits, c->t1, nullptr};
     CK(cond_gemv(g, c->stream));
@@ -1353,12 +1358,93 @@ int wam_diag_layer_deltas(wam_ctx* c, wam_state* st, int32_t episode, double* ou
   // the embedding records the latent it reads: point that record at scratch (stage stride 0)
   CK(embed_tokens(c->h, c->hq, 0, c->d_items, st->x, c->T, st->obs_emb, c->vid_w, c->vid_b, c->act_w, c->act_b,
                   c->pos, 1, c->No, c->Nv, c->vd, c->Na, c->ad, d, c->stream));
+  return WAM_OK;
+}
+
+// Output head + Euler kernel of work item 0 written to scratch only: x, x^{k+1} and v^k of a
+// stand-in item (episode 0, stage 0, stage stride 0) in three separate T-float buffers, the
+// velocity ending in `v_out`.
+int diag_final(wam_ctx* c, const float* hb, float* x_scratch, float* xn_scratch, float* v_out) {
+  StepItem s;
+  s.ep = 0;
+  s.stage = 0;
+  s.sigma = 0.0;
+  s.dsigma = 0.0;
+  TRY(upload(c, c->d_uitems, &s, sizeof(StepItem)));
+  CK(final_euler(hb, c->d_uitems, c->mods, c->mod_n, 6 * c->L * c->d, c->vout_w, c->vout_b, c->aout_w, c->aout_b,
+                 x_scratch, xn_scratch, v_out, 0, c->T, 1, c->No, c->Nv, c->vd, c->Na, c->ad, c->d, c->bf16, c->d_fhead,
+                 c->d_fconst, c->stream));
+  return WAM_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+int wam_diag_layer_deltas(wam_ctx* c, wam_state* st, int32_t episode, double* out) {
+  if (c == nullptr || st == nullptr || st->ctx != c || out == nullptr || episode < 0 || episode >= st->B)
+    return WAM_ERR_INVALID_ARG;
+  const int k = st->meta[episode].stage;
+  if (k < 0 || k >= c->K) return fail(c, WAM_ERR_BAD_STATE, "the episode has no pending denoising stage");
+  const int d = c->d, N = c->N;
+  TRY(diag_embed_item(c, st, episode));
   for (int l = 0; l < c->L; ++l) {
     CK(cudaMemcpyAsync(c->hm, c->h, size_t(N) * d * sizeof(float), cudaMemcpyDeviceToDevice, c->stream));
     TRY(run_layer(c, l, c->h, 1, nullptr, nullptr));
     double v[4];
     TRY(diag_sums(c, c->h, c->hm, int64_t(N) * d, int64_t(N) * d, int64_t(N) * d, v));
     out[l] = std::sqrt(v[3]) / std::sqrt(v[2]);
+  }
+  return WAM_OK;
+}
+
+int wam_diag_reuse_error(wam_ctx* c, wam_state* st, int32_t episode, double* e_out, double* alpha_out) {
+  if (c == nullptr || st == nullptr || st->ctx != c || e_out == nullptr || episode < 0 || episode >= st->B)
+    return WAM_ERR_INVALID_ARG;
+  const int k = st->meta[episode].stage;
+  if (k < 0 || k >= c->K) return fail(c, WAM_ERR_BAD_STATE, "the episode has no pending denoising stage");
+  const wam_config& g = c->cfg;
+  if (!(0 < g.rr_q && g.rr_q < g.rr_s && g.rr_s < g.rr_e && g.rr_e < g.n_layers))
+    return fail(c, WAM_ERR_INVALID_ARG, "the profile has no RR layer boundaries 0 < q < s < e < n_layers");
+  if (!st->meta[episode].rr_valid) return fail(c, WAM_ERR_BAD_STATE, "the episode has no retained layer state");
+  const int d = c->d, N = c->N, L = c->L, T = c->T;
+  const int q = g.rr_q, s = g.rr_s, e = g.rr_e;
+  const int split_row = c->split;
+  TRY(diag_embed_item(c, st, episode));
+  // head and probe layers: h = h_s, hq = h_q
+  for (int l = 0; l < s; ++l) TRY(run_layer(c, l, c->h, 1, nullptr, l == q ? c->hq : nullptr));
+  // Eq. 7 factors against the retained probe residual (the Eq. 8 checks are not applied)
+  const int nch = rr_num_chunks(int64_t(std::max(split_row, N - split_row)) * d);
+  CK(rr_probe_partial(c->h, c->hq, st->pa, c->d_items, 1, N, d, split_row, nch, c->d_part, c->stream));
+  CK(rr_gate(c->d_part, 1, nch, int64_t(split_row) * d, int64_t(N - split_row) * d, g.rr_alpha_min, g.rr_alpha_max,
+             g.rr_eps, g.rr_gamma_cos, g.rr_gamma_fit, c->d_gate, c->stream));
+  RRGate gates[2];
+  TRY(readback(c, gates, c->d_gate, sizeof(gates)));
+  // velocity scratch: three T-float buffers for each pass, past the h_q rows no longer needed
+  float* xs = c->d_eps;
+  float* full_v = c->hq;
+  float* full_xn = c->hq + T;
+  float* reuse_v = c->hq + 2 * T;
+  // full computation: middle and tail layers on a copy of h_s
+  CK(cudaMemcpyAsync(c->hm, c->h, size_t(N) * d * sizeof(float), cudaMemcpyDeviceToDevice, c->stream));
+  for (int l = s; l < L; ++l) TRY(run_layer(c, l, c->hm, 1, nullptr, nullptr));
+  TRY(diag_final(c, c->hm, xs, full_xn, full_v));
+  // reuse: h_e = h_s + alpha R_a per branch (Eq. 9), then the tail layers
+  RRApply ap;
+  ap.mode = kRRInject;
+  ap.cidx = 0;
+  ap.alpha0 = static_cast<float>(gates[0].alpha);
+  ap.alpha1 = static_cast<float>(gates[1].alpha);
+  TRY(upload(c, c->d_rrapply, &ap, sizeof(RRApply)));
+  CK(rr_apply(c->h, c->hm, c->hq, st->pa, st->ra, c->d_items, c->d_rrapply, 1, N, d, split_row, c->stream));
+  for (int l = e; l < L; ++l) TRY(run_layer(c, l, c->h, 1, nullptr, nullptr));
+  TRY(diag_final(c, c->h, xs, full_xn, reuse_v));
+  double v[4];
+  TRY(diag_sums(c, reuse_v, full_v, T, T, T, v));
+  *e_out = std::sqrt(v[3]) / std::sqrt(v[2]);
+  if (alpha_out != nullptr) {
+    alpha_out[0] = split_row == 0 ? 0.0 : gates[0].alpha;
+    alpha_out[1] = split_row == N ? 0.0 : gates[1].alpha;
   }
   return WAM_OK;
 }

@@ -135,6 +135,7 @@ def lib() -> ctypes.CDLL:
         "wam_diag_similarity": (ctypes.c_int, [_vp, _vp, _vp, ctypes.c_int64, _vp, _vp]),
         "wam_diag_action_rmse": (ctypes.c_int, [_vp, _vp, _vp, _i32, _i32, _i32, _vp]),
         "wam_diag_layer_deltas": (ctypes.c_int, [_vp, _vp, _i32, _vp]),
+        "wam_diag_reuse_error": (ctypes.c_int, [_vp, _vp, _i32, _vp, _vp]),
         "wam_op_attention": (ctypes.c_int, [_vp, _vp, _i32, _i32, _i32, _i32, _i32, _vp]),
         "wam_op_ln_modulate": (ctypes.c_int, [_vp, _vp, _vp, ctypes.c_int64, _vp, _i32, _i32, _i32, _i32, _vp]),
         "wam_op_last_error": (ctypes.c_char_p, []),
@@ -318,6 +319,14 @@ class Context:
         out = np.zeros(int(self.cfg["n_layers"]), dtype=np.float64)
         self._check(lib().wam_diag_layer_deltas(self.handle, st.handle, int(episode), out.ctypes.data))
         return out
+
+    def diag_reuse_error(self, st: "State", episode: int) -> tuple[float, list]:
+        """App. E: output error of residual reuse against full computation at the episode's pending
+        stage, and the Eq. 7 factor per branch."""
+        e = ctypes.c_double()
+        al = (ctypes.c_double * 2)()
+        self._check(lib().wam_diag_reuse_error(self.handle, st.handle, int(episode), ctypes.byref(e), al))
+        return e.value, [al[0], al[1]]
 
     def set_graph_replay(self, enable: bool):
         """CUDA-graph replay of the layer stack (default on); off launches every kernel."""

@@ -606,3 +606,51 @@ def test_single_branch_models_denoise_their_own_trajectory():
         want = np.concatenate([(y[a0:a1] @ W["vout_w"].astype(np.float64) + W["vout_b"]).ravel(),
                                (y[a1:] @ W["aout_w"].astype(np.float64) + W["aout_b"]).ravel()])
         assert np.allclose(v, want, atol=1e-12)
+
+
+# ----------------------------------------------------------------------------- App. E reuse error
+def test_reuse_output_error_zero_on_identical_inputs():
+    """A layer state retained from the same inputs makes alpha = 1 and h_s + R_a = h_e: the
+    reuse output equals the full one (Eq. 9 on identical inputs)."""
+    cfgd = micro_config(n_layers=6, rr_policy=1, rr_q=1, rr_s=2, rr_e=5)
+    W, cfg = _setup(cfgd, std=0.3)
+    rng = np.random.default_rng(40)
+    x = rng.standard_normal(cfg.traj_len)
+    obs = rng.standard_normal((cfg.n_obs, cfg.d_model))
+    _, layer, _ = O.velocity_rr(W, cfg, x, obs, 0.5, None, True)
+    err, alphas = O.reuse_output_error(W, cfg, x, obs, 0.5, layer)
+    assert err < 1e-12 and alphas == [1.0, 1.0]
+
+
+def test_reuse_output_error_bruteforce():
+    """E_out against a direct evaluation: embed, layers [0, s), h_s + alpha_b R_a on each
+    branch's rows with alpha_b the clamped least-squares ratio of Eq. 7 written out by loops,
+    layers [e, L), output head; the state retained at another noise level."""
+    cfgd = micro_config(n_layers=6, rr_policy=1, rr_q=1, rr_s=2, rr_e=5, rr_alpha_max=2.0)
+    W, cfg = _setup(cfgd, std=0.3)
+    rng = np.random.default_rng(41)
+    x0, x1 = rng.standard_normal(cfg.traj_len), rng.standard_normal(cfg.traj_len)
+    obs = rng.standard_normal((cfg.n_obs, cfg.d_model))
+    _, layer, _ = O.velocity_rr(W, cfg, x0, obs, 0.7, None, True)
+    err, alphas = O.reuse_output_error(W, cfg, x1, obs, 0.4, layer)
+    mods, fin = O.conditioning(W, cfg, 0.4)
+    h = O.embed(W, cfg, x1, obs)
+    for l in range(cfg.rr_q):
+        h = O.dit_layer(W, cfg, h, l, mods[l])
+    h_q = h.copy()
+    for l in range(cfg.rr_q, cfg.rr_s):
+        h = O.dit_layer(W, cfg, h, l, mods[l])
+    h_s = h.copy()
+    split = cfg.n_obs + cfg.n_video
+    for b, (a0, a1) in enumerate(((0, split), (split, cfg.n_tokens))):
+        pi = (h_s[a0:a1] - h_q[a0:a1]).ravel().tolist()
+        pa = layer.p_a[a0:a1].ravel().tolist()
+        alpha = min(max(sum(u * v for u, v in zip(pi, pa)) / sum(v * v for v in pa), 1.0), 2.0)
+        assert alphas[b] == pytest.approx(alpha, rel=1e-12)
+        h[a0:a1] = h_s[a0:a1] + alpha * layer.R_a[a0:a1]
+    for l in range(cfg.rr_e, cfg.n_layers):
+        h = O.dit_layer(W, cfg, h, l, mods[l])
+    y_reuse = O.final_velocity(W, cfg, h, fin)
+    y_full = O.velocity(W, cfg, x1, obs, 0.4)
+    want = np.linalg.norm(y_reuse - y_full) / np.linalg.norm(y_full)
+    assert err == pytest.approx(want, rel=1e-12) and err > 1e-3
