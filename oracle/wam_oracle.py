@@ -9,8 +9,8 @@ What it computes (paper: "Efficient World Action Model Inference with Adaptive I
 States", arXiv 2609.34608):
 
 * the DiT denoiser the method runs inside.  The paper cites DiT (§1) and never defines the
-  network; the builder's definition is written out in ``embed`` / ``dit_layer`` /
-  ``final_velocity`` and listed among the readings in the design doc,
+  network; the definition used here (token embedding, adaLN-modulated blocks, output heads) is
+  written out in ``embed`` / ``dit_layer`` / ``final_velocity``,
 * the Euler integration of the flow over the step schedule (§3.2 "native solver"; App. B.1,
   Table 5 and the Fast-WAM schedule values),
 * Trajectory Remapping (§3.1, Eq. 1 direction, Eq. 2 remapped init; App. B.1 Eq. 12 unit-RMS
