@@ -922,7 +922,14 @@ int wam_create(const wam_config* cfg, const float* weights, size_t n_weights, vo
   wam_ctx* c = new (std::nothrow) wam_ctx();
   if (c == nullptr) return WAM_ERR_OOM;
   std::memset(c->ring_ev, 0, sizeof(c->ring_ev));
-  const int r = create_impl(c, cfg, weights, n_weights, stream);
+  int r;
+  try {  // no exception crosses the C ABI
+    r = create_impl(c, cfg, weights, n_weights, stream);
+  } catch (const std::bad_alloc&) {
+    r = fail(c, WAM_ERR_OOM, "host allocation failed");
+  } catch (...) {
+    r = fail(c, WAM_ERR_CUDA, "unexpected host exception");
+  }
   if (r != WAM_OK) {
     std::fprintf(stderr, "wam_create: %s\n", c->err.c_str());
     destroy_impl(c);
@@ -947,7 +954,7 @@ int wam_set_stream(wam_ctx* c, void* stream) {
   return WAM_OK;
 }
 
-int wam_state_create(wam_ctx* c, int32_t batch, wam_state** out) {
+int wam_state_create(wam_ctx* c, int32_t batch, wam_state** out) try {
   if (c == nullptr || out == nullptr) return WAM_ERR_INVALID_ARG;
   *out = nullptr;
   if (batch < 1 || batch > c->Bmax) return fail(c, WAM_ERR_INVALID_ARG, "batch outside [1, batch_max]");
@@ -983,6 +990,10 @@ int wam_state_create(wam_ctx* c, int32_t batch, wam_state** out) {
   st->meta.assign(batch, EpisodeMeta());
   *out = st;
   return WAM_OK;
+} catch (const std::bad_alloc&) {
+  return fail(c, WAM_ERR_OOM, "host allocation failed");
+} catch (...) {
+  return fail(c, WAM_ERR_CUDA, "unexpected host exception");
 }
 
 void wam_state_destroy(wam_state* st) {
@@ -993,7 +1004,7 @@ void wam_state_destroy(wam_state* st) {
 }
 
 int wam_adapt_state(wam_ctx* c, wam_state* st, const float* new_obs, const int32_t* executed_shift,
-                    const int32_t* entry_stage, const float* fresh_noise, int32_t* status_out) {
+                    const int32_t* entry_stage, const float* fresh_noise, int32_t* status_out) try {
   if (c == nullptr || st == nullptr || st->ctx != c) return WAM_ERR_INVALID_ARG;
   if (new_obs == nullptr) return fail(c, WAM_ERR_INVALID_ARG, "new_obs is required");
   const int B = st->B;
@@ -1120,9 +1131,13 @@ int wam_adapt_state(wam_ctx* c, wam_state* st, const float* new_obs, const int32
   c->stats.n_bind += dstats.n_bind;
   if (status_out) std::memcpy(status_out, status.data(), sizeof(int32_t) * B);
   return WAM_OK;
+} catch (const std::bad_alloc&) {
+  return fail(c, WAM_ERR_OOM, "host allocation failed");
+} catch (...) {
+  return fail(c, WAM_ERR_CUDA, "unexpected host exception");
 }
 
-int wam_continue(wam_ctx* c, wam_state* st, const int32_t* n_steps, float* actions_out, float* video_out) {
+int wam_continue(wam_ctx* c, wam_state* st, const int32_t* n_steps, float* actions_out, float* video_out) try {
   if (c == nullptr || st == nullptr || st->ctx != c || n_steps == nullptr) return WAM_ERR_INVALID_ARG;
   std::vector<int> n(st->B);
   for (int b = 0; b < st->B; ++b) {
@@ -1138,10 +1153,14 @@ int wam_continue(wam_ctx* c, wam_state* st, const int32_t* n_steps, float* actio
   TRY(copy_out(c, st, actions_out, video_out, host_out));
   if (host_out) TRY(sync_check(c));
   return WAM_OK;
+} catch (const std::bad_alloc&) {
+  return fail(c, WAM_ERR_OOM, "host allocation failed");
+} catch (...) {
+  return fail(c, WAM_ERR_CUDA, "unexpected host exception");
 }
 
 int wam_continue_many(int32_t n, wam_ctx* const* ctxs, wam_state* const* states, const int32_t* const* n_steps,
-                      float* const* actions_out, float* const* video_out, int32_t* status_out) {
+                      float* const* actions_out, float* const* video_out, int32_t* status_out) try {
   if (n < 1 || ctxs == nullptr || states == nullptr || n_steps == nullptr) return WAM_ERR_INVALID_ARG;
   for (int i = 0; i < n; ++i) {
     if (ctxs[i] == nullptr || states[i] == nullptr || states[i]->ctx != ctxs[i] || n_steps[i] == nullptr)
@@ -1179,15 +1198,23 @@ int wam_continue_many(int32_t n, wam_ctx* const* ctxs, wam_state* const* states,
     if (first == WAM_OK) first = rc[i];
   }
   return first;
+} catch (const std::bad_alloc&) {
+  return fail((n > 0 && ctxs != nullptr ? ctxs[0] : nullptr), WAM_ERR_OOM, "host allocation failed");
+} catch (...) {
+  return fail((n > 0 && ctxs != nullptr ? ctxs[0] : nullptr), WAM_ERR_CUDA, "unexpected host exception");
 }
 
-int wam_sample_cold(wam_ctx* c, wam_state* st, const float* obs, const float* noise, int32_t n_steps, float* actions_out) {
+int wam_sample_cold(wam_ctx* c, wam_state* st, const float* obs, const float* noise, int32_t n_steps, float* actions_out) try {
   if (c == nullptr || st == nullptr || st->ctx != c || obs == nullptr || noise == nullptr) return WAM_ERR_INVALID_ARG;
   if (n_steps < 1 || n_steps > c->K) return fail(c, WAM_ERR_INVALID_ARG, "n_steps outside [1, K]");
   std::vector<int32_t> entry(st->B, WAM_ENTRY_COLD);
   TRY(wam_adapt_state(c, st, obs, nullptr, entry.data(), noise, nullptr));
   std::vector<int32_t> n(st->B, n_steps);
   return wam_continue(c, st, n.data(), actions_out, nullptr);
+} catch (const std::bad_alloc&) {
+  return fail(c, WAM_ERR_OOM, "host allocation failed");
+} catch (...) {
+  return fail(c, WAM_ERR_CUDA, "unexpected host exception");
 }
 
 int wam_get_stats(wam_ctx* c, wam_stats* out) {
@@ -1210,7 +1237,7 @@ int wam_state_log(const wam_state* st, wam_step_record* out, int32_t capacity, i
   return WAM_OK;
 }
 
-int wam_state_read(wam_ctx* c, const wam_state* st, int32_t field, int32_t index, void* out, size_t n_bytes) {
+int wam_state_read(wam_ctx* c, const wam_state* st, int32_t field, int32_t index, void* out, size_t n_bytes) try {
   if (c == nullptr || st == nullptr || out == nullptr || st->ctx != c) return WAM_ERR_INVALID_ARG;
   if (field == WAM_FIELD_META) {
     const size_t need = size_t(st->B) * 8 * sizeof(int32_t);
@@ -1230,9 +1257,13 @@ int wam_state_read(wam_ctx* c, const wam_state* st, int32_t field, int32_t index
   CK(cudaMemcpyAsync(out, p, bytes, cudaMemcpyDefault, c->stream));
   if (!is_device_ptr(out)) TRY(sync_check(c));
   return WAM_OK;
+} catch (const std::bad_alloc&) {
+  return fail(c, WAM_ERR_OOM, "host allocation failed");
+} catch (...) {
+  return fail(c, WAM_ERR_CUDA, "unexpected host exception");
 }
 
-int wam_state_write(wam_ctx* c, wam_state* st, int32_t field, int32_t index, const void* in, size_t n_bytes) {
+int wam_state_write(wam_ctx* c, wam_state* st, int32_t field, int32_t index, const void* in, size_t n_bytes) try {
   if (c == nullptr || st == nullptr || in == nullptr || st->ctx != c) return WAM_ERR_INVALID_ARG;
   if (field == WAM_FIELD_META) {
     const size_t need = size_t(st->B) * 8 * sizeof(int32_t);
@@ -1265,11 +1296,19 @@ int wam_state_write(wam_ctx* c, wam_state* st, int32_t field, int32_t index, con
   CK(cudaMemcpyAsync(p, in, bytes, cudaMemcpyDefault, c->stream));
   if (!is_device_ptr(in)) CK(cudaStreamSynchronize(c->stream));
   return WAM_OK;
+} catch (const std::bad_alloc&) {
+  return fail(c, WAM_ERR_OOM, "host allocation failed");
+} catch (...) {
+  return fail(c, WAM_ERR_CUDA, "unexpected host exception");
 }
 
-int wam_sync(wam_ctx* c) {
+int wam_sync(wam_ctx* c) try {
   if (c == nullptr) return WAM_ERR_INVALID_ARG;
   return sync_check(c);
+} catch (const std::bad_alloc&) {
+  return fail(c, WAM_ERR_OOM, "host allocation failed");
+} catch (...) {
+  return fail(c, WAM_ERR_CUDA, "unexpected host exception");
 }
 
 // ------------------------------------------------------------------- diagnostics (App. E)
@@ -1304,7 +1343,7 @@ int diag_sums(wam_ctx* c, const float* a, const float* b, int64_t n, int64_t row
 
 }  // namespace
 
-int wam_diag_similarity(wam_ctx* c, const float* a, const float* b, int64_t n, double* cos_out, double* rel_l2_out) {
+int wam_diag_similarity(wam_ctx* c, const float* a, const float* b, int64_t n, double* cos_out, double* rel_l2_out) try {
   if (c == nullptr || a == nullptr || b == nullptr || cos_out == nullptr || rel_l2_out == nullptr) return WAM_ERR_INVALID_ARG;
   double v[4];
   TRY(diag_sums(c, a, b, n, n, n, v));
@@ -1312,10 +1351,14 @@ int wam_diag_similarity(wam_ctx* c, const float* a, const float* b, int64_t n, d
   *cos_out = (na > 0.0 && nb > 0.0) ? v[0] / (na * nb) : 0.0;
   *rel_l2_out = nb > 0.0 ? dist / nb : (dist == 0.0 ? 0.0 : HUGE_VAL);
   return WAM_OK;
+} catch (const std::bad_alloc&) {
+  return fail(c, WAM_ERR_OOM, "host allocation failed");
+} catch (...) {
+  return fail(c, WAM_ERR_CUDA, "unexpected host exception");
 }
 
 int wam_diag_action_rmse(wam_ctx* c, const float* a, const float* b, int32_t n_rows, int32_t row_len, int32_t dims,
-                         double* out) {
+                         double* out) try {
   if (c == nullptr || a == nullptr || b == nullptr || out == nullptr || n_rows <= 0 || row_len <= 0 || dims <= 0 ||
       dims > row_len)
     return WAM_ERR_INVALID_ARG;
@@ -1323,6 +1366,10 @@ int wam_diag_action_rmse(wam_ctx* c, const float* a, const float* b, int32_t n_r
   TRY(diag_sums(c, a, b, int64_t(n_rows) * row_len, row_len, dims, v));
   *out = std::sqrt(v[3] / (double(n_rows) * dims));
   return WAM_OK;
+} catch (const std::bad_alloc&) {
+  return fail(c, WAM_ERR_OOM, "host allocation failed");
+} catch (...) {
+  return fail(c, WAM_ERR_CUDA, "unexpected host exception");
 }
 
 }  // extern "C"
@@ -1381,7 +1428,7 @@ int diag_final(wam_ctx* c, const float* hb, float* x_scratch, float* xn_scratch,
 
 extern "C" {
 
-int wam_diag_layer_deltas(wam_ctx* c, wam_state* st, int32_t episode, double* out) {
+int wam_diag_layer_deltas(wam_ctx* c, wam_state* st, int32_t episode, double* out) try {
   if (c == nullptr || st == nullptr || st->ctx != c || out == nullptr || episode < 0 || episode >= st->B)
     return WAM_ERR_INVALID_ARG;
   const int k = st->meta[episode].stage;
@@ -1396,9 +1443,13 @@ int wam_diag_layer_deltas(wam_ctx* c, wam_state* st, int32_t episode, double* ou
     out[l] = std::sqrt(v[3]) / std::sqrt(v[2]);
   }
   return WAM_OK;
+} catch (const std::bad_alloc&) {
+  return fail(c, WAM_ERR_OOM, "host allocation failed");
+} catch (...) {
+  return fail(c, WAM_ERR_CUDA, "unexpected host exception");
 }
 
-int wam_diag_reuse_error(wam_ctx* c, wam_state* st, int32_t episode, double* e_out, double* alpha_out) {
+int wam_diag_reuse_error(wam_ctx* c, wam_state* st, int32_t episode, double* e_out, double* alpha_out) try {
   if (c == nullptr || st == nullptr || st->ctx != c || e_out == nullptr || episode < 0 || episode >= st->B)
     return WAM_ERR_INVALID_ARG;
   const int k = st->meta[episode].stage;
@@ -1447,6 +1498,10 @@ int wam_diag_reuse_error(wam_ctx* c, wam_state* st, int32_t episode, double* e_o
     alpha_out[1] = split_row == N ? 0.0 : gates[1].alpha;
   }
   return WAM_OK;
+} catch (const std::bad_alloc&) {
+  return fail(c, WAM_ERR_OOM, "host allocation failed");
+} catch (...) {
+  return fail(c, WAM_ERR_CUDA, "unexpected host exception");
 }
 
 int wam_set_graph_replay(wam_ctx* c, int32_t enable) {
@@ -1462,16 +1517,20 @@ int wam_gemm_tile_width(const wam_ctx* c, int32_t M, int32_t N, int32_t K, int32
   return tc_gemm_plan(M, N, K, r64, false, c->num_sms).bn;
 }
 
-int wam_profile_enable(wam_ctx* c, int32_t enable) {
+int wam_profile_enable(wam_ctx* c, int32_t enable) try {
   if (c == nullptr) return WAM_ERR_INVALID_ARG;
   CK(cudaStreamSynchronize(c->stream));
   c->spans.clear();
   c->evnext = 0;
   c->prof_on = enable != 0;
   return WAM_OK;
+} catch (const std::bad_alloc&) {
+  return fail(c, WAM_ERR_OOM, "host allocation failed");
+} catch (...) {
+  return fail(c, WAM_ERR_CUDA, "unexpected host exception");
 }
 
-int wam_profile_read(wam_ctx* c, wam_kclass_timing* out) {
+int wam_profile_read(wam_ctx* c, wam_kclass_timing* out) try {
   if (c == nullptr || out == nullptr) return WAM_ERR_INVALID_ARG;
   CK(cudaStreamSynchronize(c->stream));
   for (int k = 0; k < WAM_KCLASS_COUNT; ++k) out[k] = wam_kclass_timing{0, 0.0, 0.0, 0.0};
@@ -1485,6 +1544,10 @@ int wam_profile_read(wam_ctx* c, wam_kclass_timing* out) {
     t.bytes += s.bytes;
   }
   return WAM_OK;
+} catch (const std::bad_alloc&) {
+  return fail(c, WAM_ERR_OOM, "host allocation failed");
+} catch (...) {
+  return fail(c, WAM_ERR_CUDA, "unexpected host exception");
 }
 
 }  // extern "C"
