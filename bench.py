@@ -511,7 +511,8 @@ def run_independent(dev, n_steps=50, warmup=5):
     continuations through wam_continue_many (one host thread per context, overlapping on the
     GPU; the action stream has the higher priority), as two wam_continue calls in sequence, and
     in sequence with the action branch first (the shortest observation-to-action time).
-    O2A = real observation to action chunk."""
+    O2A = real observation to action chunk (for the concurrent call, when it returns: an upper
+    bound, since the call returns once both branches are issued)."""
     import torch
 
     from paper_2609_34608_gb300 import inputs as I
@@ -565,11 +566,14 @@ def run_independent(dev, n_steps=50, warmup=5):
         calls = [(vctx, vst, K - kv, None, vout), (actx, ast, K - ca["tr_entry_stage"], aout, None)]
         if mode == "concurrent":
             W.Context.continue_many(calls)
+            if marks is not None:
+                marks[2].record(sa)      # action chunk ready (recorded once the concurrent call returns)
         else:
             for c in (calls if mode == "sequential" else calls[::-1]):
                 c[0].continue_(c[1], c[2], c[3], c[4])
+                if marks is not None and c[0] is actx:
+                    marks[2].record(sa)  # action chunk ready, before the other branch is issued
         if marks is not None:
-            marks[2].record(sa)          # action chunk ready
             sv.wait_event(marks[2])
             marks[3].record(sv)          # both branches done
 
