@@ -67,3 +67,12 @@ def test_config_struct_matches_header_size(lib):
     # 12 ints + 1 float + 4 ints + 4 ints + 5 floats + 1 float + 2 ints + 8 floats = 37 x 4 bytes
     assert ctypes.sizeof(W.Config) == 37 * 4
     assert ctypes.sizeof(W.StepRecord) == 12 * 4
+
+
+def test_every_header_function_has_a_binding_signature(lib):
+    """The Python binding declares argument and result types for every function of include/*.h
+    (no call goes through ctypes' default int conversion)."""
+    W.lib()
+    for name in W.header_functions():
+        fn = getattr(lib, name)
+        assert fn.argtypes is not None, name
