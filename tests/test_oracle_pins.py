@@ -192,6 +192,126 @@ def test_conditioning_vs_torch_linear_chain():
     assert np.allclose(fin, f.numpy(), atol=1e-13)
 
 
+def _torch_embed(W, cfg, x, obs):
+    """Token embedding from torch library modules (float64): one nn.Linear per token group,
+    concatenated, plus a learned position table looked up with nn.Embedding."""
+    d = cfg.d_model
+    g = lambda n: torch.from_numpy(np.asarray(W[n], dtype=np.float64))
+    lin = {}
+    for name, din in (("obs", d), ("vid", cfg.video_dim), ("act", cfg.action_dim)):
+        m = torch.nn.Linear(din, d, dtype=torch.float64)
+        with torch.no_grad():
+            m.weight.copy_(g(name + "_w").T)
+            m.bias.copy_(g(name + "_b"))
+        lin[name] = m
+    emb = torch.nn.Embedding(cfg.n_tokens, d, dtype=torch.float64)
+    with torch.no_grad():
+        emb.weight.copy_(g("pos"))
+        xt = torch.from_numpy(np.asarray(x, dtype=np.float64))
+        xv = xt[:cfg.video_len].reshape(cfg.n_video, cfg.video_dim)
+        xa = xt[cfg.video_len:].reshape(cfg.n_action, cfg.action_dim)
+        h = torch.cat([lin["obs"](torch.from_numpy(np.asarray(obs, dtype=np.float64))),
+                       lin["vid"](xv), lin["act"](xa)], dim=0)
+        h = h + emb(torch.arange(cfg.n_tokens))
+    return h.numpy()
+
+
+def _distinct_embedding_weights(W, rng):
+    """Biases and positions of clearly different magnitudes, so that a dropped position term,
+    a bias taken from the wrong group or rows of the wrong group all change the result."""
+    W["obs_b"][:] = rng.standard_normal(W["obs_b"].shape) * 1.0
+    W["vid_b"][:] = rng.standard_normal(W["vid_b"].shape) * 3.0 + 2.0
+    W["act_b"][:] = rng.standard_normal(W["act_b"].shape) * 5.0 - 4.0
+    W["pos"][:] = rng.standard_normal(W["pos"].shape) * 0.7
+
+
+def test_embed_vs_torch_modules():
+    W, cfg = _setup(micro_config(), std=0.3)
+    rng = np.random.default_rng(11)
+    _distinct_embedding_weights(W, rng)
+    x = rng.standard_normal(cfg.traj_len)
+    obs = rng.standard_normal((cfg.n_obs, cfg.d_model))
+    h = O.embed(W, cfg, x, obs)
+    assert h.shape == (cfg.n_tokens, cfg.d_model)
+    assert np.allclose(h, _torch_embed(W, cfg, x, obs), atol=1e-12)
+
+
+def test_embed_zero_inputs_give_bias_plus_position_per_group():
+    """Closed form: with zero trajectory and observation every row is its group's bias plus
+    its own position row."""
+    W, cfg = _setup(micro_config(), std=0.3)
+    _distinct_embedding_weights(W, np.random.default_rng(12))
+    h = O.embed(W, cfg, np.zeros(cfg.traj_len), np.zeros((cfg.n_obs, cfg.d_model)))
+    No, Nv = cfg.n_obs, cfg.n_video
+    pos = np.asarray(W["pos"], dtype=np.float64)
+    for r in range(cfg.n_tokens):
+        b = W["obs_b"] if r < No else (W["vid_b"] if r < No + Nv else W["act_b"])
+        assert np.array_equal(h[r], np.asarray(b, dtype=np.float64) + pos[r])
+
+
+def _torch_final(W, cfg, h, fin):
+    """Final layer from torch library ops: layer_norm (no affine, eps 1e-6), adaLN modulation,
+    then nn.Linear output heads on the video rows and on the action rows."""
+    g = lambda n: torch.from_numpy(np.asarray(W[n], dtype=np.float64))
+    d = cfg.d_model
+    heads = {}
+    for name, dout in (("vout", cfg.video_dim), ("aout", cfg.action_dim)):
+        m = torch.nn.Linear(d, dout, dtype=torch.float64)
+        with torch.no_grad():
+            m.weight.copy_(g(name + "_w").T)
+            m.bias.copy_(g(name + "_b"))
+        heads[name] = m
+    with torch.no_grad():
+        f = torch.from_numpy(np.asarray(fin, dtype=np.float64))
+        y = TF.layer_norm(torch.from_numpy(h), (d,), eps=1e-6) * (1 + f[1]) + f[0]
+        a0, a1 = cfg.n_obs, cfg.n_obs + cfg.n_video
+        vv = heads["vout"](y[a0:a1]).reshape(-1)
+        va = heads["aout"](y[a1:]).reshape(-1)
+    return torch.cat([vv, va]).numpy()
+
+
+def test_final_velocity_vs_torch_modules():
+    W, cfg = _setup(micro_config(), std=0.3)
+    rng = np.random.default_rng(13)
+    W["vout_b"][:] = rng.standard_normal(W["vout_b"].shape) * 2.0
+    W["aout_b"][:] = rng.standard_normal(W["aout_b"].shape) * 2.0 - 3.0
+    h = rng.standard_normal((cfg.n_tokens, cfg.d_model)) * 2.0 + 0.5
+    # shift and scale of very different size and sign: a swapped pair, or a `scale` in place
+    # of `1 + scale`, moves the result far outside the tolerance
+    fin = np.stack([rng.standard_normal(cfg.d_model) * 4.0 + 3.0,
+                    rng.standard_normal(cfg.d_model) * 0.3 - 0.6])
+    v = O.final_velocity(W, cfg, h, fin)
+    assert v.shape == (cfg.traj_len,)
+    assert np.allclose(v, _torch_final(W, cfg, h, fin), atol=1e-11)
+
+
+def test_final_velocity_closed_forms():
+    """scale = -1 removes the normalised hidden state: every video row equals shift W_ov + b_ov
+    and every action row shift W_oa + b_oa.  With scale = 0 and shift = 0 each row is
+    LN(h) W + b, which for h = a row of +-c values (zero mean, unit variance after LN) is the
+    signed column sum of W plus b."""
+    W, cfg = _setup(micro_config(), std=0.3)
+    rng = np.random.default_rng(14)
+    d = cfg.d_model
+    h = rng.standard_normal((cfg.n_tokens, d))
+    shift = rng.standard_normal(d) * 2.0
+    v = O.final_velocity(W, cfg, h, np.stack([shift, -np.ones(d)]))
+    Wv, bv = np.asarray(W["vout_w"], np.float64), np.asarray(W["vout_b"], np.float64)
+    Wa, ba = np.asarray(W["aout_w"], np.float64), np.asarray(W["aout_b"], np.float64)
+    vv = v[:cfg.video_len].reshape(cfg.n_video, cfg.video_dim)
+    va = v[cfg.video_len:].reshape(cfg.n_action, cfg.action_dim)
+    assert np.allclose(vv, np.broadcast_to(shift @ Wv + bv, vv.shape), atol=1e-12)
+    assert np.allclose(va, np.broadcast_to(shift @ Wa + ba, va.shape), atol=1e-12)
+    sign = np.where(np.arange(d) % 2 == 0, 1.0, -1.0)
+    h2 = np.broadcast_to(sign * 2.5, (cfg.n_tokens, d)).copy()
+    v2 = O.final_velocity(W, cfg, h2, np.zeros((2, d)))
+    ln = sign * (2.5 / math.sqrt(2.5 * 2.5 + 1e-6))
+    assert np.allclose(v2[:cfg.video_len].reshape(cfg.n_video, -1),
+                       np.broadcast_to(ln @ Wv + bv, (cfg.n_video, cfg.video_dim)), atol=1e-12)
+    assert np.allclose(v2[cfg.video_len:].reshape(cfg.n_action, -1),
+                       np.broadcast_to(ln @ Wa + ba, (cfg.n_action, cfg.action_dim)), atol=1e-12)
+
+
 def test_velocity_is_token_permutation_equivariant_without_positions():
     cfgd = micro_config()
     W, cfg = _setup(cfgd, std=0.3)
