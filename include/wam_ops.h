@@ -104,12 +104,14 @@ const char* wam_op_last_error(void);
 /*
  * Trajectory Remapping of `batch` finished trajectories that allocates no device memory, for
  * callers that cannot allocate: controllers whose control loop forbids allocation after
- * start-up (bounded step latency), or hosts that own all device memory.  The paper has no
- * counterpart; this is the same computation as the remap inside wam_adapt_state (Eqs. 1-2 with
- * the Eq. 12 normaliser when normalize != 0) with one executed shift and one (sigma_r,
- * sigma_b0) pair for every episode.
+ * start-up (bounded step latency), or hosts that own all device memory and hand the library
+ * none.  The paper has no counterpart: this is the remap that wam_adapt_state performs on a
+ * finished replan, for one executed shift and one (sigma_r, sigma_b0) pair shared by every
+ * episode, and it returns the same bits as that remap.
  *   x_bar, x_r, eps, out: [batch, T] float32 device buffers, T = n_video*video_dim +
- *   n_action*action_dim; eps may be NULL when shift == 0 and video_mode == 0.
+ *   n_action*action_dim (at most 2^31 - 1); eps may be NULL when shift == 0 and
+ *   video_mode == 0 (no slot takes fresh noise then).
+ *   normalize != 0 scales each branch's direction to unit RMS; 0 keeps (x_r - x_bar) / sigma_r.
  *   video_mode 0 remaps video without a shift, 1 fills it with sigma_b0 * eps.
  * Scratch: a fixed 64 KiB array inside the library (8192 float64 partial sums) holds the RMS
  * partial sums; batch * 2 * ceil(max(n_video*video_dim, n_action*action_dim) / 2048) must not

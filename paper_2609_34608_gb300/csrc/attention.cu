@@ -305,13 +305,9 @@ __global__ void __launch_bounds__(256) attn_f32_kernel(const float* __restrict__
 template <int DH>
 cudaError_t launch_bf16(const bf16* qkv, bf16* out, int B, int N, int d, int H, cudaStream_t s) {
   using C = AttnCfg<DH>;
-  static std::atomic<bool> attr_set{false};  // contexts may run on several host threads
-  if (!attr_set.load(std::memory_order_acquire)) {
-    cudaError_t e = cudaFuncSetAttribute(attn_bf16_kernel<DH>,
-                                         cudaFuncAttributeMaxDynamicSharedMemorySize, C::kSmem);
-    if (e != cudaSuccess) return e;
-    attr_set.store(true, std::memory_order_release);
-  }
+  static PerDeviceSmem smem_rec;  // contexts may run on several host threads and devices
+  const cudaError_t e = ensure_max_smem(smem_rec, attn_bf16_kernel<DH>, C::kSmem);
+  if (e != cudaSuccess) return e;
   dim3 grid((N + C::kBQ - 1) / C::kBQ, H, B);
   const float scale_log2 = 1.4426950408889634f / sqrtf(static_cast<float>(DH));
   return launch_pdl(attn_bf16_kernel<DH>, grid, dim3(128), C::kSmem, s, qkv, out, N, d, scale_log2);

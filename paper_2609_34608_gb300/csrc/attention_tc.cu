@@ -323,12 +323,9 @@ cudaError_t attention_tc(const CUtensorMap& tm_qk, const CUtensorMap& tm_vt, bf1
                          int H, int* dev_err, cudaStream_t s) {
   if (B <= 0 || N <= 0) return cudaSuccess;
   if (d / H != kDH) return cudaErrorInvalidValue;
-  static std::atomic<bool> attr_set{false};  // contexts may run on several host threads
-  if (!attr_set.load(std::memory_order_acquire)) {
-    cudaError_t e = cudaFuncSetAttribute(attn_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemAttn);
-    if (e != cudaSuccess) return e;
-    attr_set.store(true, std::memory_order_release);
-  }
+  static PerDeviceSmem smem_rec;  // contexts may run on several host threads and devices
+  const cudaError_t e = ensure_max_smem(smem_rec, attn_tc_kernel, kSmemAttn);
+  if (e != cudaSuccess) return e;
   const float scale_log2 = 1.4426950408889634f / 8.0f;  // log2(e) / sqrt(64)
   dim3 grid((N + kQ - 1) / kQ, H, B);
   return launch_pdl(attn_tc_kernel, grid, dim3(kThreadsAttn), kSmemAttn, s, tm_qk, tm_vt, out, N, d, H,

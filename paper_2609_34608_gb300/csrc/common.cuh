@@ -49,6 +49,48 @@ inline cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, s
   return cudaLaunchKernelEx(&cfg, kernel, static_cast<KArgs>(args)...);
 }
 
+// Kernel attributes (the dynamic shared-memory limit) and device properties belong to one device,
+// and a process may drive contexts on several GPUs (wam_continue_many switches devices per
+// context), so "already set" is recorded per device index.  Devices beyond 64 are simply set on
+// every launch.
+constexpr int kMaxTrackedDevices = 64;
+
+inline int current_device() {
+  int d = 0;
+  if (cudaGetDevice(&d) != cudaSuccess) d = -1;
+  return d;
+}
+
+// Largest dynamic shared-memory size already granted to one kernel, per device.
+struct PerDeviceSmem {
+  std::atomic<int> granted[kMaxTrackedDevices] = {};
+};
+
+template <typename Kernel>
+inline cudaError_t ensure_max_smem(PerDeviceSmem& rec, Kernel kernel, int bytes) {
+  const int dev = current_device();
+  const bool tracked = dev >= 0 && dev < kMaxTrackedDevices;
+  if (tracked && rec.granted[dev].load(std::memory_order_acquire) >= bytes) return cudaSuccess;
+  const cudaError_t e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
+  if (e != cudaSuccess || !tracked) return e;
+  int prev = rec.granted[dev].load(std::memory_order_relaxed);
+  while (prev < bytes && !rec.granted[dev].compare_exchange_weak(prev, bytes)) {
+  }
+  return cudaSuccess;
+}
+
+// Streaming-multiprocessor count of the current device, looked up once per device.
+inline int device_sm_count() {
+  static std::atomic<int> cached[kMaxTrackedDevices] = {};
+  const int dev = current_device();
+  const bool tracked = dev >= 0 && dev < kMaxTrackedDevices;
+  int n = tracked ? cached[dev].load(std::memory_order_relaxed) : 0;
+  if (n > 0) return n;
+  if (dev < 0 || cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n < 1) n = 1;
+  if (tracked) cached[dev].store(n, std::memory_order_relaxed);
+  return n;
+}
+
 WAM_DEV float warp_sum(float v) {
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);

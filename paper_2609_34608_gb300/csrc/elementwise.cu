@@ -1109,15 +1109,7 @@ cudaError_t final_euler(const float* h, const StepItem* items, const float* mods
                         float* head_const, cudaStream_t s) {
   if (Bw <= 0) return cudaSuccess;
   if (d % 128 != 0 || vd > 16 || ad > 16) return cudaErrorInvalidValue;  // heads padded to 16
-  static std::atomic<int> sms_cached{0};  // contexts may run on several host threads
-  int num_sms = sms_cached.load(std::memory_order_relaxed);
-  if (num_sms == 0) {
-    int dev = 0;
-    cudaGetDevice(&dev);
-    cudaDeviceGetAttribute(&num_sms, cudaDevAttrMultiProcessorCount, dev);
-    if (num_sms < 1) num_sms = 1;
-    sms_cached.store(num_sms, std::memory_order_relaxed);
-  }
+  const int num_sms = device_sm_count();
   const int64_t hstride = final_head_bytes(d);
   if (head_bf16)
     launch_pdl(final_head_prep_kernel<true>, dim3(2, Bw), dim3(256), 0, s, mods, mod_stride, fin_off, vout_w, vout_b,
@@ -1138,16 +1130,9 @@ cudaError_t final_euler(const float* h, const StepItem* items, const float* mods
   dim3 grid(vblocks + ablocks, Bw);
 #define WAM_SET_SMEM(KERNEL)                                                                       \
   {                                                                                                \
-    static std::atomic<int> smem_set{0};                                                           \
-    if (smem_set.load(std::memory_order_acquire) < static_cast<int>(smem)) {                       \
-      cudaError_t e = cudaFuncSetAttribute(KERNEL, cudaFuncAttributeMaxDynamicSharedMemorySize,    \
-                                           static_cast<int>(smem));                                \
-      if (e != cudaSuccess) return e;                                                              \
-      int prev = smem_set.load(std::memory_order_relaxed);                                         \
-      while (prev < static_cast<int>(smem) &&                                                      \
-             !smem_set.compare_exchange_weak(prev, static_cast<int>(smem)))                        \
-        ;                                                                                          \
-    }                                                                                              \
+    static PerDeviceSmem smem_rec; /* per device: contexts may run on several GPUs */             \
+    const cudaError_t e = ensure_max_smem(smem_rec, KERNEL, static_cast<int>(smem));               \
+    if (e != cudaSuccess) return e;                                                                \
   }
   if (head_bf16) {
     WAM_SET_SMEM(final_euler_tc_kernel)

@@ -472,13 +472,9 @@ template <int BN, int EPI, int KA>
 cudaError_t launch(const CUtensorMap& ta, const CUtensorMap& tb, int M, int N, int K,
                    const EpiArgs& e, const SplitArgs& sp, int num_sms, int* dev_err, cudaStream_t s) {
   using C = TileCfg<BN, KA>;
-  static std::atomic<bool> attr_set{false};  // contexts may run on several host threads
-  if (!attr_set.load(std::memory_order_acquire)) {
-    cudaError_t err = cudaFuncSetAttribute(gemm_tc_kernel<BN, EPI, KA>,
-                                           cudaFuncAttributeMaxDynamicSharedMemorySize, C::kSmemBytes);
-    if (err != cudaSuccess) return err;
-    attr_set.store(true, std::memory_order_release);
-  }
+  static PerDeviceSmem smem_rec;  // contexts may run on several host threads and devices
+  const cudaError_t err = ensure_max_smem(smem_rec, gemm_tc_kernel<BN, EPI, KA>, C::kSmemBytes);
+  if (err != cudaSuccess) return err;
   const int units = ((M + kBM - 1) / kBM) * (N / BN) * sp.splits;
   const int grid = units < num_sms ? units : num_sms;
   return launch_pdl(gemm_tc_kernel<BN, EPI, KA>, dim3(grid), dim3(kThreads), C::kSmemBytes, s, ta, tb, M, N,

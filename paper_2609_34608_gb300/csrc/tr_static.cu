@@ -14,6 +14,7 @@
 // and must be serialised by the caller.  The first call on a device looks up the array's
 // device address (cudaGetSymbolAddress, with that device current); make that first call before
 // any stream capture begins.
+#include <climits>
 #include <mutex>
 #include <string>
 
@@ -45,7 +46,11 @@ WAM_DEV double block_sum(double v, double* red) {
   return s;
 }
 
-// Sum over one chunk of one branch of ((x^r - x_bar) / sigma_r)^2 (Eq. 1 before N).
+// Sum over one chunk of one branch of (x^r - x_bar)^2 / sigma_r^2, accumulated in the same order
+// and with the same roundings as the remap of wam_adapt_state (thread t of the block takes
+// elements t, t + 256, ... of the chunk with one fused multiply-add each; the thread's sum is
+// scaled by 1 / sigma_r^2 once; then the warp and block sums), so the two entry points agree
+// bit for bit.
 __global__ void __launch_bounds__(256) tr_static_partial_kernel(const float* __restrict__ x_bar,
                                                                 const float* __restrict__ x_r,
                                                                 int T, int V, double sigma_r,
@@ -58,28 +63,31 @@ __global__ void __launch_bounds__(256) tr_static_partial_kernel(const float* __r
   const int end = min(len, (ch + 1) * kStaticChunk);
   double s = 0.0;
   for (int i = ch * kStaticChunk + threadIdx.x; i < end; i += blockDim.x) {
-    const double u = (static_cast<double>(x_r[bo + i]) - static_cast<double>(x_bar[bo + i])) / sigma_r;
-    s += u * u;
+    const double v = static_cast<double>(x_r[bo + i]) - static_cast<double>(x_bar[bo + i]);
+    s = fma(v, v, s);
   }
+  s *= 1.0 / (sigma_r * sigma_r);
   s = block_sum(s, red);
   if (threadIdx.x == 0) partial[(static_cast<int64_t>(b) * 2 + br) * nch + ch] = s;
 }
 
-// Remapped init (Eq. 2) with the unit-RMS direction (Eq. 12), the action shift and the
-// fresh-noise fill sigma_b0 * eps of uncovered slots.
+// Remapped init: retained slots get x_bar + sigma_b0 * unit-RMS direction, computed as one
+// fused multiply-add with the branch gain sigma_b0 / (sigma_r rms) (the same float64 operations
+// as the remap of wam_adapt_state); the action slots move by the executed shift and the slots
+// left uncovered (and, in video mode 1, every video slot) get sigma_b0 * eps.
 __global__ void __launch_bounds__(256) tr_static_apply_kernel(
     const float* __restrict__ x_bar, const float* __restrict__ x_r, const float* __restrict__ eps,
     float* __restrict__ out, int T, int V, int Na, int ad, int shift, double sigma_r,
     double sigma_b0, int normalize, int video_mode, int nch, const double* __restrict__ partial) {
-  __shared__ double rms[2];
-  __shared__ int zero[2];
+  __shared__ double gain[2];
   const int b = blockIdx.y;
   if (threadIdx.x < 2) {
     double s = 0.0;
     for (int c = 0; c < nch; ++c) s += partial[(static_cast<int64_t>(b) * 2 + threadIdx.x) * nch + c];
     const double ms = s / (threadIdx.x == 0 ? V : T - V);
-    rms[threadIdx.x] = normalize ? sqrt(ms) : 1.0;
-    zero[threadIdx.x] = normalize && !(ms > 0.0);
+    const double rms = normalize ? sqrt(ms) : 1.0;
+    const bool zero = normalize && !(ms > 0.0);
+    gain[threadIdx.x] = zero ? 0.0 : sigma_b0 / (sigma_r * rms);
   }
   __syncthreads();
   const int64_t bo = static_cast<int64_t>(b) * T;
@@ -95,9 +103,8 @@ __global__ void __launch_bounds__(256) tr_static_apply_kernel(
     }
     float val;
     if (src >= 0) {
-      const double u = (static_cast<double>(x_r[bo + src]) - static_cast<double>(x_bar[bo + src])) / sigma_r;
-      const double dir = zero[br] ? 0.0 : u / rms[br];
-      val = static_cast<float>(static_cast<double>(x_bar[bo + src]) + sigma_b0 * dir);
+      const double xbs = static_cast<double>(x_bar[bo + src]);
+      val = static_cast<float>(fma(gain[br], static_cast<double>(x_r[bo + src]) - xbs, xbs));
     } else {
       val = static_cast<float>(sigma_b0 * static_cast<double>(eps[bo + j]));
     }
@@ -145,8 +152,14 @@ extern "C" int wam_tr_remap_static(const float* x_bar, const float* x_r, const f
     set_op_error("invalid argument: null buffer, non-positive size, negative shift or sigma_r <= 0");
     return WAM_ERR_INVALID_ARG;
   }
-  const int V = n_video * video_dim;
-  const int T = V + n_action * action_dim;
+  const int64_t V64 = static_cast<int64_t>(n_video) * video_dim;
+  const int64_t T64 = V64 + static_cast<int64_t>(n_action) * action_dim;
+  if (T64 > INT_MAX || static_cast<int64_t>(batch) * T64 > (int64_t(1) << 40)) {
+    set_op_error("trajectory length n_video*video_dim + n_action*action_dim above 2^31 - 1 values");
+    return WAM_ERR_INVALID_ARG;
+  }
+  const int V = static_cast<int>(V64);
+  const int T = static_cast<int>(T64);
   if (eps == nullptr && (video_mode == 1 || shift > 0)) {
     set_op_error("eps is required when any slot receives fresh noise");
     return WAM_ERR_INVALID_ARG;
