@@ -12,11 +12,17 @@ Printed JSON line: `value` = action chunks/s with every input already resident i
 `latency_ms` = per-control-step p50/p99 and the observation-to-action part (rebinding + the
 steps after it); `cold` = a native cold 10-step sample; `e2e` = the same control loop through
 the C ABI with pinned host buffers (host<->device copies inside the timed region);
-`roofline` = the dominant kernel class (tcgen05 GEMM) against the measured bf16 peak;
-`ablation` = the same control steps with the layer stack launched kernel by kernel instead of
-replayed from CUDA graphs; `independent` = the separate video / action models of independent
-execution, their continuations overlapped on two streams and in sequence; `cpu_baseline` = the float64 CPU oracle on the host cores for one
-control step.
+`roofline` = the dominant kernel class (tcgen05 GEMM) against the measured burst bf16 peak,
+its time taken as its share of a profiled pass applied to the un-instrumented step;
+`kernels` = every kernel class of the profiled pass; `ablation` = the paper's Table 3 variants
+(w/o TR, w/o OR, w/o RR, w/o graph replay, native with and without graphs) and a labelled run
+with a relaxed RR gate; `serving` = 32-episode batches of the 24-block d1024 model;
+`bimanual` = the 28-block d1152 model (head dim 72, 4914 tokens, batch 8): cold 10 steps and
+the warm sweep over 1..9 retained steps with shift 25; `independent` = the separate video /
+action models of independent execution, their continuations overlapped on two streams and in
+sequence; `cpu_baseline` = the float64 CPU oracle on the host cores continuing the GPU run's
+cold sample (all cores; one core extrapolated from one forward).  `--cpu-plan` times the whole
+CPU plan (latency cold sample end to end, serving / bimanual sample-steps) and exits.
 
 Usage: python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
 Multi-GPU (torchrun): one replica per rank, no collective on the data path (the work is
@@ -72,9 +78,10 @@ def job_throughput(units_per_rank: int, world: int, ms: float) -> float:
     return units_per_rank * world / (ms * 1e-3)
 
 
-def kernel_table(prof: dict, units: int, peaks: dict) -> dict:
+def kernel_table(prof: dict, units: int, peaks: dict, tensor_peak: str = "bf16") -> dict:
     """Per kernel class: time per unit, share, and achieved rate against the measured peak
-    (TFLOP/s for the tensor-core classes, GB/s of algorithmic bytes for the HBM-bound ones)."""
+    (TFLOP/s for the tensor-core classes, GB/s of algorithmic bytes for the HBM-bound ones).
+    `tensor_peak` is "bf16" (burst: a step of a few ms) or "bf16_sus" (seconds-long runs)."""
     tot = sum(v["ms"] for v in prof.values())
     out = {}
     for k, v in prof.items():
@@ -84,7 +91,7 @@ def kernel_table(prof: dict, units: int, peaks: dict) -> dict:
         if v["ms"] > 0:
             if k in TENSOR_CLASSES:
                 row["tflops"] = v["flops"] / (v["ms"] * 1e-3) / 1e12
-                row["frac"] = row["tflops"] / peaks["bf16_sus"]
+                row["frac"] = row["tflops"] / peaks[tensor_peak]
             else:
                 row["gbs"] = v["bytes"] / (v["ms"] * 1e-3) / 1e9
                 row["frac"] = row["gbs"] / peaks["hbm"]
@@ -167,23 +174,46 @@ class ClockSampler:
 
 
 # ------------------------------------------------------------------------------ CPU oracle
-def _oracle_control_step_worker(q, cfg, seed, n_steps):
-    """Time the float64 oracle on one warm control step (a bounded sample of the workload)."""
+def _oracle_episode_from(cfg, retained):
+    """An oracle episode holding a finished replan: `retained` = dict of the stage latents
+    ("hist": {stage: x}), the bound observation and the RR layer state (p_a, R_a), taken from a
+    real cold sample; None draws a random finished replan (the reference arm's own stand-in)."""
     from oracle import wam_oracle as O
     from paper_2609_34608_gb300 import inputs as I
 
     Wd = I.make_weights(cfg)
     ocfg = O.OracleConfig.from_dict(cfg)
     K = cfg["n_steps"]
-    b0 = cfg["tr_entry_stage"]
     ep = O.OracleEpisode(Wd, ocfg)
+    if retained is None:
+        rng = np.random.default_rng(0)
+        T = ocfg.traj_len
+        b0 = cfg["tr_entry_stage"]
+        ep.hist = {K: rng.standard_normal(T), b0: rng.standard_normal(T)}
+        ep.hist_from = b0
+    else:
+        ep.hist = {int(k): np.asarray(v, np.float64) for k, v in retained["hist"].items()}
+        ep.hist_from = 0
+        if retained.get("p_a") is not None:
+            ep.layer = O.LayerState(p_a=np.asarray(retained["p_a"], np.float64),
+                                    R_a=np.asarray(retained["R_a"], np.float64))
+    ep.obs = np.asarray(retained["obs"] if retained is not None else np.zeros((cfg["n_obs"], cfg["d_model"])),
+                        np.float64)
+    ep.stage, ep.finished = K, True
+    ep.x = ep.hist[K].copy()
+    return ep
+
+
+def _oracle_control_step_worker(q, cfg, seed, n_steps, retained):
+    """Time the float64 oracle on warm control steps (a bounded sample of the workload)."""
+    from oracle import wam_oracle as O
+    from paper_2609_34608_gb300 import inputs as I
+
+    ep = _oracle_episode_from(cfg, retained)
+    K = cfg["n_steps"]
     proc = I.ObsProcess(cfg, 1, seed=seed)
-    rng = np.random.default_rng(seed)
-    T = ocfg.traj_len
-    # a finished previous replan (its stage-K and stage-r latents) to remap from
-    ep.obs = proc.obs[0].astype(np.float64)
-    ep.hist = {K: rng.standard_normal(T), b0: rng.standard_normal(T)}
-    ep.hist_from, ep.stage, ep.finished = b0, K, True
+    if retained is not None:
+        proc.obs = np.asarray(retained["obs"], np.float32)[None]
     times = []
     for t in range(n_steps):
         pred, real = proc.predicted()[0], proc.step()[0]
@@ -197,17 +227,121 @@ def _oracle_control_step_worker(q, cfg, seed, n_steps):
     q.put(times)
 
 
-def run_oracle_steps(cfg, n_steps, seed=0):
+def _oracle_forward_worker(q, cfg, n):
+    """Time n float64 oracle denoising forwards (one sample-step each) of one episode."""
+    from oracle import wam_oracle as O
+    from paper_2609_34608_gb300 import inputs as I
+
+    Wd = I.make_weights(cfg)
+    ocfg = O.OracleConfig.from_dict(cfg)
+    x, obs = I.make_noise(cfg, 1)[0], I.make_obs(cfg, 1)[0]
+    times = []
+    for _ in range(n):
+        t0 = time.perf_counter()
+        O.velocity(Wd, ocfg, x, obs, 0.5)
+        times.append(time.perf_counter() - t0)
+    q.put(times)
+
+
+def _oracle_tiny_e2e_worker(q, cfg):
+    """The tiny workload end to end: cold K-step sample, TR with the executed shift, warm
+    continuation of the retained steps."""
+    from oracle import wam_oracle as O
+    from paper_2609_34608_gb300 import inputs as I
+
+    Wd = I.make_weights(cfg)
+    ocfg = O.OracleConfig.from_dict(cfg)
+    K = cfg["n_steps"]
+    t0 = time.perf_counter()
+    ep = O.OracleEpisode(Wd, ocfg)
+    ep.sample_cold(I.make_obs(cfg, 1)[0], I.make_noise(cfg, 1)[0], K)
+    ep.adapt(I.make_obs(cfg, 1, seed=3)[0], cfg["shift"], I.make_fresh_eps(cfg, 1, 0)[0])
+    ep.advance(K - ep.stage)
+    q.put([time.perf_counter() - t0])
+
+
+def _spawn(target, args, threads):
+    """Run an oracle timing in a fresh (spawned) process with `threads` BLAS threads."""
     ctx = mp.get_context("spawn")
     q = ctx.Queue()
+    keys = ("OPENBLAS_NUM_THREADS", "OMP_NUM_THREADS", "MKL_NUM_THREADS")
+    saved = {k: os.environ.get(k) for k in keys}
+    for k in keys:
+        os.environ[k] = str(threads)
+    try:
+        p = ctx.Process(target=target, args=(q,) + tuple(args))
+        p.start()
+        out = q.get()
+        p.join()
+    finally:
+        for k, v in saved.items():
+            if v is None:
+                os.environ.pop(k, None)
+            else:
+                os.environ[k] = v
+    return out
+
+
+def run_oracle_steps(cfg, n_steps, seed=0, retained=None, threads=None):
+    threads = threads or (os.cpu_count() or 1)
+    return _spawn(_oracle_control_step_worker, (cfg, seed, n_steps, retained), threads), threads
+
+
+def cpu_baseline(retained):
+    """The oracle on the host cores, bounded to about a minute: two warm control steps of the
+    benchmarked workload continuing a real cold sample (all cores), one denoising forward of
+    that model on one core (a control step runs three), and the tiny workload end to end on
+    all cores and on one core."""
+    from paper_2609_34608_gb300 import inputs as I
+
     ncpu = os.cpu_count() or 1
-    os.environ.setdefault("OPENBLAS_NUM_THREADS", str(ncpu))
-    os.environ.setdefault("OMP_NUM_THREADS", str(ncpu))
-    p = ctx.Process(target=_oracle_control_step_worker, args=(q, cfg, seed, n_steps))
-    p.start()
-    times = q.get()
-    p.join()
-    return times, int(os.environ["OPENBLAS_NUM_THREADS"])
+    cfg = I.get_config(WORKLOAD)
+    steps, _ = run_oracle_steps(cfg, 2, retained=retained, threads=ncpu)
+    fwd1 = _spawn(_oracle_forward_worker, (cfg, 1), 1)
+    tiny = I.get_config("tiny")
+    t_all = _spawn(_oracle_tiny_e2e_worker, (tiny,), ncpu)
+    t_one = _spawn(_oracle_tiny_e2e_worker, (tiny,), 1)
+    per_step = statistics.mean(steps)
+    return {
+        "value": 1.0 / per_step, "unit": "chunks/s", "cores": ncpu, "kind": "oracle",
+        "sample": "two warm control steps (TR + 1 prefix step + OR + 2 steps, RR) continuing the GPU run's "
+                  "cold sample (its retained latents and layer state), float64 oracle, mean of the two",
+        "step_s": steps,
+        "one_core": {"forward_s": fwd1[0], "chunks_per_s_extrapolated": 1.0 / (3.0 * fwd1[0]),
+                     "what": "one denoising forward of the same model on one core; a control step runs "
+                             "three (TR and OR are below 1 % of it), so chunks/s is extrapolated"},
+        "tiny_e2e_s": {"cores_all": t_all[0], "cores_1": t_one[0],
+                       "what": "2-block d128 fp32 model: cold 8-step sample + TR (shift 1) + 4 warm steps"},
+    }
+
+
+def cpu_plan():
+    """The full CPU plan (about 10 minutes on 16 cores): the latency model's cold 10-step sample
+    end to end, the tiny workload end to end, and one sample-step of the serving and bimanual
+    models (extrapolated to their batches), each on all cores and on one core (the one-core
+    timings of the large models are extrapolated from one forward)."""
+    from paper_2609_34608_gb300 import inputs as I
+
+    ncpu = os.cpu_count() or 1
+    out = {"cores": ncpu}
+    tiny = I.get_config("tiny")
+    out["tiny_e2e_s"] = {"all": _spawn(_oracle_tiny_e2e_worker, (tiny,), ncpu)[0],
+                         "one": _spawn(_oracle_tiny_e2e_worker, (tiny,), 1)[0]}
+    lat = I.get_config("latency")
+    f_all = _spawn(_oracle_forward_worker, (lat, lat["n_steps"]), ncpu)
+    f_one = _spawn(_oracle_forward_worker, (lat, 1), 1)
+    out["latency_cold10"] = {"all_s": sum(f_all), "one_s_extrapolated": 10 * f_one[0],
+                             "chunks_per_s_all": 1.0 / sum(f_all)}
+    for name in ("serving", "bimanual"):
+        cfg = I.get_config(name)
+        fa = _spawn(_oracle_forward_worker, (cfg, 1), ncpu)[0]
+        fo = _spawn(_oracle_forward_worker, (cfg, 1), 1)[0]
+        B, K = cfg["batch"], cfg["n_steps"]
+        steps = B // 2 * K + B // 2 * 2 if name == "serving" else B * K
+        out[name] = {"sample_step_s_all": fa, "sample_step_s_one": fo, "sample_steps_per_batch": steps,
+                     "chunks_per_s_all_extrapolated": B / (steps * fa),
+                     "chunks_per_s_one_extrapolated": B / (steps * fo)}
+    return out
 
 
 # ------------------------------------------------------------------------------ reference arm
@@ -249,12 +383,6 @@ def main_ours(args):
     torch.cuda.set_device(local)
     dev = torch.device("cuda", local)
 
-    # The CPU baseline process is spawned before any GPU work.
-    cpu_times, cpu_cores = (None, None)
-    if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        from paper_2609_34608_gb300 import inputs as I0
-        cpu_times, cpu_cores = run_oracle_steps(I0.get_config(WORKLOAD), 2)
-
     from paper_2609_34608_gb300 import _build
     from paper_2609_34608_gb300 import inputs as I
     from paper_2609_34608_gb300 import wam as W
@@ -265,7 +393,6 @@ def main_ours(args):
     stream = torch.cuda.Stream(dev)
     flat = torch.from_numpy(I.flatten_weights(I.make_weights(cfg))).to(dev)
     ctx = W.Context(cfg, flat, stream=stream.cuda_stream)
-    del flat
     n_total = args.warmup + args.steps
     proc = I.ObsProcess(cfg, 1, seed=rank)
     first_obs = proc.obs.copy()
@@ -282,15 +409,17 @@ def main_ours(args):
         noise = torch.from_numpy(I.make_noise(cfg, 1)).to(dev)
         obs0 = torch.from_numpy(first_obs).to(dev)
 
-    def control_step(inp, act, ev=None):
+    def control_step(inp, act, ev=None, c=None, s=None):
+        c = c or ctx
+        s = s or st
         pred, real, eps = inp
-        s1 = ctx.adapt(st, pred, shift=shift, fresh_noise=eps)[0]
+        s1 = c.adapt(s, pred, shift=shift, fresh_noise=eps)[0]
         if s1 == W.ADAPT_TR_INIT:
-            ctx.continue_(st, 1)
+            c.continue_(s, cfg["prefix_steps"])
         if ev is not None:
             ev.record(stream)
-        s2 = ctx.adapt(st, real)[0]
-        ctx.continue_(st, K - (b0 + 1 if s2 == W.ADAPT_REBIND_ACCEPT else b0), act)
+        s2 = c.adapt(s, real)[0]
+        c.continue_(s, K - (b0 + cfg["prefix_steps"] if s2 == W.ADAPT_REBIND_ACCEPT else b0), act)
         return s1, s2
 
     def barrier():
@@ -302,6 +431,13 @@ def main_ours(args):
     st = ctx.state(1)
     with torch.cuda.stream(stream):
         ctx.sample_cold(st, obs0, noise, K, act_dev)
+    torch.cuda.synchronize(dev)
+    # the finished cold replan, kept for the CPU oracle baseline to continue from
+    retained = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        retained = {"hist": {k: ctx.read(st, W.FIELD_X_STAGE, k)[0] for k in range(K + 1)},
+                    "obs": first_obs[0], "p_a": ctx.read(st, W.FIELD_RR_P)[0], "R_a": ctx.read(st, W.FIELD_RR_R)[0]}
+    with torch.cuda.stream(stream):
         for t in range(args.warmup):
             control_step(dev_in[t], act_dev)
     ctx.reset_stats()
@@ -321,6 +457,7 @@ def main_ours(args):
     step_ms = [ev_s[i].elapsed_time(ev_s[i + 1]) for i in range(args.steps)]
     o2a_ms = [ev_m[i].elapsed_time(ev_s[i + 1]) for i in range(args.steps)]
     total_ms = slowest_rank_ms(total_ms, dist)
+    rr_log = ctx.log(st)
 
     # ---- end to end: pinned host inputs and outputs through the C ABI -----------------
     st_e = ctx.state(1)
@@ -357,23 +494,7 @@ def main_ours(args):
     torch.cuda.synchronize(dev)
     cold_ms = [a.elapsed_time(b) for a, b in cold_ms][1:]
 
-    # ---- ablation: the same control steps with every kernel launched individually ------
-    # (CUDA-graph replay of the layer stack off; the paper's Table 3 "Graph" switch)
-    st = st_keep
-    n_abl = min(args.steps, 50)
-    ctx.set_graph_replay(False)
-    a0, a1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    with torch.cuda.stream(stream):
-        a0.record(stream)
-        for i in range(n_abl):
-            control_step(dev_in[args.warmup + i], act_dev)
-        a1.record(stream)
-    torch.cuda.synchronize(dev)
-    ctx.set_graph_replay(True)
-    abl_ms = a0.elapsed_time(a1) / n_abl
-
     # ---- kernel-class timing (CUDA events on the library's stream) --------------------
-    st = st_keep
     ctx.profile_enable(True)
     nprof = min(args.steps, 20)
     with torch.cuda.stream(stream):
@@ -382,20 +503,36 @@ def main_ours(args):
     prof = ctx.profile_read()
     ctx.profile_enable(False)
 
-    serving = serving_rr = independent = None
+    # ---- Table 3 ablation of the mechanisms and the graph replay ----------------------
+    ablation = None
+    if not args.no_ablation:
+        ablation = run_table3(ctx, flat, cfg, dev, stream, dev_in, obs0, noise, min(args.steps, 20))
+    del flat
+
+    serving = serving_rr = independent = bimanual = None
     if not args.no_serving:
         ctx.close()
         serving = run_serving(dev, stream, _peaks())
         serving_rr = run_serving(dev, stream, _peaks(), relax_gate=True)
+    if not args.no_bimanual:
+        ctx.close()
+        bimanual = run_bimanual(dev, stream, _peaks())
     if not args.no_independent:
         independent = run_independent(dev)
 
     if rank != 0:
         return 0
     peaks = _peaks()
+    kt = kernel_table(prof, nprof, peaks)
     g = prof["gemm"]
-    gemm_tflops = g["flops"] / (g["ms"] * 1e-3) / 1e12 if g["ms"] > 0 else 0.0
+    # The per-launch events of the profiled pass stretch every kernel (they serialise the
+    # launches); the GEMM class's rate is taken from its share of that pass applied to the
+    # un-instrumented step time.
+    gemm_flops_step = g["flops"] / nprof
+    gemm_ms_step = kt["gemm"]["share"] * total_ms / args.steps
+    gemm_tflops = gemm_flops_step / (gemm_ms_step * 1e-3) / 1e12
     value = job_throughput(args.steps, world, total_ms)
+    accepted = [r for r in rr_log if r["rr_attempt"]]
     line = {
         "metric": METRIC, "value": value, "unit": "chunks/s", "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": total_ms / args.steps, "higher_is_better": True,
@@ -405,33 +542,198 @@ def main_ours(args):
                        "o2a_p50": float(np.percentile(o2a_ms, 50)), "o2a_p99": float(np.percentile(o2a_ms, 99))},
         "cold": {"ms_p50": float(np.percentile(cold_ms, 50)), "chunks_per_s": 1000.0 / float(np.percentile(cold_ms, 50)),
                  "what": "native cold 10-step sample of the same model, RR active after the first step"},
-        "ablation": {"graph_replay_off": {"chunks_per_s": 1000.0 / abl_ms, "ms_per_step": abl_ms, "steps": n_abl,
-                                          "what": "same control steps, every kernel launched individually"}},
         "reuse": {"r_rr": stats["n_reuse"] / max(1, stats["n_attempt"]), "f_skip": stats["b_skip"] / max(1, stats["b_dense"]),
-                  "r_or": stats["n_bind"] / max(1, stats["n_start"]), "coverage": stats["n_bind"] / max(1, stats["n_noninitial"])},
+                  "r_or": stats["n_bind"] / max(1, stats["n_start"]), "coverage": stats["n_bind"] / max(1, stats["n_noninitial"]),
+                  "rr_cos_last_step": [r["cos"] for r in accepted[-1:]],
+                  "rr_fit_last_step": [r["fit"] for r in accepted[-1:]]},
         "roofline": {"bound": "tensor", "kernel": "tcgen05 GEMM (QKV / out / MLP projections)",
-                     "achieved": gemm_tflops, "peak": peaks["bf16_sus"], "unit": "TFLOP/s",
-                     "frac": gemm_tflops / peaks["bf16_sus"], "traffic": _gemm_traffic(),
+                     "achieved": gemm_tflops, "peak": peaks["bf16"], "unit": "TFLOP/s",
+                     "frac": gemm_tflops / peaks["bf16"], "traffic": _gemm_traffic(),
                      "algorithmic_bytes_per_launch": g["bytes"] / max(1, g["launches"]),
-                     "peak_source": f"{peaks['source']} sustained bf16"},
-        "kernels": kernel_table(prof, nprof, peaks),
+                     "gemm_flops_per_step": gemm_flops_step, "gemm_ms_per_step": gemm_ms_step,
+                     "method": "GEMM FLOPs of a control step / (GEMM share of the profiled pass x the timed step time)",
+                     "event_timed_tflops": kt["gemm"]["tflops"],
+                     "peak_source": f"{peaks['source']} burst bf16 (the timed unit is a step of a few ms)"},
+        "kernels": kt,
         "gpu_launches": int(stats["n_kernel_launches"]),
         "e2e": {"value": job_throughput(args.steps, world, e2e_ms), "unit": "chunks/s", "h2d_bytes_per_step": int(h2d),
                 "d2h_bytes_per_step": int(d2h), "wall_s": e2e_wall},
         "clocks": clk,
     }
+    if ablation is not None:
+        line["ablation"] = ablation
     if serving is not None:
         line["serving"] = serving
         line["serving_rr_accept"] = serving_rr
+    if bimanual is not None:
+        line["bimanual"] = bimanual
     if independent is not None:
         line["independent"] = independent
-    if cpu_times:
-        ct = cpu_times[-1]
-        line["cpu_baseline"] = {"value": 1.0 / ct, "unit": "chunks/s", "cores": cpu_cores, "kind": "oracle",
-                                "sample": "one warm control step (TR + 1 prefix step + OR + 2 steps, RR), float64 "
-                                          "oracle; best-effort second of two runs"}
+    if retained is not None:
+        line["cpu_baseline"] = cpu_baseline(retained)
     print(json.dumps(line))
     return 0
+
+
+def run_table3(ctx, flat, cfg, dev, stream, dev_in, obs0, noise, n, warm=3):
+    """The mechanisms of the paper's ablation (Table 3, App. C) on the benchmarked workload,
+    each timed over n control steps: GPU ms per replan (all denoising work of the replan) and
+    O2A ms (real observation to action chunk; App. A).
+      full       TR + OR (1 anticipatory step) + RR, layer stack replayed from CUDA graphs
+      wo_tr      every replan from fresh noise: 8 anticipatory steps under the prediction (the
+                 same rebinding stage), OR, 2 steps under the real observation
+      wo_or      TR, then all 3 retained steps under the real observation (no prefix)
+      wo_rr      TR + OR, every step runs all layers
+      wo_graph   TR + OR + RR, every kernel launched individually
+      native / native_graph   cold 10-step sample under the real observation, all layers
+    plus `rr_relaxed`: the full variant with RR thresholds that let every check pass (on random
+    weights the d768 model's consecutive probe residuals have cosine ~0.7, below every Table 7
+    threshold, so this is the only way to time the reuse path here; not a trained model's rate)."""
+    import torch
+
+    from paper_2609_34608_gb300 import inputs as I
+    from paper_2609_34608_gb300 import wam as W
+
+    K, b0, shift, pre = cfg["n_steps"], cfg["tr_entry_stage"], cfg["shift"], cfg["prefix_steps"]
+    ctx_norr = W.Context(dict(cfg, rr_policy=0), flat, stream=stream.cuda_stream)
+    ctx_relax = W.Context(dict(cfg, rr_gamma_cos=-1.0, rr_gamma_fit=1e30), flat, stream=stream.cuda_stream)
+    act = torch.zeros((1, cfg["n_action"], cfg["action_dim"]), device=dev)
+
+    def step_full(c, s, inp, mark):
+        pred, real, eps = inp
+        if c.adapt(s, pred, shift=shift, fresh_noise=eps)[0] == W.ADAPT_TR_INIT:
+            c.continue_(s, pre)
+        mark.record(stream)
+        s2 = c.adapt(s, real)[0]
+        c.continue_(s, K - (b0 + pre if s2 == W.ADAPT_REBIND_ACCEPT else b0), act)
+
+    def step_wo_tr(c, s, inp, mark):
+        pred, real, eps = inp
+        c.adapt(s, pred, entry=W.ENTRY_COLD, fresh_noise=eps)
+        c.continue_(s, b0 + pre)
+        mark.record(stream)
+        s2 = c.adapt(s, real)[0]
+        c.continue_(s, K - (b0 + pre if s2 == W.ADAPT_REBIND_ACCEPT else 0), act)
+
+    def step_wo_or(c, s, inp, mark):
+        pred, real, eps = inp
+        mark.record(stream)
+        c.adapt(s, real, shift=shift, fresh_noise=eps)
+        c.continue_(s, K - b0, act)
+
+    def step_native(c, s, inp, mark):
+        pred, real, eps = inp
+        mark.record(stream)
+        c.sample_cold(s, real, eps, K, act)
+
+    variants = [("full", ctx, True, step_full), ("wo_tr", ctx, True, step_wo_tr), ("wo_or", ctx, True, step_wo_or),
+                ("wo_rr", ctx_norr, True, step_full), ("wo_graph", ctx, False, step_full),
+                ("native_graph", ctx_norr, True, step_native), ("native", ctx_norr, False, step_native),
+                ("rr_relaxed", ctx_relax, True, step_full)]
+    ev = lambda: torch.cuda.Event(enable_timing=True)
+    out = {}
+    for name, c, graphs, fn in variants:
+        c.set_graph_replay(graphs)
+        s = c.state(1)
+        with torch.cuda.stream(stream):
+            c.sample_cold(s, obs0, noise, K)
+            for t in range(warm):
+                fn(c, s, dev_in[t % len(dev_in)], ev())
+        c.reset_stats()
+        torch.cuda.synchronize(dev)
+        marks = [(ev(), ev(), ev()) for _ in range(n)]
+        with torch.cuda.stream(stream):
+            for i in range(n):
+                marks[i][0].record(stream)
+                fn(c, s, dev_in[(warm + i) % len(dev_in)], marks[i][1])
+                marks[i][2].record(stream)
+        torch.cuda.synchronize(dev)
+        gpu = [m[0].elapsed_time(m[2]) for m in marks]
+        o2a = [m[1].elapsed_time(m[2]) for m in marks]
+        stt = c.stats()
+        out[name] = {"gpu_ms_per_replan": statistics.mean(gpu), "o2a_ms": statistics.mean(o2a),
+                     "o2a_ms_p50": float(np.percentile(o2a, 50)), "chunks_per_s": 1000.0 / statistics.mean(gpu),
+                     "r_rr": stt["n_reuse"] / max(1, stt["n_attempt"]),
+                     "f_skip": stt["b_skip"] / max(1, stt["b_dense"]),
+                     "r_or": stt["n_bind"] / max(1, stt["n_start"])}
+        s.close()
+        c.set_graph_replay(True)
+    ctx_norr.close()
+    ctx_relax.close()
+    out["steps"] = n
+    out["what"] = ("Table 3 variants on the closed-loop workload (GPU = mean ms of one replan's work, O2A = real "
+                   "observation to action chunk, both on the device clock); rr_relaxed = full with RR thresholds "
+                   "that accept every check (labelled: random weights, not a trained model's acceptance)")
+    return out
+
+
+def run_bimanual(dev, stream, peaks, n_cold=2):
+    """The large bimanual model (28 blocks, d1152, 16 heads of dim 72; 768 obs + 4096 video +
+    50 x 14 action tokens = 4914 tokens; batch 8): a 10-step cold sample of the batch, then the
+    warm-continuation sweep over retained-step counts 1..9 with executed shift 25 (TR of the
+    finished replan to entry stage K - n, then n steps; run from n = 9 down to 1)."""
+    import torch
+
+    from paper_2609_34608_gb300 import inputs as I
+    from paper_2609_34608_gb300 import wam as W
+
+    # retained stage = entry stage (r = b0), so that each replan of the sweep (n = 9 down to 1,
+    # entry stage K - n rising) remaps a stage the previous replan produced
+    cfg = I.get_config("bimanual", tr_retain_stage=-1)
+    B, K = cfg["batch"], cfg["n_steps"]
+    flat = torch.from_numpy(I.flatten_weights(I.make_weights(cfg))).to(dev)
+    ctx = W.Context(cfg, flat, stream=stream.cuda_stream)
+    del flat
+    with torch.cuda.stream(stream):
+        obs = torch.from_numpy(I.make_obs(cfg, B)).to(dev)
+        noise = torch.from_numpy(I.make_noise(cfg, B)).to(dev)
+        eps = [torch.from_numpy(I.make_fresh_eps(cfg, B, i)).to(dev) for i in range(K)]
+        act = torch.zeros((B, cfg["n_action"], cfg["action_dim"]), device=dev)
+        st = ctx.state(B)
+        ctx.sample_cold(st, obs, noise, K, act)   # warm-up (also captures the layer graphs)
+    ev = lambda: torch.cuda.Event(enable_timing=True)
+    cold = []
+    with torch.cuda.stream(stream):
+        for _ in range(n_cold):
+            a, b = ev(), ev()
+            a.record(stream)
+            ctx.sample_cold(st, obs, noise, K, act)
+            b.record(stream)
+            cold.append((a, b))
+    torch.cuda.synchronize(dev)
+    cold_ms = statistics.mean(a.elapsed_time(b) for a, b in cold)
+    sweep = {}
+    with torch.cuda.stream(stream):
+        marks = []
+        for n in range(K - 1, 0, -1):
+            a, b = ev(), ev()
+            a.record(stream)
+            ctx.adapt(st, obs, shift=cfg["shift"], entry=K - n, fresh_noise=eps[n])
+            ctx.continue_(st, n, act)
+            b.record(stream)
+            marks.append((n, a, b))
+    torch.cuda.synchronize(dev)
+    for n, a, b in marks:
+        ms = a.elapsed_time(b)
+        sweep[str(n)] = {"ms_per_batch": ms, "chunks_per_s": B / (ms * 1e-3)}
+    ctx.profile_enable(True)
+    with torch.cuda.stream(stream):
+        ctx.sample_cold(st, obs, noise, K, act)
+    prof = ctx.profile_read()
+    ctx.profile_enable(False)
+    ctx.close()
+    kt = kernel_table(prof, 1, peaks, tensor_peak="bf16_sus")
+    return {
+        "workload": "28-block d1152 16-head (head dim 72) bf16 DiT, 768 obs + 4096 video + 50x14 action tokens, "
+                    "batch 8; cold 10-step sample, then warm continuation of n = 1..9 retained steps after TR with "
+                    "executed shift 25",
+        "cold_ms_per_batch": cold_ms, "cold_chunks_per_s": B / (cold_ms * 1e-3),
+        "warm_sweep": sweep,
+        "gemm_tflops": kt["gemm"]["tflops"], "gemm_frac": kt["gemm"]["frac"],
+        "attn_tflops": kt["attn"]["tflops"], "attn_frac": kt["attn"]["frac"],
+        "kernels_per_cold_batch": kt,
+        "peak_source": "measured sustained bf16 (a batch runs for seconds)",
+    }
 
 
 def run_serving(dev, stream, peaks, warm_batches=2, batches=3, relax_gate=False):
@@ -485,7 +787,7 @@ def run_serving(dev, stream, peaks, warm_batches=2, batches=3, relax_gate=False)
     prof = ctx.profile_read()
     stats = ctx.stats()
     ctx.close()
-    kt = kernel_table(prof, 1, peaks)
+    kt = kernel_table(prof, 1, peaks, tensor_peak="bf16_sus")
     res = {
         "workload": "24-block d1024 16-head bf16 DiT, 384 obs + 2048 video + 32x7 action tokens; batch of 32 "
                     "episodes: 16 cold (10 steps) + 16 warm (TR shift 16, 2 of 10 steps) per batch",
@@ -623,9 +925,16 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-serving", action="store_true", help="skip the batched serving section")
     ap.add_argument("--no-independent", action="store_true", help="skip the independent-execution section")
+    ap.add_argument("--no-bimanual", action="store_true", help="skip the large bimanual model section")
+    ap.add_argument("--no-ablation", action="store_true", help="skip the Table 3 ablation section")
+    ap.add_argument("--cpu-plan", action="store_true",
+                    help="only time the CPU oracle plan (all cores and one core; no GPU) and print it")
     args = ap.parse_args()
     if args.warmup < 3:
         raise SystemExit("--warmup must be >= 3")
+    if args.cpu_plan:
+        print(json.dumps({"cpu_plan": cpu_plan()}))
+        return 0
     if args.impl == "reference":
         return main_reference(args)
     return main_ours(args)
