@@ -278,6 +278,25 @@ typedef struct wam_kclass_timing {
 } wam_kclass_timing;
 /* enable != 0 starts recording (clears previous spans); reading synchronizes the stream. */
 int wam_profile_enable(wam_ctx* ctx, int32_t enable);
+
+/*
+ * One task of a fused row-chain launch (wam_set_layer_fusion), recorded while profiling is on:
+ * kind 0 out-projection, 1 LN before the MLP, 2 MLP up, 3 MLP down, 4 LN of the next block, 5 QKV
+ * projection; m = 128-row block, j = column tile (or 32-row quarter for LN); times are the GPU's
+ * global timer in ns: task taken, dependency satisfied (operands requested), epilogue start,
+ * completion published.
+ */
+typedef struct {
+  int32_t launch, cta, kind, m, j, pad;
+  uint64_t t_take, t_dep, t_epi0, t_epi1;
+} wam_chain_task;
+
+/*
+ * Copies up to `capacity` recorded chain tasks (in launch order) since profiling was enabled into
+ * out (host memory) and their count into *n_out.  Synchronises the context's stream.
+ * WAM_ERR_INVALID_ARG for null pointers.
+ */
+int wam_profile_chain_trace(wam_ctx* ctx, wam_chain_task* out, int32_t capacity, int32_t* n_out);
 int wam_profile_read(wam_ctx* ctx, wam_kclass_timing* out /* [WAM_KCLASS_COUNT] */);
 
 /*
@@ -323,6 +342,31 @@ int wam_diag_layer_deltas(wam_ctx* ctx, wam_state* state, int32_t episode,
  * Results are identical either way.
  */
 int wam_set_graph_replay(wam_ctx* ctx, int32_t enable);
+
+/*
+ * Device-side Residual Rescaling branching (default on).  When a denoising step has a single work
+ * item whose RR check is attempted and the layer stack is replayed from graphs, the whole step
+ * around the gate (layers before the probe end, the probe sums and the Eq. 8 check, the middle
+ * layers under a graph conditional node that runs them only when the check fails, the injection
+ * or refresh, and the tail layers) is one CUDA graph captured on its second use: the decision is
+ * taken on the device and the host does not wait for it.  The decisions reach the step log and
+ * the reuse statistics through a small ring copied after each call; wam_state_log and
+ * wam_get_stats wait for the copies.  enable = 0 keeps the decision on the host (a read-back per
+ * step).  Results are identical either way.  WAM_ERR_INVALID_ARG for a null context.
+ */
+int wam_set_device_branching(wam_ctx* ctx, int32_t enable);
+
+/*
+ * Fused row-chain launches (default off).  Between two attentions the work of the DiT blocks is
+ * row-local: out-projection + gated residual, LN + modulation, MLP, gated residual, then the next
+ * block's LN + modulation and QKV projection.  With enable != 0, bf16 models with the tensor-core
+ * attention and a layer range of at most 16384 rows (episodes x tokens) run these as one
+ * persistent tensor-core launch per block instead of six, with per-row-block dependencies.  The
+ * arithmetic is the same either way (identical results).  Measured on one episode of the 12-block
+ * d768 model the fused launch is slower than the separate ones, so it is off by default.
+ * Returns WAM_ERR_INVALID_ARG for a null context.
+ */
+int wam_set_layer_fusion(wam_ctx* ctx, int32_t enable);
 
 /*
  * Output tile width (64, 128 or 256 columns) the context's bf16 path uses for the GEMM

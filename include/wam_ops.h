@@ -92,9 +92,11 @@ int wam_op_gemm_qkv_vt(const void* A, const void* Wt, const float* bias, void* q
                        int32_t M, int32_t d, int32_t rows_per_item, int32_t vt_ld, void* stream);
 
 /*
- * Full bidirectional attention on tcgen05 (head dim 64): q and k from qkv [B*N, 3d] (bf16),
- * v from vt as written by wam_op_gemm_qkv_vt with vt_ld = N rounded up to a multiple of 8,
- * out [B*N, d] bf16.  softmax(q k^T / 8) v per item and head, no mask.
+ * Full bidirectional attention on tcgen05 (head dim dh = d / n_heads, 64 or 72): q and k from
+ * qkv [B*N, 3d] (bf16), v from vt as written by wam_op_gemm_qkv_vt with vt_ld = N rounded up to a
+ * multiple of 8, out [B*N, d] bf16.  softmax(q k^T / sqrt(dh)) v per item and head, no mask.
+ * The head-dim-72 path reads eight V^T rows past each head (the next head's, or nothing past the
+ * end of vt); they only feed output columns that are discarded.
  */
 int wam_op_attention_tc(const void* qkv, const void* vt, void* out, int32_t B, int32_t N,
                         int32_t d, int32_t n_heads, void* stream);

@@ -21,7 +21,7 @@ BUILD_DIR = os.path.join(HERE, "_build")
 LIB_PATH = os.path.join(HERE, "libwam_gb300.so")
 
 SOURCES = ["wam_api.cu", "ops.cu", "gemm_tc.cu", "gemm_simt.cu", "attention.cu", "elementwise.cu",
-           "tr_static.cu", "attention_tc.cu"]
+           "tr_static.cu", "attention_tc.cu", "dit_chain.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ARCH + ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "-I", INCLUDE,
                 "--expt-relaxed-constexpr"]

@@ -1,4 +1,13 @@
-// Full bidirectional attention on the fifth-generation tensor cores (head dim 64).
+// Full bidirectional attention on the fifth-generation tensor cores (head dim 64 or 72).
+//
+// Head dim 72 (the bimanual model): tcgen05 K and N come in steps of 16, so the head is padded to
+// 80.  Q and K arrive as a 128-byte-swizzled atom of columns 0..63 plus a 32-byte-swizzled atom of
+// columns 64..79, fetched through a 3-D view {72, 3 heads, rows} of the QKV buffer whose
+// out-of-range columns 72..79 TMA fills with zeros, so the fifth K step of Q K^T adds nothing
+// spurious.  The P.V product runs with N = 80 over V^T rows of the head and the next eight
+// (or zero fill at the end); O columns 72..79 are never read.  Two S buffers instead of three keep
+// S and both padded O accumulators within the 512 TMEM columns.  The description below is for
+// head dim 64; with 72 the O accumulators sit at columns 256..335 and 336..415.
 //
 // One CTA owns 128 queries of one (item, head); TMEM lane r is query r.  Per block of 128 keys:
 //   S = Q K^T    tcgen05.mma M=128 N=128 K=64 into one of three TMEM S buffers (cols 0/128/256)
@@ -28,25 +37,36 @@ namespace {
 
 constexpr int kQ = 128;
 constexpr int kKV = 128;
-constexpr int kDH = 64;
 constexpr int kThreadsAttn = 384;
 constexpr float kRescaleLog2 = 8.0f;  // lazy-rescale threshold (log2 units)
-constexpr int kQBytes = kQ * kDH * 2;    // 16 KB
-constexpr int kKBytes = kKV * kDH * 2;   // 16 KB
-constexpr int kVBytes = kDH * kKV * 2;   // 16 KB: two 8 KB atom columns (64 keys each)
-constexpr int kOffQ = 0;
-constexpr int kKVStages = 6;
-constexpr int kSBuf = 3;  // TMEM S buffers (each also holds its block's P)
-constexpr int kOffK = kOffQ + kQBytes;
-constexpr int kOffV = kOffK + kKVStages * kKBytes;
-constexpr int kOffX = kOffV + kKVStages * kVBytes;   // max / sum exchange [2][2][128] floats
-constexpr int kOffBar = kOffX + 2048;
-constexpr int kNumBars = 1 + 2 * kKVStages + 3 * kSBuf + 8;
-constexpr int kSmemAttn = kOffBar + 512 + 1024;  // barriers, TMEM slot, abort flag; alignment slack
-static_assert(kNumBars * 8 + 8 <= 512, "barrier block exceeds its reservation");
 constexpr uint32_t kTmemCols = 512;
-constexpr uint32_t kColO = 384;  // O_0 at 384..447, O_1 at 448..511
 constexpr int kSoftmaxWarps = 8;
+
+// Shape of one head dimension.  Q / K tiles: a 128-byte-swizzled atom (head columns 0..63) plus,
+// for 72, a 32-byte-swizzled atom (columns 64..79); V^T tiles: kDHP rows of 128 keys as two atom
+// columns of 64 keys.
+template <int DH>
+struct AttnShape {
+  static constexpr int kDHP = DH == 64 ? 64 : 80;       // head dim padded to the MMA's N / K step
+  static constexpr int kTailRow = DH == 64 ? 0 : 32;    // bytes per row of the 32-byte-swizzled atom
+  static constexpr int kKVStages = DH == 64 ? 6 : 5;
+  static constexpr int kSBuf = DH == 64 ? 3 : 2;        // TMEM S buffers (each also holds its P)
+  static constexpr int kQBytes = kQ * (128 + kTailRow);
+  static constexpr int kKBytes = kKV * (128 + kTailRow);
+  static constexpr int kVBytes = kDHP * kKV * 2;        // two atom columns of 64 keys
+  static constexpr int kOffQ = 0;
+  static constexpr int kOffK = kOffQ + kQBytes;
+  static constexpr int kOffV = kOffK + kKVStages * kKBytes;
+  static constexpr int kOffX = kOffV + kKVStages * kVBytes;   // max / sum exchange [2][2][128] floats
+  static constexpr int kOffBar = kOffX + 2048;
+  static constexpr int kNumBars = 1 + 2 * kKVStages + 3 * kSBuf + 8;
+  static constexpr int kSmem = kOffBar + 512 + 1024;   // barriers, TMEM slot, abort flag; alignment slack
+  static constexpr uint32_t kColO = kSBuf * kKV;        // O_0 at kColO, O_1 at kColO + kDHP
+  static_assert(kNumBars * 8 + 8 <= 512, "barrier block exceeds its reservation");
+  static_assert(kColO + 2 * kDHP <= kTmemCols, "TMEM columns");
+  static_assert(kSmem <= 232448, "shared memory");
+  static_assert(kOffK % 1024 == 0 && kKBytes % 1024 == 0 && kVBytes % 2048 == 0, "swizzle alignment");
+};
 
 WAM_DEV float ex2(float x) {
   float y;
@@ -60,9 +80,16 @@ WAM_DEV float max3(float a, float b, float c) {
   return y;
 }
 
+template <int DH>
 __global__ void __launch_bounds__(kThreadsAttn, 1)
-    attn_tc_kernel(const __grid_constant__ CUtensorMap tmQK, const __grid_constant__ CUtensorMap tmVt,
-                   bf16* __restrict__ out, int N, int d, int H, float scale_log2, int* dev_err) {
+    attn_tc_kernel(const __grid_constant__ CUtensorMap tmQK, const __grid_constant__ CUtensorMap tmQKTail,
+                   const __grid_constant__ CUtensorMap tmVt, bf16* __restrict__ out, int N, int d, int H,
+                   float scale_log2, int* dev_err) {
+  using S = AttnShape<DH>;
+  constexpr int kDHP = S::kDHP, kKVStages = S::kKVStages, kSBuf = S::kSBuf;
+  constexpr int kQBytes = S::kQBytes, kKBytes = S::kKBytes, kVBytes = S::kVBytes;
+  constexpr int kOffQ = S::kOffQ, kOffK = S::kOffK, kOffV = S::kOffV, kOffX = S::kOffX, kOffBar = S::kOffBar;
+  constexpr uint32_t kColO = S::kColO;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint64_t* bars = reinterpret_cast<uint64_t*>(smem + kOffBar);
@@ -113,15 +140,25 @@ __global__ void __launch_bounds__(kThreadsAttn, 1)
     asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmQK)) : "memory");
     asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmVt)) : "memory");
     pdl_wait();
+    // Q (or K) rows [row, row + 128) of head hh: head dim 64 through the 2-D map {3d, rows};
+    // 72 through the 3-D map {72, 3H, rows}, columns 0..63 and 64..79 (72..79 zero-filled)
+    auto load_qk = [&](uint32_t dst, int hh, int row, uint32_t bar) {
+      if constexpr (DH == 64) {
+        tma_load_2d(dst, &tmQK, hh * 64, row, bar);
+      } else {
+        tma_load_3d(dst, &tmQK, 0, hh, row, bar);
+        tma_load_3d(dst + kQ * 128, &tmQKTail, 64, hh, row, bar);
+      }
+    };
     mbar_expect_tx(smem_u32(q_full), kQBytes);
-    tma_load_2d(smem_u32(smem + kOffQ), &tmQK, h * kDH, row_base + q0, smem_u32(q_full));
-    const int vt_row = (b * H + h) * kDH;
+    load_qk(smem_u32(smem + kOffQ), h, row_base + q0, smem_u32(q_full));
+    const int vt_row = (b * H + h) * DH;
     for (int j = 0; j < nkv; ++j) {
       const int s = j % kKVStages;
       if (!mbar_wait(smem_u32(&kv_empty[s]), ((j / kKVStages) & 1) ^ 1u, abort_flag, dev_err)) break;
       const uint32_t fb = smem_u32(&kv_full[s]);
       mbar_expect_tx(fb, kKBytes + kVBytes);
-      tma_load_2d(smem_u32(smem + kOffK + s * kKBytes), &tmQK, d + h * kDH, row_base + j * kKV, fb);
+      load_qk(smem_u32(smem + kOffK + s * kKBytes), H + h, row_base + j * kKV, fb);
       tma_load_2d(smem_u32(smem + kOffV + s * kVBytes), &tmVt, j * kKV, vt_row, fb);
       tma_load_2d(smem_u32(smem + kOffV + s * kVBytes + kVBytes / 2), &tmVt, j * kKV + 64, vt_row, fb);
     }
@@ -141,8 +178,11 @@ __global__ void __launch_bounds__(kThreadsAttn, 1)
       const uint64_t dk = sw128_desc(smem_u32(smem + kOffK + ks * kKBytes));
       if (elect_one()) {
 #pragma unroll
-        for (int t = 0; t < kDH / 16; ++t)   // descriptor address field is addr >> 4: +32 B = +2
+        for (int t = 0; t < 4; ++t)   // descriptor address field is addr >> 4: +32 B = +2
           umma_bf16(tmem + s * kKV, dq + 2 * t, dk + 2 * t, idS, t > 0 ? 1u : 0u);
+        if constexpr (DH != 64)        // head columns 64..79 from the 32-byte-swizzled atoms
+          umma_bf16(tmem + s * kKV, sw32_desc(smem_u32(smem + kOffQ) + kQ * 128),
+                    sw32_desc(smem_u32(smem + kOffK + ks * kKBytes) + kKV * 128), idS, 1u);
         umma_commit(smem_u32(&s_full[s]));   // same lane as the MMAs it tracks
       }
       __syncwarp();
@@ -154,7 +194,7 @@ __global__ void __launch_bounds__(kThreadsAttn, 1)
     // producer and tells the softmax that O is up to date; s_free[buffer] hands the S buffer (and
     // the P inside it) back to the S thread.
     const int hv = warp - 2;
-    const uint32_t idO = idesc_bf16(kQ, kDH);
+    const uint32_t idO = idesc_bf16(kQ, kDHP);
     for (int j = 0; j < nkv; ++j) {
       const int sb = j % kSBuf;
       const int vs = j % kKVStages;
@@ -167,7 +207,7 @@ __global__ void __launch_bounds__(kThreadsAttn, 1)
       if (elect_one()) {
 #pragma unroll
         for (int t = 0; t < 4; ++t)
-          umma_bf16_ta(tmem + kColO + hv * kDH, tp + t * 8, dv + 2 * t, idO, (j > 0 || t > 0) ? 1u : 0u);
+          umma_bf16_ta(tmem + kColO + hv * kDHP, tp + t * 8, dv + 2 * t, idO, (j > 0 || t > 0) ? 1u : 0u);
         umma_commit(smem_u32(&s_free[sb]));   // same lane as the MMAs they track
         umma_commit(smem_u32(&kv_empty[vs]));
       }
@@ -257,12 +297,19 @@ __global__ void __launch_bounds__(kThreadsAttn, 1)
         }
         tc_fence_after();
 #pragma unroll
-        for (int c = 0; c < kDH / 32; ++c) {
+        for (int c = 0; c < 2; ++c) {
           uint32_t v[32];
-          tmem_ld32(lane_addr + kColO + half * kDH + c * 32, v);
+          tmem_ld32(lane_addr + kColO + half * kDHP + c * 32, v);
 #pragma unroll
           for (int i = 0; i < 32; ++i) v[i] = __float_as_uint(__uint_as_float(v[i]) * corr);
-          tmem_st32(lane_addr + kColO + half * kDH + c * 32, v);
+          tmem_st32(lane_addr + kColO + half * kDHP + c * 32, v);
+        }
+        if constexpr (DH != 64) {   // head columns 64..71 (72..79 are padding, never read)
+          uint32_t v[8];
+          tmem_ld8(lane_addr + kColO + half * kDHP + 64, v);
+#pragma unroll
+          for (int i = 0; i < 8; ++i) v[i] = __float_as_uint(__uint_as_float(v[i]) * corr);
+          tmem_st8(lane_addr + kColO + half * kDHP + 64, v);
         }
       }
       // 32 bf16 pairs over the first 32 columns of this thread's S half-row (already read).
@@ -286,10 +333,26 @@ __global__ void __launch_bounds__(kThreadsAttn, 1)
         tc_fence_after();
         const int q = q0 + r;
         uint32_t v0[32], v1[32];
-        tmem_ld32(lane_addr + kColO + half * 32, v0);        // O_0, this thread's 32 columns
-        tmem_ld32(lane_addr + kColO + kDH + half * 32, v1);  // O_1, same columns
+        tmem_ld32(lane_addr + kColO + half * 32, v0);         // O_0, this thread's 32 columns
+        tmem_ld32(lane_addr + kColO + kDHP + half * 32, v1);  // O_1, same columns
+        if constexpr (DH != 64) {   // head columns 64..71, written by the first thread of the row
+          uint32_t t0[8], t1[8];
+          tmem_ld8(lane_addr + kColO + 64, t0);
+          tmem_ld8(lane_addr + kColO + kDHP + 64, t1);
+          if (q < N && half == 0) {
+            float o[8];
+#pragma unroll
+            for (int e = 0; e < 8; ++e) o[e] = fmaf(__uint_as_float(t0[e]), w0, __uint_as_float(t1[e]) * w1);
+            uint4 u;
+            u.x = pack_bf16x2(o[0], o[1]);
+            u.y = pack_bf16x2(o[2], o[3]);
+            u.z = pack_bf16x2(o[4], o[5]);
+            u.w = pack_bf16x2(o[6], o[7]);
+            *reinterpret_cast<uint4*>(out + static_cast<int64_t>(row_base + q) * d + h * DH + 64) = u;
+          }
+        }
         if (q < N) {
-          uint4* dst = reinterpret_cast<uint4*>(out + static_cast<int64_t>(row_base + q) * d + h * kDH + half * 32);
+          uint4* dst = reinterpret_cast<uint4*>(out + static_cast<int64_t>(row_base + q) * d + h * DH + half * 32);
 #pragma unroll
           for (int k = 0; k < 4; ++k) {
             float o[8];
@@ -319,17 +382,45 @@ __global__ void __launch_bounds__(kThreadsAttn, 1)
 
 }  // namespace
 
-cudaError_t attention_tc(const CUtensorMap& tm_qk, const CUtensorMap& tm_vt, bf16* out, int B, int N, int d,
-                         int H, int* dev_err, cudaStream_t s) {
+int attention_tc_encode(AttnMaps* m, const void* qkv, const void* vt, int items, int N, int d, int H, int vt_ld) {
+  const int dh = H > 0 ? d / H : 0;
+  const uint64_t rows = static_cast<uint64_t>(items) * N;
+  if (H <= 0 || d != dh * H || (dh != 64 && dh != 72)) return -1;
+  m->dh = dh;
+  if (dh == 64) {
+    if (tc_encode_bf16_box(&m->qk, qkv, rows, 3 * d, 3 * d, 64, 128) != 0) return -2;
+    m->qk_tail = m->qk;
+  } else {
+    // {72 head columns, 3H heads of q | k | v, rows}: box columns past 72 are zero-filled
+    const uint64_t dims[3] = {72, static_cast<uint64_t>(3 * H), rows};
+    const uint64_t strides[2] = {72 * 2, static_cast<uint64_t>(3 * d) * 2};
+    const uint32_t box0[3] = {64, 1, 128}, box1[3] = {16, 1, 128};
+    if (tc_encode_bf16_3d(&m->qk, qkv, dims, strides, box0, 128) != 0 ||
+        tc_encode_bf16_3d(&m->qk_tail, qkv, dims, strides, box1, 32) != 0)
+      return -2;
+  }
+  const uint32_t vrows = dh == 64 ? 64 : 80;
+  if (tc_encode_bf16_box(&m->vt, vt, static_cast<uint64_t>(items) * d, vt_ld, vt_ld, 64, vrows) != 0) return -3;
+  return 0;
+}
+
+cudaError_t attention_tc(const AttnMaps& m, bf16* out, int B, int N, int d, int H, int* dev_err, cudaStream_t s) {
   if (B <= 0 || N <= 0) return cudaSuccess;
-  if (d / H != kDH) return cudaErrorInvalidValue;
-  static PerDeviceSmem smem_rec;  // contexts may run on several host threads and devices
-  const cudaError_t e = ensure_max_smem(smem_rec, attn_tc_kernel, kSmemAttn);
-  if (e != cudaSuccess) return e;
-  const float scale_log2 = 1.4426950408889634f / 8.0f;  // log2(e) / sqrt(64)
+  if (d / H != m.dh) return cudaErrorInvalidValue;
+  const float scale_log2 = 1.4426950408889634f / sqrtf(static_cast<float>(m.dh));  // log2(e) / sqrt(dh)
   dim3 grid((N + kQ - 1) / kQ, H, B);
-  return launch_pdl(attn_tc_kernel, grid, dim3(kThreadsAttn), kSmemAttn, s, tm_qk, tm_vt, out, N, d, H,
-                    scale_log2, dev_err);
+  if (m.dh == 64) {
+    static PerDeviceSmem smem_rec;  // contexts may run on several host threads and devices
+    const cudaError_t e = ensure_max_smem(smem_rec, attn_tc_kernel<64>, AttnShape<64>::kSmem);
+    if (e != cudaSuccess) return e;
+    return launch_pdl(attn_tc_kernel<64>, grid, dim3(kThreadsAttn), AttnShape<64>::kSmem, s, m.qk, m.qk_tail, m.vt,
+                      out, N, d, H, scale_log2, dev_err);
+  }
+  static PerDeviceSmem smem_rec72;
+  const cudaError_t e = ensure_max_smem(smem_rec72, attn_tc_kernel<72>, AttnShape<72>::kSmem);
+  if (e != cudaSuccess) return e;
+  return launch_pdl(attn_tc_kernel<72>, grid, dim3(kThreadsAttn), AttnShape<72>::kSmem, s, m.qk, m.qk_tail, m.vt,
+                    out, N, d, H, scale_log2, dev_err);
 }
 
 int attention_tc_vt_ld(int N) { return (N + 7) / 8 * 8; }

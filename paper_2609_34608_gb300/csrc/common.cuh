@@ -7,7 +7,10 @@
 #include <cuda_runtime.h>
 #include <stdint.h>
 
+#include "wam.h"
+
 #include <atomic>
+#include <mutex>
 
 #define WAM_DEV __device__ __forceinline__
 
@@ -66,16 +69,31 @@ struct PerDeviceSmem {
   std::atomic<int> granted[kMaxTrackedDevices] = {};
 };
 
+// Raises the kernel's limit to at least `bytes` on the current device.  The limit never shrinks:
+// another host thread may launch the same kernel with a larger size between this set and its own
+// launch.  Sets are serialised so the recorded value is always the attribute's value.
+inline std::mutex& smem_attr_mutex() {
+  static std::mutex m;
+  return m;
+}
+
 template <typename Kernel>
 inline cudaError_t ensure_max_smem(PerDeviceSmem& rec, Kernel kernel, int bytes) {
   const int dev = current_device();
   const bool tracked = dev >= 0 && dev < kMaxTrackedDevices;
   if (tracked && rec.granted[dev].load(std::memory_order_acquire) >= bytes) return cudaSuccess;
-  const cudaError_t e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
-  if (e != cudaSuccess || !tracked) return e;
-  int prev = rec.granted[dev].load(std::memory_order_relaxed);
-  while (prev < bytes && !rec.granted[dev].compare_exchange_weak(prev, bytes)) {
+  std::lock_guard<std::mutex> lock(smem_attr_mutex());
+  if (!tracked) {
+    // untracked device: never lower the limit below what the function already allows
+    int cur = 0;
+    cudaFuncAttributes fa;
+    if (cudaFuncGetAttributes(&fa, kernel) == cudaSuccess) cur = fa.maxDynamicSharedSizeBytes;
+    return cur >= bytes ? cudaSuccess : cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
   }
+  if (rec.granted[dev].load(std::memory_order_relaxed) >= bytes) return cudaSuccess;
+  const cudaError_t e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
+  if (e != cudaSuccess) return e;
+  rec.granted[dev].store(bytes, std::memory_order_release);
   return cudaSuccess;
 }
 
@@ -101,6 +119,23 @@ WAM_DEV double warp_sum_d(double v) {
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
   return v;
+}
+
+// Mean and reciprocal standard deviation (eps 1e-6) of one d-wide row held by a warp as NV4
+// float4s per lane (d = 128 NV4): the LayerNorm statistics of every LN kernel.
+template <int NV4>
+WAM_DEV void row_stats(const float4 (&v)[NV4], int d, float& mean, float& rstd) {
+  float s = 0.0f;
+#pragma unroll
+  for (int i = 0; i < NV4; ++i) s += (v[i].x + v[i].y) + (v[i].z + v[i].w);
+  mean = warp_sum(s) / d;
+  float q = 0.0f;
+#pragma unroll
+  for (int i = 0; i < NV4; ++i) {
+    const float a = v[i].x - mean, b = v[i].y - mean, c = v[i].z - mean, e = v[i].w - mean;
+    q += (a * a + b * b) + (c * c + e * e);
+  }
+  rstd = rsqrtf(warp_sum(q) / d + 1e-6f);
 }
 
 WAM_DEV float silu_f(float x) { return x / (1.0f + expf(-x)); }
@@ -174,6 +209,38 @@ GemmPlan tc_gemm_plan(int M, int N, int K, bool has64, bool can_split, int num_s
 cudaError_t tc_gemm(const GemmOperand& a, const GemmOperand& b, int M, int N, int K, int epi, const EpiArgs& e,
                     int num_sms, int* dev_err, cudaStream_t s, const SplitWorkspace* ws, GemmPlan plan);
 
+// Row-local chain of DiT blocks as one persistent tcgen05 kernel (dit_chain.cu): the "tail" of
+// block l (out-projection + gated residual, LN, MLP up, MLP down + gated residual) followed by the
+// "head" of block l+1 (LN + modulation, QKV projection with V^T), either part optional.
+struct ChainParams {
+  int M, Mt, d, dff;          // rows, 128-row blocks, model width, MLP width
+  int has_tail, has_head;
+  EpiArgs e_out, e_up, e_down, e_qkv;
+  const float* mods;          // per-item modulation rows
+  int64_t mod_stride;
+  const int* item_map;        // nullable: modulation row of local item i = item_map[i]
+  int rows_per_item;
+  int shift2_off, scale2_off;  // tail: LN before the MLP
+  int shift1_off, scale1_off;  // head: LN before attention
+  float* h;                   // fp32 residual stream [M, d]
+  float* hq;                  // nullable: the head's LN also copies h here
+  bf16* xln;                  // LN output [M, d]
+  int* ctr;                   // dit_chain_counters(max rows) ints, zero before the first launch
+  int* dev_err;
+  wam_chain_task* trace;      // nullable: per-task timestamps (profiling), task t at trace[t]
+  int trace_cap;              // tasks beyond it are not recorded
+  int trace_launch;           // launch number written into the records
+  int phase_barrier;          // 1: each kind waits for all of the previous kind (grid-wide)
+};
+// Two-atom, 128-row tensor maps of the operands (unused ones may repeat any valid map).
+struct ChainMaps {
+  const CUtensorMap *att, *xln, *u, *out_w, *up_w, *down_w, *qkv_w;
+};
+int dit_chain_counters(int max_rows);
+int dit_chain_tasks(const ChainParams& p);
+bool dit_chain_supported(int d, int dff);
+cudaError_t dit_chain(const ChainMaps& maps, const ChainParams& p, int num_sms, cudaStream_t s);
+
 // float32 SIMT GEMM (gemm_simt.cu): C = A[M,K] Wt[N,K]^T
 cudaError_t simt_gemm(const float* A, const float* Wt, int M, int N, int K, int epi,
                       const EpiArgs& e, cudaStream_t s);
@@ -184,12 +251,20 @@ cudaError_t attention_bf16(const bf16* qkv, bf16* out, int B, int N, int d, int 
 cudaError_t attention_f32(const float* qkv, float* out, int B, int N, int d, int H,
                           cudaStream_t s);
 bool attention_bf16_supported(int head_dim);
-// tcgen05 attention (attention_tc.cu), head dim 64: Q / K read from the qkv buffer through
-// tm_qk (box 64 x 128), V^T [items*heads*64, vt_ld] through tm_vt (box 64 x 64).
-cudaError_t attention_tc(const CUtensorMap& tm_qk, const CUtensorMap& tm_vt, bf16* out, int B, int N, int d,
-                         int H, int* dev_err, cudaStream_t s);
+// tcgen05 attention (attention_tc.cu), head dim 64 or 72: Q / K read from the qkv buffer
+// [items * N, 3d], V^T [items * d, vt_ld] as written by the QKV projection's epilogue.
+struct AttnMaps {
+  CUtensorMap qk, qk_tail, vt;
+  int dh;
+};
+// 0 on success; negative when the head dim is unsupported or an encoding failed.
+int attention_tc_encode(AttnMaps* m, const void* qkv, const void* vt, int items, int N, int d, int H, int vt_ld);
+cudaError_t attention_tc(const AttnMaps& m, bf16* out, int B, int N, int d, int H, int* dev_err, cudaStream_t s);
 int attention_tc_vt_ld(int N);
 int tc_encode_bf16_box(CUtensorMap* map, const void* base, uint64_t rows, uint64_t cols, uint64_t ld,
                        uint32_t box_cols, uint32_t box_rows);
+// 3-D bf16 map: dims (innermost first), byte strides of dims 1 and 2, box, swizzle 128 or 32 bytes.
+int tc_encode_bf16_3d(CUtensorMap* map, const void* base, const uint64_t (&dims)[3], const uint64_t (&strides)[2],
+                      const uint32_t (&box)[3], int swizzle_bytes);
 
 }  // namespace wam

@@ -200,21 +200,6 @@ __global__ void __launch_bounds__(256) embed_kernel(
 }
 
 // ---------------------------------------------------------------- LN modulate
-template <int NV4>
-WAM_DEV void row_stats(const float4 (&v)[NV4], int d, float& mean, float& rstd) {
-  float s = 0.0f;
-#pragma unroll
-  for (int i = 0; i < NV4; ++i) s += (v[i].x + v[i].y) + (v[i].z + v[i].w);
-  mean = warp_sum(s) / d;
-  float q = 0.0f;
-#pragma unroll
-  for (int i = 0; i < NV4; ++i) {
-    const float a = v[i].x - mean, b = v[i].y - mean, c = v[i].z - mean, e = v[i].w - mean;
-    q += (a * a + b * b) + (c * c + e * e);
-  }
-  rstd = rsqrtf(warp_sum(q) / d + 1e-6f);
-}
-
 template <int NV4, typename TO>
 __global__ void __launch_bounds__(256) ln_mod_kernel(const float* __restrict__ h,
                                                      float* __restrict__ hcopy,
@@ -886,6 +871,38 @@ __global__ void rr_gate_kernel(const double* __restrict__ partial, int Bw, int n
   out[i] = g;
 }
 
+// Device-side RR decision of a single work item (§3.3 branch rule: every non-empty branch must
+// pass Eq. 8): writes the item's apply mode and factors, appends the decision to a ring of records
+// for the host's bookkeeping, and, inside a CUDA graph, sets the conditional that runs the middle
+// layers (1 = rejected: run them and refresh; 0 = accepted: inject).
+__global__ void rr_decide_kernel(const RRGate* __restrict__ g, int has0, int has1, RRApply* __restrict__ ap,
+                                 RRDecision* __restrict__ ring, unsigned long long* __restrict__ ring_n,
+                                 int ring_cap, cudaGraphConditionalHandle handle, int set_handle) {
+  pdl_wait();
+  pdl_launch_dependents();
+  if (threadIdx.x != 0) return;
+  const bool pass = (!has0 || g[0].pass) && (!has1 || g[1].pass);
+  RRApply a;
+  a.mode = pass ? kRRInject : kRRRefresh;
+  a.cidx = 0;
+  a.alpha0 = pass ? static_cast<float>(g[0].alpha) : 0.0f;
+  a.alpha1 = pass ? static_cast<float>(g[1].alpha) : 0.0f;
+  ap[0] = a;
+  const unsigned long long n = *ring_n;
+  RRDecision r;
+  r.accept = pass ? 1 : 0;
+  r.pad = 0;
+  for (int b = 0; b < 2; ++b) {
+    const bool has = b == 0 ? has0 : has1;
+    r.alpha[b] = has ? static_cast<float>(g[b].alpha) : 0.0f;
+    r.cos[b] = has ? static_cast<float>(g[b].cos) : 0.0f;
+    r.fit[b] = has ? static_cast<float>(g[b].fit) : 0.0f;
+  }
+  ring[n % static_cast<unsigned long long>(ring_cap)] = r;
+  *ring_n = n + 1;
+  if (set_handle) cudaGraphSetConditional(handle, pass ? 0u : 1u);
+}
+
 // Accepted: h_e = h_s + alpha_branch R_a (Eq. 9).  Refresh: R_a = h_e - h_s, p_a = h_s - h_q,
 // h = h_e.  Copy-back: h = h_e (item not on an RR path).
 __global__ void __launch_bounds__(256) rr_apply_kernel(float* __restrict__ h,
@@ -1026,8 +1043,10 @@ cudaError_t gemv_launch(const CondGemv& g, cudaStream_t s) {
   const int kslice = (g.K + g.splits - 1) / g.splits;
   const size_t smem = sizeof(float) * (static_cast<size_t>(KB) * kslice + 8 * KB * CPB);
   if (smem > 200 * 1024) return cudaErrorInvalidValue;
-  cudaError_t e = cudaFuncSetAttribute(cond_gemv_kernel<TW, KB>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                       static_cast<int>(smem));
+  // The limit only ever grows (per device): contexts on other host threads launch the same kernel
+  // with other sizes, and lowering it between their set and their launch would fail that launch.
+  static PerDeviceSmem smem_rec;
+  cudaError_t e = ensure_max_smem(smem_rec, cond_gemv_kernel<TW, KB>, static_cast<int>(smem));
   if (e != cudaSuccess) return e;
   dim3 grid((g.Nout + CPB - 1) / CPB, g.splits);
   launch_pdl(cond_gemv_kernel<TW, KB>, dim3(grid), dim3(256), smem, s, g.in_part, g.in_splits, g.in_bias, g.in_act, g.features,
@@ -1216,6 +1235,12 @@ cudaError_t rr_gate(const double* partial, int Bw, int nch, int64_t n0, int64_t 
   if (Bw <= 0) return cudaSuccess;
   launch_pdl(rr_gate_kernel, dim3((Bw * 2 * 32 + 127) / 128), dim3(128), 0, s, partial, Bw, nch, n0, n1, amin, amax, eps,
                                                            gcos, gfit, out);
+  return cudaGetLastError();
+}
+
+cudaError_t rr_decide(const RRGate* g, int has0, int has1, RRApply* ap, RRDecision* ring, unsigned long long* ring_n,
+                      int ring_cap, cudaGraphConditionalHandle handle, int set_handle, cudaStream_t s) {
+  launch_pdl(rr_decide_kernel, dim3(1), dim3(32), 0, s, g, has0, has1, ap, ring, ring_n, ring_cap, handle, set_handle);
   return cudaGetLastError();
 }
 

@@ -31,6 +31,12 @@ struct RRGate {
   int32_t pad;
 };
 
+// One device-side RR decision (single work item), as the host records it in the step log.
+struct RRDecision {
+  int32_t accept, pad;
+  float alpha[2], cos[2], fit[2];
+};
+
 // RR apply mode of one item after the gate.
 enum RRMode : int32_t { kRRNone = 0, kRRInject = 1, kRRRefresh = 2, kRRCopyBack = 3 };
 struct RRApply {
@@ -108,6 +114,9 @@ cudaError_t rr_gather(float* hm, const float* h, const int* map, int nmid, int64
 // whose column (index mod row_len) is below cols.
 cudaError_t diag_partial(const float* a, const float* b, int64_t n, int64_t row_len, int64_t cols, int nblocks,
                          double* partial, cudaStream_t s);
+// The RR decision of work item 0 taken on the device (see rr_decide_kernel).
+cudaError_t rr_decide(const RRGate* g, int has0, int has1, RRApply* ap, RRDecision* ring, unsigned long long* ring_n,
+                      int ring_cap, cudaGraphConditionalHandle handle, int set_handle, cudaStream_t s);
 cudaError_t rr_apply(float* h, const float* hm, const float* hq, float* pa, float* ra,
                      const StepItem* items, const RRApply* ap, int Bw, int N, int d,
                      int split_row, cudaStream_t s);

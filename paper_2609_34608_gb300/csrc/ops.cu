@@ -159,7 +159,7 @@ int wam_op_gemm_qkv_vt(const void* A, const void* Wt, const float* bias, void* q
   const int N = 3 * d, K = d;
   int r = check_gemm_args(A, Wt, qkv, M, N, K, WAM_EPI_BF16, nullptr, rows_per_item);
   if (r != WAM_OK) return r;
-  if (vt == nullptr || rows_per_item <= 0 || vt_ld < rows_per_item || vt_ld % 8 != 0 || d % 64 != 0 || d % 128 != 0)
+  if (vt == nullptr || rows_per_item <= 0 || vt_ld < rows_per_item || vt_ld % 8 != 0 || d % 128 != 0)
     return op_fail(WAM_ERR_INVALID_ARG, "bad V^T arguments");
   if (!aligned16(A) || !aligned16(Wt) || !aligned16(qkv) || (bias && !aligned16(bias)))
     return op_fail(WAM_ERR_INVALID_ARG, "operands must be 16-byte aligned");
@@ -181,16 +181,16 @@ int wam_op_gemm_qkv_vt(const void* A, const void* Wt, const float* bias, void* q
 
 int wam_op_attention_tc(const void* qkv, const void* vt, void* out, int32_t B, int32_t N, int32_t d,
                         int32_t n_heads, void* stream) {
-  if (qkv == nullptr || vt == nullptr || out == nullptr || B < 0 || N < 0 || n_heads <= 0 || d != 64 * n_heads)
-    return op_fail(WAM_ERR_INVALID_ARG, "tcgen05 attention needs head dim 64");
+  if (qkv == nullptr || vt == nullptr || out == nullptr || B < 0 || N < 0 || n_heads <= 0 ||
+      (d != 64 * n_heads && d != 72 * n_heads))
+    return op_fail(WAM_ERR_INVALID_ARG, "tcgen05 attention needs head dim 64 or 72");
   if (!aligned16(qkv) || !aligned16(vt) || !aligned16(out)) return op_fail(WAM_ERR_INVALID_ARG, "16-byte alignment required");
   if (B == 0 || N == 0) return WAM_OK;
   const int vt_ld = attention_tc_vt_ld(N);
-  CUtensorMap tq, tv;
-  if (tc_encode_bf16_box(&tq, qkv, static_cast<uint64_t>(B) * N, 3 * d, 3 * d, 64, 128) != 0 ||
-      tc_encode_bf16_box(&tv, vt, static_cast<uint64_t>(B) * d, vt_ld, vt_ld, 64, 64) != 0)
+  AttnMaps maps;
+  if (attention_tc_encode(&maps, qkv, vt, B, N, d, n_heads, vt_ld) != 0)
     return op_fail(WAM_ERR_CUDA, "cuTensorMapEncodeTiled failed");
-  cudaError_t e = attention_tc(tq, tv, static_cast<bf16*>(out), B, N, d, n_heads, nullptr,
+  cudaError_t e = attention_tc(maps, static_cast<bf16*>(out), B, N, d, n_heads, nullptr,
                                static_cast<cudaStream_t>(stream));
   return e == cudaSuccess ? WAM_OK : op_cuda("tcgen05 attention launch", e);
 }

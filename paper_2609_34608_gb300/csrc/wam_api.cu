@@ -8,6 +8,7 @@
 #include <cmath>
 #include <cstdio>
 #include <cstring>
+#include <deque>
 #include <map>
 #include <new>
 #include <string>
@@ -28,6 +29,10 @@ constexpr size_t kSlotBytes = 16384;
 constexpr int kMaxBatch = 256;
 constexpr int kT1Splits = 8;  // K splits of the two conditioning-MLP GEMVs
 constexpr int kT2Splits = 8;
+// Largest row count (episodes x tokens) of a layer range run by the fused row-chain kernel.  Above
+// it the per-projection GEMMs pick wider tiles and fill the GPU on their own.
+constexpr int kChainMaxRows = 16384;
+constexpr int kDecCap = 1024;   // device RR decisions in flight between the GPU and the host
 
 struct LayerW {
   void* qkv_wt = nullptr;
@@ -94,12 +99,44 @@ struct wam_ctx {
   bool tc_attn = false;
   void* vt = nullptr;
   int vt_ld = 0;
-  CUtensorMap tm_qk, tm_vt;
+  AttnMaps attn_maps;
   float *t1 = nullptr, *cvec = nullptr, *mods = nullptr;
   StepItem* d_items = nullptr;
   int* d_map = nullptr;
   // conditioning once per distinct sigma of a step: those items, their modulation rows, and the
   // work item -> distinct sigma index used to broadcast the rows
+  // fused row-chain kernel (dit_chain.cu), off unless enabled: for bf16 models with the
+  // tensor-core attention when a layer range covers at most kChainMaxRows rows; its completion
+  // counters
+  bool chain_ok = false;
+  bool layer_fusion = false;
+  bool chain_phases = true;   // grid-wide phase boundaries instead of per-row-block dependencies
+  int* d_chain_ctr = nullptr;
+  // profiling: per-task records of the fused launches (allocated on first use)
+  wam_chain_task* d_trace = nullptr;
+  int trace_cap = 0, trace_used = 0, trace_launches = 0;
+  // Device-side RR branching for a single work item (§3.3 at one episode): the whole step around
+  // the gate is one CUDA graph whose conditional node runs the middle layers only when the gate
+  // rejects, so the host never waits for the decision.  Decisions come back through a ring of
+  // records copied to pinned memory after each call and folded into the step log and the reuse
+  // statistics when the host next looks (or when the ring would overflow).
+  bool dev_branch = true;
+  bool dev_branch_ok = true;
+  cudaStream_t aux_stream = nullptr;    // captures the conditional body
+  int* d_map0 = nullptr;                // {0}: item map of the single gathered item
+  RRDecision* d_dec = nullptr;          // [kDecCap] ring of decisions
+  unsigned long long* d_dec_n = nullptr;
+  RRDecision* h_dec = nullptr;          // pinned mirror of the ring
+  unsigned long long dec_queued = 0, dec_copied = 0, dec_resolved = 0;
+  struct PendingDec {
+    wam_state* st;
+    int log_idx;   // -1 once the state's log moved on
+  };
+  std::deque<PendingDec> dec_pending;
+  std::deque<std::pair<cudaEvent_t, unsigned long long>> dec_batches;   // (copy done, records up to)
+  std::map<std::tuple<const void*, const void*>, cudaGraphExec_t> rr_graphs;
+  std::map<std::tuple<const void*, const void*>, int> rr_graph_uses;
+  std::map<cudaGraphExec_t, long long> graph_kernels;   // kernels per graph (launch counting)
   // CUDA graphs of layer ranges: key (first layer, end layer, episodes, stream buffer, item map,
   // layer that also saves h_q or -1) -> executable graph, captured on a range's second use
   bool graph_replay = true;
@@ -317,7 +354,7 @@ int run_layer(wam_ctx* c, int l, float* hb, int Bw, const int* map, float* hcopy
     const double el = c->bf16 ? 2.0 : 4.0;
     Span sp(c, WAM_KCLASS_ATTN, 4.0 * Bw * double(c->N) * c->N * d, el * 4.0 * M * d);
     if (c->tc_attn)
-      CK(attention_tc(c->tm_qk, c->tm_vt, static_cast<bf16*>(c->att), Bw, c->N, d, c->H, c->d_err, c->stream));
+      CK(attention_tc(c->attn_maps, static_cast<bf16*>(c->att), Bw, c->N, d, c->H, c->d_err, c->stream));
     else if (c->bf16)
       CK(attention_bf16(static_cast<const bf16*>(c->qkv), static_cast<bf16*>(c->att), Bw, c->N, d, c->H, c->stream));
     else
@@ -333,6 +370,82 @@ int run_layer(wam_ctx* c, int l, float* hb, int Bw, const int* map, float* hcopy
   return WAM_OK;
 }
 
+// The row-local work between two attentions as one fused launch: the tail of layer `lt`
+// (out-projection .. MLP down) and / or the head of layer `lh` (LN + QKV), -1 for none.
+int run_chain(wam_ctx* c, int lt, int lh, float* hb, int Bw, const int* map, float* hcopy) {
+  const int M = Bw * c->N, d = c->d;
+  ChainParams p;
+  std::memset(&p, 0, sizeof(p));
+  p.M = M;
+  p.Mt = (M + 127) / 128;
+  p.d = d;
+  p.dff = c->dff;
+  p.has_tail = lt >= 0;
+  p.has_head = lh >= 0;
+  p.mods = c->mods;
+  p.mod_stride = c->mod_n;
+  p.item_map = map;
+  p.rows_per_item = c->N;
+  p.h = hb;
+  p.hq = hcopy;
+  p.xln = static_cast<bf16*>(c->xln);
+  p.ctr = c->d_chain_ctr;
+  p.dev_err = c->d_err;
+  p.phase_barrier = c->chain_phases ? 1 : 0;
+  ChainMaps maps{&c->tm_att.r128_k2, &c->tm_xln.r128_k2, &c->tm_u.r128_k2, &c->tm_xln.r128_k2,
+                 &c->tm_xln.r128_k2, &c->tm_xln.r128_k2, &c->tm_xln.r128_k2};
+  double flops = 0.0, bytes = 0.0;
+  if (lt >= 0) {
+    LayerW& w = c->layers[lt];
+    const int base = lt * 6 * d;
+    p.e_out = epi_args(w.out_b, hb, c->mods + base + 2 * d, c->mod_n, c->N, map);
+    p.e_up = epi_args(w.up_b, c->u, nullptr, 0, c->N, nullptr);
+    p.e_down = epi_args(w.down_b, hb, c->mods + base + 5 * d, c->mod_n, c->N, map);
+    p.shift2_off = base + 3 * d;
+    p.scale2_off = base + 4 * d;
+    maps.out_w = &w.tm_out.r64_k2;     // 64-column tiles of the d-wide projections
+    maps.up_w = &w.tm_up.r128_k2;
+    maps.down_w = &w.tm_down.r64_k2;
+    flops += 2.0 * M * (double(d) * d + 2.0 * double(d) * c->dff);
+    bytes += 2.0 * (double(d) * d + 2.0 * double(d) * c->dff) + double(M) * (2.0 * d + 16.0 * d + 4.0 * c->dff);
+  }
+  if (lh >= 0) {
+    LayerW& w = c->layers[lh];
+    const int base = lh * 6 * d;
+    p.e_qkv = epi_args(w.qkv_b, c->qkv, nullptr, 0, c->N, nullptr);
+    p.e_qkv.vt = static_cast<bf16*>(c->vt);
+    p.e_qkv.vt_ld = c->vt_ld;
+    p.shift1_off = base;
+    p.scale1_off = base + d;
+    maps.qkv_w = &w.tm_qkv.r128_k2;
+    flops += 2.0 * M * 3.0 * double(d) * d;
+    bytes += 6.0 * double(d) * d + double(M) * (4.0 * d + 4.0 * d + 6.0 * d + (hcopy ? 4.0 * d : 0.0));
+  }
+  if (c->prof_on && c->d_trace != nullptr) {
+    const int n = dit_chain_tasks(p);
+    p.trace = c->d_trace + c->trace_used;
+    p.trace_cap = std::max(0, std::min(n, c->trace_cap - c->trace_used));
+    p.trace_launch = c->trace_launches++;
+    c->trace_used += p.trace_cap;
+  }
+  Span sp(c, WAM_KCLASS_GEMM, flops, bytes);
+  CK(dit_chain(maps, p, c->num_sms, c->stream));
+  return WAM_OK;
+}
+
+int run_attention(wam_ctx* c, int Bw) {
+  const int M = Bw * c->N, d = c->d;
+  const double el = c->bf16 ? 2.0 : 4.0;
+  Span sp(c, WAM_KCLASS_ATTN, 4.0 * Bw * double(c->N) * c->N * d, el * 4.0 * M * d);
+  if (c->tc_attn)
+    CK(attention_tc(c->attn_maps, static_cast<bf16*>(c->att), Bw, c->N, d, c->H, c->d_err, c->stream));
+  else if (c->bf16)
+    CK(attention_bf16(static_cast<const bf16*>(c->qkv), static_cast<bf16*>(c->att), Bw, c->N, d, c->H, c->stream));
+  else
+    CK(attention_f32(static_cast<const float*>(c->qkv), static_cast<float*>(c->att), Bw, c->N, d, c->H, c->stream));
+  return WAM_OK;
+}
+
 // Layers [l0, l1) of the episodes in hb (item map `map`, or none), saving h_q at layer `hq_layer`
 // (or -1).  The ~7 launches per layer have fixed arguments for a given key, so a range is
 // captured into a CUDA graph on its second use (the first runs eagerly, which also sets every
@@ -340,15 +453,29 @@ int run_layer(wam_ctx* c, int l, float* hb, int Bw, const int* map, float* hcopy
 // per-kernel launch gaps.  Profiling (per-kernel events) and a failed capture run eagerly.
 int run_layers(wam_ctx* c, int l0, int l1, float* hb, int Bw, const int* map, int hq_layer) {
   if (l0 >= l1) return WAM_OK;
+  const bool fused = c->chain_ok && c->layer_fusion && Bw * c->N <= kChainMaxRows;
   auto eager = [&]() -> int {
-    for (int l = l0; l < l1; ++l) TRY(run_layer(c, l, hb, Bw, map, l == hq_layer ? c->hq : nullptr));
+    if (!fused) {
+      for (int l = l0; l < l1; ++l) TRY(run_layer(c, l, hb, Bw, map, l == hq_layer ? c->hq : nullptr));
+      return WAM_OK;
+    }
+    // head of l0, then per layer: attention, and the tail of l fused with the head of l + 1
+    TRY(run_chain(c, -1, l0, hb, Bw, map, l0 == hq_layer ? c->hq : nullptr));
+    for (int l = l0; l < l1; ++l) {
+      TRY(run_attention(c, Bw));
+      const int nx = l + 1 < l1 ? l + 1 : -1;
+      TRY(run_chain(c, l, nx, hb, Bw, map, nx >= 0 && nx == hq_layer ? c->hq : nullptr));
+    }
     return WAM_OK;
   };
   if (!c->graph_replay || !c->graphs_ok || c->prof_on) return eager();
-  const auto key = std::make_tuple(l0, l1, Bw, static_cast<const void*>(hb), static_cast<const void*>(map), hq_layer);
+  // the fused and unfused launch sequences of one range are different graphs
+  const auto key = std::make_tuple(l0, l1, fused ? -Bw : Bw, static_cast<const void*>(hb), static_cast<const void*>(map),
+                                   hq_layer);
   const auto hit = c->layer_graphs.find(key);
   if (hit != c->layer_graphs.end()) {
     CK(cudaGraphLaunch(hit->second, c->stream));
+    c->stats.n_kernel_launches += c->graph_kernels[hit->second];
     return WAM_OK;
   }
   if (++c->layer_graph_uses[key] < 2) return eager();
@@ -358,13 +485,14 @@ int run_layers(wam_ctx* c, int l0, int l1, float* hb, int Bw, const int* map, in
     c->graphs_ok = false;
     return eager();
   }
-  int rc = WAM_OK;
-  for (int l = l0; l < l1 && rc == WAM_OK; ++l) rc = run_layer(c, l, hb, Bw, map, l == hq_layer ? c->hq : nullptr);
+  const long long k0 = c->stats.n_kernel_launches;
+  const int rc = eager();
   const cudaError_t ec = cudaStreamEndCapture(c->stream, &g);
   cudaGraphExec_t ex = nullptr;
   if (rc == WAM_OK && ec == cudaSuccess && g != nullptr && cudaGraphInstantiate(&ex, g, 0) == cudaSuccess) {
     cudaGraphDestroy(g);
     c->layer_graphs[key] = ex;
+    c->graph_kernels[ex] = c->stats.n_kernel_launches - k0;   // counted once while capturing
     CK(cudaGraphLaunch(ex, c->stream));
     return WAM_OK;
   }
@@ -374,6 +502,188 @@ int run_layers(wam_ctx* c, int l0, int l1, float* hb, int Bw, const int* map, in
   c->err.clear();
   c->graphs_ok = false;
   return eager();
+}
+
+// Folds device RR decisions whose copies have landed (all of them when `block`) into the step log
+// and the reuse statistics (App. D.2): until then a device-decided step counts as evaluated in
+// full.
+int resolve_decisions(wam_ctx* c, bool block) {
+  const int e = c->cfg.rr_e, sq = c->cfg.rr_s;
+  while (!c->dec_batches.empty()) {
+    auto& b = c->dec_batches.front();
+    if (block) {
+      CK(cudaEventSynchronize(b.first));
+    } else {
+      const cudaError_t q = cudaEventQuery(b.first);
+      if (q == cudaErrorNotReady) {
+        cudaGetLastError();
+        break;
+      }
+      if (q != cudaSuccess) return fail_cuda(c, "RR decision copy", q);
+    }
+    for (; c->dec_resolved < b.second; ++c->dec_resolved) {
+      const RRDecision& r = c->h_dec[c->dec_resolved % kDecCap];
+      const wam_ctx::PendingDec pd = c->dec_pending.front();
+      c->dec_pending.pop_front();
+      if (r.accept) {
+        c->stats.n_reuse++;
+        c->stats.b_skip += e - sq;
+        c->stats.n_layer_evals -= e - sq;
+      }
+      if (pd.st != nullptr && pd.log_idx >= 0 && pd.log_idx < static_cast<int>(pd.st->log.size())) {
+        wam_step_record& rec = pd.st->log[pd.log_idx];
+        rec.rr_accept = r.accept;
+        for (int br = 0; br < 2; ++br) {
+          rec.alpha[br] = r.alpha[br];
+          rec.cos[br] = r.cos[br];
+          rec.fit[br] = r.fit[br];
+        }
+      }
+    }
+    cudaEventDestroy(b.first);
+    c->dec_batches.pop_front();
+  }
+  return WAM_OK;
+}
+
+// Copies the decision records of this call's device-branched steps to the host ring.
+int queue_decision_copy(wam_ctx* c) {
+  if (c->dec_queued == c->dec_copied) return WAM_OK;
+  const unsigned long long a = c->dec_copied, b = c->dec_queued;
+  const size_t sz = sizeof(RRDecision);
+  const size_t i0 = a % kDecCap, i1 = b % kDecCap;
+  if (i0 < i1 || b - a == 0) {
+    CK(cudaMemcpyAsync(c->h_dec + i0, c->d_dec + i0, sz * (i1 - i0), cudaMemcpyDeviceToHost, c->stream));
+  } else {   // wraps around the ring
+    CK(cudaMemcpyAsync(c->h_dec + i0, c->d_dec + i0, sz * (kDecCap - i0), cudaMemcpyDeviceToHost, c->stream));
+    if (i1 > 0) CK(cudaMemcpyAsync(c->h_dec, c->d_dec, sz * i1, cudaMemcpyDeviceToHost, c->stream));
+  }
+  cudaEvent_t ev;
+  CK(cudaEventCreateWithFlags(&ev, cudaEventDisableTiming));
+  CK(cudaEventRecord(ev, c->stream));
+  c->dec_batches.emplace_back(ev, b);
+  c->dec_copied = b;
+  return WAM_OK;
+}
+
+// One RR step of a single work item with the decision on the device: layers [0, s) (saving
+// h_q), the probe and gate, the decision, the middle layers under a graph conditional (rejected
+// only), the injection or refresh, layers [e, L).  Captured on the second use per state and
+// replayed.  Returns WAM_OK with *done = false when the caller should run the host-branching
+// path instead (first use, or capture not possible).
+int rr_step_device(wam_ctx* c, wam_state* st, int nch, bool* done) {
+  *done = false;
+  const int N = c->N, d = c->d, L = c->L;
+  const int q = c->cfg.rr_q, s = c->cfg.rr_s, e = c->cfg.rr_e, split = c->split;
+  const auto key = std::make_tuple(static_cast<const void*>(st->pa), static_cast<const void*>(st->ra));
+  auto hit = c->rr_graphs.find(key);
+  if (hit == c->rr_graphs.end()) {
+    if (++c->rr_graph_uses[key] < 2) return WAM_OK;
+    if (c->aux_stream == nullptr) {
+      if (cudaStreamCreateWithFlags(&c->aux_stream, cudaStreamNonBlocking) != cudaSuccess) {
+        cudaGetLastError();
+        c->dev_branch_ok = false;
+        return WAM_OK;
+      }
+    }
+    const long long k0 = c->stats.n_kernel_launches;
+    cudaGraph_t g = nullptr;
+    if (cudaStreamBeginCapture(c->stream, cudaStreamCaptureModeThreadLocal) != cudaSuccess) {
+      cudaGetLastError();
+      c->dev_branch_ok = false;
+      return WAM_OK;
+    }
+    int rc = WAM_OK;
+    bool capture_ok = true;
+    for (int l = 0; l < s && rc == WAM_OK; ++l) rc = run_layer(c, l, c->h, 1, nullptr, l == q ? c->hq : nullptr);
+    if (rc == WAM_OK) {
+      Span sp(c, WAM_KCLASS_RR_PROBE, 0.0, 12.0 * double(N) * d);
+      capture_ok = rr_probe_partial(c->h, c->hq, st->pa, c->d_items, 1, N, d, split, nch, c->d_part, c->stream) ==
+                   cudaSuccess;
+    }
+    if (rc == WAM_OK && capture_ok) {
+      Span sp(c, WAM_KCLASS_RR_PROBE);
+      capture_ok = rr_gate(c->d_part, 1, nch, int64_t(split) * d, int64_t(N - split) * d, c->cfg.rr_alpha_min,
+                           c->cfg.rr_alpha_max, c->cfg.rr_eps, c->cfg.rr_gamma_cos, c->cfg.rr_gamma_fit, c->d_gate,
+                           c->stream) == cudaSuccess;
+    }
+    cudaGraph_t cg = nullptr;
+    const cudaGraphNode_t* deps = nullptr;
+    size_t nd = 0;
+    cudaStreamCaptureStatus cs;
+    cudaGraphConditionalHandle hdl = 0;
+    if (rc == WAM_OK && capture_ok)
+      capture_ok = cudaStreamGetCaptureInfo(c->stream, &cs, nullptr, &cg, &deps, nullptr, &nd) == cudaSuccess &&
+                   cudaGraphConditionalHandleCreate(&hdl, cg, 0, 0) == cudaSuccess;
+    if (rc == WAM_OK && capture_ok) {
+      Span sp(c, WAM_KCLASS_RR_PROBE);
+      capture_ok = rr_decide(c->d_gate, split > 0, split < N, c->d_rrapply, c->d_dec, c->d_dec_n, kDecCap, hdl, 1,
+                             c->stream) == cudaSuccess;
+    }
+    cudaGraphNode_t cn = nullptr;
+    cudaGraph_t body = nullptr;
+    if (rc == WAM_OK && capture_ok) {
+      cudaGraphNodeParams cp = {};
+      cp.type = cudaGraphNodeTypeConditional;
+      cp.conditional.handle = hdl;
+      cp.conditional.type = cudaGraphCondTypeIf;
+      cp.conditional.size = 1;
+      capture_ok = cudaStreamGetCaptureInfo(c->stream, &cs, nullptr, &cg, &deps, nullptr, &nd) == cudaSuccess &&
+                   cudaGraphAddNode(&cn, cg, deps, nullptr, nd, &cp) == cudaSuccess &&
+                   cudaStreamUpdateCaptureDependencies(c->stream, &cn, nullptr, 1, cudaStreamSetCaptureDependencies) ==
+                       cudaSuccess;
+      body = capture_ok ? cp.conditional.phGraph_out[0] : nullptr;
+    }
+    if (rc == WAM_OK && capture_ok) {
+      // the rejected branch: gather the item, run the middle layers on it
+      capture_ok = cudaStreamBeginCaptureToGraph(c->aux_stream, body, nullptr, nullptr, 0,
+                                                 cudaStreamCaptureModeThreadLocal) == cudaSuccess;
+      if (capture_ok) {
+        cudaStream_t main = c->stream;
+        c->stream = c->aux_stream;
+        {
+          Span sp(c, WAM_KCLASS_RR_APPLY, 0.0, 8.0 * double(N) * d);
+          if (rr_gather(c->hm, c->h, c->d_map0, 1, int64_t(N) * d, c->stream) != cudaSuccess) capture_ok = false;
+        }
+        for (int l = s; l < e && rc == WAM_OK && capture_ok; ++l) rc = run_layer(c, l, c->hm, 1, c->d_map0, nullptr);
+        c->stream = main;
+        cudaGraph_t bo = nullptr;
+        if (cudaStreamEndCapture(c->aux_stream, &bo) != cudaSuccess) capture_ok = false;
+      }
+    }
+    if (rc == WAM_OK && capture_ok) {
+      Span sp(c, WAM_KCLASS_RR_APPLY, 0.0, 24.0 * double(N) * d);
+      capture_ok = rr_apply(c->h, c->hm, c->hq, st->pa, st->ra, c->d_items, c->d_rrapply, 1, N, d, split, c->stream) ==
+                   cudaSuccess;
+    }
+    for (int l = e; l < L && rc == WAM_OK && capture_ok; ++l) rc = run_layer(c, l, c->h, 1, nullptr, nullptr);
+    const cudaError_t ec = cudaStreamEndCapture(c->stream, &g);
+    cudaGraphExec_t ex = nullptr;
+    if (rc == WAM_OK && capture_ok && ec == cudaSuccess && g != nullptr &&
+        cudaGraphInstantiate(&ex, g, 0) == cudaSuccess) {
+      cudaGraphDestroy(g);
+      hit = c->rr_graphs.emplace(key, ex).first;
+      c->graph_kernels[ex] = c->stats.n_kernel_launches - k0;
+      c->stats.n_kernel_launches = k0;   // counted again when launched below
+    } else {
+      // nothing of the capture ran: use the host-branching path from now on
+      if (g != nullptr) cudaGraphDestroy(g);
+      cudaGetLastError();
+      c->err.clear();
+      c->stats.n_kernel_launches = k0;
+      c->dev_branch_ok = false;
+      return WAM_OK;
+    }
+  }
+  if (c->dec_queued - c->dec_resolved >= kDecCap) {
+    TRY(queue_decision_copy(c));
+    TRY(resolve_decisions(c, true));
+  }
+  CK(cudaGraphLaunch(hit->second, c->stream));
+  c->stats.n_kernel_launches += c->graph_kernels[hit->second];
+  c->dec_queued++;
+  *done = true;
+  return WAM_OK;
 }
 
 int obs_embed(wam_ctx* c, wam_state* st) {
@@ -408,6 +718,10 @@ int run_steps(wam_ctx* c, wam_state* st, const std::vector<int>& n) {
   TRY(obs_embed(c, st));
   int max_n = 0;
   for (int b = 0; b < B; ++b) max_n = std::max(max_n, n[b]);
+  // decisions of earlier calls whose copies have landed; the rest lose their log entry
+  TRY(resolve_decisions(c, false));
+  for (auto& pd : c->dec_pending)
+    if (pd.st == st) pd.log_idx = -1;
   st->log.clear();
   std::vector<StepItem> items, uitems;
   std::vector<int> uidx;
@@ -492,7 +806,15 @@ int run_steps(wam_ctx* c, wam_state* st, const std::vector<int>& n) {
       }
     }
     std::vector<int> accepted(Bw, 0);
-    if (!any_rr) {
+    bool dev_step = false;   // this step's RR decision is taken on the device (work item 0)
+    if (any_rr && Bw == 1 && gate_ok[0] && c->dev_branch && c->dev_branch_ok && c->graph_replay && c->graphs_ok &&
+        !c->prof_on) {
+      const int nch = rr_num_chunks(int64_t(std::max(split_row, N - split_row)) * d);
+      TRY(rr_step_device(c, st, nch, &dev_step));
+    }
+    if (dev_step) {
+      // layers, gate, middle layers or injection and the tail all ran in the step's graph
+    } else if (!any_rr) {
       TRY(run_layers(c, 0, L, c->h, Bw, nullptr, -1));
     } else {
       TRY(run_layers(c, 0, s, c->h, Bw, nullptr, q));
@@ -572,6 +894,7 @@ int run_steps(wam_ctx* c, wam_state* st, const std::vector<int>& n) {
           rec.fit[br] = static_cast<float>(gates[2 * w + br].fit);
         }
       }
+      if (dev_step) c->dec_pending.push_back(wam_ctx::PendingDec{st, static_cast<int>(st->log.size())});
       st->log.push_back(rec);
       c->stats.n_episode_steps++;
       c->stats.n_layer_evals += accepted[w] ? (L - (e - s)) : L;
@@ -590,7 +913,7 @@ int run_steps(wam_ctx* c, wam_state* st, const std::vector<int>& n) {
       if (m.stage == c->K) m.finished = 1;
     }
   }
-  return WAM_OK;
+  return queue_decision_copy(c);
 }
 
 int copy_out(wam_ctx* c, wam_state* st, float* actions_out, float* video_out, bool& host_out) {
@@ -825,6 +1148,12 @@ int create_impl(wam_ctx* c, const wam_config* cfg, const float* weights, size_t 
   TRY(dalloc(c, c->allocs, &c->d_fconst, size_t(c->Bmax) * 64));
   TRY(dalloc(c, c->allocs, &c->d_err, 1));
   CK(cudaMemset(c->d_err, 0, sizeof(int)));
+  TRY(dalloc(c, c->allocs, &c->d_map0, 1));
+  CK(cudaMemset(c->d_map0, 0, sizeof(int)));
+  TRY(dalloc(c, c->allocs, &c->d_dec, kDecCap));
+  TRY(dalloc(c, c->allocs, &c->d_dec_n, 1));
+  CK(cudaMemset(c->d_dec_n, 0, sizeof(unsigned long long)));
+  CK(cudaHostAlloc(reinterpret_cast<void**>(&c->h_dec), sizeof(RRDecision) * kDecCap, cudaHostAllocDefault));
   // scratch for the float64 partial sums of TR / OR / RR reductions
   const int split = c->split;
   const size_t p_tr = size_t(c->Bmax) * 2 * tr_num_chunks(c->T, c->V);
@@ -838,16 +1167,21 @@ int create_impl(wam_ctx* c, const wam_config* cfg, const float* weights, size_t 
     TRY(encode(c, &c->tm_u, c->u, rows, c->dff));
     TRY(encode(c, &c->tm_obs_lp, c->obs_lp, size_t(c->Bmax) * c->No, c->d));
     TRY(encode(c, &c->tm_obs_w, c->obs_wt, c->d, c->d));
-    c->tc_attn = c->d / c->H == 64;
+    c->tc_attn = c->d / c->H == 64 || c->d / c->H == 72;
     if (c->tc_attn) {
       c->vt_ld = attention_tc_vt_ld(c->N);
       uint8_t* vt = nullptr;
       TRY(dalloc(c, c->allocs, &vt, size_t(c->Bmax) * c->d * c->vt_ld * 2));
       CK(cudaMemsetAsync(vt, 0, size_t(c->Bmax) * c->d * c->vt_ld * 2, c->stream));
       c->vt = vt;
-      if (tc_encode_bf16_box(&c->tm_qk, c->qkv, rows, 3 * c->d, 3 * c->d, 64, 128) != 0 ||
-          tc_encode_bf16_box(&c->tm_vt, c->vt, size_t(c->Bmax) * c->d, c->vt_ld, c->vt_ld, 64, 64) != 0)
+      if (attention_tc_encode(&c->attn_maps, c->qkv, c->vt, c->Bmax, c->N, c->d, c->H, c->vt_ld) != 0)
         return fail(c, WAM_ERR_CUDA, "cuTensorMapEncodeTiled failed for the attention operands");
+    }
+    c->chain_ok = c->tc_attn && dit_chain_supported(c->d, c->dff) && c->d % 128 == 0;
+    if (c->chain_ok) {
+      const int nctr = dit_chain_counters(static_cast<int>(rows));
+      TRY(dalloc(c, c->allocs, &c->d_chain_ctr, nctr));
+      CK(cudaMemsetAsync(c->d_chain_ctr, 0, sizeof(int) * nctr, c->stream));
     }
     for (LayerW& w : c->layers) {
       TRY(encode(c, &w.tm_qkv, w.qkv_wt, 3 * c->d, c->d));
@@ -870,6 +1204,12 @@ void destroy_impl(wam_ctx* c) {
   if (!c->allocs.empty()) cudaStreamSynchronize(c->stream);
   for (auto& kv : c->layer_graphs) cudaGraphExecDestroy(kv.second);
   c->layer_graphs.clear();
+  for (auto& kv : c->rr_graphs) cudaGraphExecDestroy(kv.second);
+  c->rr_graphs.clear();
+  for (auto& b : c->dec_batches) cudaEventDestroy(b.first);
+  c->dec_batches.clear();
+  if (c->aux_stream) cudaStreamDestroy(c->aux_stream);
+  if (c->h_dec) cudaFreeHost(c->h_dec);
   for (void* p : c->allocs) cudaFree(p);
   c->allocs.clear();
   if (c->ring) {
@@ -998,7 +1338,22 @@ int wam_state_create(wam_ctx* c, int32_t batch, wam_state** out) try {
 
 void wam_state_destroy(wam_state* st) {
   if (st == nullptr) return;
-  if (st->ctx) cudaStreamSynchronize(st->ctx->stream);
+  if (st->ctx) {
+    cudaStreamSynchronize(st->ctx->stream);
+    resolve_decisions(st->ctx, true);
+    for (auto& pd : st->ctx->dec_pending)
+      if (pd.st == st) pd.st = nullptr;
+    // graphs that embed this state's buffers
+    for (auto it = st->ctx->rr_graphs.begin(); it != st->ctx->rr_graphs.end();) {
+      if (std::get<0>(it->first) == st->pa) {
+        cudaGraphExecDestroy(it->second);
+        st->ctx->rr_graph_uses.erase(it->first);
+        it = st->ctx->rr_graphs.erase(it);
+      } else {
+        ++it;
+      }
+    }
+  }
   for (void* p : st->allocs) cudaFree(p);
   delete st;
 }
@@ -1219,18 +1574,23 @@ int wam_sample_cold(wam_ctx* c, wam_state* st, const float* obs, const float* no
 
 int wam_get_stats(wam_ctx* c, wam_stats* out) {
   if (c == nullptr || out == nullptr) return WAM_ERR_INVALID_ARG;
+  TRY(resolve_decisions(c, true));
   *out = c->stats;
   return WAM_OK;
 }
 
 int wam_reset_stats(wam_ctx* c) {
   if (c == nullptr) return WAM_ERR_INVALID_ARG;
+  // decisions of steps already run belong to the counts being cleared
+  TRY(queue_decision_copy(c));
+  TRY(resolve_decisions(c, true));
   std::memset(&c->stats, 0, sizeof(c->stats));
   return WAM_OK;
 }
 
 int wam_state_log(const wam_state* st, wam_step_record* out, int32_t capacity, int32_t* n_out) {
   if (st == nullptr || n_out == nullptr || (capacity > 0 && out == nullptr)) return WAM_ERR_INVALID_ARG;
+  if (st->ctx != nullptr) TRY(resolve_decisions(st->ctx, true));
   const int n = std::min<int>(capacity, static_cast<int>(st->log.size()));
   if (n > 0) std::memcpy(out, st->log.data(), sizeof(wam_step_record) * n);
   *n_out = static_cast<int32_t>(st->log.size());
@@ -1510,6 +1870,18 @@ int wam_set_graph_replay(wam_ctx* c, int32_t enable) {
   return WAM_OK;
 }
 
+int wam_set_device_branching(wam_ctx* c, int32_t enable) {
+  if (c == nullptr) return WAM_ERR_INVALID_ARG;
+  c->dev_branch = enable != 0;
+  return WAM_OK;
+}
+
+int wam_set_layer_fusion(wam_ctx* c, int32_t enable) {
+  if (c == nullptr) return WAM_ERR_INVALID_ARG;
+  c->layer_fusion = enable != 0;
+  return WAM_OK;
+}
+
 int wam_gemm_tile_width(const wam_ctx* c, int32_t M, int32_t N, int32_t K, int32_t epilogue) {
   if (c == nullptr || M < 0 || N <= 0 || K <= 0) return WAM_ERR_INVALID_ARG;
   if (!c->bf16) return WAM_ERR_UNSUPPORTED;
@@ -1523,9 +1895,28 @@ int wam_profile_enable(wam_ctx* c, int32_t enable) try {
   c->spans.clear();
   c->evnext = 0;
   c->prof_on = enable != 0;
+  if (c->prof_on && c->chain_ok && c->d_trace == nullptr) {
+    constexpr int kTraceRecords = 1 << 18;   // 16 MB of task records
+    TRY(dalloc(c, c->allocs, &c->d_trace, kTraceRecords));
+    c->trace_cap = kTraceRecords;
+  }
+  if (c->d_trace != nullptr) CK(cudaMemsetAsync(c->d_trace, 0, sizeof(wam_chain_task) * c->trace_cap, c->stream));
+  c->trace_used = 0;
+  c->trace_launches = 0;
   return WAM_OK;
 } catch (const std::bad_alloc&) {
   return fail(c, WAM_ERR_OOM, "host allocation failed");
+} catch (...) {
+  return fail(c, WAM_ERR_CUDA, "unexpected host exception");
+}
+
+int wam_profile_chain_trace(wam_ctx* c, wam_chain_task* out, int32_t capacity, int32_t* n_out) try {
+  if (c == nullptr || n_out == nullptr || (out == nullptr && capacity > 0) || capacity < 0) return WAM_ERR_INVALID_ARG;
+  CK(cudaStreamSynchronize(c->stream));
+  const int n = std::min(capacity, c->trace_used);
+  if (n > 0) CK(cudaMemcpy(out, c->d_trace, sizeof(wam_chain_task) * n, cudaMemcpyDeviceToHost));
+  *n_out = capacity == 0 ? c->trace_used : n;
+  return WAM_OK;
 } catch (...) {
   return fail(c, WAM_ERR_CUDA, "unexpected host exception");
 }

@@ -132,6 +132,9 @@ def lib() -> ctypes.CDLL:
         "wam_op_gemm_workspace_bytes": (ctypes.c_size_t, []),
         "wam_gemm_tile_width": (ctypes.c_int, [_vp, _i32, _i32, _i32, _i32]),
         "wam_set_graph_replay": (ctypes.c_int, [_vp, _i32]),
+        "wam_set_layer_fusion": (ctypes.c_int, [_vp, _i32]),
+        "wam_set_device_branching": (ctypes.c_int, [_vp, _i32]),
+        "wam_profile_chain_trace": (ctypes.c_int, [_vp, _vp, _i32, ctypes.POINTER(_i32)]),
         "wam_diag_similarity": (ctypes.c_int, [_vp, _vp, _vp, ctypes.c_int64, _vp, _vp]),
         "wam_diag_action_rmse": (ctypes.c_int, [_vp, _vp, _vp, _i32, _i32, _i32, _vp]),
         "wam_diag_layer_deltas": (ctypes.c_int, [_vp, _vp, _i32, _vp]),
@@ -332,6 +335,15 @@ class Context:
         """CUDA-graph replay of the layer stack (default on); off launches every kernel."""
         self._check(lib().wam_set_graph_replay(self.handle, 1 if enable else 0))
 
+    def set_device_branching(self, enable: bool):
+        """RR decision of a single work item taken on the device inside the step's CUDA graph
+        (default on); off reads the gate statistics back to the host every step."""
+        self._check(lib().wam_set_device_branching(self.handle, 1 if enable else 0))
+
+    def set_layer_fusion(self, enable: bool):
+        """Fused row-chain launches between attentions (default on); off launches each kernel."""
+        self._check(lib().wam_set_layer_fusion(self.handle, 1 if enable else 0))
+
     def gemm_tile_width(self, M: int, N: int, K: int, epilogue: int) -> int:
         """Output tile width the context uses for this GEMM shape (chosen from the shape alone)."""
         r = lib().wam_gemm_tile_width(self.handle, M, N, K, epilogue)
@@ -376,6 +388,17 @@ class Context:
 
     def profile_enable(self, on: bool = True):
         self._check(lib().wam_profile_enable(self.handle, 1 if on else 0))
+
+    def profile_chain_trace(self) -> np.ndarray:
+        """Per-task records of the fused row-chain launches since profiling was enabled: a numpy
+        structured array (launch, cta, kind, m, j, t_take, t_dep, t_epi0, t_epi1; times in ns)."""
+        n = _i32()
+        self._check(lib().wam_profile_chain_trace(self.handle, None, 0, ctypes.byref(n)))
+        dt = np.dtype([("launch", "<i4"), ("cta", "<i4"), ("kind", "<i4"), ("m", "<i4"), ("j", "<i4"),
+                       ("pad", "<i4"), ("t_take", "<u8"), ("t_dep", "<u8"), ("t_epi0", "<u8"), ("t_epi1", "<u8")])
+        out = np.zeros(max(1, n.value), dtype=dt)
+        self._check(lib().wam_profile_chain_trace(self.handle, out.ctypes.data, n.value, ctypes.byref(n)))
+        return out[: n.value]
 
     def profile_read(self) -> dict:
         arr = (KClassTiming * len(KCLASSES))()

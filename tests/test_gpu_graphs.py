@@ -55,3 +55,55 @@ def test_graph_replay_is_bit_identical(wamlib, precision, relax):
     assert sa["n_reuse"] == sb["n_reuse"]
     if relax:
         assert sa["n_reuse"] > 0   # the injection path (middle layers skipped) ran
+
+
+def _closed_loop_b1(cfg, device_branching, rounds=4):
+    """Batch-1 closed loop: cold sample, then TR + one prefix step + OR + the rest, repeated."""
+    Wd = I.make_weights(cfg)
+    ctx = W.Context(cfg, I.flatten_weights(Wd))
+    ctx.set_device_branching(device_branching)
+    K, b0 = cfg["n_steps"], int(cfg["tr_entry_stage"])
+    st = ctx.state(1)
+    proc = I.ObsProcess(cfg, 1, seed=4)
+    ctx.sample_cold(st, proc.obs.copy(), I.make_noise(cfg, 1), K)
+    outs, logs = [], []
+    for r in range(rounds):
+        pred, real = proc.predicted(), proc.step()
+        s1 = ctx.adapt(st, pred, shift=int(cfg["shift"]), fresh_noise=I.make_fresh_eps(cfg, 1, r))[0]
+        if s1 == W.ADAPT_TR_INIT:
+            ctx.continue_(st, 1)
+            logs += ctx.log(st)
+        ctx.adapt(st, real)
+        act = np.zeros((1, cfg["n_action"], cfg["action_dim"]), np.float32)
+        ctx.continue_(st, K - int(ctx.read(st, W.FIELD_META)[0][0]), act)
+        logs += ctx.log(st)
+        outs += [ctx.read(st, W.FIELD_X).copy(), act, ctx.read(st, W.FIELD_RR_P).copy()]
+    stats = ctx.stats()
+    ctx.close()
+    return outs, logs, stats
+
+
+@pytest.mark.parametrize("precision", ["fp32", "bf16"])
+@pytest.mark.parametrize("gate", ["relaxed", "strict", "default"])
+def test_device_branching_matches_host_branching(wamlib, precision, gate):
+    """The RR decision taken on the device inside the step's graph (conditional middle layers)
+    gives the same latents, actions, layer state, step log and reuse statistics as the host
+    decision, on the accept path (relaxed gate), the reject path (strict gate) and a mix."""
+    over = {"relaxed": dict(rr_gamma_cos=-1.0, rr_gamma_fit=1e30),
+            "strict": dict(rr_gamma_cos=0.99999, rr_gamma_fit=1e-6), "default": {}}[gate]
+    if precision == "bf16":
+        cfg = I.get_config("tiny", **SMALL_BF16, **over)
+    else:
+        cfg = I.get_config("tiny_rr", **over)
+    a, la, sa = _closed_loop_b1(cfg, True)
+    b, lb, sb = _closed_loop_b1(cfg, False)
+    for x, y in zip(a, b):
+        assert np.array_equal(x, y)
+    assert la == lb
+    for k in ("n_reuse", "n_attempt", "b_skip", "b_dense", "n_layer_evals", "n_bind"):
+        assert sa[k] == sb[k], k
+    if gate == "relaxed":
+        assert sa["n_reuse"] == sa["n_attempt"] > 0
+    if gate == "strict":
+        assert sa["n_reuse"] == 0 and sa["n_attempt"] > 0
+    assert sa["n_kernel_launches"] > 0

@@ -74,8 +74,8 @@ def test_gemm_tcgen05_matches_reference(wamlib, M, N, K, epi):
 
 # (M, N, K, tile width, K ranges): every kernel variant the planner can choose, incl. K splits.
 PLAN_CASES = [
-    (1392, 768, 3072, 128, 2),   # MLP down-projection of the 12-block d768 model, one episode
-    (1392, 768, 768, 128, 2),    # its attention out-projection
+    (1392, 768, 3072, 128, 2),   # MLP down-projection widths of the 12-block d768 model (ragged M)
+    (1392, 768, 768, 128, 2),    # its attention out-projection widths
     (1392, 768, 3072, 64, 1),
     (300, 768, 3072, 64, 4),
     (129, 256, 192, 128, 3),     # K = 192: one-atom stages, three ranges, ragged M
@@ -213,16 +213,18 @@ def test_ln_modulate_matches_oracle(wamlib, prec, d):
     assert np.max(np.abs(_f64(out) - ref)) <= tol * np.max(np.abs(ref))
 
 
-TC_ATTN_CASES = [(1, 1, 2), (1, 56, 2), (2, 128, 2), (1, 129, 4), (1, 1296, 12), (2, 300, 2), (1, 2464, 4),
-                 (2, 2464, 16), (8, 600, 8), (20, 130, 8)]
+TC_ATTN_CASES = [(1, 1, 2, 64), (1, 56, 2, 64), (2, 128, 2, 64), (1, 129, 4, 64), (1, 1296, 12, 64),
+                 (2, 300, 2, 64), (1, 2464, 4, 64), (2, 2464, 16, 64), (8, 600, 8, 64), (20, 130, 8, 64),
+                 # head dim 72 (the bimanual model: 16 heads, d 1152), ragged and multi-item
+                 (1, 1, 16, 72), (1, 200, 16, 72), (2, 130, 16, 72), (1, 4914, 16, 72), (3, 600, 16, 72)]
 
 
-@pytest.mark.parametrize("B,N,H", TC_ATTN_CASES)
-def test_attention_tcgen05_matches_oracle(wamlib, B, N, H):
+@pytest.mark.parametrize("B,N,H,dh", TC_ATTN_CASES)
+def test_attention_tcgen05_matches_oracle(wamlib, B, N, H, dh):
     """QKV projection writing V^T, then the tcgen05 attention, against the oracle's attention of
     the same bf16 q, k, v."""
-    rng = np.random.default_rng(B * 100 + N + H)
-    d = 64 * H
+    rng = np.random.default_rng(B * 100 + N + H + dh)
+    d = dh * H
     dev = torch.device("cuda")
     x = _bf16(rng.standard_normal((B * N, d)))
     Wt = _bf16(rng.standard_normal((3 * d, d)) / np.sqrt(d))
@@ -237,7 +239,7 @@ def test_attention_tcgen05_matches_oracle(wamlib, B, N, H):
     proj = torch.from_numpy(_f64(x) @ _f64(Wt).T + bias.double().numpy())
     qk = _f64(qkv)[:, :2 * d]
     assert np.max(np.abs(qk - proj.numpy()[:, :2 * d])) <= 2e-2 * np.max(np.abs(proj.numpy()))
-    v_from_vt = _f64(vt).reshape(B, H, 64, vt_ld)[..., :N].transpose(0, 3, 1, 2).reshape(B * N, d)
+    v_from_vt = _f64(vt).reshape(B, H, dh, vt_ld)[..., :N].transpose(0, 3, 1, 2).reshape(B * N, d)
     assert np.max(np.abs(v_from_vt - proj.numpy()[:, 2 * d:])) <= 2e-2 * np.max(np.abs(proj.numpy()))
     got = _f64(out)
     for b in range(B):
