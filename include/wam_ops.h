@@ -44,6 +44,11 @@ int wam_op_gemm_bf16(const void* A, const void* Wt, const float* bias, void* C, 
  *              order, so results do not depend on timing.  Needs: the K stages (K / 128 for
  *              64- / 128-wide tiles when K % 128 == 0, else K / 64) divisible by k_splits, and all
  *              tiles x k_splits units in one wave (at most the SM count).
+ *   cluster    0 = the library's rule, 1 = single CTAs, 2 = clusters of two CTAs on adjacent
+ *              column tiles of the same row block, each loading half of the shared A tile with
+ *              TMA multicast into both (64- / 128-wide tiles, an even number of column tiles,
+ *              K % 128 == 0, no K split; otherwise single CTAs).  The accumulation order is the
+ *              same either way.
  *   workspace  device buffer of wam_op_gemm_workspace_bytes() bytes, 16-byte aligned, zero-filled
  *              before its first use (every call leaves it reusable); NULL = no splitting.  Calls
  *              sharing a workspace must be ordered (same stream).
@@ -52,7 +57,8 @@ int wam_op_gemm_bf16(const void* A, const void* Wt, const float* bias, void* C, 
 int wam_op_gemm_bf16_plan(const void* A, const void* Wt, const float* bias, void* C, int32_t M,
                           int32_t N, int32_t K, int32_t epilogue, const float* gate,
                           int64_t gate_stride, int32_t rows_per_item, int32_t tile_n,
-                          int32_t k_splits, void* workspace, size_t workspace_bytes, void* stream);
+                          int32_t k_splits, int32_t cluster, void* workspace, size_t workspace_bytes,
+                          void* stream);
 
 /* Bytes of the split-K workspace of wam_op_gemm_bf16_plan on the current device. */
 size_t wam_op_gemm_workspace_bytes(void);

@@ -195,6 +195,7 @@ int tc_encode_gemm_operand(GemmOperand* op, const void* base, uint64_t rows, uin
 struct GemmPlan {
   int bn;
   int splits;
+  int mc = 0;   // CTAs per cluster sharing the A tile by multicast: 1 or 2; 0 = by the shape rule
 };
 // Device scratch of split-K: fp32 partial tiles, then one int ticket counter per output tile.
 // The counters must be zero before the first use; every GEMM leaves them zero.

@@ -15,6 +15,12 @@
 // The accumulator is double buffered in TMEM (2 x BN columns) so the epilogue of one tile
 // overlaps the main loop of the next.
 //
+// Clusters of two (MC = 2, no K split; explicit plans only): the two CTAs of a cluster take the
+// same 128-row block and adjacent column tiles, so they read the same A tile.  Each loads one
+// 64-row half of it with TMA multicast into both CTAs' shared memory (the L2 serves A once per
+// pair); a stage is refilled only after both CTAs' MMAs consumed it (their commits arrive on both
+// CTAs' empty barriers).
+//
 // K split: a projection with too few output tiles to fill the GPU is cut into `splits` work units
 // per tile, each over a contiguous range of K.  A unit's epilogue stores its fp32 partial tile to
 // a workspace and takes a ticket from the tile's counter; the unit that takes the last ticket
@@ -34,6 +40,32 @@
 
 namespace wam {
 namespace {
+
+// ---- cluster helpers ----
+WAM_DEV uint32_t cluster_rank() {
+  uint32_t r;
+  asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+  return r;
+}
+WAM_DEV void cluster_sync() {
+  asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::: "memory");
+}
+// 2-D TMA load delivered to the same shared-memory offset (and mbarrier offset) of every CTA in
+// cta_mask.
+WAM_DEV void tma_load_2d_mc(uint32_t dst, const CUtensorMap* map, int x, int y, uint32_t bar, uint16_t cta_mask) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes.multicast::cluster"
+      " [%0], [%1, {%2, %3}], [%4], %5;" ::"r"(dst),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(bar), "h"(cta_mask)
+      : "memory");
+}
+// Arrive on the mbarrier at this offset in every CTA of cta_mask once this thread's MMAs completed.
+WAM_DEV void umma_commit_mc(uint32_t bar, uint16_t cta_mask) {
+  asm volatile(
+      "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64 [%0], %1;" ::"r"(bar),
+      "h"(cta_mask)
+      : "memory");
+}
 
 constexpr int kBM = 128;
 constexpr int kBK = 64;           // 64 bf16 = 128 bytes = one swizzle row
@@ -64,11 +96,12 @@ struct SplitArgs {
   int* counters;    // [tiles] tickets, zero between launches
 };
 
-template <int BN, int EPI, int KA>
+template <int BN, int EPI, int KA, int MC>
 __global__ void __launch_bounds__(kThreads, 1)
     gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                    int M, int N, int K, EpiArgs e, SplitArgs sp, int* dev_err) {
   using C = TileCfg<BN, KA>;
+  static_assert(MC == 1 || MC == 2, "cluster size");
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint8_t* tiles = smem;
@@ -90,12 +123,32 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int num_n = N / BN;
   const int num_mn = num_m * num_n;
   const int splits = sp.splits;
-  const int num_units = num_mn * splits;
   const int num_k = K / (kBK * KA) / splits;   // stages per work unit
+  // With clusters a unit is a pair of adjacent column tiles of one row block, one per CTA; the
+  // cluster walks the units (first = cluster index, stride = clusters), both CTAs in lockstep.
+  const int rank = MC == 2 ? static_cast<int>(cluster_rank()) : 0;
+  const int num_units = MC == 2 ? num_mn / 2 : num_mn * splits;
+  const int unit0 = MC == 2 ? static_cast<int>(blockIdx.x) / 2 : static_cast<int>(blockIdx.x);
+  const int unit_stride = MC == 2 ? static_cast<int>(gridDim.x) / 2 : static_cast<int>(gridDim.x);
   // unit u: output tile mn = u % num_mn (m fastest), K range u / num_mn
-  auto unit_mt = [&](int u) { return (u % num_mn) % num_m; };
-  auto unit_nt = [&](int u) { return (u % num_mn) / num_m; };
-  auto unit_kb0 = [&](int u) { return (u / num_mn) * num_k; };
+  auto unit_mt = [&](int u) { return MC == 2 ? u % num_m : (u % num_mn) % num_m; };
+  auto unit_nt = [&](int u) { return MC == 2 ? 2 * (u / num_m) + rank : (u % num_mn) / num_m; };
+  auto unit_kb0 = [&](int u) { return MC == 2 ? 0 : (u / num_mn) * num_k; };
+  // A tile of a stage: one request per operand (MC = 1), or this CTA's 64-row half of each K-atom
+  // multicast to both CTAs (the other half arrives from the peer)
+  auto load_a = [&](uint32_t dst, const CUtensorMap* map, int row, int atom, uint32_t bar) {
+    if constexpr (MC == 1) {
+      if constexpr (KA == 1)
+        tma_load_2d(dst, map, atom * kBK, row, bar);
+      else
+        tma_load_3d(dst, map, 0, row, atom, bar);
+    } else {
+#pragma unroll
+      for (int a = 0; a < KA; ++a)
+        tma_load_2d_mc(dst + a * kTileBytesA + rank * (kTileBytesA / 2), map, (atom + a) * kBK, row + rank * 64, bar,
+                       0x3);
+    }
+  };
   // K-atoms [atom, atom + KA) of rows [row, row + box): one 2-D box {64, rows} for one atom, one
   // 3-D box {64, rows, 2} for two
   auto load_k = [&](uint32_t dst, const CUtensorMap* map, int row, int atom, uint32_t bar) {
@@ -108,7 +161,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   if (threadIdx.x == 0) {
     for (int s = 0; s < C::kStages; ++s) {
       mbar_init(smem_u32(&full[s]), 1);
-      mbar_init(smem_u32(&empty[s]), 1);
+      mbar_init(smem_u32(&empty[s]), MC);   // with clusters: both CTAs' MMAs release the stage
     }
     for (int a = 0; a < 2; ++a) {
       mbar_init(smem_u32(&tfull[a]), 1);
@@ -130,6 +183,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   }
   tc_fence_before();
   __syncthreads();
+  if constexpr (MC == 2) cluster_sync();   // the peer's barriers exist before any multicast
   tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
   pdl_launch_dependents();
@@ -140,7 +194,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmB)) : "memory");
     // The weight operand does not depend on earlier kernels: its first stages are requested
     // before waiting for them, overlapping the previous kernel's tail.
-    const int u0 = blockIdx.x;
+    const int u0 = unit0;
     const int pre = u0 < num_units ? (num_k < C::kStages ? num_k : C::kStages) : 0;
     for (int s = 0; s < pre; ++s) {
       const uint32_t fb = smem_u32(&full[s]);
@@ -158,7 +212,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     for (int s = 0; s < C::kStages; ++s) issued[s] = 0, issued_phase[s] = 0;
     bool ok = true;
     bool first = true;
-    for (int unit = blockIdx.x; ok && unit < num_units; unit += gridDim.x) {
+    for (int unit = unit0; ok && unit < num_units; unit += unit_stride) {
       const int mt = unit_mt(unit);
       const int nt = unit_nt(unit);
       const int kb0 = unit_kb0(unit);
@@ -176,7 +230,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           for (int h = 0; h < BN / C::kBoxB; ++h)
             load_k(b_dst + h * C::kBoxBytesB, &tmB, nt * BN + h * C::kBoxB, (kb0 + kb) * KA, fb);
         }
-        load_k(a_dst, &tmA, mt * kBM, (kb0 + kb) * KA, fb);
+        load_a(a_dst, &tmA, mt * kBM, (kb0 + kb) * KA, fb);
         issued[stage] = 1;
         issued_phase[stage] = phase;
         if (++stage == C::kStages) {
@@ -205,7 +259,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     int it = 0;
     bool ok = true;
     bool issued_any = false;
-    for (int unit = blockIdx.x; ok && unit < num_units; unit += gridDim.x, ++it) {
+    for (int unit = unit0; ok && unit < num_units; unit += unit_stride, ++it) {
       const int acc = it & 1;
       const uint32_t acc_phase = (it >> 1) & 1;
       if (!mbar_wait(smem_u32(&tempty[acc]), acc_phase ^ 1u, abort_flag, dev_err)) {
@@ -236,7 +290,10 @@ __global__ void __launch_bounds__(kThreads, 1)
           }
         }
         issued_any = true;
-        umma_commit(smem_u32(&empty[stage]));
+        if constexpr (MC == 2)
+          umma_commit_mc(smem_u32(&empty[stage]), 0x3);
+        else
+          umma_commit(smem_u32(&empty[stage]));
         if (++stage == C::kStages) {
           stage = 0;
           phase ^= 1u;
@@ -267,7 +324,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       return r;
     };
     const int r_local = quarter * 32 + lane;   // tile row of this thread
-    for (int unit = blockIdx.x; unit < num_units; unit += gridDim.x, ++it) {
+    for (int unit = unit0; unit < num_units; unit += unit_stride, ++it) {
       const int acc = it & 1;
       const uint32_t acc_phase = (it >> 1) & 1;
       // One lane waits; the warp then proceeds together (tcgen05.ld is warp-collective).
@@ -360,6 +417,8 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   tc_fence_before();
   __syncthreads();
+  // no CTA of a cluster leaves while its peer may still multicast into it or arrive on its barriers
+  if constexpr (MC == 2) cluster_sync();
   if (warp == 1) {
     __syncwarp();
     tc_fence_after();
@@ -383,28 +442,49 @@ PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
   return fn;
 }
 
-template <int BN, int EPI, int KA>
+template <int BN, int EPI, int KA, int MC>
 cudaError_t launch(const CUtensorMap& ta, const CUtensorMap& tb, int M, int N, int K,
                    const EpiArgs& e, const SplitArgs& sp, int num_sms, int* dev_err, cudaStream_t s) {
   using C = TileCfg<BN, KA>;
   static PerDeviceSmem smem_rec;  // contexts may run on several host threads and devices
-  const cudaError_t err = ensure_max_smem(smem_rec, gemm_tc_kernel<BN, EPI, KA>, C::kSmemBytes);
+  const cudaError_t err = ensure_max_smem(smem_rec, gemm_tc_kernel<BN, EPI, KA, MC>, C::kSmemBytes);
   if (err != cudaSuccess) return err;
   const int units = ((M + kBM - 1) / kBM) * (N / BN) * sp.splits;
-  const int grid = units < num_sms ? units : num_sms;
-  return launch_pdl(gemm_tc_kernel<BN, EPI, KA>, dim3(grid), dim3(kThreads), C::kSmemBytes, s, ta, tb, M, N,
-                    K, e, sp, dev_err);
+  if constexpr (MC == 1) {
+    const int grid = units < num_sms ? units : num_sms;
+    return launch_pdl(gemm_tc_kernel<BN, EPI, KA, 1>, dim3(grid), dim3(kThreads), C::kSmemBytes, s, ta, tb, M, N,
+                      K, e, sp, dev_err);
+  } else {
+    // one cluster of two CTAs per pair of column tiles, at most one CTA per SM
+    const int pairs = units / 2;
+    const int grid = 2 * (pairs < num_sms / 2 ? pairs : num_sms / 2);
+    cudaLaunchAttribute attr[2];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    attr[1].id = cudaLaunchAttributeClusterDimension;
+    attr[1].val.clusterDim.x = 2;
+    attr[1].val.clusterDim.y = 1;
+    attr[1].val.clusterDim.z = 1;
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(grid);
+    cfg.blockDim = dim3(kThreads);
+    cfg.dynamicSmemBytes = C::kSmemBytes;
+    cfg.stream = s;
+    cfg.attrs = attr;
+    cfg.numAttrs = 2;
+    return cudaLaunchKernelEx(&cfg, gemm_tc_kernel<BN, EPI, KA, 2>, ta, tb, M, N, K, e, sp, dev_err);
+  }
 }
 
-template <int BN, int KA>
+template <int BN, int KA, int MC>
 cudaError_t dispatch_epi(const CUtensorMap& ta, const CUtensorMap& tb, int M, int N, int K, int epi,
                          const EpiArgs& e, const SplitArgs& sp, int num_sms, int* dev_err, cudaStream_t s) {
   switch (epi) {
-    case kEpiBf16: return launch<BN, kEpiBf16, KA>(ta, tb, M, N, K, e, sp, num_sms, dev_err, s);
-    case kEpiGeluBf16: return launch<BN, kEpiGeluBf16, KA>(ta, tb, M, N, K, e, sp, num_sms, dev_err, s);
-    case kEpiResidF32: return launch<BN, kEpiResidF32, KA>(ta, tb, M, N, K, e, sp, num_sms, dev_err, s);
-    case kEpiF32: return launch<BN, kEpiF32, KA>(ta, tb, M, N, K, e, sp, num_sms, dev_err, s);
-    case kEpiQkvVt: return launch<BN, kEpiQkvVt, KA>(ta, tb, M, N, K, e, sp, num_sms, dev_err, s);
+    case kEpiBf16: return launch<BN, kEpiBf16, KA, MC>(ta, tb, M, N, K, e, sp, num_sms, dev_err, s);
+    case kEpiGeluBf16: return launch<BN, kEpiGeluBf16, KA, MC>(ta, tb, M, N, K, e, sp, num_sms, dev_err, s);
+    case kEpiResidF32: return launch<BN, kEpiResidF32, KA, MC>(ta, tb, M, N, K, e, sp, num_sms, dev_err, s);
+    case kEpiF32: return launch<BN, kEpiF32, KA, MC>(ta, tb, M, N, K, e, sp, num_sms, dev_err, s);
+    case kEpiQkvVt: return launch<BN, kEpiQkvVt, KA, MC>(ta, tb, M, N, K, e, sp, num_sms, dev_err, s);
     default: return cudaErrorInvalidValue;
   }
 }
@@ -463,14 +543,21 @@ size_t tc_gemm_workspace_bytes(int num_sms) {
 // ones cannot fill the SMs (more CTAs in flight hide the operand latency), 256-wide tiles win once
 // they fill four waves (fewest operand bytes per flop), 128-wide tiles in between.  K splitting
 // changes the summation order, so it is only used when asked for.
+// Clusters are not chosen by the rule: measured on the three models' projections at 1 to 32
+// episodes, the pair never beat the best single-CTA plan (at one episode the main loop is bound by
+// the latency of the operand round trip, not by the bytes the L2 delivers; at large M the 256-wide
+// single tiles move fewer bytes than 128-wide pairs).  They stay available through explicit plans.
 GemmPlan tc_gemm_plan(int M, int N, int K, bool has64, bool can_split, int num_sms) {
-  (void)K;
   (void)can_split;
+  (void)K;
   const long m_tiles = (M + kBM - 1) / kBM;
   const long tiles128 = m_tiles * (N / 128);
-  if (has64 && tiles128 < num_sms) return GemmPlan{64, 1};
-  if (N % 256 == 0 && (tiles128 / 2) >= 4L * num_sms) return GemmPlan{256, 1};
-  return GemmPlan{128, 1};
+  int bn = 128;
+  if (has64 && tiles128 < num_sms)
+    bn = 64;
+  else if (N % 256 == 0 && (tiles128 / 2) >= 4L * num_sms)
+    bn = 256;
+  return GemmPlan{bn, 1, 1};
 }
 
 cudaError_t tc_gemm(const GemmOperand& a, const GemmOperand& b, int M, int N, int K, int epi, const EpiArgs& e,
@@ -479,6 +566,12 @@ cudaError_t tc_gemm(const GemmOperand& a, const GemmOperand& b, int M, int N, in
   if (K % kBK != 0 || N % 128 != 0) return cudaErrorInvalidValue;
   if (plan.bn == 0) plan = tc_gemm_plan(M, N, K, b.r64, ws != nullptr && ws->ws != nullptr, num_sms);
   const int bn = plan.bn;
+  // clusters need a K split of 1, two K-atoms per stage, an even number of column tiles and the
+  // A operand's 64-row boxes; otherwise the plan runs without
+  int mc = plan.mc == 0 ? tc_gemm_plan(M, N, K, b.r64, false, num_sms).mc : plan.mc;
+  if (mc == 2 && !(plan.splits <= 1 && bn <= 128 && K % (2 * kBK) == 0 && (N / bn) % 2 == 0 && a.r64 &&
+                   num_sms >= 2))
+    mc = 1;
   if ((bn != 64 && bn != 128 && bn != 256) || N % bn != 0 || (bn == 64 && !b.r64)) return cudaErrorInvalidValue;
   const int ka = pick_ka(bn, K);
   if (ka == 2 && !(a.k2 && b.k2)) return cudaErrorInvalidValue;
@@ -492,16 +585,20 @@ cudaError_t tc_gemm(const GemmOperand& a, const GemmOperand& b, int M, int N, in
     sp.ws = ws->ws;
     sp.counters = ws->counters;
   }
+  if (mc == 2) {   // A halves through the 64-row one-atom boxes
+    if (bn == 64) return dispatch_epi<64, 2, 2>(a.r64_k1, b.r64_k2, M, N, K, epi, e, sp, num_sms, dev_err, s);
+    return dispatch_epi<128, 2, 2>(a.r64_k1, b.r128_k2, M, N, K, epi, e, sp, num_sms, dev_err, s);
+  }
   const CUtensorMap& ta = ka == 2 ? a.r128_k2 : a.r128_k1;
   if (bn == 64) {
     const CUtensorMap& tb = ka == 2 ? b.r64_k2 : b.r64_k1;
-    return ka == 2 ? dispatch_epi<64, 2>(ta, tb, M, N, K, epi, e, sp, num_sms, dev_err, s)
-                   : dispatch_epi<64, 1>(ta, tb, M, N, K, epi, e, sp, num_sms, dev_err, s);
+    return ka == 2 ? dispatch_epi<64, 2, 1>(ta, tb, M, N, K, epi, e, sp, num_sms, dev_err, s)
+                   : dispatch_epi<64, 1, 1>(ta, tb, M, N, K, epi, e, sp, num_sms, dev_err, s);
   }
-  if (bn == 256) return dispatch_epi<256, 1>(ta, b.r128_k1, M, N, K, epi, e, sp, num_sms, dev_err, s);
+  if (bn == 256) return dispatch_epi<256, 1, 1>(ta, b.r128_k1, M, N, K, epi, e, sp, num_sms, dev_err, s);
   const CUtensorMap& tb = ka == 2 ? b.r128_k2 : b.r128_k1;
-  return ka == 2 ? dispatch_epi<128, 2>(ta, tb, M, N, K, epi, e, sp, num_sms, dev_err, s)
-                 : dispatch_epi<128, 1>(ta, tb, M, N, K, epi, e, sp, num_sms, dev_err, s);
+  return ka == 2 ? dispatch_epi<128, 2, 1>(ta, tb, M, N, K, epi, e, sp, num_sms, dev_err, s)
+                 : dispatch_epi<128, 1, 1>(ta, tb, M, N, K, epi, e, sp, num_sms, dev_err, s);
 }
 
 int tc_encode_bf16_box(CUtensorMap* map, const void* base, uint64_t rows, uint64_t cols, uint64_t ld,

@@ -58,8 +58,8 @@ const char* wam_op_last_error(void) { return g_op_err.c_str(); }
 int wam_op_gemm_bf16(const void* A, const void* Wt, const float* bias, void* C, int32_t M, int32_t N,
                      int32_t K, int32_t epilogue, const float* gate, int64_t gate_stride,
                      int32_t rows_per_item, void* stream) {
-  return wam_op_gemm_bf16_plan(A, Wt, bias, C, M, N, K, epilogue, gate, gate_stride, rows_per_item, 0, 0, nullptr, 0,
-                               stream);
+  return wam_op_gemm_bf16_plan(A, Wt, bias, C, M, N, K, epilogue, gate, gate_stride, rows_per_item, 0, 0, 0, nullptr,
+                               0, stream);
 }
 
 size_t wam_op_gemm_workspace_bytes(void) {
@@ -71,8 +71,8 @@ size_t wam_op_gemm_workspace_bytes(void) {
 
 int wam_op_gemm_bf16_plan(const void* A, const void* Wt, const float* bias, void* C, int32_t M, int32_t N,
                           int32_t K, int32_t epilogue, const float* gate, int64_t gate_stride,
-                          int32_t rows_per_item, int32_t tile_n, int32_t k_splits, void* workspace,
-                          size_t workspace_bytes, void* stream) {
+                          int32_t rows_per_item, int32_t tile_n, int32_t k_splits, int32_t cluster,
+                          void* workspace, size_t workspace_bytes, void* stream) {
   int r = check_gemm_args(A, Wt, C, M, N, K, epilogue, gate, rows_per_item);
   if (r != WAM_OK) return r;
   if (K % 64 != 0 || N % 128 != 0) return op_fail(WAM_ERR_UNSUPPORTED, "needs K % 64 == 0 and N % 128 == 0");
@@ -82,6 +82,7 @@ int wam_op_gemm_bf16_plan(const void* A, const void* Wt, const float* bias, void
   if (tile_n != 0 && tile_n != 64 && tile_n != 128 && tile_n != 256)
     return op_fail(WAM_ERR_INVALID_ARG, "tile_n must be 0, 64, 128 or 256");
   if (k_splits < 0 || k_splits > 4) return op_fail(WAM_ERR_INVALID_ARG, "k_splits must be 0 .. 4");
+  if (cluster < 0 || cluster > 2) return op_fail(WAM_ERR_INVALID_ARG, "cluster must be 0, 1 or 2");
   int dev = 0, sms = 0;
   cudaError_t e = cudaGetDevice(&dev);
   if (e == cudaSuccess) e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
@@ -90,7 +91,7 @@ int wam_op_gemm_bf16_plan(const void* A, const void* Wt, const float* bias, void
   if (workspace != nullptr && (workspace_bytes < need || !aligned16(workspace)))
     return op_fail(WAM_ERR_INVALID_ARG, "workspace smaller than wam_op_gemm_workspace_bytes() or unaligned");
   GemmOperand ta, tb;
-  if (tc_encode_gemm_operand(&ta, A, static_cast<uint64_t>(M > 0 ? M : 1), K, false) != 0 ||
+  if (tc_encode_gemm_operand(&ta, A, static_cast<uint64_t>(M > 0 ? M : 1), K, true) != 0 ||
       tc_encode_gemm_operand(&tb, Wt, N, K, true) != 0)
     return op_fail(WAM_ERR_CUDA, "cuTensorMapEncodeTiled failed");
   SplitWorkspace ws{nullptr, nullptr, 0};
@@ -100,7 +101,7 @@ int wam_op_gemm_bf16_plan(const void* A, const void* Wt, const float* bias, void
                         reinterpret_cast<int*>(static_cast<uint8_t*>(workspace) + need - counters_bytes),
                         need - counters_bytes};
   }
-  const GemmPlan plan{tile_n, tile_n == 0 ? 0 : (k_splits < 1 ? 1 : k_splits)};
+  const GemmPlan plan{tile_n, tile_n == 0 ? 0 : (k_splits < 1 ? 1 : k_splits), cluster};
   if (plan.bn == 0 && k_splits > 1) return op_fail(WAM_ERR_INVALID_ARG, "k_splits needs an explicit tile_n");
   e = tc_gemm(ta, tb, M, N, K, epilogue, make_epi(bias, C, gate, gate_stride, rows_per_item), sms, nullptr,
               static_cast<cudaStream_t>(stream), workspace != nullptr ? &ws : nullptr, plan);

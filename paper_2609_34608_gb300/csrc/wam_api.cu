@@ -1162,10 +1162,11 @@ int create_impl(wam_ctx* c, const wam_config* cfg, const float* weights, size_t 
   c->part_doubles = std::max(p_tr, std::max(p_or, p_rr));
   TRY(dalloc(c, c->allocs, &c->d_part, c->part_doubles));
   if (c->bf16) {
-    TRY(encode(c, &c->tm_xln, c->xln, rows, c->d));
-    TRY(encode(c, &c->tm_att, c->att, rows, c->d));
-    TRY(encode(c, &c->tm_u, c->u, rows, c->dff));
-    TRY(encode(c, &c->tm_obs_lp, c->obs_lp, size_t(c->Bmax) * c->No, c->d));
+    // A operands also with 64-row boxes: the clustered GEMM multicasts 64-row halves of A
+    TRY(encode(c, &c->tm_xln, c->xln, rows, c->d, true));
+    TRY(encode(c, &c->tm_att, c->att, rows, c->d, true));
+    TRY(encode(c, &c->tm_u, c->u, rows, c->dff, true));
+    TRY(encode(c, &c->tm_obs_lp, c->obs_lp, size_t(c->Bmax) * c->No, c->d, true));
     TRY(encode(c, &c->tm_obs_w, c->obs_wt, c->d, c->d));
     c->tc_attn = c->d / c->H == 64 || c->d / c->H == 72;
     if (c->tc_attn) {

@@ -128,7 +128,7 @@ def lib() -> ctypes.CDLL:
         "wam_op_gemm_bf16": (ctypes.c_int, [_vp, _vp, _vp, _vp, _i32, _i32, _i32, _i32, _vp, ctypes.c_int64, _i32, _vp]),
         "wam_op_gemm_f32": (ctypes.c_int, [_vp, _vp, _vp, _vp, _i32, _i32, _i32, _i32, _vp, ctypes.c_int64, _i32, _vp]),
         "wam_op_gemm_bf16_plan": (ctypes.c_int, [_vp, _vp, _vp, _vp, _i32, _i32, _i32, _i32, _vp, ctypes.c_int64, _i32,
-                                                 _i32, _i32, _vp, ctypes.c_size_t, _vp]),
+                                                 _i32, _i32, _i32, _vp, ctypes.c_size_t, _vp]),
         "wam_op_gemm_workspace_bytes": (ctypes.c_size_t, []),
         "wam_gemm_tile_width": (ctypes.c_int, [_vp, _i32, _i32, _i32, _i32]),
         "wam_set_graph_replay": (ctypes.c_int, [_vp, _i32]),
@@ -419,13 +419,14 @@ def op_gemm_bf16(A, Wt, bias, C, M, N, K, epilogue, gate=None, gate_stride=0, ro
 
 
 def op_gemm_bf16_plan(A, Wt, bias, C, M, N, K, epilogue, tile_n, k_splits, workspace=None, gate=None,
-                      gate_stride=0, rows_per_item=1, stream=None):
-    """wam_op_gemm_bf16 with an explicit output tile width and K split (workspace: a zero-filled
-    device buffer of gemm_workspace_bytes() bytes, needed when k_splits > 1)."""
+                      gate_stride=0, rows_per_item=1, stream=None, cluster=0):
+    """wam_op_gemm_bf16 with an explicit output tile width, K split and cluster size (0 = the
+    library's rule, 1 = single CTAs, 2 = pairs sharing the A tile); workspace: a zero-filled device
+    buffer of gemm_workspace_bytes() bytes, needed when k_splits > 1."""
     nbytes = 0 if workspace is None else workspace.numel() * workspace.element_size()
     _op_check(lib().wam_op_gemm_bf16_plan(ptr(A), ptr(Wt), ptr(bias), ptr(C), M, N, K, epilogue, ptr(gate),
-                                          gate_stride, rows_per_item, tile_n, k_splits, ptr(workspace), nbytes,
-                                          stream))
+                                          gate_stride, rows_per_item, tile_n, k_splits, cluster, ptr(workspace),
+                                          nbytes, stream))
 
 
 def gemm_workspace_bytes():

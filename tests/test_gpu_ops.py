@@ -99,6 +99,25 @@ def test_gemm_plans_match_reference(wamlib, M, N, K, tile_n, k_splits, epi):
     assert int(ws[ws.numel() - 4 * n_sms:].count_nonzero()) == 0
 
 
+# (M, N, K, tile width): shapes where the two-CTA clusters apply (even column-tile count)
+CLUSTER_CASES = [(1296, 768, 768, 64), (1296, 3072, 768, 128), (1296, 768, 3072, 64), (1296, 2304, 768, 128),
+                 (129, 256, 256, 128), (1, 256, 128, 64), (2600, 1024, 1024, 64)]
+
+
+@pytest.mark.parametrize("M,N,K,tile_n", CLUSTER_CASES)
+@pytest.mark.parametrize("epi", [W.EPI_GELU_BF16, W.EPI_RESID_F32])
+def test_gemm_clusters_match_reference_and_single_ctas(wamlib, M, N, K, tile_n, epi):
+    """Clusters of two CTAs sharing the A tile by multicast: the reference within tolerance, and the
+    single-CTA kernel bit for bit (same accumulation order)."""
+    outs = []
+    for cluster in (2, 1):
+        def run(A, Wt, b, C, gate, rpi):
+            W.op_gemm_bf16_plan(A, Wt, b, C, M, N, K, epi, tile_n, 1, gate=gate, gate_stride=N + 4,
+                                rows_per_item=rpi, cluster=cluster)
+        outs.append(_check_gemm(M, N, K, epi, run).cpu())
+    assert torch.equal(outs[0], outs[1])
+
+
 def test_gemm_split_is_deterministic(wamlib):
     """A K-split result does not depend on which unit finished last: repeated runs agree bit for bit."""
     M, N, K = 1392, 768, 3072
