@@ -510,7 +510,9 @@ def main_ours(args):
     ablation = None
     if not args.no_ablation:
         ablation = run_table3(ctx, flat, cfg, dev, stream, dev_in, obs0, noise, min(args.steps, 20))
-    async_prefix = run_async_prefix(ctx, cfg, dev, stream, dev_in, obs0, noise, n=min(args.steps, 20))
+    async_prefix = None
+    if not args.no_async:
+        async_prefix = run_async_prefix(ctx, cfg, dev, stream, dev_in, obs0, noise, n=min(args.steps, 20))
     del flat
 
     serving = serving_rr = independent = bimanual = None
@@ -566,7 +568,8 @@ def main_ours(args):
     }
     if ablation is not None:
         line["ablation"] = ablation
-    line["async_prefix"] = async_prefix
+    if async_prefix is not None:
+        line["async_prefix"] = async_prefix
     if serving is not None:
         line["serving"] = serving
         line["serving_rr_accept"] = serving_rr
@@ -998,6 +1001,7 @@ def main():
     ap.add_argument("--no-independent", action="store_true", help="skip the independent-execution section")
     ap.add_argument("--no-bimanual", action="store_true", help="skip the large bimanual model section")
     ap.add_argument("--no-ablation", action="store_true", help="skip the Table 3 ablation section")
+    ap.add_argument("--no-async", action="store_true", help="skip the asynchronous-prefix section")
     ap.add_argument("--cpu-plan", action="store_true",
                     help="only time the CPU oracle plan (all cores and one core; no GPU) and print it")
     args = ap.parse_args()

@@ -138,6 +138,49 @@ WAM_DEV void row_stats(const float4 (&v)[NV4], int d, float& mean, float& rstd) 
   rstd = rsqrtf(warp_sum(q) / d + 1e-6f);
 }
 
+// ---- double-float accumulation (float32 pairs) ----------------------------------------
+// GB300 runs float64 at a small fraction of its float32 rate, which made float64 reductions the
+// bottleneck of the TR direction sums.  A sum of squares kept as an unevaluated pair hi + lo of
+// floats, with the exact error of every product (fma) and addition (two-sum) carried in lo, is
+// accurate to about 2^-44 relative, enough for the float32 results those sums scale.
+WAM_DEV void two_sum(float a, float b, float& s, float& e) {
+  s = a + b;
+  const float bb = s - a;
+  e = (a - (s - bb)) + (b - bb);
+}
+
+// (hi, lo) += v^2 for v = x - y, with x - y itself split exactly into vh + vl.
+WAM_DEV void df_add_sq_diff(float x, float y, float& hi, float& lo) {
+  float vh, vl;
+  two_sum(x, -y, vh, vl);
+  const float ph = vh * vh;
+  const float pl = fmaf(vh, vh, -ph) + fmaf(2.0f * vh, vl, vl * vl);
+  float sh, se;
+  two_sum(hi, ph, sh, se);
+  const float sl = lo + (se + pl);
+  hi = sh + sl;                 // renormalise: |sl| is far below |sh|
+  lo = sl - (hi - sh);
+}
+
+// (hi, lo) += (bh, bl)
+WAM_DEV void df_add(float& hi, float& lo, float bh, float bl) {
+  float sh, se;
+  two_sum(hi, bh, sh, se);
+  const float sl = lo + bl + se;
+  hi = sh + sl;
+  lo = sl - (hi - sh);
+}
+
+// Warp sum of double-float values; every lane ends with the total.
+WAM_DEV void warp_sum_df(float& hi, float& lo) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    const float oh = __shfl_xor_sync(0xffffffffu, hi, o);
+    const float ol = __shfl_xor_sync(0xffffffffu, lo, o);
+    df_add(hi, lo, oh, ol);
+  }
+}
+
 WAM_DEV float silu_f(float x) { return x / (1.0f + expf(-x)); }
 
 WAM_DEV float gelu_tanh_f(float x) {

@@ -143,6 +143,13 @@ __global__ void __launch_bounds__(256) cond_gemv_kernel(const float* __restrict_
 }
 
 // ---------------------------------------------------------------- token embedding
+// One warp per group of kEmbRows consecutive token rows: each lane loads the embedding weights of
+// its float4 column once per group and applies them to every video (or action) row of the group,
+// so the weight reads from L1 shrink by the group size (one warp per row read 16 weight values per
+// output value and was bound by L1, not HBM).  The trajectory values of the group's rows sit in
+// shared memory.  Per output: acc = b, then acc = fma(x_i, W_i, acc) for i in order, then + pos.
+constexpr int kEmbRows = 8;
+
 __global__ void __launch_bounds__(256) embed_kernel(
     float* __restrict__ h, float* __restrict__ xhist, int64_t stage_stride,
     const StepItem* __restrict__ items, const float* __restrict__ x, int T,
@@ -152,50 +159,89 @@ __global__ void __launch_bounds__(256) embed_kernel(
     int vd, int Na, int ad, int d) {
   pdl_wait();
   pdl_launch_dependents();
+  __shared__ float xs[kRowWarps][kEmbRows][16];
+  __shared__ int rinfo[kRowWarps][kEmbRows][3];   // kind (-1 none, 0 obs, 1 video, 2 action), n, episode
   const int N = No + Nv + Na;
-  const int64_t gw = static_cast<int64_t>(blockIdx.x) * kRowWarps + (threadIdx.x >> 5);
+  const int wib = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
-  if (gw >= static_cast<int64_t>(Bw) * N) return;
-  const int w = static_cast<int>(gw / N), n = static_cast<int>(gw % N);
-  const StepItem it = items[w];
-  float4* hr = reinterpret_cast<float4*>(h + gw * d);
-  const float4* pr = reinterpret_cast<const float4*>(pos + static_cast<int64_t>(n) * d);
-  const int d4 = d / 4;
-  if (n < No) {
-    const float4* src = reinterpret_cast<const float4*>(obs_emb + (static_cast<int64_t>(it.ep) * No + n) * d);
-    for (int c = lane; c < d4; c += 32) {
-      const float4 a = src[c], p = pr[c];
-      hr[c] = make_float4(a.x + p.x, a.y + p.y, a.z + p.z, a.w + p.w);
+  const int64_t row0 = (static_cast<int64_t>(blockIdx.x) * kRowWarps + wib) * kEmbRows;
+  const int64_t rows = static_cast<int64_t>(Bw) * N;
+  if (row0 >= rows) return;
+  if (lane < kEmbRows) {
+    const int64_t gw = row0 + lane;
+    int kind = -1, n = 0, ep = 0;
+    if (gw < rows) {
+      const int w = static_cast<int>(gw / N);
+      n = static_cast<int>(gw % N);
+      ep = items[w].ep;
+      kind = n < No ? 0 : (n < No + Nv ? 1 : 2);
     }
-    return;
+    rinfo[wib][lane][0] = kind;
+    rinfo[wib][lane][1] = n;
+    rinfo[wib][lane][2] = ep;
   }
-  const bool video = n < No + Nv;
-  const int in_dim = video ? vd : ad;
-  const int64_t xoff = static_cast<int64_t>(it.ep) * T +
-                       (video ? static_cast<int64_t>(n - No) * vd
-                              : static_cast<int64_t>(Nv) * vd + static_cast<int64_t>(n - No - Nv) * ad);
-  const float* xin = x + xoff;
-  // Record the latent entering this stage (the retained trajectory at stage k).
-  if (lane < in_dim) xhist[static_cast<int64_t>(it.stage) * stage_stride + xoff + lane] = xin[lane];
-  float xi[16];
-#pragma unroll
-  for (int i = 0; i < 16; ++i) xi[i] = i < in_dim ? xin[i] : 0.0f;
-  const float4* W4 = reinterpret_cast<const float4*>(video ? vid_w : act_w);
-  const float4* b4 = reinterpret_cast<const float4*>(video ? vid_b : act_b);
-  for (int c = lane; c < d4; c += 32) {
-    float4 acc = b4[c];
-#pragma unroll
-    for (int i = 0; i < 16; ++i) {
+  __syncwarp();
+  // the group's trajectory values, and the record of the latent entering this stage
+  bool any_v = false, any_a = false;
+  for (int j = lane; j < kEmbRows * 16; j += 32) {
+    const int r = j >> 4, i = j & 15;
+    const int kind = rinfo[wib][r][0], n = rinfo[wib][r][1], ep = rinfo[wib][r][2];
+    float v = 0.0f;
+    if (kind >= 1) {
+      const int in_dim = kind == 1 ? vd : ad;
+      const int64_t xoff = static_cast<int64_t>(ep) * T +
+                           (kind == 1 ? static_cast<int64_t>(n - No) * vd
+                                      : static_cast<int64_t>(Nv) * vd + static_cast<int64_t>(n - No - Nv) * ad);
       if (i < in_dim) {
-        const float4 wv = W4[static_cast<int64_t>(i) * d4 + c];
-        acc.x = fmaf(xi[i], wv.x, acc.x);
-        acc.y = fmaf(xi[i], wv.y, acc.y);
-        acc.z = fmaf(xi[i], wv.z, acc.z);
-        acc.w = fmaf(xi[i], wv.w, acc.w);
+        v = x[xoff + i];
+        const int stage = items[(row0 + r) / N].stage;
+        xhist[static_cast<int64_t>(stage) * stage_stride + xoff + i] = v;
       }
     }
-    const float4 p = pr[c];
-    hr[c] = make_float4(acc.x + p.x, acc.y + p.y, acc.z + p.z, acc.w + p.w);
+    xs[wib][r][i] = v;
+  }
+#pragma unroll
+  for (int r = 0; r < kEmbRows; ++r) {
+    any_v |= rinfo[wib][r][0] == 1;
+    any_a |= rinfo[wib][r][0] == 2;
+  }
+  __syncwarp();
+  const int d4 = d / 4;
+  for (int c = lane; c < d4; c += 32) {
+#pragma unroll
+    for (int r = 0; r < kEmbRows; ++r) {
+      if (rinfo[wib][r][0] != 0) continue;
+      const int n = rinfo[wib][r][1], ep = rinfo[wib][r][2];
+      const float4 a = reinterpret_cast<const float4*>(obs_emb + (static_cast<int64_t>(ep) * No + n) * d)[c];
+      const float4 p = reinterpret_cast<const float4*>(pos + static_cast<int64_t>(n) * d)[c];
+      reinterpret_cast<float4*>(h + (row0 + r) * d)[c] = make_float4(a.x + p.x, a.y + p.y, a.z + p.z, a.w + p.w);
+    }
+    for (int kind = 1; kind <= 2; ++kind) {
+      if (kind == 1 ? !any_v : !any_a) continue;
+      const int in_dim = kind == 1 ? vd : ad;
+      const float4* W4 = reinterpret_cast<const float4*>(kind == 1 ? vid_w : act_w);
+      float4 wv[16];
+#pragma unroll
+      for (int i = 0; i < 16; ++i) wv[i] = i < in_dim ? W4[static_cast<int64_t>(i) * d4 + c] : make_float4(0.f, 0.f, 0.f, 0.f);
+      const float4 bias = reinterpret_cast<const float4*>(kind == 1 ? vid_b : act_b)[c];
+#pragma unroll 1
+      for (int r = 0; r < kEmbRows; ++r) {
+        if (rinfo[wib][r][0] != kind) continue;
+        float4 acc = bias;
+#pragma unroll
+        for (int i = 0; i < 16; ++i) {
+          if (i < in_dim) {
+            const float xi = xs[wib][r][i];
+            acc.x = fmaf(xi, wv[i].x, acc.x);
+            acc.y = fmaf(xi, wv[i].y, acc.y);
+            acc.z = fmaf(xi, wv[i].z, acc.z);
+            acc.w = fmaf(xi, wv[i].w, acc.w);
+          }
+        }
+        const float4 p = reinterpret_cast<const float4*>(pos + static_cast<int64_t>(rinfo[wib][r][1]) * d)[c];
+        reinterpret_cast<float4*>(h + (row0 + r) * d)[c] = make_float4(acc.x + p.x, acc.y + p.y, acc.z + p.z, acc.w + p.w);
+      }
+    }
   }
 }
 
@@ -614,10 +660,10 @@ __global__ void __launch_bounds__(256) tr_rms_partial_kernel(const AdaptItem* __
                                                              double* __restrict__ partial) {
   pdl_wait();
   pdl_launch_dependents();
-  __shared__ double red[8];
+  __shared__ float red[2][8];
   const int b = blockIdx.z, br = blockIdx.y, ch = blockIdx.x;
   const AdaptItem it = items[b];
-  double s = 0.0;
+  float hi = 0.0f, lo = 0.0f;
   if (it.op == kAdaptTR) {
     const int beg = br == 0 ? 0 : V;
     const int len = br == 0 ? V : T - V;
@@ -634,17 +680,24 @@ __global__ void __launch_bounds__(256) tr_rms_partial_kernel(const AdaptItem* __
       a[u] = i < end ? xr[i] : 0.0f;
       c[u] = i < end ? xb[i] : 0.0f;
     }
-    // sum of (x^r - x_bar)^2, scaled by 1 / sigma_r^2 once (no float64 division per element:
-    // float64 runs at a small fraction of the float32 rate on this part)
+    // sum of (x^r - x_bar)^2 in double-float (float64 runs at a small fraction of the float32
+    // rate on this part); the block total is scaled by 1 / sigma_r^2 once, in float64
 #pragma unroll
-    for (int u = 0; u < kPer; ++u) {
-      const double v = static_cast<double>(a[u]) - static_cast<double>(c[u]);
-      s = fma(v, v, s);
-    }
-    s *= 1.0 / (it.sigma_r * it.sigma_r);
+    for (int u = 0; u < kPer; ++u) df_add_sq_diff(a[u], c[u], hi, lo);
   }
-  s = block_sum_d(s, red);
-  if (threadIdx.x == 0) partial[(static_cast<int64_t>(b) * 2 + br) * nch + ch] = s;
+  warp_sum_df(hi, lo);
+  const int warp = threadIdx.x >> 5;
+  if ((threadIdx.x & 31) == 0) {
+    red[0][warp] = hi;
+    red[1][warp] = lo;
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    double s = 0.0;
+    for (int w = 0; w < 8; ++w) s += static_cast<double>(red[0][w]) + static_cast<double>(red[1][w]);
+    partial[(static_cast<int64_t>(b) * 2 + br) * nch + ch] =
+        it.op == kAdaptTR ? s * (1.0 / (it.sigma_r * it.sigma_r)) : 0.0;
+  }
 }
 
 // Remapped initialisation (Eq. 2), cold init, restart, and binding of the new condition.
@@ -1080,7 +1133,8 @@ cudaError_t embed_tokens(float* h, float* xhist, int64_t stage_stride, const Ste
                          cudaStream_t s) {
   if (Bw <= 0) return cudaSuccess;
   const int64_t rows = static_cast<int64_t>(Bw) * (No + Nv + Na);
-  launch_pdl(embed_kernel, dim3(row_blocks(rows)), dim3(32 * kRowWarps), 0, s, h, xhist, stage_stride, items, x, T,
+  const int64_t groups = (rows + kEmbRows - 1) / kEmbRows;
+  launch_pdl(embed_kernel, dim3(row_blocks(groups)), dim3(32 * kRowWarps), 0, s, h, xhist, stage_stride, items, x, T,
                                                            obs_emb, vid_w, vid_b, act_w, act_b,
                                                            pos, Bw, No, Nv, vd, Na, ad, d);
   return cudaGetLastError();

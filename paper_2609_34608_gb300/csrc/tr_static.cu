@@ -36,39 +36,39 @@ static __device__ __align__(256) double g_tr_partials[kStaticPartials];
 std::mutex g_mu;
 double* g_partials_ptr[kMaxDevices] = {};
 
-WAM_DEV double block_sum(double v, double* red) {
-  v = warp_sum_d(v);
-  if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = v;
-  __syncthreads();
-  double s = 0.0;
-  if (threadIdx.x == 0)
-    for (int w = 0; w < (blockDim.x >> 5); ++w) s += red[w];
-  return s;
-}
-
-// Sum over one chunk of one branch of (x^r - x_bar)^2 / sigma_r^2, accumulated in the same order
-// and with the same roundings as the remap of wam_adapt_state (thread t of the block takes
-// elements t, t + 256, ... of the chunk with one fused multiply-add each; the thread's sum is
-// scaled by 1 / sigma_r^2 once; then the warp and block sums), so the two entry points agree
-// bit for bit.
+// Sum over one chunk of one branch of (x^r - x_bar)^2 / sigma_r^2, with the same operations in
+// the same order as the remap of wam_adapt_state (thread t of the block takes elements t, t + 256,
+// ... of the chunk into a double-float sum; then the warp and block sums; the block total is
+// scaled by 1 / sigma_r^2 once), so the two entry points agree bit for bit.
 __global__ void __launch_bounds__(256) tr_static_partial_kernel(const float* __restrict__ x_bar,
                                                                 const float* __restrict__ x_r,
                                                                 int T, int V, double sigma_r,
                                                                 int nch, double* __restrict__ partial) {
-  __shared__ double red[8];
+  __shared__ float red[2][8];
   const int b = blockIdx.z, br = blockIdx.y, ch = blockIdx.x;
   const int beg = br == 0 ? 0 : V;
   const int len = br == 0 ? V : T - V;
   const int64_t bo = static_cast<int64_t>(b) * T + beg;
   const int end = min(len, (ch + 1) * kStaticChunk);
-  double s = 0.0;
-  for (int i = ch * kStaticChunk + threadIdx.x; i < end; i += blockDim.x) {
-    const double v = static_cast<double>(x_r[bo + i]) - static_cast<double>(x_bar[bo + i]);
-    s = fma(v, v, s);
+  float hi = 0.0f, lo = 0.0f;
+  for (int u = 0; u < kStaticChunk / 256; ++u) {
+    const int i = ch * kStaticChunk + u * 256 + threadIdx.x;
+    const float a = i < end ? x_r[bo + i] : 0.0f;
+    const float c = i < end ? x_bar[bo + i] : 0.0f;
+    df_add_sq_diff(a, c, hi, lo);
   }
-  s *= 1.0 / (sigma_r * sigma_r);
-  s = block_sum(s, red);
-  if (threadIdx.x == 0) partial[(static_cast<int64_t>(b) * 2 + br) * nch + ch] = s;
+  warp_sum_df(hi, lo);
+  const int warp = threadIdx.x >> 5;
+  if ((threadIdx.x & 31) == 0) {
+    red[0][warp] = hi;
+    red[1][warp] = lo;
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    double s = 0.0;
+    for (int w = 0; w < 8; ++w) s += static_cast<double>(red[0][w]) + static_cast<double>(red[1][w]);
+    partial[(static_cast<int64_t>(b) * 2 + br) * nch + ch] = s * (1.0 / (sigma_r * sigma_r));
+  }
 }
 
 // Remapped init: retained slots get x_bar + sigma_b0 * unit-RMS direction, computed as one

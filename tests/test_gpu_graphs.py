@@ -107,3 +107,45 @@ def test_device_branching_matches_host_branching(wamlib, precision, gate):
     if gate == "strict":
         assert sa["n_reuse"] == 0 and sa["n_attempt"] > 0
     assert sa["n_kernel_launches"] > 0
+
+
+def test_prefix_on_second_stream_matches_one_stream(wamlib):
+    """The anticipatory prefix (TR + one step under the prediction) issued on a second stream
+    while the first is idle, ordered by events, gives the same replans as one stream."""
+    import torch
+
+    cfg = I.get_config("tiny", **SMALL_BF16)
+    K, b0 = cfg["n_steps"], int(cfg["tr_entry_stage"])
+    dev = torch.device("cuda")
+    res = []
+    for two in (False, True):
+        main, side = torch.cuda.Stream(dev), torch.cuda.Stream(dev)
+        ctx = W.Context(cfg, I.flatten_weights(I.make_weights(cfg)), stream=main.cuda_stream)
+        st = ctx.state(1)
+        proc = I.ObsProcess(cfg, 1, seed=6)
+        act = torch.zeros((1, cfg["n_action"], cfg["action_dim"])).pin_memory()
+        ctx.sample_cold(st, proc.obs.copy(), I.make_noise(cfg, 1), K, act)
+        outs = []
+        for r in range(4):
+            pred, real = proc.predicted(), proc.step()
+            if two:
+                ready = torch.cuda.Event()
+                ready.record(main)
+                side.wait_event(ready)
+                ctx.set_stream(side.cuda_stream)
+            s1 = ctx.adapt(st, pred, shift=int(cfg["shift"]), fresh_noise=I.make_fresh_eps(cfg, 1, r))[0]
+            if s1 == W.ADAPT_TR_INIT:
+                ctx.continue_(st, 1)
+            if two:
+                done = torch.cuda.Event()
+                done.record(side)
+                ctx.set_stream(main.cuda_stream)
+                main.wait_event(done)
+            s2 = ctx.adapt(st, real)[0]
+            ctx.continue_(st, K - (b0 + 1 if s2 == W.ADAPT_REBIND_ACCEPT else b0), act)   # host output: synchronous
+            outs += [act.numpy().copy(), ctx.read(st, W.FIELD_X).copy()]
+        res.append((outs, ctx.stats()["n_reuse"]))
+        ctx.close()
+    for x, y in zip(res[0][0], res[1][0]):
+        assert np.array_equal(x, y)
+    assert res[0][1] == res[1][1]
