@@ -16,7 +16,10 @@ the C ABI with pinned host buffers (host<->device copies inside the timed region
 its time taken as its share of a profiled pass applied to the un-instrumented step;
 `kernels` = every kernel class of the profiled pass; `ablation` = the paper's Table 3 variants
 (w/o TR, w/o OR, w/o RR, w/o graph replay, native with and without graphs) and a labelled run
-with a relaxed RR gate; `serving` = 32-episode batches of the 24-block d1024 model;
+with a relaxed RR gate; `seeds` = the closed-loop rollout over seeds 0..3 (its own observation
+process per seed), each seed's warm control steps against cold 10-step samples under the same
+observations; `async_prefix` = the anticipatory prefix on a second stream during a modelled
+action-execution window (O2A and GPU time per replan); `serving` = 32-episode batches of the 24-block d1024 model;
 `bimanual` = the 28-block d1152 model (head dim 72, 4914 tokens, batch 8): cold 10 steps and
 the warm sweep over 1..9 retained steps with shift 25; `independent` = the separate video /
 action models of independent execution, their continuations overlapped on two streams and in
@@ -510,6 +513,9 @@ def main_ours(args):
     ablation = None
     if not args.no_ablation:
         ablation = run_table3(ctx, flat, cfg, dev, stream, dev_in, obs0, noise, min(args.steps, 20))
+    seeds = None
+    if not args.no_seeds:
+        seeds = run_seeds(ctx, cfg, dev, stream, min(args.steps, 200))
     async_prefix = None
     if not args.no_async:
         async_prefix = run_async_prefix(ctx, cfg, dev, stream, dev_in, obs0, noise, n=min(args.steps, 20))
@@ -568,6 +574,8 @@ def main_ours(args):
     }
     if ablation is not None:
         line["ablation"] = ablation
+    if seeds is not None:
+        line["seeds"] = seeds
     if async_prefix is not None:
         line["async_prefix"] = async_prefix
     if serving is not None:
@@ -677,6 +685,79 @@ def run_table3(ctx, flat, cfg, dev, stream, dev_in, obs0, noise, n, warm=3):
     out["what"] = ("Table 3 variants on the closed-loop workload (GPU = mean ms of one replan's work, O2A = real "
                    "observation to action chunk, both on the device clock); rr_relaxed = full with RR thresholds "
                    "that accept every check (labelled: random weights, not a trained model's acceptance)")
+    return out
+
+
+def run_seeds(ctx, cfg, dev, stream, n, seeds=(0, 1, 2, 3), warm=3):
+    """The closed-loop rollout over several seeds: per seed, its own observation process
+    (o' = 0.9 o + sqrt(0.19) N(0,1), prediction 0.9 o), initial noise and fresh-noise draws, one
+    cold replan, then n control steps (TR shift, 1 anticipatory step, OR, the remaining steps with
+    RR), each timed on the device; beside it the cold 10-step sample under the same real
+    observations, so every seed reports warm versus cold."""
+    import torch
+
+    from paper_2609_34608_gb300 import inputs as I
+    from paper_2609_34608_gb300 import wam as W
+
+    K, b0, shift, pre = cfg["n_steps"], cfg["tr_entry_stage"], cfg["shift"], cfg["prefix_steps"]
+    act = torch.zeros((1, cfg["n_action"], cfg["action_dim"]), device=dev)
+    ev = lambda: torch.cuda.Event(enable_timing=True)
+    out = {}
+    for seed in seeds:
+        proc = I.ObsProcess(cfg, 1, seed=seed)
+        with torch.cuda.stream(stream):
+            obs0 = torch.from_numpy(proc.obs.copy()).to(dev)
+            noise = torch.from_numpy(I.make_noise(cfg, 1, seed=1 + seed)).to(dev)
+            inp = []
+            for t in range(warm + n):
+                pred = proc.predicted()
+                real = proc.step()
+                eps = I.make_fresh_eps(cfg, 1, 100000 * seed + t)
+                inp.append(tuple(torch.from_numpy(a).to(dev) for a in (pred, real, eps)))
+        st, st_c = ctx.state(1), ctx.state(1)
+        with torch.cuda.stream(stream):
+            ctx.sample_cold(st, obs0, noise, K, act)
+            for t in range(warm):
+                pred, real, eps = inp[t]
+                if ctx.adapt(st, pred, shift=shift, fresh_noise=eps)[0] == W.ADAPT_TR_INIT:
+                    ctx.continue_(st, pre)
+                s2 = ctx.adapt(st, real)[0]
+                ctx.continue_(st, K - (b0 + pre if s2 == W.ADAPT_REBIND_ACCEPT else b0), act)
+        ctx.reset_stats()
+        torch.cuda.synchronize(dev)
+        warm_ev = [(ev(), ev()) for _ in range(n)]
+        cold_ev = [(ev(), ev()) for _ in range(n)]
+        with torch.cuda.stream(stream):
+            for i in range(n):
+                pred, real, eps = inp[warm + i]
+                warm_ev[i][0].record(stream)
+                if ctx.adapt(st, pred, shift=shift, fresh_noise=eps)[0] == W.ADAPT_TR_INIT:
+                    ctx.continue_(st, pre)
+                s2 = ctx.adapt(st, real)[0]
+                ctx.continue_(st, K - (b0 + pre if s2 == W.ADAPT_REBIND_ACCEPT else b0), act)
+                warm_ev[i][1].record(stream)
+        stt = ctx.stats()
+        with torch.cuda.stream(stream):
+            for i in range(n):
+                pred, real, eps = inp[warm + i]
+                cold_ev[i][0].record(stream)
+                ctx.sample_cold(st_c, real, eps, K, act)
+                cold_ev[i][1].record(stream)
+        torch.cuda.synchronize(dev)
+        w = [a.elapsed_time(b) for a, b in warm_ev]
+        c = [a.elapsed_time(b) for a, b in cold_ev]
+        out[f"seed_{seed}"] = {"chunks_per_s": 1000.0 * n / sum(w), "ms_p50": float(np.percentile(w, 50)),
+                               "ms_p99": float(np.percentile(w, 99)),
+                               "cold_chunks_per_s": 1000.0 * n / sum(c), "cold_ms_p50": float(np.percentile(c, 50)),
+                               "speedup_vs_cold": sum(c) / sum(w),
+                               "r_or": stt["n_bind"] / max(1, stt["n_start"]),
+                               "r_rr": stt["n_reuse"] / max(1, stt["n_attempt"])}
+        st.close()
+        st_c.close()
+        del inp
+    out["steps_per_seed"] = n
+    out["what"] = ("closed-loop rollout per seed (own observation process, noise and fresh-noise draws): n warm "
+                   "control steps and, under the same real observations, n cold 10-step samples; device time")
     return out
 
 
@@ -1002,6 +1083,7 @@ def main():
     ap.add_argument("--no-bimanual", action="store_true", help="skip the large bimanual model section")
     ap.add_argument("--no-ablation", action="store_true", help="skip the Table 3 ablation section")
     ap.add_argument("--no-async", action="store_true", help="skip the asynchronous-prefix section")
+    ap.add_argument("--no-seeds", action="store_true", help="skip the per-seed closed-loop rollouts")
     ap.add_argument("--cpu-plan", action="store_true",
                     help="only time the CPU oracle plan (all cores and one core; no GPU) and print it")
     args = ap.parse_args()

@@ -110,8 +110,25 @@ __global__ void __launch_bounds__(256) cond_gemv_kernel(const float* __restrict_
 #pragma unroll
       for (int c = 0; c < CPT; ++c) acc[bi][c] = 0.0f;
     if (col0 < Nout) {
-#pragma unroll 4
-      for (int kk = kw0; kk < kw1; ++kk) {
+      // eight weight rows in flight per thread before their first use (the weights stream from
+      // HBM once per step; fewer loads in flight left the read latency-bound at one item)
+      constexpr int kBatch = 8;
+      int kk = kw0;
+      for (; kk + kBatch <= kw1; kk += kBatch) {
+        float w[kBatch][CPT];
+#pragma unroll
+        for (int u = 0; u < kBatch; ++u) WVec<TW>::load(W, static_cast<int64_t>(k_beg + kk + u) * Nout + col0, w[u]);
+#pragma unroll
+        for (int u = 0; u < kBatch; ++u) {
+#pragma unroll
+          for (int bi = 0; bi < KB; ++bi) {
+            const float xv = sx[bi * kslice + kk + u];
+#pragma unroll
+            for (int c = 0; c < CPT; ++c) acc[bi][c] = fmaf(xv, w[u][c], acc[bi][c]);
+          }
+        }
+      }
+      for (; kk < kw1; ++kk) {
         float w[CPT];
         WVec<TW>::load(W, static_cast<int64_t>(k_beg + kk) * Nout + col0, w);
 #pragma unroll
@@ -143,11 +160,12 @@ __global__ void __launch_bounds__(256) cond_gemv_kernel(const float* __restrict_
 }
 
 // ---------------------------------------------------------------- token embedding
-// One warp per group of kEmbRows consecutive token rows: each lane loads the embedding weights of
-// its float4 column once per group and applies them to every video (or action) row of the group,
-// so the weight reads from L1 shrink by the group size (one warp per row read 16 weight values per
-// output value and was bound by L1, not HBM).  The trajectory values of the group's rows sit in
-// shared memory.  Per output: acc = b, then acc = fma(x_i, W_i, acc) for i in order, then + pos.
+// One warp per group of kEmbRows consecutive token rows and one 128-column slice (blockIdx.y): each
+// lane loads the embedding weights of its float4 column once and applies them to every video (or
+// action) row of the group, so the weight reads from L1 shrink by the group size (one warp per row
+// read 16 weight values per output value and was bound by L1, not HBM).  The trajectory values of
+// the group's rows sit in shared memory; the slice-0 warps record them in the stage history.  Per
+// output: acc = b, then acc = fma(x_i, W_i, acc) for i in order, then + pos.
 constexpr int kEmbRows = 8;
 
 __global__ void __launch_bounds__(256) embed_kernel(
@@ -194,8 +212,10 @@ __global__ void __launch_bounds__(256) embed_kernel(
                                       : static_cast<int64_t>(Nv) * vd + static_cast<int64_t>(n - No - Nv) * ad);
       if (i < in_dim) {
         v = x[xoff + i];
-        const int stage = items[(row0 + r) / N].stage;
-        xhist[static_cast<int64_t>(stage) * stage_stride + xoff + i] = v;
+        if (blockIdx.y == 0) {
+          const int stage = items[(row0 + r) / N].stage;
+          xhist[static_cast<int64_t>(stage) * stage_stride + xoff + i] = v;
+        }
       }
     }
     xs[wib][r][i] = v;
@@ -207,7 +227,8 @@ __global__ void __launch_bounds__(256) embed_kernel(
   }
   __syncwarp();
   const int d4 = d / 4;
-  for (int c = lane; c < d4; c += 32) {
+  const int c = blockIdx.y * 32 + lane;
+  if (c < d4) {
 #pragma unroll
     for (int r = 0; r < kEmbRows; ++r) {
       if (rinfo[wib][r][0] != 0) continue;
@@ -1134,7 +1155,7 @@ cudaError_t embed_tokens(float* h, float* xhist, int64_t stage_stride, const Ste
   if (Bw <= 0) return cudaSuccess;
   const int64_t rows = static_cast<int64_t>(Bw) * (No + Nv + Na);
   const int64_t groups = (rows + kEmbRows - 1) / kEmbRows;
-  launch_pdl(embed_kernel, dim3(row_blocks(groups)), dim3(32 * kRowWarps), 0, s, h, xhist, stage_stride, items, x, T,
+  launch_pdl(embed_kernel, dim3(row_blocks(groups), (d / 4 + 31) / 32), dim3(32 * kRowWarps), 0, s, h, xhist, stage_stride, items, x, T,
                                                            obs_emb, vid_w, vid_b, act_w, act_b,
                                                            pos, Bw, No, Nv, vd, Na, ad, d);
   return cudaGetLastError();

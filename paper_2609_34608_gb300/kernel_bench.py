@@ -1,7 +1,7 @@
 """Single-kernel timing through the C ABI (include/wam_ops.h), for kernel tuning and ncu captures.
 
     python -m paper_2609_34608_gb300.kernel_bench gemm M N K [--iters I]
-    python -m paper_2609_34608_gb300.kernel_bench attn B N H [--iters I] [--impl tc|mma]
+    python -m paper_2609_34608_gb300.kernel_bench attn B N H [--iters I] [--impl tc|mma] [--head-dim 64|72]
     python -m paper_2609_34608_gb300.kernel_bench step CONFIG [--batch B] [--rounds R] [--relax-gate]
     python -m paper_2609_34608_gb300.kernel_bench sweep CONFIG B1 B2 ... [--relax-gate]
 
@@ -68,9 +68,11 @@ def bench_gemm(M: int, N: int, K: int, iters: int) -> dict:
     return {"kernel": "gemm_tc", "M": M, "N": N, "K": K, "us": us, "tflops": 2.0 * M * N * K / us / 1e6}
 
 
-def bench_attn(B: int, N: int, H: int, iters: int, impl: str) -> dict:
+def bench_attn(B: int, N: int, H: int, iters: int, impl: str, head_dim: int = 64) -> dict:
     dev = torch.device("cuda")
-    d = 64 * H
+    if head_dim != 64 and impl != "tc":
+        raise ValueError("the mma.sync attention takes head dim 64 only")
+    d = head_dim * H
     qkv = torch.randn(B * N, 3 * d, device=dev).to(torch.bfloat16)
     out = torch.empty(B * N, d, device=dev, dtype=torch.bfloat16)
     if impl == "tc":
@@ -80,7 +82,7 @@ def bench_attn(B: int, N: int, H: int, iters: int, impl: str) -> dict:
     else:
         fn = lambda st: W.op_attention(qkv, out, B, N, d, H, "bf16", stream=st)
     us = _time(fn, iters)
-    return {"kernel": f"attention_{impl}", "B": B, "N": N, "H": H, "us": us,
+    return {"kernel": f"attention_{impl}", "B": B, "N": N, "H": H, "head_dim": head_dim, "us": us,
             "tflops": 4.0 * B * N * N * d / us / 1e6}
 
 
@@ -169,6 +171,7 @@ def main() -> None:
     ap.add_argument("dims", nargs="+")
     ap.add_argument("--iters", type=int, default=20)
     ap.add_argument("--impl", choices=["tc", "mma"], default="tc")
+    ap.add_argument("--head-dim", type=int, choices=[64, 72], default=64)
     ap.add_argument("--batch", type=int, default=1)
     ap.add_argument("--rounds", type=int, default=1)
     ap.add_argument("--relax-gate", action="store_true")
@@ -177,7 +180,7 @@ def main() -> None:
     if a.kind == "gemm":
         print(json.dumps(bench_gemm(*map(int, a.dims), a.iters)))
     elif a.kind == "attn":
-        print(json.dumps(bench_attn(*map(int, a.dims), a.iters, a.impl)))
+        print(json.dumps(bench_attn(*map(int, a.dims), a.iters, a.impl, a.head_dim)))
     elif a.kind == "sweep":
         for row in bench_sweep(a.dims[0], [int(b) for b in a.dims[1:]], a.relax_gate):
             print(json.dumps(row))
