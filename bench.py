@@ -81,23 +81,33 @@ def job_throughput(units_per_rank: int, world: int, ms: float) -> float:
     return units_per_rank * world / (ms * 1e-3)
 
 
-def kernel_table(prof: dict, units: int, peaks: dict, tensor_peak: str = "bf16") -> dict:
+def kernel_table(prof: dict, units: int, peaks: dict, tensor_peak: str = "bf16", step_ms: float | None = None) -> dict:
     """Per kernel class: time per unit, share, and achieved rate against the measured peak
     (TFLOP/s for the tensor-core classes, GB/s of algorithmic bytes for the HBM-bound ones).
-    `tensor_peak` is "bf16" (burst: a step of a few ms) or "bf16_sus" (seconds-long runs)."""
+    `tensor_peak` is "bf16" (burst: a step of a few ms) or "bf16_sus" (seconds-long runs).
+    The profiled pass brackets every launch with CUDA events, which serialises launches that
+    would otherwise overlap their prologues, so its spans add up to more than an un-instrumented
+    unit; with `step_ms` (the un-instrumented time per unit) each class also gets its share of
+    that time (`ms_in_step`, which sum to step_ms) and the rate over it (`*_in_step`)."""
     tot = sum(v["ms"] for v in prof.values())
     out = {}
     for k, v in prof.items():
         if v["launches"] == 0:
             continue
         row = {"ms_per_unit": v["ms"] / units, "share": v["ms"] / tot if tot else 0.0, "launches": v["launches"]}
-        if v["ms"] > 0:
+        spans = [("", v["ms"] / units)]
+        if step_ms is not None:
+            row["ms_in_step"] = row["share"] * step_ms
+            spans.append(("_in_step", row["ms_in_step"]))
+        for suffix, ms in spans:
+            if ms <= 0:
+                continue
             if k in TENSOR_CLASSES:
-                row["tflops"] = v["flops"] / (v["ms"] * 1e-3) / 1e12
-                row["frac"] = row["tflops"] / peaks[tensor_peak]
+                row["tflops" + suffix] = v["flops"] / units / (ms * 1e-3) / 1e12
+                row["frac" + suffix] = row["tflops" + suffix] / peaks[tensor_peak]
             else:
-                row["gbs"] = v["bytes"] / (v["ms"] * 1e-3) / 1e9
-                row["frac"] = row["gbs"] / peaks["hbm"]
+                row["gbs" + suffix] = v["bytes"] / units / (ms * 1e-3) / 1e9
+                row["frac" + suffix] = row["gbs" + suffix] / peaks["hbm"]
         out[k] = row
     return out
 
@@ -535,14 +545,14 @@ def main_ours(args):
     if rank != 0:
         return 0
     peaks = _peaks()
-    kt = kernel_table(prof, nprof, peaks)
+    kt = kernel_table(prof, nprof, peaks, step_ms=total_ms / args.steps)
     g = prof["gemm"]
     # The per-launch events of the profiled pass stretch every kernel (they serialise the
     # launches); the GEMM class's rate is taken from its share of that pass applied to the
     # un-instrumented step time.
     gemm_flops_step = g["flops"] / nprof
-    gemm_ms_step = kt["gemm"]["share"] * total_ms / args.steps
-    gemm_tflops = gemm_flops_step / (gemm_ms_step * 1e-3) / 1e12
+    gemm_ms_step = kt["gemm"]["ms_in_step"]
+    gemm_tflops = kt["gemm"]["tflops_in_step"]
     value = job_throughput(args.steps, world, total_ms)
     accepted = [r for r in rr_log if r["rr_attempt"]]
     line = {

@@ -85,7 +85,9 @@ struct TileCfg {
   static constexpr int kStages = (192 * 1024) / kStageBytes;    // 2 .. 8
   static constexpr int kTmemCols = 2 * BN;
   static constexpr int kBarrierBytes = 256;
-  static constexpr int kSmemBytes = kStages * kStageBytes + kBarrierBytes + 1024;
+  // the epilogue's staged bias and gate row of a tile, one copy per TMEM accumulator
+  static constexpr int kEpiStageBytes = 2 * 2 * BN * 4;
+  static constexpr int kSmemBytes = kStages * kStageBytes + kBarrierBytes + kEpiStageBytes + 1024;
   static_assert(kStages >= 2 && kStages <= 8, "stage count");
   static_assert((2 * kStages + 7) * 8 + 12 <= kBarrierBytes, "barrier block");
 };
@@ -116,6 +118,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(rbar + 1);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
   volatile int* last_flag = abort_flag + 1;
+  float* epi_stage = reinterpret_cast<float*>(reinterpret_cast<uint8_t*>(bars) + C::kBarrierBytes);
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
@@ -324,9 +327,41 @@ __global__ void __launch_bounds__(kThreads, 1)
       return r;
     };
     const int r_local = quarter * 32 + lane;   // tile row of this thread
+    const int t_epi = static_cast<int>(threadIdx.x) - 64;   // 0 .. 127
     for (int unit = unit0; unit < num_units; unit += unit_stride, ++it) {
       const int acc = it & 1;
       const uint32_t acc_phase = (it >> 1) & 1;
+      const int mt = unit_mt(unit);
+      const int nt = unit_nt(unit);
+      const int row = mt * kBM + r_local;
+      // Everything the tail reads besides the accumulator is fetched while the main loop runs:
+      // the tile's bias and (gated residual) the gate row of its first row's item into shared
+      // memory, and this thread's residual values of the first 64 columns into registers.
+      float* sb = epi_stage + acc * 2 * BN;   // [bias BN][gate BN]
+      int item0 = 0;
+      float4 hb0[8], hb1[8];
+      if (splits == 1) {
+        if constexpr (EPI == kEpiResidF32) {
+          item0 = (mt * kBM) / e.rows_per_item;
+          if (e.item_map != nullptr) item0 = e.item_map[item0];
+        }
+        for (int c = t_epi; c < BN; c += 128) {
+          if (e.bias != nullptr) sb[c] = e.bias[nt * BN + c];
+          if constexpr (EPI == kEpiResidF32) sb[BN + c] = e.gate[item0 * e.gate_stride + nt * BN + c];
+        }
+        if constexpr (EPI == kEpiResidF32) {
+          if (row < M) {
+            const float4* h4 = reinterpret_cast<const float4*>(static_cast<const float*>(e.C) +
+                                                               static_cast<int64_t>(row) * N + nt * BN);
+#pragma unroll
+            for (int j = 0; j < 8; ++j) {
+              hb0[j] = h4[j];
+              hb1[j] = h4[8 + j];
+            }
+          }
+        }
+        if (!ep_sync()) break;   // the staged values are visible to every epilogue thread
+      }
       // One lane waits; the warp then proceeds together (tcgen05.ld is warp-collective).
       int ok = 1;
       if (lane == 0) ok = mbar_wait(smem_u32(&tfull[acc]), acc_phase, abort_flag, dev_err) ? 1 : 0;
@@ -334,16 +369,59 @@ __global__ void __launch_bounds__(kThreads, 1)
       __syncwarp();
       if (!ok) break;
       tc_fence_after();
-      const int mt = unit_mt(unit);
-      const int nt = unit_nt(unit);
-      const int row = mt * kBM + r_local;
       const uint32_t taddr = tmem_base + (static_cast<uint32_t>(quarter * 32) << 16) + acc * BN;
       if (splits == 1) {
-#pragma unroll 1
-        for (int c = 0; c < BN / 32; ++c) {
+        int item = item0;
+        if constexpr (EPI == kEpiResidF32) {
+          if (row < M) {
+            item = row / e.rows_per_item;
+            if (e.item_map != nullptr) item = e.item_map[item];
+          }
+        }
+        const bool own_gate = EPI == kEpiResidF32 && item != item0;   // a tile spanning two items
+        EpiArgs es = e;
+        es.bias = e.bias != nullptr ? sb - nt * BN : nullptr;          // es.bias + col hits the stage
+        // the tail of one 32-column chunk; hb = this thread's residual values of it
+        auto chunk = [&](int c, const float4 (&hb)[8]) {
           uint32_t r[32];
           tmem_ld32(taddr + c * 32, r);
-          if (row < M) epilogue32<EPI>(e, N, row, nt * BN + c * 32, r);
+          if (row >= M) return;
+#pragma unroll
+          for (int half = 0; half < 2; ++half) {
+            const int col = nt * BN + c * 32 + half * 16;
+            EpiIn in;
+            if (es.bias != nullptr) {
+#pragma unroll
+              for (int j = 0; j < 4; ++j) in.b[j] = reinterpret_cast<const float4*>(es.bias + col)[j];
+            }
+            if constexpr (EPI == kEpiResidF32) {
+              const float4* g4 = own_gate ? reinterpret_cast<const float4*>(e.gate + item * e.gate_stride + col)
+                                          : reinterpret_cast<const float4*>(sb + BN + (col - nt * BN));
+#pragma unroll
+              for (int j = 0; j < 4; ++j) {
+                in.g[j] = g4[j];
+                in.h[j] = hb[half * 4 + j];
+              }
+            }
+            epi_store16<EPI>(es, N, row, col, r + half * 16, in);
+          }
+        };
+        auto reload = [&](int c, float4 (&hb)[8]) {
+          if constexpr (EPI == kEpiResidF32) {
+            if (row < M && c < BN / 32) {
+              const float4* h4 = reinterpret_cast<const float4*>(static_cast<const float*>(e.C) +
+                                                                 static_cast<int64_t>(row) * N + nt * BN + c * 32);
+#pragma unroll
+              for (int j = 0; j < 8; ++j) hb[j] = h4[j];
+            }
+          }
+        };
+#pragma unroll 1
+        for (int c = 0; c < BN / 32; c += 2) {
+          chunk(c, hb0);
+          reload(c + 2, hb0);
+          chunk(c + 1, hb1);
+          reload(c + 3, hb1);
         }
         tc_fence_before();
         mbar_arrive(smem_u32(&tempty[acc]));
