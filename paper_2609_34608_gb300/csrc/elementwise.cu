@@ -282,9 +282,18 @@ __global__ void __launch_bounds__(256) ln_mod_kernel(const float* __restrict__ h
   const int lane = threadIdx.x & 31;
   if (row >= M) return;
   const float4* hr = reinterpret_cast<const float4*>(h + row * d);
-  float4 v[NV4];
+  int item = static_cast<int>(row / rows_per_item);
+  if (item_map != nullptr) item = item_map[item];
+  const float* shift = mods + item * mod_stride + shift_off;
+  const float* scale = mods + item * mod_stride + scale_off;
+  // the row and its modulation are requested together: one memory round trip, not two
+  float4 v[NV4], sh[NV4], sc[NV4];
 #pragma unroll
-  for (int i = 0; i < NV4; ++i) v[i] = hr[lane + 32 * i];
+  for (int i = 0; i < NV4; ++i) {
+    v[i] = hr[lane + 32 * i];
+    sh[i] = *reinterpret_cast<const float4*>(shift + (lane + 32 * i) * 4);
+    sc[i] = *reinterpret_cast<const float4*>(scale + (lane + 32 * i) * 4);
+  }
   if (hcopy != nullptr) {
     float4* cr = reinterpret_cast<float4*>(hcopy + row * d);
 #pragma unroll
@@ -292,19 +301,13 @@ __global__ void __launch_bounds__(256) ln_mod_kernel(const float* __restrict__ h
   }
   float mean, rstd;
   row_stats<NV4>(v, d, mean, rstd);
-  int item = static_cast<int>(row / rows_per_item);
-  if (item_map != nullptr) item = item_map[item];
-  const float* shift = mods + item * mod_stride + shift_off;
-  const float* scale = mods + item * mod_stride + scale_off;
 #pragma unroll
   for (int i = 0; i < NV4; ++i) {
     const int c = (lane + 32 * i) * 4;
-    const float4 sh = *reinterpret_cast<const float4*>(shift + c);
-    const float4 sc = *reinterpret_cast<const float4*>(scale + c);
-    Act<TO>::store4(out + row * d + c, fmaf((v[i].x - mean) * rstd, 1.0f + sc.x, sh.x),
-                    fmaf((v[i].y - mean) * rstd, 1.0f + sc.y, sh.y),
-                    fmaf((v[i].z - mean) * rstd, 1.0f + sc.z, sh.z),
-                    fmaf((v[i].w - mean) * rstd, 1.0f + sc.w, sh.w));
+    Act<TO>::store4(out + row * d + c, fmaf((v[i].x - mean) * rstd, 1.0f + sc[i].x, sh[i].x),
+                    fmaf((v[i].y - mean) * rstd, 1.0f + sc[i].y, sh[i].y),
+                    fmaf((v[i].z - mean) * rstd, 1.0f + sc[i].z, sh[i].z),
+                    fmaf((v[i].w - mean) * rstd, 1.0f + sc[i].w, sh[i].w));
   }
 }
 

@@ -103,8 +103,6 @@ struct wam_ctx {
   float *t1 = nullptr, *cvec = nullptr, *mods = nullptr;
   StepItem* d_items = nullptr;
   int* d_map = nullptr;
-  // conditioning once per distinct sigma of a step: those items, their modulation rows, and the
-  // work item -> distinct sigma index used to broadcast the rows
   // fused row-chain kernel (dit_chain.cu), off unless enabled: for bf16 models with the
   // tensor-core attention when a layer range covers at most kChainMaxRows rows; its completion
   // counters
@@ -143,6 +141,9 @@ struct wam_ctx {
   bool graphs_ok = true;
   std::map<std::tuple<int, int, int, const void*, const void*, int>, cudaGraphExec_t> layer_graphs;
   std::map<std::tuple<int, int, int, const void*, const void*, int>, int> layer_graph_uses;
+  // conditioning once per distinct sigma of a call: those sigmas (capacity Ucap = max(batch,
+  // steps)), their modulation rows, and the work item -> row index a step gathers with
+  int Ucap = 0;
   StepItem* d_uitems = nullptr;
   int* d_uidx = nullptr;
   float* mods_u = nullptr;
@@ -725,6 +726,49 @@ int run_steps(wam_ctx* c, wam_state* st, const std::vector<int>& n) {
   st->log.clear();
   std::vector<StepItem> items, uitems;
   std::vector<int> uidx;
+  // The conditioning depends on sigma alone (exact equality: equal sigmas give bit-identical
+  // modulations), and every stage each episode runs in this call is known now, so one pass over
+  // the conditioning weights computes the modulation rows of all distinct sigmas of the call;
+  // each step then gathers its work items' rows (none to gather with one item and one sigma).
+  for (int b = 0; b < B; ++b)
+    for (int j = 0; j < n[b]; ++j) {
+      const int k = st->meta[b].stage + j;
+      if (k < 0 || k >= c->K) continue;
+      bool seen = false;
+      for (const StepItem& u : uitems) seen = seen || u.sigma == c->sigma[k];
+      if (seen) continue;
+      StepItem it;
+      it.ep = b;
+      it.stage = k;
+      it.sigma = c->sigma[k];
+      it.dsigma = c->sigma[k + 1] - c->sigma[k];
+      uitems.push_back(it);
+    }
+  const int U = static_cast<int>(uitems.size());
+  if (U > c->Ucap) return fail(c, WAM_ERR_INVALID_ARG, "more distinct noise levels than denoising steps");
+  const bool cond_in_place = B == 1 && U == 1;
+  if (U > 0) {
+    TRY(upload(c, c->d_uitems, uitems.data(), sizeof(StepItem) * U));
+    float* cond_out = cond_in_place ? c->mods : c->mods_u;
+    // features -> W1 (split K) -> SiLU -> W2 (split K) -> SiLU -> every layer's modulation; each
+    // stage reduces the previous stage's K-split partial rows in a fixed order
+    {
+      Span sp(c, WAM_KCLASS_COND, 2.0 * U * 256 * d, 4.0 * 256 * d);
+      const CondGemv g{nullptr, 0, nullptr, 0, 1, c->d_uitems, c->t_w1, false, 256, d, U, kT1Splits, c->t1, nullptr};
+      CK(cond_gemv(g, c->stream));
+    }
+    {
+      Span sp(c, WAM_KCLASS_COND, 2.0 * U * d * d, 4.0 * d * d);
+      const CondGemv g{c->t1, kT1Splits, c->t_b1, 1, 0, c->d_uitems, c->t_w2, false, d, d, U, kT2Splits, c->cvec, nullptr};
+      CK(cond_gemv(g, c->stream));
+    }
+    {
+      Span sp(c, WAM_KCLASS_COND, 2.0 * U * d * c->mod_n, (c->bf16 ? 2.0 : 4.0) * d * c->mod_n);
+      const CondGemv g{c->cvec, kT2Splits, c->t_b2, 1, 0, c->d_uitems, c->mod_w, c->bf16, d, static_cast<int>(c->mod_n),
+                       U, 1, cond_out, c->mod_b};
+      CK(cond_gemv(g, c->stream));
+    }
+  }
   std::vector<int> rr_path, gate_ok;
   std::vector<RRGate> gates(2 * B);
   std::vector<RRApply> ap(B);
@@ -743,44 +787,18 @@ int run_steps(wam_ctx* c, wam_state* st, const std::vector<int>& n) {
     }
     const int Bw = static_cast<int>(items.size());
     TRY(upload(c, c->d_items, items.data(), sizeof(StepItem) * Bw));
-    // The conditioning depends on sigma alone, so it is computed once per distinct sigma of the
-    // step (exact equality: equal sigmas give bit-identical modulations) and its rows are then
-    // broadcast to the work items that share it.
-    uitems.clear();
-    uidx.assign(Bw, 0);
-    for (int w = 0; w < Bw; ++w) {
-      int j = 0;
-      while (j < static_cast<int>(uitems.size()) && uitems[j].sigma != items[w].sigma) ++j;
-      if (j == static_cast<int>(uitems.size())) uitems.push_back(items[w]);
-      uidx[w] = j;
-    }
-    const int U = static_cast<int>(uitems.size());
-    const bool share = U < Bw;
-    const StepItem* cond_items = c->d_items;
-    if (share) {
-      TRY(upload(c, c->d_uitems, uitems.data(), sizeof(StepItem) * U));
+    // this step's modulation rows: work item w takes the call's row of its sigma
+    if (!cond_in_place) {
+      uidx.assign(Bw, 0);
+      for (int w = 0; w < Bw; ++w)
+        for (int j = 0; j < U; ++j)
+          if (uitems[j].sigma == items[w].sigma) {
+            uidx[w] = j;
+            break;
+          }
       TRY(upload(c, c->d_uidx, uidx.data(), sizeof(int) * Bw));
-      cond_items = c->d_uitems;
-    }
-    // conditioning: features -> W1 (split K) -> SiLU -> W2 (split K) -> SiLU -> every layer's
-    // modulation; each stage reduces the previous stage's K-split partial rows in a fixed order
-    {
-      Span sp(c, WAM_KCLASS_COND, 2.0 * U * 256 * d, 4.0 * 256 * d);
-      const CondGemv g{nullptr, 0, nullptr, 0, 1, cond_items, c->t_w1, false, 256, d, U, kT1Splits, c->t1, nullptr};
-      CK(cond_gemv(g, c->stream));
-    }
-    {
-      Span sp(c, WAM_KCLASS_COND, 2.0 * U * d * d, 4.0 * d * d);
-      const CondGemv g{c->t1, kT1Splits, c->t_b1, 1, 0, cond_items, c->t_w2, false, d, d, U, kT2Splits, c->cvec, nullptr};
-      CK(cond_gemv(g, c->stream));
-    }
-    {
-      Span sp(c, WAM_KCLASS_COND, 2.0 * U * d * c->mod_n,
-              (c->bf16 ? 2.0 : 4.0) * d * c->mod_n + (share ? 8.0 * Bw * c->mod_n : 0.0));
-      const CondGemv g{c->cvec, kT2Splits, c->t_b2, 1, 0, cond_items, c->mod_w, c->bf16, d, static_cast<int>(c->mod_n),
-                       U, 1, share ? c->mods_u : c->mods, c->mod_b};
-      CK(cond_gemv(g, c->stream));
-      if (share) CK(rr_gather(c->mods, c->mods_u, c->d_uidx, Bw, c->mod_n, c->stream));
+      Span sp(c, WAM_KCLASS_COND, 0.0, 8.0 * Bw * c->mod_n);
+      CK(rr_gather(c->mods, c->mods_u, c->d_uidx, Bw, c->mod_n, c->stream));
     }
     {
       Span sp(c, WAM_KCLASS_EMBED, 0.0, 4.0 * Bw * double(N) * d * 2.0);
@@ -1131,14 +1149,15 @@ int create_impl(wam_ctx* c, const wam_config* cfg, const float* weights, size_t 
   c->att = att;
   c->u = u;
   c->obs_lp = olp;
-  TRY(dalloc(c, c->allocs, &c->t1, size_t(kT1Splits) * c->Bmax * c->d));
-  TRY(dalloc(c, c->allocs, &c->cvec, size_t(kT2Splits) * c->Bmax * c->d));
+  c->Ucap = std::max(c->Bmax, c->K);
+  TRY(dalloc(c, c->allocs, &c->t1, size_t(kT1Splits) * c->Ucap * c->d));
+  TRY(dalloc(c, c->allocs, &c->cvec, size_t(kT2Splits) * c->Ucap * c->d));
   TRY(dalloc(c, c->allocs, &c->mods, size_t(c->Bmax) * c->mod_n));
   TRY(dalloc(c, c->allocs, &c->d_items, c->Bmax));
   TRY(dalloc(c, c->allocs, &c->d_map, c->Bmax));
-  TRY(dalloc(c, c->allocs, &c->d_uitems, c->Bmax));
+  TRY(dalloc(c, c->allocs, &c->d_uitems, c->Ucap));
   TRY(dalloc(c, c->allocs, &c->d_uidx, c->Bmax));
-  TRY(dalloc(c, c->allocs, &c->mods_u, size_t(c->Bmax) * c->mod_n));
+  TRY(dalloc(c, c->allocs, &c->mods_u, size_t(c->Ucap) * c->mod_n));
   TRY(dalloc(c, c->allocs, &c->d_rrapply, c->Bmax));
   TRY(dalloc(c, c->allocs, &c->d_gate, 2 * c->Bmax));
   TRY(dalloc(c, c->allocs, &c->d_adapt, c->Bmax));
