@@ -11,7 +11,11 @@
 //   warp 1      MMA issuer: one thread issues tcgen05.mma (M=128, N=BN for one-atom stages, else
 //               N=min(BN,128), K=16) and commits
 //               smem-slot / accumulator-ready mbarriers; also owns the TMEM allocation
-//   warps 2..5  epilogue: tcgen05.ld 32x32b per TMEM lane quarter, fused tail, 16-byte stores
+//   warps 2..5  epilogue: tcgen05.ld 32x32b per TMEM lane quarter (one row per lane), fused
+//               tail, then each warp's 32 x 32 block goes through a swizzled shared-memory
+//               transpose so that 8 (fp32) or 4 (bf16) lanes store each 32-column row segment.
+//               What the tail reads besides the accumulator (bias, the gate row, the residual)
+//               is fetched while the main loop still runs.
 // The accumulator is double buffered in TMEM (2 x BN columns) so the epilogue of one tile
 // overlaps the main loop of the next.
 //
@@ -85,9 +89,11 @@ struct TileCfg {
   static constexpr int kStages = (192 * 1024) / kStageBytes;    // 2 .. 8
   static constexpr int kTmemCols = 2 * BN;
   static constexpr int kBarrierBytes = 256;
-  // the epilogue's staged bias and gate row of a tile, one copy per TMEM accumulator
+  // the epilogue's staged bias and gate row of a tile, one copy per TMEM accumulator, and each
+  // epilogue warp's 32 x 32 fp32 block for the transpose ahead of the coalesced stores
   static constexpr int kEpiStageBytes = 2 * 2 * BN * 4;
-  static constexpr int kSmemBytes = kStages * kStageBytes + kBarrierBytes + kEpiStageBytes + 1024;
+  static constexpr int kEpiScratchBytes = 4 * 4096;
+  static constexpr int kSmemBytes = kStages * kStageBytes + kBarrierBytes + kEpiStageBytes + kEpiScratchBytes + 1024;
   static_assert(kStages >= 2 && kStages <= 8, "stage count");
   static_assert((2 * kStages + 7) * 8 + 12 <= kBarrierBytes, "barrier block");
 };
@@ -119,6 +125,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
   volatile int* last_flag = abort_flag + 1;
   float* epi_stage = reinterpret_cast<float*>(reinterpret_cast<uint8_t*>(bars) + C::kBarrierBytes);
+  uint8_t* epi_scratch = reinterpret_cast<uint8_t*>(epi_stage) + C::kEpiStageBytes;
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
@@ -336,7 +343,8 @@ __global__ void __launch_bounds__(kThreads, 1)
       const int row = mt * kBM + r_local;
       // Everything the tail reads besides the accumulator is fetched while the main loop runs:
       // the tile's bias and (gated residual) the gate row of its first row's item into shared
-      // memory, and this thread's residual values of the first 64 columns into registers.
+      // memory, and the residual values this thread stores in the first 64 columns into registers
+      // (in the layout of the coalesced stores: 8 lanes per 32-column row segment).
       float* sb = epi_stage + acc * 2 * BN;   // [bias BN][gate BN]
       int item0 = 0;
       float4 hb0[8], hb1[8];
@@ -350,13 +358,14 @@ __global__ void __launch_bounds__(kThreads, 1)
           if constexpr (EPI == kEpiResidF32) sb[BN + c] = e.gate[item0 * e.gate_stride + nt * BN + c];
         }
         if constexpr (EPI == kEpiResidF32) {
-          if (row < M) {
-            const float4* h4 = reinterpret_cast<const float4*>(static_cast<const float*>(e.C) +
-                                                               static_cast<int64_t>(row) * N + nt * BN);
 #pragma unroll
-            for (int j = 0; j < 8; ++j) {
-              hb0[j] = h4[j];
-              hb1[j] = h4[8 + j];
+          for (int i = 0; i < 8; ++i) {
+            const int trow = mt * kBM + quarter * 32 + i * 4 + (lane >> 3);
+            if (trow < M) {
+              const float4* h4 = reinterpret_cast<const float4*>(static_cast<const float*>(e.C) +
+                                                                 static_cast<int64_t>(trow) * N + nt * BN) + (lane & 7);
+              hb0[i] = h4[0];
+              hb1[i] = h4[8];
             }
           }
         }
@@ -371,48 +380,138 @@ __global__ void __launch_bounds__(kThreads, 1)
       tc_fence_after();
       const uint32_t taddr = tmem_base + (static_cast<uint32_t>(quarter * 32) << 16) + acc * BN;
       if (splits == 1) {
-        int item = item0;
-        if constexpr (EPI == kEpiResidF32) {
-          if (row < M) {
-            item = row / e.rows_per_item;
-            if (e.item_map != nullptr) item = e.item_map[item];
-          }
-        }
-        const bool own_gate = EPI == kEpiResidF32 && item != item0;   // a tile spanning two items
         EpiArgs es = e;
         es.bias = e.bias != nullptr ? sb - nt * BN : nullptr;          // es.bias + col hits the stage
-        // the tail of one 32-column chunk; hb = this thread's residual values of it
+        uint8_t* wscr = epi_scratch + (warp - 2) * 4096;               // this warp's transpose block
+        const int row0 = mt * kBM + quarter * 32;                       // first row of this warp
+        // every row of this warp belongs to the item whose gate row was staged
+        bool one_item = true;
+        if constexpr (EPI == kEpiResidF32) {
+          const int last = (row0 + 31 < M ? row0 + 31 : M - 1);
+          one_item = (mt * kBM) / e.rows_per_item == last / e.rows_per_item;
+        }
+        // The tail of one 32-column chunk.  The accumulator arrives one row per lane; the stores
+        // leave one 32 x 32 block per warp through shared memory so that 8 (fp32) or 4 (bf16)
+        // lanes write each row segment, i.e. whole cache lines per store instruction.  Both
+        // shared-memory passes use a 16-byte-piece XOR swizzle: conflict-free.  hb = the residual
+        // values of this chunk in the store layout.
         auto chunk = [&](int c, const float4 (&hb)[8]) {
           uint32_t r[32];
           tmem_ld32(taddr + c * 32, r);
-          if (row >= M) return;
+          const int col_c = nt * BN + c * 32;
+          if constexpr (EPI == kEpiResidF32 || EPI == kEpiF32) {
 #pragma unroll
-          for (int half = 0; half < 2; ++half) {
-            const int col = nt * BN + c * 32 + half * 16;
-            EpiIn in;
-            if (es.bias != nullptr) {
+            for (int pc = 0; pc < 8; ++pc)
+              *reinterpret_cast<uint4*>(wscr + lane * 128 + ((pc ^ (lane & 7)) * 16)) =
+                  make_uint4(r[4 * pc], r[4 * pc + 1], r[4 * pc + 2], r[4 * pc + 3]);
+            __syncwarp();
+            const int pc = lane & 7;
+            float4 vv[8];
 #pragma unroll
-              for (int j = 0; j < 4; ++j) in.b[j] = reinterpret_cast<const float4*>(es.bias + col)[j];
+            for (int i = 0; i < 8; ++i) {
+              const int rr = i * 4 + (lane >> 3);
+              vv[i] = *reinterpret_cast<const float4*>(wscr + rr * 128 + ((pc ^ (rr & 7)) * 16));
             }
-            if constexpr (EPI == kEpiResidF32) {
-              const float4* g4 = own_gate ? reinterpret_cast<const float4*>(e.gate + item * e.gate_stride + col)
-                                          : reinterpret_cast<const float4*>(sb + BN + (col - nt * BN));
+            __syncwarp();   // the block is free for the next chunk
+            float4 b4 = make_float4(0.0f, 0.0f, 0.0f, 0.0f);
+            if (es.bias != nullptr) b4 = *reinterpret_cast<const float4*>(es.bias + col_c + pc * 4);
+            float4 g0 = make_float4(0.0f, 0.0f, 0.0f, 0.0f);
+            if constexpr (EPI == kEpiResidF32) g0 = *reinterpret_cast<const float4*>(sb + BN + c * 32 + pc * 4);
 #pragma unroll
-              for (int j = 0; j < 4; ++j) {
-                in.g[j] = g4[j];
-                in.h[j] = hb[half * 4 + j];
+            for (int i = 0; i < 8; ++i) {
+              const int grow = row0 + i * 4 + (lane >> 3);
+              float4 v = vv[i];
+              if (grow < M) {
+                if (es.bias != nullptr) {
+                  v.x += b4.x;
+                  v.y += b4.y;
+                  v.z += b4.z;
+                  v.w += b4.w;
+                }
+                float4* dst = reinterpret_cast<float4*>(static_cast<float*>(e.C) + static_cast<int64_t>(grow) * N + col_c) + pc;
+                if constexpr (EPI == kEpiResidF32) {
+                  float4 g = g0;
+                  if (!one_item) {
+                    int item = grow / e.rows_per_item;
+                    if (e.item_map != nullptr) item = e.item_map[item];
+                    if (item != item0) g = __ldg(reinterpret_cast<const float4*>(e.gate + item * e.gate_stride + col_c) + pc);
+                  }
+                  float4 h = hb[i];
+                  h.x = fmaf(g.x, v.x, h.x);
+                  h.y = fmaf(g.y, v.y, h.y);
+                  h.z = fmaf(g.z, v.z, h.z);
+                  h.w = fmaf(g.w, v.w, h.w);
+                  *dst = h;
+                } else {
+                  *dst = v;
+                }
               }
             }
-            epi_store16<EPI>(es, N, row, col, r + half * 16, in);
+          } else {
+            const int d3 = N / 3;
+            if (EPI == kEpiQkvVt && col_c >= 2 * d3) {
+              // V columns: written transposed into V^T straight from the row layout (lanes hold
+              // consecutive tokens, so each store instruction covers 64 contiguous bytes)
+              if (row < M) {
+#pragma unroll
+                for (int half = 0; half < 2; ++half) {
+                  EpiIn in;
+                  if (es.bias != nullptr) {
+#pragma unroll
+                    for (int j = 0; j < 4; ++j) in.b[j] = reinterpret_cast<const float4*>(es.bias + col_c + half * 16)[j];
+                  }
+                  epi_store16<EPI>(es, N, row, col_c + half * 16, r + half * 16, in);
+                }
+              }
+              return;
+            }
+            float v[32];
+#pragma unroll
+            for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
+            if (es.bias != nullptr) {
+#pragma unroll
+              for (int j = 0; j < 8; ++j) {
+                const float4 b = reinterpret_cast<const float4*>(es.bias + col_c)[j];
+                v[4 * j] += b.x;
+                v[4 * j + 1] += b.y;
+                v[4 * j + 2] += b.z;
+                v[4 * j + 3] += b.w;
+              }
+            }
+            if constexpr (EPI == kEpiGeluBf16) {
+#pragma unroll
+              for (int i = 0; i < 32; ++i) v[i] = gelu_tanh_bf16tail(v[i]);
+            }
+#pragma unroll
+            for (int pc = 0; pc < 4; ++pc)
+              *reinterpret_cast<uint4*>(wscr + lane * 64 + ((pc ^ ((lane >> 1) & 3)) * 16)) = pack_bf16x8(v + 8 * pc);
+            __syncwarp();
+            const int pc = lane & 3;
+            uint4 uu[4];
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+              const int rr = i * 8 + (lane >> 2);
+              uu[i] = *reinterpret_cast<const uint4*>(wscr + rr * 64 + ((pc ^ ((rr >> 1) & 3)) * 16));
+            }
+            __syncwarp();   // the block is free for the next chunk
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+              const int grow = row0 + i * 8 + (lane >> 2);
+              if (grow < M)
+                reinterpret_cast<uint4*>(static_cast<bf16*>(e.C) + static_cast<int64_t>(grow) * N + col_c)[pc] = uu[i];
+            }
           }
         };
         auto reload = [&](int c, float4 (&hb)[8]) {
           if constexpr (EPI == kEpiResidF32) {
-            if (row < M && c < BN / 32) {
-              const float4* h4 = reinterpret_cast<const float4*>(static_cast<const float*>(e.C) +
-                                                                 static_cast<int64_t>(row) * N + nt * BN + c * 32);
+            if (c < BN / 32) {
 #pragma unroll
-              for (int j = 0; j < 8; ++j) hb[j] = h4[j];
+              for (int i = 0; i < 8; ++i) {
+                const int trow = row0 + i * 4 + (lane >> 3);
+                if (trow < M)
+                  hb[i] = reinterpret_cast<const float4*>(static_cast<const float*>(e.C) + static_cast<int64_t>(trow) * N +
+                                                          nt * BN + c * 32)[lane & 7];
+              }
             }
           }
         };
