@@ -140,9 +140,12 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int num_units = MC == 2 ? num_mn / 2 : num_mn * splits;
   const int unit0 = MC == 2 ? static_cast<int>(blockIdx.x) / 2 : static_cast<int>(blockIdx.x);
   const int unit_stride = MC == 2 ? static_cast<int>(gridDim.x) / 2 : static_cast<int>(gridDim.x);
-  // unit u: output tile mn = u % num_mn (m fastest), K range u / num_mn
-  auto unit_mt = [&](int u) { return MC == 2 ? u % num_m : (u % num_mn) % num_m; };
-  auto unit_nt = [&](int u) { return MC == 2 ? 2 * (u / num_m) + rank : (u % num_mn) / num_m; };
+  // unit u: output tile mn = u % num_mn, K range u / num_mn.  Column tiles vary fastest, so the
+  // CTAs running at the same time share A row blocks (each read from DRAM about once) while the
+  // weight matrix, a few MB, stays in L2; with rows fastest a tall activation operand was
+  // streamed from DRAM once per column tile.
+  auto unit_mt = [&](int u) { return MC == 2 ? u / (num_n / 2) : (u % num_mn) / num_n; };
+  auto unit_nt = [&](int u) { return MC == 2 ? 2 * (u % (num_n / 2)) + rank : (u % num_mn) % num_n; };
   auto unit_kb0 = [&](int u) { return MC == 2 ? 0 : (u / num_mn) * num_k; };
   // A tile of a stage: one request per operand (MC = 1), or this CTA's 64-row half of each K-atom
   // multicast to both CTAs (the other half arrives from the peer)
