@@ -47,8 +47,11 @@ int wam_op_gemm_bf16(const void* A, const void* Wt, const float* bias, void* C, 
  *   cluster    0 = the library's rule, 1 = single CTAs, 2 = clusters of two CTAs on adjacent
  *              column tiles of the same row block, each loading half of the shared A tile with
  *              TMA multicast into both (64- / 128-wide tiles, an even number of column tiles,
- *              K % 128 == 0, no K split; otherwise single CTAs).  The accumulation order is the
- *              same either way.
+ *              K % 128 == 0, no K split; otherwise single CTAs); 3 = pairs of CTAs (a cluster of
+ *              two) running one 256-row MMA (tcgen05 cta_group::2): each CTA loads 128 rows of A and
+ *              tile_n / 2 rows of the weight and holds its 128 x tile_n accumulator (tile_n 128 or
+ *              256, K % 128 == 0, no K split; WAM_ERR_UNSUPPORTED otherwise).  The accumulation
+ *              order over K is the same for every choice.
  *   workspace  device buffer of wam_op_gemm_workspace_bytes() bytes, 16-byte aligned, zero-filled
  *              before its first use (every call leaves it reusable); NULL = no splitting.  Calls
  *              sharing a workspace must be ordered (same stream).

@@ -71,21 +71,103 @@ WAM_DEV void umma_commit_mc(uint32_t bar, uint16_t cta_mask) {
       : "memory");
 }
 
+// ---- two-SM (CTA pair) MMA helpers ----
+// The shared::cluster address of offset `saddr` in the shared memory of cluster CTA `rank`.
+WAM_DEV uint32_t cluster_addr(uint32_t saddr, uint32_t rank) {
+  uint32_t r;
+  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(saddr), "r"(rank));
+  return r;
+}
+// TMA loads into this CTA's shared memory whose completion is signalled on an mbarrier of either
+// CTA of the pair (`bar`: a shared::cluster address), so the pair's first CTA sees both halves.
+WAM_DEV void tma_load_2d_pair(uint32_t dst, const CUtensorMap* map, int x, int y, uint32_t bar) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.cta_group::2.shared::cluster.global.mbarrier::complete_tx::bytes"
+      " [%0], [%1, {%2, %3}], [%4];" ::"r"(dst),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(bar)
+      : "memory");
+}
+WAM_DEV void tma_load_3d_pair(uint32_t dst, const CUtensorMap* map, int x, int y, int z, uint32_t bar) {
+  asm volatile(
+      "cp.async.bulk.tensor.3d.cta_group::2.shared::cluster.global.mbarrier::complete_tx::bytes"
+      " [%0], [%1, {%2, %3, %4}], [%5];" ::"r"(dst),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(z), "r"(bar)
+      : "memory");
+}
+// One MMA of the pair, issued by its first CTA: D is 256 x N, rows 0..127 in the first CTA's TMEM
+// and rows 128..255 in the second's (same TMEM address); A rows 0..127 / 128..255 and B columns
+// 0..N/2-1 / N/2..N-1 are read at the same shared-memory offsets of the first / second CTA.
+WAM_DEV void umma_bf16_pair(uint32_t d_tmem, uint64_t a, uint64_t b, uint32_t idesc, uint32_t acc) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "setp.ne.b32 p, %4, 0;\n\t"
+      "tcgen05.mma.cta_group::2.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
+      "l"(a), "l"(b), "r"(idesc), "r"(acc)
+      : "memory");
+}
+// Arrive on the mbarrier at offset `bar` of every CTA in cta_mask once the pair's MMAs issued by
+// this thread completed.
+WAM_DEV void umma_commit_pair_mc(uint32_t bar, uint16_t cta_mask) {
+  asm volatile(
+      "tcgen05.commit.cta_group::2.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64 [%0], %1;" ::"r"(bar),
+      "h"(cta_mask)
+      : "memory");
+}
+WAM_DEV void umma_commit_pair(uint32_t bar) {
+  asm volatile("tcgen05.commit.cta_group::2.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(bar) : "memory");
+}
+// Arrive (release, cluster scope) on an mbarrier given by its shared::cluster address.
+WAM_DEV void mbar_arrive_cluster(uint32_t cbar) {
+  asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];" ::"r"(cbar) : "memory");
+}
+// Bounded wait (as mbar_wait) with cluster-scope acquire: for barriers the peer CTA arrives on.
+WAM_DEV bool mbar_wait_cluster(uint32_t bar, uint32_t parity, volatile int* abort_flag, int* dev_err) {
+  auto try_wait = [&]() -> bool {
+    uint32_t ok;
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "mbarrier.try_wait.parity.acquire.cluster.shared::cta.b64 p, [%1], %2;\n\t"
+        "selp.u32 %0, 1, 0, p;\n\t}"
+        : "=r"(ok)
+        : "r"(bar), "r"(parity)
+        : "memory");
+    return ok != 0;
+  };
+  if (try_wait()) return true;
+  const uint64_t t0 = globaltimer_ns();
+  for (uint32_t i = 1;; ++i) {
+    if (try_wait()) return true;
+    if ((i & 63u) == 0) {
+      if (*abort_flag) return false;
+      if (globaltimer_ns() - t0 > kWaitLimitNs) {
+        *abort_flag = 1;
+        if (dev_err != nullptr) atomicOr(dev_err, kDevErrTimeout);
+        return false;
+      }
+    }
+  }
+}
+
 constexpr int kBM = 128;
 constexpr int kBK = 64;           // 64 bf16 = 128 bytes = one swizzle row
 constexpr int kThreads = 192;
 constexpr int kTileBytesA = kBM * kBK * 2;  // 16 KB
 constexpr int kBoxRows = 128;               // TMA box rows of the A operand and wide B tiles
 
-template <int BN, int KA>
+// CG = 2: a CTA pair runs one 256-row MMA (tcgen05 cta_group::2); each CTA holds 128 rows of A,
+// BN / 2 rows of B and its 128 rows x BN columns of the accumulator.
+template <int BN, int KA, int CG = 1>
 struct TileCfg {
-  static constexpr int kBoxB = BN < kBoxRows ? BN : kBoxRows;  // rows per B request
+  static constexpr int kBRows = BN / CG;                        // B rows this CTA loads
+  static constexpr int kBoxB = kBRows < kBoxRows ? kBRows : kBoxRows;  // rows per B request
   // One atom per stage: the B boxes lie back to back, so one MMA spans all BN columns.  Two atoms:
-  // each box holds both atoms of its rows ([atom][rows]), so each box gets its own MMA.
-  static constexpr int kMmaN = KA == 1 ? BN : kBoxB;
+  // each box holds both atoms of its rows ([atom][rows]), so each box gets its own MMA.  A pair's
+  // B half is one box, and one MMA spans both halves.
+  static constexpr int kMmaN = (KA == 1 || CG == 2) ? BN : kBoxB;
   static constexpr int kBytesA = KA * kTileBytesA;              // [KA atoms][128 rows][128 B]
   static constexpr int kBoxBytesB = KA * kBoxB * kBK * 2;       // [KA atoms][kBoxB rows][128 B]
-  static constexpr int kStageBytes = kBytesA + (BN / kBoxB) * kBoxBytesB;
+  static constexpr int kStageBytes = kBytesA + (kBRows / kBoxB) * kBoxBytesB;
+  static_assert(CG == 1 || (CG == 2 && kBRows == kBoxB && BN <= 256), "a pair's B half is one box");
   static constexpr int kStages = (192 * 1024) / kStageBytes;    // 2 .. 8
   static constexpr int kTmemCols = 2 * BN;
   static constexpr int kBarrierBytes = 256;
@@ -104,12 +186,15 @@ struct SplitArgs {
   int* counters;    // [tiles] tickets, zero between launches
 };
 
-template <int BN, int EPI, int KA, int MC>
+template <int BN, int EPI, int KA, int MC, int CG = 1>
 __global__ void __launch_bounds__(kThreads, 1)
     gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                    int M, int N, int K, EpiArgs e, SplitArgs sp, int* dev_err) {
-  using C = TileCfg<BN, KA>;
+  using C = TileCfg<BN, KA, CG>;
   static_assert(MC == 1 || MC == 2, "cluster size");
+  static_assert(CG == 1 || (CG == 2 && MC == 1), "CTA-pair MMAs do not combine with multicast clusters");
+  constexpr bool kPair = CG == 2;
+  constexpr int kRowsPerUnit = kBM * CG;   // output rows of a work unit
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint8_t* tiles = smem;
@@ -129,17 +214,24 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
-  const int num_m = (M + kBM - 1) / kBM;
+  const int num_m = (M + kRowsPerUnit - 1) / kRowsPerUnit;
   const int num_n = N / BN;
   const int num_mn = num_m * num_n;
   const int splits = sp.splits;
   const int num_k = K / (kBK * KA) / splits;   // stages per work unit
   // With clusters a unit is a pair of adjacent column tiles of one row block, one per CTA; the
   // cluster walks the units (first = cluster index, stride = clusters), both CTAs in lockstep.
-  const int rank = MC == 2 ? static_cast<int>(cluster_rank()) : 0;
+  // With CTA pairs (CG = 2) a unit is a 256-row x BN tile: this CTA holds its rows
+  // [128 rank, 128 rank + 128) and loads B rows [rank BN/2, (rank + 1) BN/2) of the column tile;
+  // the pair walks the units in lockstep like a cluster.
+  const int rank = (MC == 2 || kPair) ? static_cast<int>(cluster_rank()) : 0;
   const int num_units = MC == 2 ? num_mn / 2 : num_mn * splits;
-  const int unit0 = MC == 2 ? static_cast<int>(blockIdx.x) / 2 : static_cast<int>(blockIdx.x);
-  const int unit_stride = MC == 2 ? static_cast<int>(gridDim.x) / 2 : static_cast<int>(gridDim.x);
+  const int unit0 = (MC == 2 || kPair) ? static_cast<int>(blockIdx.x) / 2 : static_cast<int>(blockIdx.x);
+  const int unit_stride = (MC == 2 || kPair) ? static_cast<int>(gridDim.x) / 2 : static_cast<int>(gridDim.x);
+  const bool leader = !kPair || rank == 0;   // the CTA that issues a pair's MMAs
+  const int b_row_off = kPair ? rank * C::kBRows : 0;
+  // first output (and A) row of unit tile row mt held by this CTA
+  auto tile_row = [&](int mt) { return mt * kRowsPerUnit + (kPair ? rank * kBM : 0); };
   // unit u: output tile mn = u % num_mn, K range u / num_mn.  Column tiles vary fastest, so the
   // CTAs running at the same time share A row blocks (each read from DRAM about once) while the
   // weight matrix, a few MB, stays in L2; with rows fastest a tall activation operand was
@@ -150,7 +242,12 @@ __global__ void __launch_bounds__(kThreads, 1)
   // A tile of a stage: one request per operand (MC = 1), or this CTA's 64-row half of each K-atom
   // multicast to both CTAs (the other half arrives from the peer)
   auto load_a = [&](uint32_t dst, const CUtensorMap* map, int row, int atom, uint32_t bar) {
-    if constexpr (MC == 1) {
+    if constexpr (kPair) {
+      if constexpr (KA == 1)
+        tma_load_2d_pair(dst, map, atom * kBK, row, bar);
+      else
+        tma_load_3d_pair(dst, map, 0, row, atom, bar);
+    } else if constexpr (MC == 1) {
       if constexpr (KA == 1)
         tma_load_2d(dst, map, atom * kBK, row, bar);
       else
@@ -165,10 +262,16 @@ __global__ void __launch_bounds__(kThreads, 1)
   // K-atoms [atom, atom + KA) of rows [row, row + box): one 2-D box {64, rows} for one atom, one
   // 3-D box {64, rows, 2} for two
   auto load_k = [&](uint32_t dst, const CUtensorMap* map, int row, int atom, uint32_t bar) {
-    if constexpr (KA == 1)
+    if constexpr (kPair) {
+      if constexpr (KA == 1)
+        tma_load_2d_pair(dst, map, atom * kBK, row, bar);
+      else
+        tma_load_3d_pair(dst, map, 0, row, atom, bar);
+    } else if constexpr (KA == 1) {
       tma_load_2d(dst, map, atom * kBK, row, bar);
-    else
+    } else {
       tma_load_3d(dst, map, 0, row, atom, bar);
+    }
   };
 
   if (threadIdx.x == 0) {
@@ -178,7 +281,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     for (int a = 0; a < 2; ++a) {
       mbar_init(smem_u32(&tfull[a]), 1);
-      mbar_init(smem_u32(&tempty[a]), 128);
+      mbar_init(smem_u32(&tempty[a]), 128 * CG);   // pairs: both CTAs' epilogue threads
     }
     mbar_init(smem_u32(drain), 1);
     mbar_init(smem_u32(epbar), 128);
@@ -188,15 +291,25 @@ __global__ void __launch_bounds__(kThreads, 1)
     asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
   }
   if (warp == 1) {
-    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
-                     smem_u32(tmem_slot)),
-                 "r"(C::kTmemCols)
-                 : "memory");
-    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+    if constexpr (kPair) {
+      // one warp of each CTA of the pair allocates the same columns in both CTAs' TMEM
+      asm volatile("tcgen05.alloc.cta_group::2.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
+                       smem_u32(tmem_slot)),
+                   "r"(C::kTmemCols)
+                   : "memory");
+      asm volatile("tcgen05.relinquish_alloc_permit.cta_group::2.sync.aligned;" ::: "memory");
+    } else {
+      asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
+                       smem_u32(tmem_slot)),
+                   "r"(C::kTmemCols)
+                   : "memory");
+      asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+    }
   }
   tc_fence_before();
   __syncthreads();
-  if constexpr (MC == 2) cluster_sync();   // the peer's barriers exist before any multicast
+  // the peer's barriers exist before any multicast or any copy signalling them
+  if constexpr (MC == 2 || kPair) cluster_sync();
   tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
   pdl_launch_dependents();
@@ -209,13 +322,20 @@ __global__ void __launch_bounds__(kThreads, 1)
     // before waiting for them, overlapping the previous kernel's tail.
     const int u0 = unit0;
     const int pre = u0 < num_units ? (num_k < C::kStages ? num_k : C::kStages) : 0;
+    // A stage's copies signal its full barrier; with CTA pairs both CTAs' copies signal the first
+    // CTA's barrier, whose MMA thread consumes the stage of both, and only that CTA arms it (with
+    // the bytes of both CTAs).
+    auto full_bar = [&](int st) -> uint32_t {
+      return kPair ? cluster_addr(smem_u32(&full[st]), 0) : smem_u32(&full[st]);
+    };
     for (int s = 0; s < pre; ++s) {
-      const uint32_t fb = smem_u32(&full[s]);
+      const uint32_t fb = full_bar(s);
       const uint32_t b_dst = smem_u32(tiles + s * C::kStageBytes) + C::kBytesA;
-      mbar_expect_tx(fb, C::kStageBytes);
+      if (leader) mbar_expect_tx(smem_u32(&full[s]), CG * C::kStageBytes);
 #pragma unroll
-      for (int h = 0; h < BN / C::kBoxB; ++h)
-        load_k(b_dst + h * C::kBoxBytesB, &tmB, unit_nt(u0) * BN + h * C::kBoxB, (unit_kb0(u0) + s) * KA, fb);
+      for (int h = 0; h < C::kBRows / C::kBoxB; ++h)
+        load_k(b_dst + h * C::kBoxBytesB, &tmB, unit_nt(u0) * BN + b_row_off + h * C::kBoxB, (unit_kb0(u0) + s) * KA,
+               fb);
     }
     pdl_wait();
     int stage = 0;
@@ -234,16 +354,16 @@ __global__ void __launch_bounds__(kThreads, 1)
           ok = false;
           break;
         }
-        const uint32_t fb = smem_u32(&full[stage]);
+        const uint32_t fb = full_bar(stage);
         const uint32_t a_dst = smem_u32(tiles + stage * C::kStageBytes);
         const uint32_t b_dst = a_dst + C::kBytesA;
         if (!(first && kb < pre)) {
-          mbar_expect_tx(fb, C::kStageBytes);
+          if (leader) mbar_expect_tx(smem_u32(&full[stage]), CG * C::kStageBytes);
 #pragma unroll
-          for (int h = 0; h < BN / C::kBoxB; ++h)
-            load_k(b_dst + h * C::kBoxBytesB, &tmB, nt * BN + h * C::kBoxB, (kb0 + kb) * KA, fb);
+          for (int h = 0; h < C::kBRows / C::kBoxB; ++h)
+            load_k(b_dst + h * C::kBoxBytesB, &tmB, nt * BN + b_row_off + h * C::kBoxB, (kb0 + kb) * KA, fb);
         }
-        load_a(a_dst, &tmA, mt * kBM, (kb0 + kb) * KA, fb);
+        load_a(a_dst, &tmA, tile_row(mt), (kb0 + kb) * KA, fb);
         issued[stage] = 1;
         issued_phase[stage] = phase;
         if (++stage == C::kStages) {
@@ -253,7 +373,13 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
       first = false;
     }
-    if (!ok) {
+    if (!ok && !leader) {
+      // The second CTA of a pair cannot observe its copies (they signal the first CTA's barriers):
+      // give them time to land before the CTA releases its shared memory.
+      const uint64_t t0 = globaltimer_ns();
+      while (globaltimer_ns() - t0 < 200000ull) {
+      }
+    } else if (!ok) {
       // Drain: let every copy this thread issued land before the CTA releases its smem.
       for (int s = 0; s < C::kStages; ++s) {
         if (!issued[s]) continue;
@@ -263,10 +389,10 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
       }
     }
-  } else if (warp == 1 && lane == 0) {
-    // ---------------- MMA issuer ----------------
+  } else if (warp == 1 && lane == 0 && leader) {
+    // ---------------- MMA issuer (with CTA pairs: the first CTA's, for both) ----------------
     pdl_wait();
-    const uint32_t idesc = idesc_bf16(kBM, C::kMmaN);
+    const uint32_t idesc = idesc_bf16(kRowsPerUnit, C::kMmaN);
     int stage = 0;
     uint32_t phase = 0;
     int it = 0;
@@ -275,7 +401,9 @@ __global__ void __launch_bounds__(kThreads, 1)
     for (int unit = unit0; ok && unit < num_units; unit += unit_stride, ++it) {
       const int acc = it & 1;
       const uint32_t acc_phase = (it >> 1) & 1;
-      if (!mbar_wait(smem_u32(&tempty[acc]), acc_phase ^ 1u, abort_flag, dev_err)) {
+      const bool drained = kPair ? mbar_wait_cluster(smem_u32(&tempty[acc]), acc_phase ^ 1u, abort_flag, dev_err)
+                                 : mbar_wait(smem_u32(&tempty[acc]), acc_phase ^ 1u, abort_flag, dev_err);
+      if (!drained) {
         ok = false;
         break;
       }
@@ -296,14 +424,21 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
           for (int k = 0; k < kBK / 16; ++k) {
 #pragma unroll
-            for (int h = 0; h < BN / C::kMmaN; ++h)
-              umma_bf16(d_tmem + h * C::kMmaN, da + ((a * kTileBytesA + k * 32) >> 4),
-                        db + ((h * C::kBoxBytesB + a * C::kBoxB * 128 + k * 32) >> 4), idesc,
-                        (kb | a | k) != 0 ? 1u : 0u);
+            for (int h = 0; h < BN / C::kMmaN; ++h) {
+              if constexpr (kPair)
+                umma_bf16_pair(d_tmem, da + ((a * kTileBytesA + k * 32) >> 4), db + ((a * C::kBoxB * 128 + k * 32) >> 4),
+                               idesc, (kb | a | k) != 0 ? 1u : 0u);
+              else
+                umma_bf16(d_tmem + h * C::kMmaN, da + ((a * kTileBytesA + k * 32) >> 4),
+                          db + ((h * C::kBoxBytesB + a * C::kBoxB * 128 + k * 32) >> 4), idesc,
+                          (kb | a | k) != 0 ? 1u : 0u);
+            }
           }
         }
         issued_any = true;
-        if constexpr (MC == 2)
+        if constexpr (kPair)
+          umma_commit_pair_mc(smem_u32(&empty[stage]), 0x3);   // both CTAs' stage buffers are free
+        else if constexpr (MC == 2)
           umma_commit_mc(smem_u32(&empty[stage]), 0x3);
         else
           umma_commit(smem_u32(&empty[stage]));
@@ -313,11 +448,17 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
       }
       if (!ok) break;
-      umma_commit(smem_u32(&tfull[acc]));
+      if constexpr (kPair)
+        umma_commit_pair_mc(smem_u32(&tfull[acc]), 0x3);   // both CTAs' halves of the accumulator
+      else
+        umma_commit(smem_u32(&tfull[acc]));
     }
     if (!ok && issued_any) {
       // Drain: wait for every MMA this thread issued before TMEM is released.
-      umma_commit(smem_u32(drain));
+      if constexpr (kPair)
+        umma_commit_pair(smem_u32(drain));
+      else
+        umma_commit(smem_u32(drain));
       const uint64_t t0 = globaltimer_ns();
       while (!mbar_try_wait(smem_u32(drain), 0) && globaltimer_ns() - t0 < kWaitLimitNs) {
       }
@@ -343,7 +484,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       const uint32_t acc_phase = (it >> 1) & 1;
       const int mt = unit_mt(unit);
       const int nt = unit_nt(unit);
-      const int row = mt * kBM + r_local;
+      const int row = tile_row(mt) + r_local;
       // Everything the tail reads besides the accumulator is fetched while the main loop runs:
       // the tile's bias and (gated residual) the gate row of its first row's item into shared
       // memory, and the residual values this thread stores in the first 64 columns into registers
@@ -353,7 +494,8 @@ __global__ void __launch_bounds__(kThreads, 1)
       float4 hb0[8], hb1[8];
       if (splits == 1) {
         if constexpr (EPI == kEpiResidF32) {
-          item0 = (mt * kBM) / e.rows_per_item;
+          // (the second CTA of a pair may hold only rows past M: clamp to a real row's item)
+          item0 = (tile_row(mt) < M ? tile_row(mt) : M - 1) / e.rows_per_item;
           if (e.item_map != nullptr) item0 = e.item_map[item0];
         }
         for (int c = t_epi; c < BN; c += 128) {
@@ -363,7 +505,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         if constexpr (EPI == kEpiResidF32) {
 #pragma unroll
           for (int i = 0; i < 8; ++i) {
-            const int trow = mt * kBM + quarter * 32 + i * 4 + (lane >> 3);
+            const int trow = tile_row(mt) + quarter * 32 + i * 4 + (lane >> 3);
             if (trow < M) {
               const float4* h4 = reinterpret_cast<const float4*>(static_cast<const float*>(e.C) +
                                                                  static_cast<int64_t>(trow) * N + nt * BN) + (lane & 7);
@@ -386,12 +528,12 @@ __global__ void __launch_bounds__(kThreads, 1)
         EpiArgs es = e;
         es.bias = e.bias != nullptr ? sb - nt * BN : nullptr;          // es.bias + col hits the stage
         uint8_t* wscr = epi_scratch + (warp - 2) * 4096;               // this warp's transpose block
-        const int row0 = mt * kBM + quarter * 32;                       // first row of this warp
+        const int row0 = tile_row(mt) + quarter * 32;                       // first row of this warp
         // every row of this warp belongs to the item whose gate row was staged
         bool one_item = true;
         if constexpr (EPI == kEpiResidF32) {
           const int last = (row0 + 31 < M ? row0 + 31 : M - 1);
-          one_item = (mt * kBM) / e.rows_per_item == last / e.rows_per_item;
+          one_item = (tile_row(mt)) / e.rows_per_item == last / e.rows_per_item;
         }
         // The tail of one 32-column chunk.  The accumulator arrives one row per lane; the stores
         // leave one 32 x 32 block per warp through shared memory so that 8 (fp32) or 4 (bf16)
@@ -526,9 +668,13 @@ __global__ void __launch_bounds__(kThreads, 1)
           reload(c + 3, hb1);
         }
         tc_fence_before();
-        mbar_arrive(smem_u32(&tempty[acc]));
+        if constexpr (kPair)
+          mbar_arrive_cluster(cluster_addr(smem_u32(&tempty[acc]), 0));   // the MMA thread's barrier
+        else
+          mbar_arrive(smem_u32(&tempty[acc]));
         continue;
       }
+      if constexpr (kPair) break;   // pairs never split K
       // ---- K split: publish this unit's partial, then the last unit of the tile finishes it ----
       const int mn = unit % num_mn;
       const int ks = unit / num_mn;
@@ -598,13 +744,17 @@ __global__ void __launch_bounds__(kThreads, 1)
   tc_fence_before();
   __syncthreads();
   // no CTA of a cluster leaves while its peer may still multicast into it or arrive on its barriers
-  if constexpr (MC == 2) cluster_sync();
+  // (pairs: nor while the first CTA's MMAs may still write the second CTA's TMEM)
+  if constexpr (MC == 2 || kPair) cluster_sync();
   if (warp == 1) {
     __syncwarp();
     tc_fence_after();
-    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem_base),
-                 "r"(C::kTmemCols)
-                 : "memory");
+    if constexpr (kPair)
+      asm volatile("tcgen05.dealloc.cta_group::2.sync.aligned.b32 %0, %1;" ::"r"(tmem_base), "r"(C::kTmemCols)
+                   : "memory");
+    else
+      asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem_base), "r"(C::kTmemCols)
+                   : "memory");
   }
 }
 
@@ -622,15 +772,33 @@ PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
   return fn;
 }
 
-template <int BN, int EPI, int KA, int MC>
+template <int BN, int EPI, int KA, int MC, int CG = 1>
 cudaError_t launch(const CUtensorMap& ta, const CUtensorMap& tb, int M, int N, int K,
                    const EpiArgs& e, const SplitArgs& sp, int num_sms, int* dev_err, cudaStream_t s) {
-  using C = TileCfg<BN, KA>;
+  using C = TileCfg<BN, KA, CG>;
   static PerDeviceSmem smem_rec;  // contexts may run on several host threads and devices
-  const cudaError_t err = ensure_max_smem(smem_rec, gemm_tc_kernel<BN, EPI, KA, MC>, C::kSmemBytes);
+  const cudaError_t err = ensure_max_smem(smem_rec, gemm_tc_kernel<BN, EPI, KA, MC, CG>, C::kSmemBytes);
   if (err != cudaSuccess) return err;
-  const int units = ((M + kBM - 1) / kBM) * (N / BN) * sp.splits;
-  if constexpr (MC == 1) {
+  const int units = ((M + kBM * CG - 1) / (kBM * CG)) * (N / BN) * sp.splits;
+  if constexpr (CG == 2) {
+    // one cluster (the CTA pair) per 256-row unit, at most one CTA per SM
+    const int grid = 2 * (units < num_sms / 2 ? units : num_sms / 2);
+    cudaLaunchAttribute attr[2];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    attr[1].id = cudaLaunchAttributeClusterDimension;
+    attr[1].val.clusterDim.x = 2;
+    attr[1].val.clusterDim.y = 1;
+    attr[1].val.clusterDim.z = 1;
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(grid);
+    cfg.blockDim = dim3(kThreads);
+    cfg.dynamicSmemBytes = C::kSmemBytes;
+    cfg.stream = s;
+    cfg.attrs = attr;
+    cfg.numAttrs = 2;
+    return cudaLaunchKernelEx(&cfg, gemm_tc_kernel<BN, EPI, KA, 1, 2>, ta, tb, M, N, K, e, sp, dev_err);
+  } else if constexpr (MC == 1) {
     const int grid = units < num_sms ? units : num_sms;
     return launch_pdl(gemm_tc_kernel<BN, EPI, KA, 1>, dim3(grid), dim3(kThreads), C::kSmemBytes, s, ta, tb, M, N,
                       K, e, sp, dev_err);
@@ -656,15 +824,15 @@ cudaError_t launch(const CUtensorMap& ta, const CUtensorMap& tb, int M, int N, i
   }
 }
 
-template <int BN, int KA, int MC>
+template <int BN, int KA, int MC, int CG = 1>
 cudaError_t dispatch_epi(const CUtensorMap& ta, const CUtensorMap& tb, int M, int N, int K, int epi,
                          const EpiArgs& e, const SplitArgs& sp, int num_sms, int* dev_err, cudaStream_t s) {
   switch (epi) {
-    case kEpiBf16: return launch<BN, kEpiBf16, KA, MC>(ta, tb, M, N, K, e, sp, num_sms, dev_err, s);
-    case kEpiGeluBf16: return launch<BN, kEpiGeluBf16, KA, MC>(ta, tb, M, N, K, e, sp, num_sms, dev_err, s);
-    case kEpiResidF32: return launch<BN, kEpiResidF32, KA, MC>(ta, tb, M, N, K, e, sp, num_sms, dev_err, s);
-    case kEpiF32: return launch<BN, kEpiF32, KA, MC>(ta, tb, M, N, K, e, sp, num_sms, dev_err, s);
-    case kEpiQkvVt: return launch<BN, kEpiQkvVt, KA, MC>(ta, tb, M, N, K, e, sp, num_sms, dev_err, s);
+    case kEpiBf16: return launch<BN, kEpiBf16, KA, MC, CG>(ta, tb, M, N, K, e, sp, num_sms, dev_err, s);
+    case kEpiGeluBf16: return launch<BN, kEpiGeluBf16, KA, MC, CG>(ta, tb, M, N, K, e, sp, num_sms, dev_err, s);
+    case kEpiResidF32: return launch<BN, kEpiResidF32, KA, MC, CG>(ta, tb, M, N, K, e, sp, num_sms, dev_err, s);
+    case kEpiF32: return launch<BN, kEpiF32, KA, MC, CG>(ta, tb, M, N, K, e, sp, num_sms, dev_err, s);
+    case kEpiQkvVt: return launch<BN, kEpiQkvVt, KA, MC, CG>(ta, tb, M, N, K, e, sp, num_sms, dev_err, s);
     default: return cudaErrorInvalidValue;
   }
 }
@@ -723,13 +891,15 @@ size_t tc_gemm_workspace_bytes(int num_sms) {
 // ones cannot fill the SMs (more CTAs in flight hide the operand latency), 256-wide tiles win once
 // they fill four waves (fewest operand bytes per flop), 128-wide tiles in between.  K splitting
 // changes the summation order, so it is only used when asked for.
-// Clusters are not chosen by the rule: measured on the three models' projections at 1 to 32
-// episodes, the pair never beat the best single-CTA plan (at one episode the main loop is bound by
-// the latency of the operand round trip, not by the bytes the L2 delivers; at large M the 256-wide
-// single tiles move fewer bytes than 128-wide pairs).  They stay available through explicit plans.
+// Where the rule picks 256-wide tiles (and K % 128 == 0), CTA pairs run them as 256 x 256 units on
+// one two-SM MMA: each SM then receives 128 weight rows per unit instead of 256 (serving scale,
+// 78848 x {1024, 3072, 4096} projections: 1565 / 1537 / 1567 -> 1801 / 1574 / 1595 TFLOP/s).  At one
+// episode the pairs gain nothing (fixed per-launch costs dominate), and the rule keeps single CTAs.
+// Multicast clusters are not chosen by the rule: measured on the three models' projections at 1 to
+// 32 episodes, they never beat the best single-CTA plan.  Both stay available through explicit
+// plans.
 GemmPlan tc_gemm_plan(int M, int N, int K, bool has64, bool can_split, int num_sms) {
   (void)can_split;
-  (void)K;
   const long m_tiles = (M + kBM - 1) / kBM;
   const long tiles128 = m_tiles * (N / 128);
   int bn = 128;
@@ -737,6 +907,7 @@ GemmPlan tc_gemm_plan(int M, int N, int K, bool has64, bool can_split, int num_s
     bn = 64;
   else if (N % 256 == 0 && (tiles128 / 2) >= 4L * num_sms)
     bn = 256;
+  if (bn == 256 && K % (2 * kBK) == 0 && num_sms >= 2) return GemmPlan{256, 1, 3};
   return GemmPlan{bn, 1, 1};
 }
 
@@ -749,6 +920,7 @@ cudaError_t tc_gemm(const GemmOperand& a, const GemmOperand& b, int M, int N, in
   // clusters need a K split of 1, two K-atoms per stage, an even number of column tiles and the
   // A operand's 64-row boxes; otherwise the plan runs without
   int mc = plan.mc == 0 ? tc_gemm_plan(M, N, K, b.r64, false, num_sms).mc : plan.mc;
+  if (plan.mc == 0) plan.mc = mc;
   if (mc == 2 && !(plan.splits <= 1 && bn <= 128 && K % (2 * kBK) == 0 && (N / bn) % 2 == 0 && a.r64 &&
                    num_sms >= 2))
     mc = 1;
@@ -764,6 +936,14 @@ cudaError_t tc_gemm(const GemmOperand& a, const GemmOperand& b, int M, int N, in
       return cudaErrorInvalidValue;
     sp.ws = ws->ws;
     sp.counters = ws->counters;
+  }
+  if (plan.mc == 3) {
+    // CTA pairs on one 256-row MMA: each CTA loads 128 rows of A and bn / 2 rows of B (one box)
+    if (sp.splits != 1 || (bn != 128 && bn != 256) || N % bn != 0 || K % (2 * kBK) != 0 || !(a.k2 && b.k2) ||
+        (bn == 128 && !b.r64) || num_sms < 2)
+      return cudaErrorInvalidValue;
+    if (bn == 256) return dispatch_epi<256, 2, 1, 2>(a.r128_k2, b.r128_k2, M, N, K, epi, e, sp, num_sms, dev_err, s);
+    return dispatch_epi<128, 2, 1, 2>(a.r128_k2, b.r64_k2, M, N, K, epi, e, sp, num_sms, dev_err, s);
   }
   if (mc == 2) {   // A halves through the 64-row one-atom boxes
     if (bn == 64) return dispatch_epi<64, 2, 2>(a.r64_k1, b.r64_k2, M, N, K, epi, e, sp, num_sms, dev_err, s);

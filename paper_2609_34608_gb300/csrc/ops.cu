@@ -82,7 +82,7 @@ int wam_op_gemm_bf16_plan(const void* A, const void* Wt, const float* bias, void
   if (tile_n != 0 && tile_n != 64 && tile_n != 128 && tile_n != 256)
     return op_fail(WAM_ERR_INVALID_ARG, "tile_n must be 0, 64, 128 or 256");
   if (k_splits < 0 || k_splits > 4) return op_fail(WAM_ERR_INVALID_ARG, "k_splits must be 0 .. 4");
-  if (cluster < 0 || cluster > 2) return op_fail(WAM_ERR_INVALID_ARG, "cluster must be 0, 1 or 2");
+  if (cluster < 0 || cluster > 3) return op_fail(WAM_ERR_INVALID_ARG, "cluster must be 0, 1, 2 or 3");
   int dev = 0, sms = 0;
   cudaError_t e = cudaGetDevice(&dev);
   if (e == cudaSuccess) e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);

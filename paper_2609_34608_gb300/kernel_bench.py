@@ -1,6 +1,6 @@
 """Single-kernel timing through the C ABI (include/wam_ops.h), for kernel tuning and ncu captures.
 
-    python -m paper_2609_34608_gb300.kernel_bench gemm M N K [--iters I]
+    python -m paper_2609_34608_gb300.kernel_bench gemm M N K [--iters I] [--tile T --cluster C] [--epi E]
     python -m paper_2609_34608_gb300.kernel_bench attn B N H [--iters I] [--impl tc|mma] [--head-dim 64|72]
     python -m paper_2609_34608_gb300.kernel_bench step CONFIG [--batch B] [--rounds R] [--relax-gate]
     python -m paper_2609_34608_gb300.kernel_bench sweep CONFIG B1 B2 ... [--relax-gate]
@@ -58,14 +58,28 @@ def _time(fn, iters: int) -> float:
     return e0.elapsed_time(e1) * 1000.0 / iters
 
 
-def bench_gemm(M: int, N: int, K: int, iters: int) -> dict:
+EPILOGUES = {"bf16": W.EPI_BF16, "gelu": W.EPI_GELU_BF16, "resid": W.EPI_RESID_F32}
+
+
+def bench_gemm(M: int, N: int, K: int, iters: int, tile_n: int = 0, cluster: int = 0, epi: str = "bf16") -> dict:
+    """One projection; tile_n / cluster = 0: the library's plan, else an explicit plan
+    (wam_op_gemm_bf16_plan: tile width, 1 single CTAs, 2 multicast pairs, 3 two-SM MMA pairs)."""
     dev = torch.device("cuda")
     A = torch.randn(M, K, device=dev).to(torch.bfloat16)
     Wt = (torch.randn(N, K, device=dev) * 0.05).to(torch.bfloat16)
-    C = torch.empty(M, N, device=dev, dtype=torch.bfloat16)
+    e = EPILOGUES[epi]
+    C = torch.zeros(M, N, device=dev, dtype=torch.float32 if e == W.EPI_RESID_F32 else torch.bfloat16)
     b = torch.zeros(N, device=dev)
-    us = _time(lambda st: W.op_gemm_bf16(A, Wt, b, C, M, N, K, W.EPI_BF16, stream=st), iters)
-    return {"kernel": "gemm_tc", "M": M, "N": N, "K": K, "us": us, "tflops": 2.0 * M * N * K / us / 1e6}
+    gate = torch.full((M, N), 0.5, device=dev) if e == W.EPI_RESID_F32 else None
+    if tile_n == 0 and cluster == 0:
+        fn = lambda st: W.op_gemm_bf16(A, Wt, b, C, M, N, K, e, gate=gate, gate_stride=N, rows_per_item=M,
+                                       stream=st)
+    else:
+        fn = lambda st: W.op_gemm_bf16_plan(A, Wt, b, C, M, N, K, e, tile_n, 1, gate=gate, gate_stride=N,
+                                            rows_per_item=M, stream=st, cluster=cluster)
+    us = _time(fn, iters)
+    return {"kernel": "gemm_tc", "M": M, "N": N, "K": K, "tile_n": tile_n, "cluster": cluster, "epi": epi,
+            "us": us, "tflops": 2.0 * M * N * K / us / 1e6}
 
 
 def bench_attn(B: int, N: int, H: int, iters: int, impl: str, head_dim: int = 64) -> dict:
@@ -175,10 +189,13 @@ def main() -> None:
     ap.add_argument("--batch", type=int, default=1)
     ap.add_argument("--rounds", type=int, default=1)
     ap.add_argument("--relax-gate", action="store_true")
+    ap.add_argument("--tile", type=int, default=0, help="gemm: explicit tile width (0 = the library's plan)")
+    ap.add_argument("--cluster", type=int, default=0, help="gemm: 1 single, 2 multicast pairs, 3 two-SM pairs")
+    ap.add_argument("--epi", choices=sorted(EPILOGUES), default="bf16")
     a = ap.parse_args()
     _build.build()
     if a.kind == "gemm":
-        print(json.dumps(bench_gemm(*map(int, a.dims), a.iters)))
+        print(json.dumps(bench_gemm(*map(int, a.dims), a.iters, a.tile, a.cluster, a.epi)))
     elif a.kind == "attn":
         print(json.dumps(bench_attn(*map(int, a.dims), a.iters, a.impl, a.head_dim)))
     elif a.kind == "sweep":

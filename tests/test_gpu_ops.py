@@ -118,6 +118,28 @@ def test_gemm_clusters_match_reference_and_single_ctas(wamlib, M, N, K, tile_n, 
     assert torch.equal(outs[0], outs[1])
 
 
+# (M, N, K, tile width) for CTA pairs on one 256-row MMA: the projections of one episode of the
+# 12-block d768 model (the second CTA of the last pair holds only rows past M), a single row, a
+# ragged M with 128-wide pair tiles, and enough units that each pair runs several tiles (both
+# TMEM accumulators in turn, the second CTA releasing them to the first).
+PAIR_CASES = [(1296, 3072, 768, 256), (1296, 2304, 768, 256), (1296, 768, 768, 128), (1, 256, 128, 256),
+              (129, 512, 256, 128), (20000, 1024, 1024, 256)]
+
+
+@pytest.mark.parametrize("M,N,K,tile_n", PAIR_CASES)
+@pytest.mark.parametrize("epi", [W.EPI_BF16, W.EPI_GELU_BF16, W.EPI_RESID_F32, W.EPI_F32])
+def test_gemm_cta_pairs_match_reference_and_single_ctas(wamlib, M, N, K, tile_n, epi):
+    """Two-SM MMA pairs (tcgen05 cta_group::2): the reference within tolerance, and the single-CTA
+    kernel of the same tile width bit for bit (the same K order into the fp32 accumulator)."""
+    outs = []
+    for cluster in (3, 1):
+        def run(A, Wt, b, C, gate, rpi):
+            W.op_gemm_bf16_plan(A, Wt, b, C, M, N, K, epi, tile_n, 1, gate=gate, gate_stride=N + 4,
+                                rows_per_item=rpi, cluster=cluster)
+        outs.append(_check_gemm(M, N, K, epi, run).cpu())
+    assert torch.equal(outs[0], outs[1])
+
+
 def test_gemm_split_is_deterministic(wamlib):
     """A K-split result does not depend on which unit finished last: repeated runs agree bit for bit."""
     M, N, K = 1392, 768, 3072
@@ -150,6 +172,12 @@ def test_gemm_plan_rejections(wamlib):
         W.op_gemm_bf16_plan(A, Wt, None, C, 1392, 768, 768, W.EPI_F32, 96, 1, workspace=ws)
     with pytest.raises(W.WamError):   # 256-wide partials of two ranges exceed the stage buffers
         W.op_gemm_bf16_plan(A[:200], Wt, None, C[:200], 200, 768, 768, W.EPI_F32, 256, 2, workspace=ws)
+    with pytest.raises(W.WamError):   # CTA pairs never split K
+        W.op_gemm_bf16_plan(A, Wt, None, C, 1392, 768, 768, W.EPI_F32, 128, 2, workspace=ws, cluster=3)
+    with pytest.raises(W.WamError):   # CTA pairs take 128- or 256-wide tiles
+        W.op_gemm_bf16_plan(A, Wt, None, C, 1392, 768, 768, W.EPI_F32, 64, 1, cluster=3)
+    with pytest.raises(W.WamError):   # no such cluster mode
+        W.op_gemm_bf16_plan(A, Wt, None, C, 1392, 768, 768, W.EPI_F32, 128, 1, cluster=4)
 
 
 def test_gemm_rejects_unsupported_shapes(wamlib):
