@@ -149,6 +149,19 @@ WAM_DEV void two_sum(float a, float b, float& s, float& e) {
   e = (a - (s - bb)) + (b - bb);
 }
 
+// x_b + g (x_r - x_b) for a float64 gain g given as gh = float(g), gl = float(g - gh): the
+// difference split exactly by two_sum, the product's rounding error recovered by fma, one final
+// rounding.  Within one float32 ulp of the float64 evaluation (Eq. 2's remap), on the float32 pipe.
+WAM_DEV float df_remap(float xr, float xb, float gh, float gl) {
+  float dh, dl;
+  two_sum(xr, -xb, dh, dl);
+  const float ph = __fmul_rn(gh, dh);   // never contracted into the sum below
+  const float pl = fmaf(gh, dl, fmaf(gl, dh, fmaf(gh, dh, -ph)));
+  float sh, se;
+  two_sum(xb, ph, sh, se);
+  return sh + (se + pl);
+}
+
 // (hi, lo) += v^2 for v = x - y, with x - y itself split exactly into vh + vl.
 WAM_DEV void df_add_sq_diff(float x, float y, float& hi, float& lo) {
   float vh, vl;

@@ -71,15 +71,16 @@ __global__ void __launch_bounds__(256) tr_static_partial_kernel(const float* __r
   }
 }
 
-// Remapped init: retained slots get x_bar + sigma_b0 * unit-RMS direction, computed as one
-// fused multiply-add with the branch gain sigma_b0 / (sigma_r rms) (the same float64 operations
-// as the remap of wam_adapt_state); the action slots move by the executed shift and the slots
-// left uncovered (and, in video mode 1, every video slot) get sigma_b0 * eps.
+// Remapped init: retained slots get x_bar + sigma_b0 * unit-RMS direction, computed as
+// x_bar + g (x_r - x_bar) with the branch gain g = sigma_b0 / (sigma_r rms) in double-float
+// arithmetic (the same operations as the remap of wam_adapt_state); the action slots move by the
+// executed shift and the slots left uncovered (and, in video mode 1, every video slot) get
+// sigma_b0 * eps.
 __global__ void __launch_bounds__(256) tr_static_apply_kernel(
     const float* __restrict__ x_bar, const float* __restrict__ x_r, const float* __restrict__ eps,
     float* __restrict__ out, int T, int V, int Na, int ad, int shift, double sigma_r,
     double sigma_b0, int normalize, int video_mode, int nch, const double* __restrict__ partial) {
-  __shared__ double gain[2];
+  __shared__ float gain_hi[2], gain_lo[2];
   const int b = blockIdx.y;
   if (threadIdx.x < 2) {
     double s = 0.0;
@@ -87,7 +88,9 @@ __global__ void __launch_bounds__(256) tr_static_apply_kernel(
     const double ms = s / (threadIdx.x == 0 ? V : T - V);
     const double rms = normalize ? sqrt(ms) : 1.0;
     const bool zero = normalize && !(ms > 0.0);
-    gain[threadIdx.x] = zero ? 0.0 : sigma_b0 / (sigma_r * rms);
+    const double gain = zero ? 0.0 : sigma_b0 / (sigma_r * rms);
+    gain_hi[threadIdx.x] = static_cast<float>(gain);
+    gain_lo[threadIdx.x] = static_cast<float>(gain - static_cast<double>(gain_hi[threadIdx.x]));
   }
   __syncthreads();
   const int64_t bo = static_cast<int64_t>(b) * T;
@@ -103,8 +106,7 @@ __global__ void __launch_bounds__(256) tr_static_apply_kernel(
     }
     float val;
     if (src >= 0) {
-      const double xbs = static_cast<double>(x_bar[bo + src]);
-      val = static_cast<float>(fma(gain[br], static_cast<double>(x_r[bo + src]) - xbs, xbs));
+      val = df_remap(x_r[bo + src], x_bar[bo + src], gain_hi[br], gain_lo[br]);
     } else {
       val = static_cast<float>(sigma_b0 * static_cast<double>(eps[bo + j]));
     }

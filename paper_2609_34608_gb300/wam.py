@@ -341,7 +341,7 @@ class Context:
         self._check(lib().wam_set_device_branching(self.handle, 1 if enable else 0))
 
     def set_layer_fusion(self, enable: bool):
-        """Fused row-chain launches between attentions (default on); off launches each kernel."""
+        """Fused row-chain launches between attentions (default off); off launches each kernel."""
         self._check(lib().wam_set_layer_fusion(self.handle, 1 if enable else 0))
 
     def gemm_tile_width(self, M: int, N: int, K: int, epilogue: int) -> int:
