@@ -61,7 +61,11 @@ template <> struct WVec<float> {
   }
 };
 
-template <typename TW, int KB>
+// LPR lanes share one weight row piece of CPB = LPR * CPT columns; with LPR = 16 a warp works on
+// two rows at a time (its half-warps take alternate rows of its K range) and a block covers half as
+// many columns, so the bf16 modulation weight spreads over twice as many blocks (at one episode 222
+// blocks of 256 columns filled 1.5 waves of the SMs and left the read latency-bound).
+template <typename TW, int KB, int LPR>
 __global__ void __launch_bounds__(256) cond_gemv_kernel(const float* __restrict__ in_part, int in_splits,
                                                         const float* __restrict__ in_bias, int in_act,
                                                         int features, const StepItem* __restrict__ items,
@@ -71,14 +75,16 @@ __global__ void __launch_bounds__(256) cond_gemv_kernel(const float* __restrict_
   pdl_wait();
   pdl_launch_dependents();
   constexpr int CPT = WVec<TW>::kCPT;
-  constexpr int CPB = 32 * CPT;
+  constexpr int CPB = LPR * CPT;
+  constexpr int HW = 32 / LPR;            // rows a warp works on at a time
   extern __shared__ float smem[];
   float* sx = smem;                       // [KB][kslice]
   float* red = smem + KB * kslice;        // [8][KB][CPB]
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int sub = lane / LPR, lc = lane % LPR;
   const int k_beg = blockIdx.y * kslice;
   const int k_len = max(0, min(K, k_beg + kslice) - k_beg);
-  const int col0 = blockIdx.x * CPB + lane * CPT;
+  const int col0 = blockIdx.x * CPB + lc * CPT;
   const int kw = (k_len + 7) / 8;
   const int kw0 = warp * kw, kw1 = min(k_len, kw0 + kw);
   const int64_t part_stride = static_cast<int64_t>(Bw) * K;
@@ -113,22 +119,22 @@ __global__ void __launch_bounds__(256) cond_gemv_kernel(const float* __restrict_
       // eight weight rows in flight per thread before their first use (the weights stream from
       // HBM once per step; fewer loads in flight left the read latency-bound at one item)
       constexpr int kBatch = 8;
-      int kk = kw0;
-      for (; kk + kBatch <= kw1; kk += kBatch) {
+      int kk = kw0 + sub;
+      for (; kk + HW * (kBatch - 1) < kw1; kk += HW * kBatch) {
         float w[kBatch][CPT];
 #pragma unroll
-        for (int u = 0; u < kBatch; ++u) WVec<TW>::load(W, static_cast<int64_t>(k_beg + kk + u) * Nout + col0, w[u]);
+        for (int u = 0; u < kBatch; ++u) WVec<TW>::load(W, static_cast<int64_t>(k_beg + kk + HW * u) * Nout + col0, w[u]);
 #pragma unroll
         for (int u = 0; u < kBatch; ++u) {
 #pragma unroll
           for (int bi = 0; bi < KB; ++bi) {
-            const float xv = sx[bi * kslice + kk + u];
+            const float xv = sx[bi * kslice + kk + HW * u];
 #pragma unroll
             for (int c = 0; c < CPT; ++c) acc[bi][c] = fmaf(xv, w[u][c], acc[bi][c]);
           }
         }
       }
-      for (; kk < kw1; ++kk) {
+      for (; kk < kw1; kk += HW) {
         float w[CPT];
         WVec<TW>::load(W, static_cast<int64_t>(k_beg + kk) * Nout + col0, w);
 #pragma unroll
@@ -139,10 +145,18 @@ __global__ void __launch_bounds__(256) cond_gemv_kernel(const float* __restrict_
         }
       }
     }
+    if constexpr (HW == 2) {   // the half-warps' alternate rows, combined in a fixed order
 #pragma unroll
-    for (int bi = 0; bi < KB; ++bi)
+      for (int bi = 0; bi < KB; ++bi)
 #pragma unroll
-      for (int c = 0; c < CPT; ++c) red[(warp * KB + bi) * CPB + lane * CPT + c] = acc[bi][c];
+        for (int c = 0; c < CPT; ++c) acc[bi][c] += __shfl_xor_sync(0xffffffffu, acc[bi][c], 16);
+    }
+    if (sub == 0) {
+#pragma unroll
+      for (int bi = 0; bi < KB; ++bi)
+#pragma unroll
+        for (int c = 0; c < CPT; ++c) red[(warp * KB + bi) * CPB + lc * CPT + c] = acc[bi][c];
+    }
     __syncthreads();
     for (int i = threadIdx.x; i < nb * CPB; i += 256) {
       const int bi = i / CPB, cc = i - bi * CPB;
@@ -1134,17 +1148,18 @@ __global__ void copy2d_kernel(const float* __restrict__ in, int64_t spitch, TO* 
 
 template <typename TW, int KB>
 cudaError_t gemv_launch(const CondGemv& g, cudaStream_t s) {
-  constexpr int CPB = 32 * WVec<TW>::kCPT;
+  constexpr int LPR = sizeof(TW) == 2 ? 16 : 32;   // the bf16 modulation weight: half-warp rows
+  constexpr int CPB = LPR * WVec<TW>::kCPT;
   const int kslice = (g.K + g.splits - 1) / g.splits;
   const size_t smem = sizeof(float) * (static_cast<size_t>(KB) * kslice + 8 * KB * CPB);
   if (smem > 200 * 1024) return cudaErrorInvalidValue;
   // The limit only ever grows (per device): contexts on other host threads launch the same kernel
   // with other sizes, and lowering it between their set and their launch would fail that launch.
   static PerDeviceSmem smem_rec;
-  cudaError_t e = ensure_max_smem(smem_rec, cond_gemv_kernel<TW, KB>, static_cast<int>(smem));
+  cudaError_t e = ensure_max_smem(smem_rec, cond_gemv_kernel<TW, KB, LPR>, static_cast<int>(smem));
   if (e != cudaSuccess) return e;
   dim3 grid((g.Nout + CPB - 1) / CPB, g.splits);
-  launch_pdl(cond_gemv_kernel<TW, KB>, dim3(grid), dim3(256), smem, s, g.in_part, g.in_splits, g.in_bias, g.in_act, g.features,
+  launch_pdl(cond_gemv_kernel<TW, KB, LPR>, dim3(grid), dim3(256), smem, s, g.in_part, g.in_splits, g.in_bias, g.in_act, g.features,
                                                    g.items, static_cast<const TW*>(g.W), g.K, g.Nout, g.Bw,
                                                    kslice, g.out, g.out_bias);
   return cudaGetLastError();
