@@ -225,15 +225,16 @@ template <> struct Act<bf16> {
 // ---- GEMM epilogue description (shared by the tensor-core and SIMT GEMMs) ---------------
 enum EpiMode { kEpiBf16 = 0, kEpiGeluBf16 = 1, kEpiResidF32 = 2, kEpiF32 = 3, kEpiQkvVt = 4 };
 
+// Every field has a default, so an EpiArgs that names only what its epilogue uses is complete.
 struct EpiArgs {
-  const float* bias;     // [N] or null
-  void* C;               // output (bf16 or f32, row-major, leading dim N)
-  const float* gate;     // RESID: gate rows
-  int64_t gate_stride;   // floats between gate rows of consecutive items
-  int rows_per_item;     // rows of one item (tokens of one episode)
-  const int* item_map;   // nullable: gate row of local item i = item_map[i]
-  bf16* vt;              // QKV_VT: V^T destination [items * heads * 64, vt_ld]
-  int vt_ld;             // QKV_VT: padded token count (row length of V^T)
+  const float* bias = nullptr;    // [N] or null
+  void* C = nullptr;              // output (bf16 or f32, row-major, leading dim N)
+  const float* gate = nullptr;    // RESID: gate rows
+  int64_t gate_stride = 0;        // floats between gate rows of consecutive items
+  int rows_per_item = 1;          // rows of one item (tokens of one episode)
+  const int* item_map = nullptr;  // nullable: gate row of local item i = item_map[i]
+  bf16* vt = nullptr;             // QKV_VT: V^T destination [items * heads * 64, vt_ld]
+  int vt_ld = 0;                  // QKV_VT: padded token count (row length of V^T)
 };
 
 // ---- internal interfaces -----------------------------------------------------------------
