@@ -43,7 +43,7 @@ struct LayerW {
   float* out_b = nullptr;
   float* up_b = nullptr;
   float* down_b = nullptr;
-  GemmOperand tm_qkv, tm_out, tm_up, tm_down;   // out / down also with 64-row boxes
+  GemmOperand tm_qkv, tm_out, tm_up, tm_down;   // also with 64-row boxes
 };
 
 struct ProfSpan {
@@ -1204,9 +1204,10 @@ int create_impl(wam_ctx* c, const wam_config* cfg, const float* weights, size_t 
       CK(cudaMemsetAsync(c->d_chain_ctr, 0, sizeof(int) * nctr, c->stream));
     }
     for (LayerW& w : c->layers) {
-      TRY(encode(c, &w.tm_qkv, w.qkv_wt, 3 * c->d, c->d));
+      // every weight also with 64-row boxes: 64-wide tiles and the B halves of 128-wide CTA pairs
+      TRY(encode(c, &w.tm_qkv, w.qkv_wt, 3 * c->d, c->d, true));
       TRY(encode(c, &w.tm_out, w.out_wt, c->d, c->d, true));
-      TRY(encode(c, &w.tm_up, w.up_wt, c->dff, c->d));
+      TRY(encode(c, &w.tm_up, w.up_wt, c->dff, c->d, true));
       TRY(encode(c, &w.tm_down, w.down_wt, c->d, c->dff, true));
     }
   }
@@ -1905,8 +1906,8 @@ int wam_set_layer_fusion(wam_ctx* c, int32_t enable) {
 int wam_gemm_tile_width(const wam_ctx* c, int32_t M, int32_t N, int32_t K, int32_t epilogue) {
   if (c == nullptr || M < 0 || N <= 0 || K <= 0) return WAM_ERR_INVALID_ARG;
   if (!c->bf16) return WAM_ERR_UNSUPPORTED;
-  const bool r64 = epilogue == kEpiResidF32;   // the projections encoded with 64-row boxes
-  return tc_gemm_plan(M, N, K, r64, false, c->num_sms).bn;
+  (void)epilogue;   // every projection's weight has 64-row boxes
+  return tc_gemm_plan(M, N, K, true, false, c->num_sms).bn;
 }
 
 int wam_profile_enable(wam_ctx* c, int32_t enable) try {
