@@ -371,7 +371,8 @@ int wam_set_layer_fusion(wam_ctx* ctx, int32_t enable);
 /*
  * Output tile width (64, 128 or 256 columns) the context's bf16 path uses for the GEMM
  * [M, K] x [K, N] with the given epilogue (WAM_EPI_*, or 4 for the QKV projection that also
- * writes V^T), chosen from the shape alone: 64 while 128-wide tiles cannot fill the SMs, 256 from
+ * writes V^T), chosen from the shape alone: 64 (residual projections, WAM_EPI_RESID_F32) while
+ * 128-wide tiles cannot fill the SMs, 256 from
  * four waves of 256-wide tiles on, else 128.  When K % 128 == 0, 256-wide tiles, and 128-wide
  * tiles that fill four waves, run on CTA pairs sharing one two-SM MMA.  Every width and pairing
  * sums K in the same order, so the choice affects speed only.  Returns WAM_ERR_INVALID_ARG for a

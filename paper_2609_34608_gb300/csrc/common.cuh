@@ -262,7 +262,8 @@ struct SplitWorkspace {
   size_t ws_bytes;
 };
 size_t tc_gemm_workspace_bytes(int num_sms);
-GemmPlan tc_gemm_plan(int M, int N, int K, bool has64, bool can_split, int num_sms);
+// allow64: 64-wide tiles may be chosen; pairs64: the weight has 64-row boxes (128-wide CTA pairs)
+GemmPlan tc_gemm_plan(int M, int N, int K, bool allow64, bool pairs64, int num_sms);
 // ws == nullptr: no K split.  plan.bn == 0: chosen by tc_gemm_plan.
 cudaError_t tc_gemm(const GemmOperand& a, const GemmOperand& b, int M, int N, int K, int epi, const EpiArgs& e,
                     int num_sms, int* dev_err, cudaStream_t s, const SplitWorkspace* ws, GemmPlan plan);

@@ -898,19 +898,18 @@ size_t tc_gemm_workspace_bytes(int num_sms) {
 // Multicast clusters are not chosen by the rule: measured on the three models' projections at 1 to
 // 32 episodes, they never beat the best single-CTA plan.  Both stay available through explicit
 // plans.
-GemmPlan tc_gemm_plan(int M, int N, int K, bool has64, bool can_split, int num_sms) {
-  (void)can_split;
+GemmPlan tc_gemm_plan(int M, int N, int K, bool allow64, bool pairs64, int num_sms) {
   const long m_tiles = (M + kBM - 1) / kBM;
   const long tiles128 = m_tiles * (N / 128);
   int bn = 128;
-  if (has64 && tiles128 < num_sms)
+  if (allow64 && tiles128 < num_sms)
     bn = 64;
   else if (N % 256 == 0 && (tiles128 / 2) >= 4L * num_sms)
     bn = 256;
   if (bn == 256 && K % (2 * kBK) == 0 && num_sms >= 2) return GemmPlan{256, 1, 3};
   // 128-wide tiles over many waves (N not a multiple of 256, e.g. the d1152 model's QKV and
   // MLP down-projection at 8 episodes: 1226 / 1214 -> 1294 / 1386 TFLOP/s) run as pairs too
-  if (bn == 128 && has64 && K % (2 * kBK) == 0 && tiles128 >= 4L * num_sms && num_sms >= 2) return GemmPlan{128, 1, 3};
+  if (bn == 128 && pairs64 && K % (2 * kBK) == 0 && tiles128 >= 4L * num_sms && num_sms >= 2) return GemmPlan{128, 1, 3};
   return GemmPlan{bn, 1, 1};
 }
 
@@ -918,11 +917,11 @@ cudaError_t tc_gemm(const GemmOperand& a, const GemmOperand& b, int M, int N, in
                     int num_sms, int* dev_err, cudaStream_t s, const SplitWorkspace* ws, GemmPlan plan) {
   if (M <= 0) return cudaSuccess;
   if (K % kBK != 0 || N % 128 != 0) return cudaErrorInvalidValue;
-  if (plan.bn == 0) plan = tc_gemm_plan(M, N, K, b.r64, ws != nullptr && ws->ws != nullptr, num_sms);
+  if (plan.bn == 0) plan = tc_gemm_plan(M, N, K, b.r64, b.r64, num_sms);
   const int bn = plan.bn;
   // clusters need a K split of 1, two K-atoms per stage, an even number of column tiles and the
   // A operand's 64-row boxes; otherwise the plan runs without
-  int mc = plan.mc == 0 ? tc_gemm_plan(M, N, K, b.r64, false, num_sms).mc : plan.mc;
+  int mc = plan.mc == 0 ? tc_gemm_plan(M, N, K, b.r64, b.r64, num_sms).mc : plan.mc;
   if (plan.mc == 0) plan.mc = mc;
   if (mc == 2 && !(plan.splits <= 1 && bn <= 128 && K % (2 * kBK) == 0 && (N / bn) % 2 == 0 && a.r64 &&
                    num_sms >= 2))

@@ -322,7 +322,7 @@ int gemm(wam_ctx* c, const GemmOperand* ta, const void* A, const GemmOperand* tb
   Span sp(c, WAM_KCLASS_GEMM, 2.0 * M * N * K, in_b * (double(M) * K + double(N) * K) + out_b * double(M) * N);
   if (c->bf16) {
     CK(tc_gemm(*ta, *tb, M, N, K, epi, e, c->num_sms, c->d_err, c->stream, nullptr,
-               tc_gemm_plan(M, N, K, tb->r64, false, c->num_sms)));
+               tc_gemm_plan(M, N, K, epi == kEpiResidF32, tb->r64, c->num_sms)));
   } else {
     CK(simt_gemm(static_cast<const float*>(A), static_cast<const float*>(Wt), M, N, K, epi, e, c->stream));
   }
@@ -1906,8 +1906,9 @@ int wam_set_layer_fusion(wam_ctx* c, int32_t enable) {
 int wam_gemm_tile_width(const wam_ctx* c, int32_t M, int32_t N, int32_t K, int32_t epilogue) {
   if (c == nullptr || M < 0 || N <= 0 || K <= 0) return WAM_ERR_INVALID_ARG;
   if (!c->bf16) return WAM_ERR_UNSUPPORTED;
-  (void)epilogue;   // every projection's weight has 64-row boxes
-  return tc_gemm_plan(M, N, K, true, false, c->num_sms).bn;
+  // 64-wide tiles for the residual projections (measured faster there at small M), 64-row weight
+  // boxes for every projection (128-wide CTA pairs)
+  return tc_gemm_plan(M, N, K, epilogue == kEpiResidF32, true, c->num_sms).bn;
 }
 
 int wam_profile_enable(wam_ctx* c, int32_t enable) try {
