@@ -19,6 +19,16 @@
 // The accumulator is double buffered in TMEM (2 x BN columns) so the epilogue of one tile
 // overlaps the main loop of the next.
 //
+// CTA pairs (CG = 2, no K split; chosen by the shape rule from four waves of tiles on): a cluster
+// of two CTAs computes a 256-row x BN unit with one tcgen05.mma.cta_group::2 per K step, M = 256.
+// Each CTA loads its 128 rows of A and BN / 2 rows of the weight tile to the same shared-memory
+// offsets, and both CTAs' copies signal the first CTA's full barrier (TMA .cta_group::2), which
+// that CTA arms with the bytes of both.  Only the first CTA issues MMAs; its commits arrive on
+// both CTAs' stage and accumulator barriers by multicast.  Each CTA's epilogue reads its own
+// 128 x BN accumulator, and the second CTA releases it to the MMA thread by a remote arrival.
+// Per output tile an SM thus receives half the weight rows of a single-CTA tile.  The TMEM
+// allocation is collective over the pair.
+//
 // Clusters of two (MC = 2, no K split; explicit plans only): the two CTAs of a cluster take the
 // same 128-row block and adjacent column tiles, so they read the same A tile.  Each loads one
 // 64-row half of it with TMA multicast into both CTAs' shared memory (the L2 serves A once per
