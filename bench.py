@@ -147,15 +147,33 @@ class ClockSampler:
               "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
               "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
 
-    def __init__(self, gpu_index: int):
+    def __init__(self, gpu_index: int, interval_ms: int = 25):
+        """nvidia-smi polling every interval_ms; the timed region of a control-step run lasts tens of
+        milliseconds, so the interval is short and start() waits for the first sample."""
         self.proc = None
         self.path = tempfile.mktemp(suffix=".csv")
         try:
             self.proc = subprocess.Popen(
                 ["nvidia-smi", f"--id={gpu_index}", f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
-                 "-lms", "200"], stdout=open(self.path, "w"), stderr=subprocess.DEVNULL)
+                 "-lms", str(interval_ms)], stdout=open(self.path, "w"), stderr=subprocess.DEVNULL)
         except Exception:
             self.proc = None
+
+    def wait_first_sample(self, timeout_s: float = 5.0) -> bool:
+        """Block until nvidia-smi has written its first sample (it takes a while to start)."""
+        if self.proc is None:
+            return False
+        t0 = time.time()
+        while time.time() - t0 < timeout_s:
+            try:
+                if os.path.getsize(self.path) > 0:
+                    return True
+            except OSError:
+                pass
+            if self.proc.poll() is not None:
+                return False
+            time.sleep(0.005)
+        return False
 
     def stop(self):
         if self.proc is None:
@@ -460,6 +478,7 @@ def main_ours(args):
     ev_s = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps + 1)]
     ev_m = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
     clocks = ClockSampler(local)
+    clocks.wait_first_sample()
     barrier()
     with torch.cuda.stream(stream):
         ev_s[0].record(stream)
