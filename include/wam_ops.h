@@ -66,6 +66,19 @@ int wam_op_gemm_bf16_plan(const void* A, const void* Wt, const float* bias, void
 /* Bytes of the split-K workspace of wam_op_gemm_bf16_plan on the current device. */
 size_t wam_op_gemm_workspace_bytes(void);
 
+/*
+ * The plan the library's shape rule picks for a bf16 projection [M, K] x [K, N] on a GPU with
+ * num_sms SMs (what wam_op_gemm_bf16 and the context's projections run): *tile_n = 64, 128 or 256
+ * output columns per tile, *cta_pairs = 1 when the tiles run on CTA pairs sharing one two-SM MMA.
+ * residual != 0 for a projection whose weight has 64-row boxes and may take 64-wide tiles (the
+ * gated-residual projections of a context; every call of wam_op_gemm_bf16).  Host arithmetic
+ * only: no device is touched, so it answers on a machine without a GPU.
+ * Returns WAM_ERR_INVALID_ARG for M < 1, N or K not multiples of 128 / 64, num_sms < 1 or null
+ * outputs.
+ */
+int wam_op_gemm_plan(int32_t M, int32_t N, int32_t K, int32_t residual, int32_t num_sms, int32_t* tile_n,
+                     int32_t* cta_pairs);
+
 /* Same contraction in float32 SIMT (the library's fp32 precision mode). */
 int wam_op_gemm_f32(const float* A, const float* Wt, const float* bias, float* C, int32_t M,
                     int32_t N, int32_t K, int32_t epilogue, const float* gate,

@@ -69,6 +69,18 @@ size_t wam_op_gemm_workspace_bytes(void) {
   return tc_gemm_workspace_bytes(sms);
 }
 
+int wam_op_gemm_plan(int32_t M, int32_t N, int32_t K, int32_t residual, int32_t num_sms, int32_t* tile_n,
+                     int32_t* cta_pairs) {
+  if (M < 1 || N < 128 || N % 128 != 0 || K < 64 || K % 64 != 0 || num_sms < 1 || tile_n == nullptr ||
+      cta_pairs == nullptr)
+    return op_fail(WAM_ERR_INVALID_ARG, "bad GEMM plan query");
+  // a context's projections: 64-wide tiles for the residual ones, 64-row boxes on every weight
+  const GemmPlan p = tc_gemm_plan(M, N, K, residual != 0, true, num_sms);
+  *tile_n = p.bn;
+  *cta_pairs = p.mc == 3 ? 1 : 0;
+  return WAM_OK;
+}
+
 int wam_op_gemm_bf16_plan(const void* A, const void* Wt, const float* bias, void* C, int32_t M, int32_t N,
                           int32_t K, int32_t epilogue, const float* gate, int64_t gate_stride,
                           int32_t rows_per_item, int32_t tile_n, int32_t k_splits, int32_t cluster,

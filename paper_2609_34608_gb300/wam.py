@@ -130,6 +130,7 @@ def lib() -> ctypes.CDLL:
         "wam_op_gemm_bf16_plan": (ctypes.c_int, [_vp, _vp, _vp, _vp, _i32, _i32, _i32, _i32, _vp, ctypes.c_int64, _i32,
                                                  _i32, _i32, _i32, _vp, ctypes.c_size_t, _vp]),
         "wam_op_gemm_workspace_bytes": (ctypes.c_size_t, []),
+        "wam_op_gemm_plan": (ctypes.c_int, [_i32, _i32, _i32, _i32, _i32, _vp, _vp]),
         "wam_gemm_tile_width": (ctypes.c_int, [_vp, _i32, _i32, _i32, _i32]),
         "wam_set_graph_replay": (ctypes.c_int, [_vp, _i32]),
         "wam_set_layer_fusion": (ctypes.c_int, [_vp, _i32]),
@@ -431,6 +432,13 @@ def op_gemm_bf16_plan(A, Wt, bias, C, M, N, K, epilogue, tile_n, k_splits, works
 
 def gemm_workspace_bytes():
     return int(lib().wam_op_gemm_workspace_bytes())
+
+
+def gemm_plan(M, N, K, residual, num_sms):
+    """The shape rule's plan for a bf16 projection (host only): (tile width, on CTA pairs)."""
+    tn, pairs = _i32(), _i32()
+    _op_check(lib().wam_op_gemm_plan(M, N, K, 1 if residual else 0, num_sms, ctypes.byref(tn), ctypes.byref(pairs)))
+    return tn.value, bool(pairs.value)
 
 
 def op_gemm_f32(A, Wt, bias, C, M, N, K, epilogue, gate=None, gate_stride=0, rows_per_item=1, stream=None):

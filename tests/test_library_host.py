@@ -76,3 +76,38 @@ def test_every_header_function_has_a_binding_signature(lib):
     for name in W.header_functions():
         fn = getattr(lib, name)
         assert fn.argtypes is not None, name
+
+
+# (rows, N, K, residual) -> (tile width, CTA pairs) on the 152 SMs of a GB300: the plans the shape
+# rule gives the three models' projections.  One episode of the d768 model stays on single CTAs
+# (its launches are bound by fixed costs); 32 serving episodes run 256-wide pairs; at 8 bimanual
+# episodes N = 3456 / 1152 rule out 256-wide tiles, so the 128-wide tiles that fill four waves pair.
+GEMM_PLANS = [
+    ((1296, 768, 768, True), (64, False)),      # one episode: attention out-projection
+    ((1296, 3072, 768, False), (128, False)),   # MLP up
+    ((1296, 768, 3072, True), (64, False)),     # MLP down
+    ((1296, 2304, 768, False), (128, False)),   # QKV
+    ((78848, 3072, 1024, False), (256, True)),  # 32 serving episodes: QKV
+    ((78848, 4096, 1024, False), (256, True)),  # MLP up
+    ((78848, 1024, 4096, True), (256, True)),   # MLP down
+    ((39312, 3456, 1152, False), (128, True)),  # 8 bimanual episodes: QKV
+    ((39312, 1152, 4608, True), (128, True)),   # MLP down
+    ((39312, 4608, 1152, False), (256, True)),  # MLP up
+    ((272, 2304, 768, False), (128, False)),    # a small non-residual projection keeps 128-wide tiles
+    ((272, 768, 768, True), (64, False)),       # ... and a small residual one takes 64-wide tiles
+    ((78848, 1024, 192, False), (256, False)),  # K % 128 != 0: no pairs
+]
+
+
+@pytest.mark.parametrize("shape,plan", GEMM_PLANS)
+def test_gemm_shape_rule(lib, shape, plan):
+    M, N, K, resid = shape
+    tile, pairs = W.gemm_plan(M, N, K, resid, 152)
+    assert (tile, pairs) == plan
+    assert N % tile == 0
+
+
+def test_gemm_plan_query_rejects_bad_sizes(lib):
+    for bad in ((0, 768, 768), (1296, 100, 768), (1296, 768, 96)):
+        with pytest.raises(W.WamError):
+            W.gemm_plan(*bad, True, 152)
